@@ -1,0 +1,194 @@
+/*
+ * retrace.h — C ABI of libretrace, the GB300 (sm_103a) per-round hot path of
+ * ReTrace: Rejected-Trajectory Conditioning for Speculative Decoding
+ * (arXiv 2608.29748).
+ *
+ * One ReTrace decoding round (Algorithm 1 of the paper) is, on the data path:
+ *
+ *   1. greedy verification of a K-token draft block against the target's
+ *      verify logits (Algorithm 1 "Verify" step; greedy decoding = top-k 1,
+ *      Appendix "Evaluation Protocol"): row-wise argmax, first mismatch,
+ *      accepted length A, committed tokens and the correction/bonus token;
+ *   2. alignment of the rejected suffix (Eq. 3-5) and target-aware
+ *      correction r = m + beta * W_c [m; u]   (Eq. 6-7);
+ *   3. gated residual conditioning of the next block's drafter inputs
+ *      e~ = e + (W_v r) .* sigmoid(W_g [e; r])   (Eq. 8).
+ *
+ * Index conventions (0-based; the paper is 1-based).
+ *   K      draft tokens per block (the paper's block size "B").
+ *   B      number of independent sequences in the batch.
+ *   V      vocabulary size;  d  hidden size (target and drafter share it).
+ *   logits[b, i, :] for i = 0..K is the target's distribution at draft slot i:
+ *          row i scores draft token i, row K scores the bonus position.
+ *   hD[b, k, :]  drafter final-layer state of draft slot k   (paper h^D_{t,k+1}).
+ *   hT[b, k, :]  target final-layer state at the position of draft slot k
+ *                (paper h^T_{t,k+1}); its logits score slot k+1.
+ *   A_b          accepted length, 0..K.  First rejected slot is A_b (paper r_t = A_t+1).
+ *   n_b = max(0, K-1-A_b)   number of carried rows (Eq. 4 range, Algorithm 1 reset rule).
+ *   For j < n_b:  m[b,j] = hD[b, A_b+1+j]  (Eq. 4),  u[b,j] = hT[b, A_b+j]  (Eq. 5).
+ *   Rows j >= n_b carry nothing: m = u = r = 0 and e~[b,j] = e[b,j].
+ *   e[b, j, :] for j = 0..K-1 are the drafter inputs of the K proposal positions
+ *   (paper positions 1..K); the anchor (paper position 0) is never modified.
+ *
+ * Weight layout follows y = W x as the equations write it (row-major [out, in]):
+ *   W_c [d, 2d]  columns 0..d-1 act on m, d..2d-1 on u              (Eq. 6)
+ *   W_v [d, d]                                                     (Eq. 8)
+ *   W_g [d, 2d]  columns 0..d-1 act on e, d..2d-1 on r              (Eq. 8)
+ *   No biases: the equations have none.
+ *
+ * Precision.  RETRACE_BF16: every floating tensor (logits, hD, hT, e, weights,
+ * r, e~) is bfloat16; products accumulate in fp32; r is rounded once to bf16
+ * (round-to-nearest-even) before the gate projection; the gate, sigmoid and
+ * residual run in fp32; e~ is rounded once to bf16.  RETRACE_F32: fp32
+ * everywhere, plain FFMA accumulation (no TF32).
+ *
+ * Conventions common to every entry point.
+ *   Ownership   every pointer is caller-owned DEVICE memory unless stated; the
+ *               library allocates no device memory.  Scratch comes from the
+ *               caller's workspace `ws` (size from retrace_workspace_bytes).
+ *   Layout      row-major, last dimension contiguous.  16-byte alignment of
+ *               every tensor base enables the vector paths; unaligned inputs
+ *               take a scalar path on the GPU.  Outputs must not overlap inputs.
+ *   Async       all work is enqueued on `stream` (NULL = legacy default stream);
+ *               no entry point synchronises the host except
+ *               retrace_workspace_check.
+ *   Workspace   `ws` must be zeroed once by retrace_workspace_init before its
+ *               first use.  Every successful call leaves the workspace ready for
+ *               the next call.  Calls sharing one workspace must be ordered on
+ *               one stream (or otherwise serialised); after an error status,
+ *               call retrace_workspace_init again.
+ *   Errors      arguments are checked on the host before anything is enqueued;
+ *               a bad argument returns a status and enqueues nothing.  A CUDA
+ *               launch error returns RETRACE_ERR_CUDA.  Kernels never trap: a
+ *               device-side wait that exceeds its bound sets a flag in `ws`
+ *               that retrace_workspace_check reports.  retrace_last_error()
+ *               gives a thread-local message for the last failing call.
+ *   Semantics   NaN logits are outside the contract (result unspecified).  A
+ *               draft token outside [0, V) never matches, so the block is
+ *               rejected there.  Ties in the argmax resolve to the lowest
+ *               vocabulary index; -0 and +0 compare equal.
+ */
+#ifndef RETRACE_H_
+#define RETRACE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  RETRACE_OK = 0,
+  RETRACE_ERR_INVALID_ARG = 1, /* null pointer, negative size, bad stride        */
+  RETRACE_ERR_UNSUPPORTED = 2, /* valid but not implemented (e.g. strided e)    */
+  RETRACE_ERR_WORKSPACE = 3,   /* ws missing, misaligned or smaller than needed  */
+  RETRACE_ERR_CUDA = 4,        /* a CUDA runtime call or launch failed           */
+  RETRACE_ERR_DEVICE = 5       /* a kernel reported a bounded-wait expiry        */
+} retrace_status;
+
+typedef enum { RETRACE_F32 = 0, RETRACE_BF16 = 1 } retrace_dtype;
+
+/* Thread-local, NUL-terminated description of the last non-OK status returned
+ * on this thread ("" if none).  Owned by the library; valid until the next call
+ * on the same thread. */
+const char* retrace_last_error(void);
+
+/* Library version string, e.g. "retrace 0.1.0 sm_103a". */
+const char* retrace_version(void);
+
+/* Bytes of workspace that every entry point below needs for a batch of this
+ * shape (one size covers verify, align_refine, gate_fuse and round).  Pure host
+ * arithmetic; returns 0 for invalid shapes (negative sizes or V < 1). */
+size_t retrace_workspace_bytes(int B, int K, int V, int d, retrace_dtype dtype);
+
+/* Zero `ws_bytes` bytes of the workspace on `stream` (cudaMemsetAsync).  Must
+ * precede the first use of a workspace and follow any non-OK status. */
+retrace_status retrace_workspace_init(void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* Synchronises `stream`, then reads the device status word of `ws` into
+ * *device_flags (0 = no kernel reported a problem; bit 0 = a bounded wait in a
+ * tensor-core kernel expired).  Returns RETRACE_ERR_DEVICE if any bit is set. */
+retrace_status retrace_workspace_check(const void* ws, size_t ws_bytes,
+                                       uint32_t* device_flags, cudaStream_t stream);
+
+/* Greedy verification of one draft block per sequence (Algorithm 1, Verify and
+ * commit steps; greedy = top_k 1).
+ *   logits        [B, K+1, V] of `dtype`; element (b,i,v) at
+ *                 b*logits_batch_stride + i*logits_row_stride + v (elements).
+ *                 Requires logits_row_stride >= V and
+ *                 logits_batch_stride >= (K+1)*logits_row_stride.
+ *   draft         [B, K] int32 draft tokens.
+ *   accept_len    [B] int32 out: A_b = first i < K with argmax(logits[b,i]) !=
+ *                 draft[b,i], else K.
+ *   committed     [B, K+1] int32 out: draft[b, 0..A_b-1], then the correction
+ *                 (A_b < K) or bonus (A_b = K) token argmax(logits[b, A_b]);
+ *                 positions after A_b are -1.
+ *   bonus         [B] int32 out: argmax(logits[b, A_b]) (= committed[b, A_b]).
+ *   target_argmax [B, K+1] int32 out, optional (NULL to skip).
+ * B = 0 is a no-op.  K >= 0, V >= 1. */
+retrace_status retrace_verify(const void* logits, retrace_dtype dtype, int B, int K, int V,
+                              int64_t logits_row_stride, int64_t logits_batch_stride,
+                              const int32_t* draft, int32_t* accept_len, int32_t* committed,
+                              int32_t* bonus, int32_t* target_argmax, void* ws,
+                              size_t ws_bytes, cudaStream_t stream);
+
+/* Rejected-trajectory alignment and target-aware correction (Eq. 3-7,
+ * Algorithm 1 carry/reset steps).
+ *   hD, hT      [B, K, d] of `dtype`, contiguous.
+ *   accept_len  [B] int32 (device), values in [0, K]; values outside are
+ *               clamped to that range.
+ *   Wc          [d, 2d] of `dtype`, row-major.
+ *   beta        correction strength (1.0 at inference; 0 gives the "raw
+ *               conditioning" ablation).
+ *   r_out       [B, K, d] of `dtype` out: r[b,j] = m + beta*W_c[m;u] for
+ *               j < n_b, zero rows for j >= n_b (Eq. 4-5 zero padding).
+ *   n_out       [B] int32 out: n_b = max(0, K-1-A_b).
+ * K >= 1, d >= 1. */
+retrace_status retrace_align_refine(const void* hD, const void* hT, retrace_dtype dtype, int B,
+                                    int K, int d, const int32_t* accept_len, const void* Wc,
+                                    float beta, void* r_out, int32_t* n_out, void* ws,
+                                    size_t ws_bytes, cudaStream_t stream);
+
+/* Gated residual conditioning (Eq. 8).
+ *   e           drafter inputs of the K proposal positions.  Two layouts:
+ *               (e_batch_stride, e_pos_stride) = (0, 0): one vector [d]
+ *               broadcast to every position (the DFlash mask embedding);
+ *               (K*d, d): dense [B, K, d].  Other strides: UNSUPPORTED.
+ *   r, n        [B, K, d] corrected signal and [B] row counts, as produced
+ *               by retrace_align_refine; rows j >= n_b of r are not read.
+ *   Wv [d, d], Wg [d, 2d] of `dtype`.
+ *   e_out       [B, K, d] out: e + (Wv r) .* sigmoid(Wg [e; r]) for j < n_b,
+ *               e bit-exactly for j >= n_b.
+ * K >= 1, d >= 1. */
+retrace_status retrace_gate_fuse(const void* e, int64_t e_batch_stride, int64_t e_pos_stride,
+                                 const void* r, const int32_t* n, const void* Wv, const void* Wg,
+                                 retrace_dtype dtype, int B, int K, int d, void* e_out,
+                                 void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* One full round on one stream: verify, then align/refine and gated fusion of
+ * the rejected suffix into the next block's inputs (Algorithm 1).  Arguments
+ * have the meaning given above; r stays inside `ws` (compacted to the R =
+ * sum_b n_b conditioned rows) and is not returned.  No host synchronisation.
+ *   n_out          [B] int32 out, optional (NULL to skip).
+ *   target_argmax  [B, K+1] int32 out, optional.
+ *   phase_events   optional array of 4 cudaEvent_t recorded on `stream`
+ *                  before verification, after it, after the correction
+ *                  projection and after the gated fusion (NULL to skip).
+ * K >= 1, V >= 1, d >= 1. */
+retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
+                             int64_t logits_batch_stride, const int32_t* draft, const void* hD,
+                             const void* hT, const void* e, int64_t e_batch_stride,
+                             int64_t e_pos_stride, const void* Wc, const void* Wv, const void* Wg,
+                             float beta, retrace_dtype dtype, int B, int K, int V, int d,
+                             int32_t* accept_len, int32_t* committed, int32_t* bonus,
+                             int32_t* target_argmax, int32_t* n_out, void* e_out, void* ws,
+                             size_t ws_bytes, const cudaEvent_t* phase_events,
+                             cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RETRACE_H_ */

@@ -1,0 +1,23 @@
+"""CPU oracle of the ReTrace round (test infrastructure only).
+
+Imported only by the tests, ``__graft_entry__.smoke()`` and the CPU-baseline
+legs of ``bench.py``; the product path never uses it.
+"""
+
+from .retrace_oracle import (  # noqa: F401
+    accepted_length,
+    align,
+    bf16_bits_to_f64,
+    bf16_ulp,
+    carried_rows,
+    commit,
+    conditioned_rows,
+    correct,
+    f64_to_bf16_bits,
+    gate_fuse,
+    retrace_round,
+    round_to_bf16,
+    sigmoid,
+    target_argmax,
+    verify,
+)

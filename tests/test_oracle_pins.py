@@ -1,0 +1,406 @@
+"""Pins of the CPU oracle against facts fixed outside it (no GPU).
+
+Each test checks the oracle against something other than itself: the
+paper's Fig. 3 worked example, brute force on tiny inputs (tests/brute_force.py,
+which takes different routes: a stable sort for the argmax, a search over
+every candidate accepted length, explicit split sums for the projections),
+closed forms (closed gate, zero correction, half-open gate), invariants of
+prefix verification, and an independent bf16 conversion (torch's).
+``test_planted_mistakes_are_caught`` plants plausible mistakes in the oracle
+and checks that these pins fail on each.
+"""
+
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import brute_force as bf
+import oracle
+from oracle import retrace_oracle as orc
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# ---------------------------------------------------------------------------
+# bfloat16 format
+# ---------------------------------------------------------------------------
+
+
+def test_bf16_decode_matches_torch_on_every_pattern():
+    bits = np.arange(1 << 16, dtype=np.uint32).astype(np.uint16)
+    ours = oracle.bf16_bits_to_f64(bits)
+    ref = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).double().numpy()
+    finite = np.isfinite(ref)
+    assert np.array_equal(ours[finite], ref[finite])
+    assert np.array_equal(np.isnan(ours), np.isnan(ref))
+
+
+def test_round_to_bf16_known_values():
+    h = 2.0 ** -8  # half an ulp of bf16 at 1.0
+    cases = [
+        (1.0, 1.0),
+        (1.0 + h, 1.0),  # tie -> even (1.0)
+        (1.0 + 3 * h, 1.0 + 4 * h),  # tie -> even (1 + 2^-6)
+        (1.0 + h + 2.0 ** -30, 1.0 + 2 * h),  # just above the tie -> up
+        (-(1.0 + h), -1.0),
+        (2.0 ** -133, 2.0 ** -133),  # smallest subnormal
+        (2.0 ** -134, 0.0),  # tie between 0 and 2^-133 -> even (0)
+        (3 * 2.0 ** -134, 2.0 ** -132),  # 1.5 quanta -> 2 quanta
+        (255.0 * 2.0 ** 120, 255.0 * 2.0 ** 120),  # largest finite
+        (2.0 ** 128 * (1 - 2.0 ** -9), math.inf),  # tie at the top -> rounds up to overflow
+        (0.0, 0.0),
+    ]
+    for x, want in cases:
+        got = oracle.round_to_bf16(np.array([x]))[0]
+        assert got == want, (x, got, want)
+
+
+def test_round_to_bf16_matches_torch_float32_conversion():
+    # torch rounds binary32 -> bf16 to nearest even; on binary32 inputs the
+    # oracle's float64 rounding must agree exactly.
+    rng = np.random.default_rng(7)
+    x32 = (rng.standard_normal(200_000) * np.exp(rng.uniform(-20, 20, 200_000))).astype(np.float32)
+    ref = torch.from_numpy(x32).to(torch.bfloat16).double().numpy()
+    ours = oracle.round_to_bf16(x32.astype(np.float64))
+    assert np.array_equal(ours, ref)
+
+
+# ---------------------------------------------------------------------------
+# Verification
+# ---------------------------------------------------------------------------
+
+
+def test_argmax_lowest_index_on_ties_brute_force():
+    rng = np.random.default_rng(1)
+    values = np.array([-1.0, -0.0, 0.0, 0.5, 1.0, 1.0])
+    for _ in range(400):
+        K1 = int(rng.integers(1, 5))
+        V = int(rng.integers(1, 40))
+        logits = rng.choice(values, size=(1, K1, V))
+        t = oracle.target_argmax(logits)[0]
+        for i in range(K1):
+            assert t[i] == bf.argmax_by_sort(list(logits[0, i])), (logits[0, i], t[i])
+
+
+def test_argmax_signed_zero_and_all_equal_rows():
+    row = np.array([[[-0.0, 0.0, -0.0, -1.0], [-3.0, -3.0, -3.0, -3.0]]])
+    assert list(oracle.target_argmax(row)[0]) == [0, 0]
+    neg_inf = np.full((1, 1, 5), -np.inf)
+    assert oracle.target_argmax(neg_inf)[0, 0] == 0
+
+
+def test_accept_len_brute_force():
+    rng = np.random.default_rng(2)
+    for _ in range(500):
+        K = int(rng.integers(0, 9))
+        t = rng.integers(0, 3, size=(1, K + 1))
+        draft = rng.integers(0, 3, size=(1, K))
+        assert oracle.accepted_length(t, draft)[0] == bf.accept_len_by_search(list(t[0]), list(draft[0]))
+
+
+def test_verification_invariants():
+    """Rejected tokens are never committed; committed = target-argmax prefix + bonus."""
+    rng = np.random.default_rng(3)
+    for _ in range(300):
+        B, K, V = int(rng.integers(1, 4)), int(rng.integers(1, 8)), int(rng.integers(2, 6))
+        logits = rng.integers(-2, 3, size=(B, K + 1, V)).astype(np.float64)
+        draft = rng.integers(-1, V + 1, size=(B, K))  # includes out-of-range tokens
+        out = oracle.verify(logits, draft)
+        t, A, committed, bonus = out["target_argmax"], out["accept_len"], out["committed"], out["bonus"]
+        for b in range(B):
+            a = int(A[b])
+            assert 0 <= a <= K
+            # committed tokens are exactly the target's choices up to and including slot A
+            assert list(committed[b, : a + 1]) == list(t[b, : a + 1])
+            assert list(committed[b, :a]) == list(draft[b, :a])
+            assert all(x == -1 for x in committed[b, a + 1 :])
+            assert bonus[b] == t[b, a]
+            if a < K:  # the first rejected draft token is not what gets committed there
+                assert committed[b, a] != draft[b, a]
+            # out-of-range draft tokens can never be accepted
+            for i in range(a):
+                assert 0 <= draft[b, i] < V
+
+
+def _fig3():
+    with open(os.path.join(GOLDEN, "fig3_worked_example.json")) as f:
+        fx = json.load(f)
+    vocab = fx["vocab"]
+    tok = {w: i for i, w in enumerate(vocab)}
+    return fx, vocab, tok
+
+
+@pytest.mark.parametrize("unstated_choice", ["<unstated>", "but", ",", "he"])
+def test_fig3_worked_example(unstated_choice):
+    fx, vocab, tok = _fig3()
+    K, V, d = len(fx["draft"]), len(vocab), 3
+    draft = np.array([[tok[w] for w in fx["draft"]]])
+    logits = np.zeros((1, K + 1, V))
+    for i, w in enumerate(fx["target_choice_per_slot"]):
+        logits[0, i, tok[unstated_choice if w == "<unstated>" else w]] = 1.0
+    out = oracle.verify(logits, draft)
+    exp = fx["expected"]
+    A = int(out["accept_len"][0])
+    assert A == exp["accept_len"]
+    assert A + 1 == exp["first_rejected_slot_paper_1based"]
+    assert [vocab[x] for x in out["committed"][0, : A + 1]] == exp["committed"]
+    assert vocab[out["bonus"][0]] == exp["correction_token"]
+    n = oracle.carried_rows(out["accept_len"], K)
+    assert int(n[0]) == exp["carried_rows"]
+    # hD row k encodes the draft token of slot k; the carried rows must be the
+    # states of the rejected suffix "but he", shifted to the block start.
+    hD = np.zeros((1, K, d))
+    for k in range(K):
+        hD[0, k, 0] = draft[0, k]
+    hT = np.zeros((1, K, d))
+    m, _ = oracle.align(hD, hT, out["accept_len"])
+    carried = [vocab[int(m[0, j, 0])] for j in range(int(n[0]))]
+    assert carried == exp["carried_draft_tokens"]
+    assert not m[0, int(n[0]) :].any()
+
+
+def test_reset_rule_and_initial_state():
+    K = 6
+    A = np.array([0, 1, K - 2, K - 1, K])
+    assert list(oracle.carried_rows(A, K)) == [K - 1, K - 2, 1, 0, 0]
+
+
+def test_align_pairs_draft_and_target_states_of_the_same_slot():
+    """u_j is the target state whose logits score the slot that m_j drafted (Eq. 5)."""
+    rng = np.random.default_rng(4)
+    for _ in range(50):
+        B, K, d = 3, int(rng.integers(1, 9)), 2
+        A = rng.integers(0, K + 1, size=B)
+        hD = np.zeros((B, K, d))
+        hT = np.zeros((B, K, d))
+        for k in range(K):
+            hD[:, k, 0] = k + 1  # drafter state of slot k (label = slot + 1)
+            hT[:, k, 0] = k + 2  # target state at slot k scores slot k + 1
+        m, u = oracle.align(hD, hT, A)
+        n = oracle.carried_rows(A, K)
+        for b in range(B):
+            for j in range(K):
+                if j < n[b]:
+                    assert m[b, j, 0] == u[b, j, 0] == A[b] + 1 + j + 1
+                else:
+                    assert m[b, j, 0] == u[b, j, 0] == 0
+
+
+# ---------------------------------------------------------------------------
+# Projections and gate: brute force and closed forms
+# ---------------------------------------------------------------------------
+
+
+def _tiny(rng, B, K, V, d):
+    logits = rng.standard_normal((B, K + 1, V))
+    draft = rng.integers(0, V, size=(B, K))
+    for b in range(B):  # plant an accepted prefix so the suffix is exercised
+        a = int(rng.integers(0, K + 1))
+        for i in range(a):
+            logits[b, i, draft[b, i]] = logits[b, i].max() + 1
+    return dict(
+        logits=logits,
+        draft=draft,
+        hD=rng.standard_normal((B, K, d)),
+        hT=rng.standard_normal((B, K, d)),
+        e=rng.standard_normal((B, K, d)) * 0.1,
+        Wc=rng.standard_normal((d, 2 * d)) / math.sqrt(d),
+        Wv=rng.standard_normal((d, d)) / math.sqrt(d),
+        Wg=rng.standard_normal((d, 2 * d)) / math.sqrt(d),
+        beta=float(rng.uniform(0.25, 1.5)),
+    )
+
+
+def _check_round_against_brute(x, dtype="f32"):
+    out = oracle.retrace_round(
+        x["logits"], x["draft"], x["hD"], x["hT"], x["e"], x["Wc"], x["Wv"], x["Wg"], x["beta"], dtype
+    )
+    B, K = x["draft"].shape
+    rnd = (lambda r: list(oracle.round_to_bf16(np.array(r)))) if dtype == "bf16" else None
+    for b in range(B):
+        ref = bf.round_brute(
+            x["logits"][b].tolist(),
+            x["draft"][b].tolist(),
+            x["hD"][b].tolist(),
+            x["hT"][b].tolist(),
+            x["e"][b].tolist(),
+            x["Wc"].tolist(),
+            x["Wv"].tolist(),
+            x["Wg"].tolist(),
+            x["beta"],
+            rnd=rnd,
+        )
+        assert list(out["target_argmax"][b]) == ref["t"]
+        assert out["accept_len"][b] == ref["A"]
+        assert list(out["committed"][b, : ref["A"] + 1]) == ref["committed"]
+        assert out["bonus"][b] == ref["bonus"]
+        assert out["n"][b] == ref["n"]
+        np.testing.assert_allclose(out["e_tilde"][b], np.array(ref["e_tilde"]), rtol=1e-12, atol=1e-12)
+
+
+def test_round_brute_force_random_tiny_shapes():
+    rng = np.random.default_rng(5)
+    for _ in range(150):
+        B, K, V, d = int(rng.integers(1, 3)), int(rng.integers(1, 9)), int(rng.integers(1, 65)), int(rng.integers(1, 9))
+        _check_round_against_brute(_tiny(rng, B, K, V, d))
+
+
+def test_round_brute_force_bf16_rounding_point():
+    rng = np.random.default_rng(6)
+    for _ in range(40):
+        _check_round_against_brute(_tiny(rng, 2, 5, 16, 6), dtype="bf16")
+
+
+def test_closed_gate_reproduces_mask_input_exactly():
+    """W_v = 0 (the paper's initialisation) gives e~ = e bit-for-bit."""
+    rng = np.random.default_rng(8)
+    x = _tiny(rng, 3, 6, 20, 8)
+    x["Wv"] = np.zeros_like(x["Wv"])
+    out = oracle.retrace_round(**{k: x[k] for k in ("logits", "draft", "hD", "hT", "e", "Wc", "Wv", "Wg", "beta")}, dtype="f32")
+    assert np.array_equal(out["e_tilde"], x["e"])
+
+
+def test_half_open_gate_and_identity_value_projection():
+    """W_g = 0 gives sigmoid = 1/2; with W_v = I and beta = 0: e~ = e + m/2 exactly."""
+    rng = np.random.default_rng(9)
+    B, K, d = 2, 7, 5
+    x = _tiny(rng, B, K, 12, d)
+    x["Wg"] = np.zeros_like(x["Wg"])
+    x["Wv"] = np.eye(d)
+    x["beta"] = 0.0
+    out = oracle.retrace_round(**{k: x[k] for k in ("logits", "draft", "hD", "hT", "e", "Wc", "Wv", "Wg", "beta")}, dtype="f32")
+    A, n = out["accept_len"], out["n"]
+    for b in range(B):
+        for j in range(K):
+            if j < n[b]:
+                want = x["e"][b, j] + 0.5 * x["hD"][b, A[b] + 1 + j]
+            else:
+                want = x["e"][b, j]
+            assert np.array_equal(out["e_tilde"][b, j], want)
+
+
+def test_zero_correction_keeps_the_aligned_draft_state():
+    """W_c = 0 (or beta = 0) gives r = m (Eq. 7)."""
+    rng = np.random.default_rng(10)
+    x = _tiny(rng, 2, 6, 10, 4)
+    A = oracle.verify(x["logits"], x["draft"])["accept_len"]
+    m, u = oracle.align(x["hD"], x["hT"], A)
+    assert np.array_equal(oracle.correct(m, u, np.zeros_like(x["Wc"]), 1.0, False), m)
+    assert np.array_equal(oracle.correct(m, u, x["Wc"], 0.0, False), m)
+
+
+def test_sigmoid_reference_values():
+    z = np.array([0.0, 1.0, -1.0, 40.0, -40.0, -800.0, 800.0])
+    want = np.array([0.5, 1 / (1 + math.exp(-1)), math.exp(-1) / (1 + math.exp(-1)), 1 / (1 + math.exp(-40)),
+                     math.exp(-40) / (1 + math.exp(-40)), 0.0, 1.0])
+    np.testing.assert_allclose(oracle.sigmoid(z), want, rtol=1e-15, atol=0)
+
+
+def test_conditioned_rows_agree_with_full_round():
+    rng = np.random.default_rng(11)
+    x = _tiny(rng, 3, 8, 30, 6)
+    e_vec = x["e"][0, 0]
+    for dtype in ("f32", "bf16"):
+        out = oracle.retrace_round(x["logits"], x["draft"], x["hD"], x["hT"], e_vec, x["Wc"], x["Wv"], x["Wg"], x["beta"], dtype)
+        rows = [(b, j) for b in range(3) for j in range(8)]
+        got = oracle.conditioned_rows(rows, out["accept_len"], x["hD"], x["hT"], e_vec, x["Wc"], x["Wv"], x["Wg"], x["beta"], dtype)
+        full = out["e_tilde_rounded"] if dtype == "bf16" else out["e_tilde"]
+        np.testing.assert_allclose(got, full.reshape(-1, 6), rtol=1e-13, atol=1e-13)
+
+
+# ---------------------------------------------------------------------------
+# Planted mistakes: every one must make at least one pin above fail
+# ---------------------------------------------------------------------------
+
+
+def _pins():
+    return [
+        test_argmax_lowest_index_on_ties_brute_force,
+        test_accept_len_brute_force,
+        lambda: test_fig3_worked_example("<unstated>"),
+        test_reset_rule_and_initial_state,
+        test_align_pairs_draft_and_target_states_of_the_same_slot,
+        test_round_brute_force_random_tiny_shapes,
+        test_closed_gate_reproduces_mask_input_exactly,
+        test_half_open_gate_and_identity_value_projection,
+        test_zero_correction_keeps_the_aligned_draft_state,
+        test_sigmoid_reference_values,
+    ]
+
+
+def _mut_argmax_last(logits):
+    lg = np.asarray(logits, dtype=np.float64)
+    return (lg.shape[-1] - 1 - np.argmax(lg[..., ::-1], axis=-1)).astype(np.int64)
+
+
+def _mut_align_u_shift(hD, hT, A):
+    hD = np.asarray(hD, float)
+    hT = np.asarray(hT, float)
+    B, K, d = hD.shape
+    n = orc.carried_rows(A, K)
+    m = np.zeros_like(hD)
+    u = np.zeros_like(hT)
+    for b in range(B):
+        for j in range(int(n[b])):
+            m[b, j] = hD[b, A[b] + 1 + j]
+            u[b, j] = hT[b, min(A[b] + 1 + j, K - 1)]  # off by one: hT of the drafted slot
+    return m, u
+
+
+def _mut_align_keep_rejected(hD, hT, A):
+    hD = np.asarray(hD, float)
+    hT = np.asarray(hT, float)
+    B, K, d = hD.shape
+    n = orc.carried_rows(A, K)
+    m = np.zeros_like(hD)
+    u = np.zeros_like(hT)
+    for b in range(B):
+        for j in range(int(n[b])):
+            m[b, j] = hD[b, A[b] + j]  # includes the first rejected slot
+            u[b, j] = hT[b, A[b] + j]
+    return m, u
+
+
+MUTATIONS = {
+    "argmax picks the last maximum": ("target_argmax", _mut_argmax_last),
+    "accept length counts all matches": (
+        "accepted_length",
+        lambda t, draft: np.array([int(np.sum(np.asarray(t)[b, : np.asarray(draft).shape[1]] == np.asarray(draft)[b])) for b in range(np.asarray(draft).shape[0])]),
+    ),
+    "carry kept at A = K-1": ("carried_rows", lambda A, K: np.maximum(0, K - np.asarray(A))),
+    "u taken at the drafted slot": ("align", _mut_align_u_shift),
+    "first rejected state carried": ("align", _mut_align_keep_rejected),
+    "beta dropped": ("correct", lambda m, u, Wc, beta, rr: m + np.concatenate([m, u], -1) @ np.asarray(Wc).T),
+    "W_c transposed halves": (
+        "correct",
+        lambda m, u, Wc, beta, rr: m + beta * np.concatenate([u, m], -1) @ np.asarray(Wc).T,
+    ),
+    "gate sign flipped": ("sigmoid", lambda z: 1.0 / (1.0 + np.exp(np.asarray(z, float)))),
+    "W_v transposed": (
+        "gate_fuse",
+        lambda e, r, n, Wv, Wg: orc.__dict__["_orig_gate_fuse"](e, r, n, np.asarray(Wv).T, Wg),
+    ),
+    "gate ignores e": (
+        "gate_fuse",
+        lambda e, r, n, Wv, Wg: orc.__dict__["_orig_gate_fuse"](e, r, n, Wv, np.concatenate([np.zeros_like(np.asarray(Wg)[:, : np.asarray(Wv).shape[0]]), np.asarray(Wg)[:, np.asarray(Wv).shape[0]:]], 1)),
+    ),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_planted_mistakes_are_caught(name, monkeypatch):
+    attr, fn = MUTATIONS[name]
+    monkeypatch.setitem(orc.__dict__, "_orig_gate_fuse", orc.gate_fuse)
+    monkeypatch.setattr(orc, attr, fn)
+    monkeypatch.setattr(oracle, attr, fn, raising=False)
+    caught = 0
+    for pin in _pins():
+        try:
+            pin()
+        except Exception:  # an assertion or a crash: either way the pin notices
+            caught += 1
+    assert caught > 0, f"no pin detects the planted mistake: {name}"
