@@ -1,0 +1,440 @@
+"""Benchmark of one ReTrace round (verify + align/refine + gated fusion) on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config 5]
+
+A step is one retrace_round over one batch of the serving workload (default:
+B=256 sequences, K=16 drafts, V=151936, d=4096, bf16; synthetic seeded
+inputs resident in HBM).  L2 is flushed (256 MB write) before every timed
+step and each step is timed on its stream with CUDA events; `value` is
+rounds/s over the K timed steps, max over ranks.  Under torchrun every rank
+runs its own batch on its own GPU (sequences are independent, so the ranks
+shard the batch dimension with no data-path collective: weak scaling).
+
+Also reported on the same JSON line:
+  roofline      the verification kernel (HBM-bound): algorithmic bytes per launch
+                / its CUDA-event duration, against the measured HBM copy peak;
+  roofline_conditioning   the two projection kernels (tensor-bound) against the
+                measured sustained bf16 peak;
+  e2e           the same metric through the public API with host buffers: the
+                step's inputs copied from pinned host memory and its outputs
+                read back inside the timed region;
+  cpu_baseline  the CPU oracle timed on a bounded sample of the workload
+                (rank 0, N = 1 only);
+  clocks        nvidia-smi samples taken during the timed region.
+`--impl reference` times the CPU oracle itself on this workload (the paper
+has no code to run) and prints the same line with "impl": "reference".
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2608_29748_gb300.workloads import CONFIGS, RoundConfig, make_round_inputs  # noqa: E402
+
+METRIC = "verify+ReTrace rounds/sec at 1 GB300; logits HBM GB/s and % of roofline"
+UNIT = "rounds/s"
+KERNELS_PER_ROUND = 4  # verify, correction GEMM, gate-bias GEMV, gate GEMM
+L2_FLUSH_BYTES = 256 << 20
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (host side; testable with gloo on CPU)
+# ---------------------------------------------------------------------------
+
+
+def dist_env() -> tuple[int, int, int]:
+    """(rank, local_rank, world_size) from the torchrun environment."""
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+def shard_seed(base_seed: int, rank: int) -> int:
+    """Each rank draws its own batch: independent sequences, no shared data."""
+    return base_seed + 7919 * rank
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    if world <= 1:
+        return x
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int) -> None:
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def aggregate_value(rounds_per_rank: int, world: int, seconds_max: float) -> float:
+    """Whole-job rounds/s: rounds of all ranks over the slowest rank's time."""
+    return rounds_per_rank * world / seconds_max
+
+
+# ---------------------------------------------------------------------------
+# measurement helpers
+# ---------------------------------------------------------------------------
+
+
+def load_peaks() -> dict:
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": p["hbm_gbs"], "bf16_tflops": p["bf16_tflops"],
+                "bf16_tflops_sustained": p["bf16_tflops_sustained"], "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms while running."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self) -> dict | None:
+        if not self.path or not os.path.exists(self.path):
+            return None
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, flags in rows for i, f in enumerate(flags) if f.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+def cpu_threads() -> int:
+    for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(var, "").isdigit():
+            return int(os.environ[var])
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:  # pragma: no cover
+        return os.cpu_count() or 1
+
+
+def prepare_oracle_sample(cfg: RoundConfig, sample_B: int, seed: int) -> dict:
+    """Host float64 inputs for `sample_B` sequences drawn like `cfg` (weights at full size)."""
+    from oracle import bf16_bits_to_f64  # test infrastructure: CPU-baseline legs only
+    from paper_2608_29748_gb300.workloads import as_bits_numpy
+
+    sub = RoundConfig(cfg.name + f"-sample{sample_B}", sample_B, cfg.K, cfg.V, cfg.d, cfg.dtype, cfg.logits_std,
+                      cfg.prefix, cfg.prefix_p, cfg.ties, cfg.seed_offset)
+    x = make_round_inputs(sub, device="cpu", seed=seed)
+
+    def f64(t):
+        return bf16_bits_to_f64(as_bits_numpy(t)) if t.dtype == torch.bfloat16 else t.double().numpy()
+
+    host = {k: f64(x[k]) for k in ("logits", "hD", "hT", "e", "Wc", "Wv", "Wg")}
+    host.update(draft=x["draft"].numpy(), beta=x["beta"], dtype=cfg.dtype, B=sample_B)
+    return host
+
+
+def time_oracle(host: dict) -> float:
+    """Seconds the CPU oracle takes for one round over the prepared sample."""
+    from oracle import retrace_round as oracle_round_fn  # test infrastructure: CPU-baseline legs only
+
+    t0 = time.perf_counter()
+    oracle_round_fn(host["logits"], host["draft"], host["hD"], host["hT"], host["e"], host["Wc"], host["Wv"],
+                    host["Wg"], host["beta"], host["dtype"])
+    return time.perf_counter() - t0
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+
+def verify_bytes(cfg: RoundConfig, n: np.ndarray) -> int:
+    """Algorithmic bytes of one verification launch in a fused round."""
+    es = cfg.elem_bytes
+    B, K, V, d = cfg.B, cfg.K, cfg.V, cfg.d
+    logits = B * (K + 1) * V * es
+    tokens_in = B * K * 4
+    tokens_out = B * (K + 1) * 4 + 3 * B * 4  # committed; accept_len, bonus, n
+    copies = int(np.sum(K - n)) * d * es  # unconditioned rows of e~ written
+    return logits + tokens_in + tokens_out + copies
+
+
+def conditioning_flops(cfg: RoundConfig, R: int, dense_e: bool) -> int:
+    d = cfg.d
+    f = 2 * R * (2 * d) * d  # c = W_c [m; u]
+    f += 2 * R * d * (2 * d)  # [v; g_r] = [W_v; W_g,r] r
+    f += 2 * R * d * d if dense_e else 2 * d * d  # W_g,e e (per row, or once for a broadcast e)
+    return f
+
+
+def run_gpu(args) -> dict | None:
+    from paper_2608_29748_gb300 import binding as rt
+
+    rank, local_rank, world = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    cfg = CONFIGS[args.config]
+    peaks = load_peaks()
+
+    x = make_round_inputs(cfg, device=dev, seed=shard_seed(42 + 1000 * cfg.seed_offset, rank))
+    ws = rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype, device=dev)
+    out = rt.RoundBuffers(cfg.B, cfg.K, cfg.d, cfg.torch_dtype, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    for _ in range(args.warmup):
+        rt.run_round(x, ws, out=out)
+    torch.cuda.synchronize(dev)
+
+    steps = args.steps
+    phase = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
+    for evs in phase:
+        for e in evs:
+            e.record(stream)  # materialise the CUDA events before the timed region
+    torch.cuda.synchronize(dev)
+
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local_rank) as clocks:
+        t_wall0 = time.perf_counter()
+        for i in range(steps):
+            flush.fill_(i & 0xFF)  # L2 flush: a 256 MB write between timed steps
+            rt.run_round(x, ws, out=out, phase_events=phase[i])
+        torch.cuda.synchronize(dev)
+        t_wall = time.perf_counter() - t_wall0
+    barrier(world)
+
+    step_ms = [phase[i][0].elapsed_time(phase[i][3]) for i in range(steps)]
+    verify_ms = [phase[i][0].elapsed_time(phase[i][1]) for i in range(steps)]
+    cond_ms = [phase[i][1].elapsed_time(phase[i][3]) for i in range(steps)]
+    round_s = sum(step_ms) / 1e3
+    round_s_max = max_over_ranks(round_s, world, dev)
+    value = aggregate_value(steps, world, round_s_max)
+
+    n = out.n.cpu().numpy().astype(np.int64)
+    R = int(n.sum())
+    vbytes = verify_bytes(cfg, n)
+    v_avg_s = statistics.mean(verify_ms) / 1e3
+    v_gbs = vbytes / v_avg_s / 1e9
+    cflops = conditioning_flops(cfg, R, dense_e=False)
+    c_avg_s = statistics.mean(cond_ms) / 1e3
+    c_tflops = cflops / c_avg_s / 1e12
+    flags = ws.check()
+
+    # ---- end to end through the public API with host buffers ----
+    e2e = run_e2e(rt, cfg, x, ws, dev, min(steps, args.e2e_steps), world)
+
+    line = {
+        "metric": METRIC,
+        "value": round(value, 3),
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(statistics.mean(step_ms), 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16" if cfg.dtype == "bf16" else "f32",
+        "data": "synthetic (seeded; Qwen3-8B / DFlash-b16 shapes, random-init fusion weights)",
+        "config": {
+            "workload": f"{cfg.name}: B={cfg.B} K={cfg.K} V={cfg.V} d={cfg.d} {cfg.dtype}, "
+                        f"prefix {cfg.prefix}({cfg.prefix_p or ''}) capped at K",
+            "B": cfg.B, "K": cfg.K, "V": cfg.V, "d": cfg.d,
+            "conditioned_rows_R": R,
+            "l2": "flushed before every timed step (256 MB write, outside the per-step events)",
+            "parallelism": f"replicas x{world} (batch-sharded, no collective)",
+        },
+        "roofline": {
+            "kernel": "verify_kernel (argmax/compare/commit + copy of unconditioned rows)",
+            "bound": "hbm",
+            "achieved": round(v_gbs, 1),
+            "peak": peaks["hbm_gbs"],
+            "unit": "GB/s",
+            "frac": round(v_gbs / peaks["hbm_gbs"], 4),
+            "peak_source": peaks["source"] + " HBM copy bandwidth",
+            "algorithmic_bytes": vbytes,
+            "avg_launch_us": round(v_avg_s * 1e6, 2),
+            "traffic": None,
+        },
+        "roofline_conditioning": {
+            "kernels": "tc_cond_kernel<0> + gate_bias_kernel + tc_cond_kernel<1>",
+            "bound": "tensor",
+            "achieved": round(c_tflops, 2),
+            "peak": peaks["bf16_tflops_sustained"],
+            "unit": "TFLOP/s",
+            "frac": round(c_tflops / peaks["bf16_tflops_sustained"], 4),
+            "peak_source": peaks["source"] + " sustained bf16 (cuBLAS)",
+            "algorithmic_flops": cflops,
+            "avg_us": round(c_avg_s * 1e6, 2),
+        },
+        "logits_gbs": round(cfg.logits_bytes() / v_avg_s / 1e9, 1),
+        "e2e": e2e,
+        "gpu_launches": KERNELS_PER_ROUND * steps,
+        "wall_s_timed_region": round(t_wall, 4),
+        "device_status_flags": flags,
+        "impl": "ours",
+    }
+    cs = clocks.summary()
+    line["clocks"] = cs
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(cfg, args)
+    return line if rank == 0 else None
+
+
+def run_e2e(rt, cfg, x, ws, dev, steps, world) -> dict:
+    """Rounds/s with the step's inputs in pinned host memory and the outputs read back."""
+    names = ["logits", "draft", "hD", "hT"]
+    host = {k: x[k].cpu().pin_memory() for k in names}
+    dev_in = {k: torch.empty_like(x[k]) for k in names}
+    rest = {k: x[k] for k in ("e", "Wc", "Wv", "Wg", "beta", "cfg")}  # model parameters stay resident
+    out = rt.RoundBuffers(cfg.B, cfg.K, cfg.d, cfg.torch_dtype, device=dev)
+    out_host = {k: torch.empty(getattr(out, k).shape, dtype=getattr(out, k).dtype).pin_memory()
+                for k in ("accept_len", "committed", "bonus", "n", "e_out")}
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        for k in names:
+            dev_in[k].copy_(host[k], non_blocking=True)
+        rt.run_round({**dev_in, **rest}, ws, out=out)
+        for k, h in out_host.items():
+            h.copy_(getattr(out, k), non_blocking=True)
+
+    step()
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for _ in range(steps):
+        step()
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    secs = max_over_ranks(start.elapsed_time(end) / 1e3, world, dev)
+    h2d = sum(h.numel() * h.element_size() for h in host.values())
+    d2h = sum(h.numel() * h.element_size() for h in out_host.values())
+    return {"value": round(aggregate_value(steps, world, secs), 3), "unit": UNIT,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps}
+
+
+def cpu_baseline(cfg: RoundConfig, args) -> dict:
+    host = prepare_oracle_sample(cfg, args.cpu_sample, seed=1234)
+    secs = time_oracle(host)
+    rounds = host["B"] / cfg.B
+    return {"value": round(rounds / secs, 6), "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
+            "sample": f"{host['B']} of {cfg.B} sequences of {cfg.name}, full-size weights; one round of the "
+                      f"sample took {secs:.2f} s, scaled by {host['B']}/{cfg.B} to rounds/s"}
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the CPU oracle on the same workload
+# ---------------------------------------------------------------------------
+
+
+def run_reference(args) -> dict | None:
+    rank, _, world = dist_env()
+    if rank != 0:
+        return None
+    cfg = CONFIGS[args.config]
+    host = prepare_oracle_sample(cfg, args.ref_sample, seed=500)
+    for _ in range(min(args.warmup, 1)):
+        time_oracle(host)
+    total = sum(time_oracle(host) for _ in range(args.steps))
+    value = args.steps * (host["B"] / cfg.B) / total
+    return {
+        "metric": METRIC, "value": round(value, 6), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(1e3 * total / args.steps, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{cfg.name}: B={cfg.B} K={cfg.K} V={cfg.V} d={cfg.d} {cfg.dtype}",
+                   "sample_per_step": f"{args.ref_sample} of {cfg.B} sequences (full-size weights)"},
+        "impl": "reference",
+        "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
+                         "sample": f"{args.ref_sample} of {cfg.B} sequences per step, {args.steps} steps, "
+                                   f"scaled by {args.ref_sample}/{cfg.B} to rounds/s"},
+        "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", type=int, default=5, choices=sorted(CONFIGS))
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-sample", type=int, default=32, help="sequences in the CPU-baseline sample")
+    ap.add_argument("--ref-sample", type=int, default=2, help="sequences per step in the reference arm")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args(argv)
+
+
+def main(argv=None) -> None:
+    args = parse_args(argv)
+    if args.warmup < 3 and args.impl == "ours":
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    line = run_reference(args) if args.impl == "reference" else run_gpu(args)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+    _, _, world = dist_env()
+    if world > 1 and args.impl == "ours":
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

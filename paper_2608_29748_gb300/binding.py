@@ -1,0 +1,216 @@
+"""Thin ctypes binding over libretrace (the C ABI in include/retrace.h).
+
+Argument marshalling only: every step of the round runs in the library's CUDA
+kernels.  Tensors are torch CUDA tensors used as device buffers; the functions
+carry the C entry points' names.  If the library has not been built the
+import fails loudly -- there is no fallback path.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+RETRACE_F32 = 0
+RETRACE_BF16 = 1
+
+_STATUS = {
+    0: "RETRACE_OK",
+    1: "RETRACE_ERR_INVALID_ARG",
+    2: "RETRACE_ERR_UNSUPPORTED",
+    3: "RETRACE_ERR_WORKSPACE",
+    4: "RETRACE_ERR_CUDA",
+    5: "RETRACE_ERR_DEVICE",
+}
+
+
+class RetraceError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{_STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+def _load() -> ctypes.CDLL:
+    path = _build.LIB_PATH
+    if not os.path.exists(path):
+        raise ImportError(
+            f"libretrace.so is not built ({path}); run `python -m paper_2608_29748_gb300.build` "
+            "or __graft_entry__.build() first"
+        )
+    lib = ctypes.CDLL(path)
+    P, I, I64, SZ, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_size_t, ctypes.c_float
+    lib.retrace_last_error.restype = ctypes.c_char_p
+    lib.retrace_version.restype = ctypes.c_char_p
+    lib.retrace_workspace_bytes.argtypes = [I, I, I, I, I]
+    lib.retrace_workspace_bytes.restype = SZ
+    lib.retrace_workspace_init.argtypes = [P, SZ, P]
+    lib.retrace_workspace_check.argtypes = [P, SZ, ctypes.POINTER(ctypes.c_uint32), P]
+    lib.retrace_verify.argtypes = [P, I, I, I, I, I64, I64, P, P, P, P, P, P, SZ, P]
+    lib.retrace_align_refine.argtypes = [P, P, I, I, I, I, P, P, F, P, P, P, SZ, P]
+    lib.retrace_gate_fuse.argtypes = [P, I64, I64, P, P, P, P, I, I, I, I, P, P, SZ, P]
+    lib.retrace_round.argtypes = [P, I64, I64, P, P, P, P, I64, I64, P, P, P, F, I, I, I, I, I,
+                                  P, P, P, P, P, P, P, SZ, P, P]
+    for name in ("retrace_workspace_init", "retrace_workspace_check", "retrace_verify",
+                 "retrace_align_refine", "retrace_gate_fuse", "retrace_round"):
+        getattr(lib, name).restype = I
+    return lib
+
+
+lib = _load()
+
+
+def _check(status: int) -> None:
+    if status != 0:
+        raise RetraceError(status, lib.retrace_last_error().decode())
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return RETRACE_BF16
+    if t.dtype == torch.float32:
+        return RETRACE_F32
+    raise TypeError(f"unsupported floating dtype {t.dtype}")
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("libretrace takes CUDA tensors")
+    return t.data_ptr()
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+def retrace_workspace_bytes(B: int, K: int, V: int, d: int, dtype: torch.dtype) -> int:
+    code = RETRACE_BF16 if dtype == torch.bfloat16 else RETRACE_F32
+    return int(lib.retrace_workspace_bytes(B, K, V, d, code))
+
+
+class Workspace:
+    """Caller-owned device workspace sized for (B, K, V, d, dtype), zeroed once."""
+
+    def __init__(self, B, K, V, d, dtype, device=None, stream=None):
+        self.nbytes = retrace_workspace_bytes(B, K, V, d, dtype)
+        if self.nbytes == 0:
+            raise ValueError("invalid workspace shape")
+        self.buf = torch.empty(self.nbytes + 256, dtype=torch.uint8, device=device or "cuda")
+        base = self.buf.data_ptr()
+        self.ptr = (base + 255) // 256 * 256
+        retrace_workspace_init(self, stream)
+
+    def check(self, stream=None) -> int:
+        return retrace_workspace_check(self, stream)
+
+
+def retrace_workspace_init(ws: Workspace, stream=None) -> None:
+    _check(lib.retrace_workspace_init(ws.ptr, ws.nbytes, _stream(stream)))
+
+
+def retrace_workspace_check(ws: Workspace, stream=None) -> int:
+    flags = ctypes.c_uint32(0)
+    st = lib.retrace_workspace_check(ws.ptr, ws.nbytes, ctypes.byref(flags), _stream(stream))
+    if st not in (0, 5):
+        _check(st)
+    return int(flags.value)
+
+
+def _int32(t: torch.Tensor, name: str) -> None:
+    if t.dtype != torch.int32:
+        raise TypeError(f"{name} must be int32")
+
+
+def retrace_verify(logits, draft, accept_len, committed, bonus, ws, target_argmax=None, stream=None):
+    """Greedy verification (see include/retrace.h).  logits [B, K+1, V], last dim contiguous."""
+    B, K1, V = logits.shape
+    if logits.stride(2) != 1:
+        raise ValueError("logits: vocabulary dimension must be contiguous")
+    for t, n in ((draft, "draft"), (accept_len, "accept_len"), (committed, "committed"), (bonus, "bonus")):
+        _int32(t, n)
+    _check(lib.retrace_verify(_ptr(logits), _dtype_code(logits), B, K1 - 1, V, logits.stride(1),
+                              logits.stride(0), _ptr(draft), _ptr(accept_len), _ptr(committed),
+                              _ptr(bonus), _ptr(target_argmax), ws.ptr, ws.nbytes, _stream(stream)))
+
+
+def retrace_align_refine(hD, hT, accept_len, Wc, beta, r_out, n_out, ws, stream=None):
+    """Alignment + target-aware correction: r_out [B, K, d], n_out [B]."""
+    B, K, d = hD.shape
+    for t in (hD, hT, Wc, r_out):
+        if not t.is_contiguous():
+            raise ValueError("hD, hT, Wc and r_out must be contiguous")
+    _check(lib.retrace_align_refine(_ptr(hD), _ptr(hT), _dtype_code(hD), B, K, d, _ptr(accept_len),
+                                    _ptr(Wc), float(beta), _ptr(r_out), _ptr(n_out), ws.ptr,
+                                    ws.nbytes, _stream(stream)))
+
+
+def _e_strides(e: torch.Tensor, B: int, K: int, d: int):
+    if e.dim() == 1:
+        return 0, 0
+    if e.shape != (B, K, d) or not e.is_contiguous():
+        raise ValueError("e must be a [d] vector or a contiguous [B, K, d] tensor")
+    return K * d, d
+
+
+def retrace_gate_fuse(e, r, n, Wv, Wg, e_out, ws, stream=None):
+    """Gated residual conditioning: e_out [B, K, d]."""
+    B, K, d = r.shape
+    ebs, eps = _e_strides(e, B, K, d)
+    _check(lib.retrace_gate_fuse(_ptr(e), ebs, eps, _ptr(r), _ptr(n), _ptr(Wv), _ptr(Wg),
+                                 _dtype_code(r), B, K, d, _ptr(e_out), ws.ptr, ws.nbytes,
+                                 _stream(stream)))
+
+
+def retrace_round(logits, draft, hD, hT, e, Wc, Wv, Wg, beta, accept_len, committed, bonus, e_out,
+                  ws, n_out=None, target_argmax=None, phase_events=None, stream=None):
+    """One fused round on one stream (see include/retrace.h)."""
+    B, K1, V = logits.shape
+    K = K1 - 1
+    d = hD.shape[2]
+    if logits.stride(2) != 1:
+        raise ValueError("logits: vocabulary dimension must be contiguous")
+    ebs, eps = _e_strides(e, B, K, d)
+    ev = None
+    if phase_events is not None:
+        ev = (ctypes.c_void_p * 4)(*[x._as_parameter_.value for x in phase_events])
+    _check(lib.retrace_round(_ptr(logits), logits.stride(1), logits.stride(0), _ptr(draft), _ptr(hD),
+                             _ptr(hT), _ptr(e), ebs, eps, _ptr(Wc), _ptr(Wv), _ptr(Wg), float(beta),
+                             _dtype_code(logits), B, K, V, d, _ptr(accept_len), _ptr(committed),
+                             _ptr(bonus), _ptr(target_argmax), _ptr(n_out), _ptr(e_out), ws.ptr,
+                             ws.nbytes, ctypes.cast(ev, ctypes.c_void_p) if ev is not None else None,
+                             _stream(stream)))
+
+
+class RoundBuffers:
+    """Device outputs of one round for a (B, K, d) shape."""
+
+    def __init__(self, B, K, d, dtype, device="cuda"):
+        self.accept_len = torch.empty(B, dtype=torch.int32, device=device)
+        self.committed = torch.empty(B, K + 1, dtype=torch.int32, device=device)
+        self.bonus = torch.empty(B, dtype=torch.int32, device=device)
+        self.n = torch.empty(B, dtype=torch.int32, device=device)
+        self.e_out = torch.empty(B, K, d, dtype=dtype, device=device)
+
+
+def run_round(x: dict, ws: Workspace, out: RoundBuffers | None = None, target_argmax=None,
+              phase_events=None, stream=None) -> RoundBuffers:
+    """retrace_round over a dict of device tensors (keys as in workloads.make_round_inputs)."""
+    logits = x["logits"]
+    B, K1, _ = logits.shape
+    d = x["hD"].shape[2]
+    if out is None:
+        out = RoundBuffers(B, K1 - 1, d, logits.dtype, logits.device)
+    retrace_round(logits, x["draft"], x["hD"], x["hT"], x["e"], x["Wc"], x["Wv"], x["Wg"], x["beta"],
+                  out.accept_len, out.committed, out.bonus, out.e_out, ws, n_out=out.n,
+                  target_argmax=target_argmax, phase_events=phase_events, stream=stream)
+    return out
+
+
+def version() -> str:
+    return lib.retrace_version().decode()

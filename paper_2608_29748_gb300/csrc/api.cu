@@ -1,0 +1,313 @@
+// C ABI of libretrace (declared in include/retrace.h): argument checks,
+// workspace layout, tensor-map encoding and the launch sequence of a round.
+#include <stdarg.h>
+#include <stdio.h>
+
+#include "internal.h"
+
+namespace retrace {
+
+cudaError_t launch_correct_simt(const CorrectArgs& a, retrace_dtype dtype, cudaStream_t stream);
+cudaError_t launch_gate_simt(const GateArgs& a, retrace_dtype dtype, cudaStream_t stream);
+cudaError_t launch_correct_tc(const CorrectArgs& a, uint32_t* status, cudaStream_t stream);
+cudaError_t launch_gate_tc(const GateArgs& a, uint32_t* status, cudaStream_t stream);
+
+cudaError_t device_info(DeviceInfo* out) {
+  static int sm_cache[64] = {0};
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  int& sm = sm_cache[dev & 63];
+  if (sm == 0) {
+    err = cudaDeviceGetAttribute(&sm, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+  }
+  out->device = dev;
+  out->sm_count = sm;
+  return cudaSuccess;
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// bf16 2D tensor [rows, inner], 128-byte swizzle, box {box_inner, box_rows}.
+CUresult encode_tensor_map_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
+                              uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return CUDA_ERROR_NOT_FOUND;
+  const cuuint64_t dims[2] = {inner, rows};
+  const cuuint64_t strides[1] = {row_stride_bytes};
+  const cuuint32_t box[2] = {box_inner, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+}  // namespace retrace
+
+using namespace retrace;
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+retrace_status fail(retrace_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+retrace_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(RETRACE_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define RT_CUDA(expr, what)                      \
+  do {                                           \
+    cudaError_t e_ = (expr);                     \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+size_t elem_size(retrace_dtype t) { return t == RETRACE_BF16 ? 2 : 4; }
+bool dtype_ok(retrace_dtype t) { return t == RETRACE_BF16 || t == RETRACE_F32; }
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+retrace_status check_ws(const void* ws, size_t ws_bytes, size_t need) {
+  if (!ws) return fail(RETRACE_ERR_WORKSPACE, "workspace pointer is NULL");
+  if (((uintptr_t)ws & 255u) != 0) return fail(RETRACE_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  if (ws_bytes < need)
+    return fail(RETRACE_ERR_WORKSPACE, "workspace too small: %zu bytes given, %zu needed", ws_bytes, need);
+  return RETRACE_OK;
+}
+
+retrace_status check_verify_args(const void* logits, retrace_dtype dtype, int B, int K, int V,
+                                 int64_t rs, int64_t bs, const int32_t* draft,
+                                 const int32_t* accept_len, const int32_t* committed,
+                                 const int32_t* bonus) {
+  if (!dtype_ok(dtype)) return fail(RETRACE_ERR_INVALID_ARG, "unknown dtype %d", (int)dtype);
+  if (B < 0 || K < 0 || V < 1) return fail(RETRACE_ERR_INVALID_ARG, "bad shape B=%d K=%d V=%d", B, K, V);
+  if (K > kMaxK) return fail(RETRACE_ERR_UNSUPPORTED, "K=%d exceeds the supported maximum %d", K, kMaxK);
+  if (B == 0) return RETRACE_OK;
+  if (!logits || !draft || !accept_len || !committed || !bonus)
+    return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
+  if (rs < V) return fail(RETRACE_ERR_INVALID_ARG, "logits_row_stride %lld < V %d", (long long)rs, V);
+  if (bs < (int64_t)(K + 1) * rs)
+    return fail(RETRACE_ERR_INVALID_ARG, "logits_batch_stride %lld < (K+1)*row_stride", (long long)bs);
+  return RETRACE_OK;
+}
+
+retrace_status check_cond_shape(retrace_dtype dtype, int B, int K, int d) {
+  if (!dtype_ok(dtype)) return fail(RETRACE_ERR_INVALID_ARG, "unknown dtype %d", (int)dtype);
+  if (B < 0 || K < 1 || d < 1) return fail(RETRACE_ERR_INVALID_ARG, "bad shape B=%d K=%d d=%d", B, K, d);
+  if (K > kMaxK) return fail(RETRACE_ERR_UNSUPPORTED, "K=%d exceeds the supported maximum %d", K, kMaxK);
+  if ((long long)B * K * (long long)d >= (1LL << 31) * 8LL)
+    return fail(RETRACE_ERR_UNSUPPORTED, "B*K*d too large");
+  if ((long long)B * K >= (1LL << 31)) return fail(RETRACE_ERR_UNSUPPORTED, "B*K too large");
+  return RETRACE_OK;
+}
+
+retrace_status e_mode(int64_t ebs, int64_t eps, int K, int d, int* dense) {
+  if (ebs == 0 && eps == 0) {
+    *dense = 0;
+    return RETRACE_OK;
+  }
+  if (eps == d && ebs == (int64_t)K * d) {
+    *dense = 1;
+    return RETRACE_OK;
+  }
+  return fail(RETRACE_ERR_UNSUPPORTED,
+              "e strides (%lld, %lld): only (0, 0) (broadcast) or (K*d, d) (dense) are supported",
+              (long long)ebs, (long long)eps);
+}
+
+uint32_t* status_word(void* ws) { return reinterpret_cast<uint32_t*>(ws); }
+
+}  // namespace
+
+extern "C" {
+
+const char* retrace_last_error(void) { return g_err; }
+
+const char* retrace_version(void) { return "retrace 0.1.0 sm_103a"; }
+
+size_t retrace_workspace_bytes(int B, int K, int V, int d, retrace_dtype dtype) {
+  if (B < 0 || K < 0 || V < 1 || d < 0 || !dtype_ok(dtype)) return 0;
+  return ws_layout(B, K, d, elem_size(dtype)).total;
+}
+
+retrace_status retrace_workspace_init(void* ws, size_t ws_bytes, cudaStream_t stream) {
+  g_err[0] = '\0';
+  if (!ws || ws_bytes == 0) return fail(RETRACE_ERR_INVALID_ARG, "NULL or empty workspace");
+  RT_CUDA(cudaMemsetAsync(ws, 0, ws_bytes, stream), "cudaMemsetAsync(workspace)");
+  return RETRACE_OK;
+}
+
+retrace_status retrace_workspace_check(const void* ws, size_t ws_bytes, uint32_t* device_flags,
+                                       cudaStream_t stream) {
+  g_err[0] = '\0';
+  if (!ws || ws_bytes < 4 || !device_flags) return fail(RETRACE_ERR_INVALID_ARG, "bad arguments");
+  RT_CUDA(cudaStreamSynchronize(stream), "cudaStreamSynchronize");
+  RT_CUDA(cudaMemcpy(device_flags, ws, 4, cudaMemcpyDeviceToHost), "cudaMemcpy(status)");
+  if (*device_flags) return fail(RETRACE_ERR_DEVICE, "device status flags 0x%x", *device_flags);
+  return RETRACE_OK;
+}
+
+retrace_status retrace_verify(const void* logits, retrace_dtype dtype, int B, int K, int V,
+                              int64_t logits_row_stride, int64_t logits_batch_stride,
+                              const int32_t* draft, int32_t* accept_len, int32_t* committed,
+                              int32_t* bonus, int32_t* target_argmax, void* ws, size_t ws_bytes,
+                              cudaStream_t stream) {
+  g_err[0] = '\0';
+  retrace_status st = check_verify_args(logits, dtype, B, K, V, logits_row_stride,
+                                        logits_batch_stride, draft, accept_len, committed, bonus);
+  if (st != RETRACE_OK || B == 0) return st;
+  const WsLayout L = ws_layout(B, K, 0, elem_size(dtype));
+  if ((st = check_ws(ws, ws_bytes, L.ge)) != RETRACE_OK) return st;
+  VerifyArgs a{};
+  a.logits = logits;
+  a.B = B;
+  a.K = K;
+  a.V = V;
+  a.row_stride = logits_row_stride;
+  a.batch_stride = logits_batch_stride;
+  a.draft = draft;
+  a.accept_len = accept_len;
+  a.committed = committed;
+  a.bonus = bonus;
+  a.target_argmax = target_argmax;
+  a.keys = reinterpret_cast<unsigned long long*>((char*)ws + L.keys);
+  a.tickets = reinterpret_cast<uint32_t*>((char*)ws + L.tickets);
+  RT_CUDA(launch_verify(a, dtype, stream), "verify kernel launch");
+  return RETRACE_OK;
+}
+
+retrace_status retrace_align_refine(const void* hD, const void* hT, retrace_dtype dtype, int B, int K,
+                                    int d, const int32_t* accept_len, const void* Wc, float beta,
+                                    void* r_out, int32_t* n_out, void* ws, size_t ws_bytes,
+                                    cudaStream_t stream) {
+  g_err[0] = '\0';
+  retrace_status st = check_cond_shape(dtype, B, K, d);
+  if (st != RETRACE_OK || B == 0) return st;
+  if (!hD || !hT || !accept_len || !Wc || !r_out || !n_out)
+    return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
+  const WsLayout L = ws_layout(B, K, d, elem_size(dtype));
+  if ((st = check_ws(ws, ws_bytes, L.keys)) != RETRACE_OK) return st;
+  const RowSource rows{accept_len, 1};
+  RT_CUDA(launch_fill_rows(B, K, d, rows, n_out, r_out, nullptr, 0, nullptr, dtype, stream),
+          "fill kernel launch");
+  CorrectArgs a{hD, hT, Wc, beta, B, K, d, rows, r_out, 0};
+  const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) && aligned16(r_out);
+  RT_CUDA(tc ? launch_correct_tc(a, status_word(ws), stream) : launch_correct_simt(a, dtype, stream),
+          "correction kernel launch");
+  return RETRACE_OK;
+}
+
+retrace_status retrace_gate_fuse(const void* e, int64_t e_batch_stride, int64_t e_pos_stride,
+                                 const void* r, const int32_t* n, const void* Wv, const void* Wg,
+                                 retrace_dtype dtype, int B, int K, int d, void* e_out, void* ws,
+                                 size_t ws_bytes, cudaStream_t stream) {
+  g_err[0] = '\0';
+  retrace_status st = check_cond_shape(dtype, B, K, d);
+  if (st != RETRACE_OK || B == 0) return st;
+  if (!e || !r || !n || !Wv || !Wg || !e_out) return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
+  int dense = 0;
+  if ((st = e_mode(e_batch_stride, e_pos_stride, K, d, &dense)) != RETRACE_OK) return st;
+  const WsLayout L = ws_layout(B, K, d, elem_size(dtype));
+  if ((st = check_ws(ws, ws_bytes, L.r)) != RETRACE_OK) return st;
+  float* ge = reinterpret_cast<float*>((char*)ws + L.ge);
+  const RowSource rows{n, 0};
+  RT_CUDA(launch_fill_rows(B, K, d, rows, nullptr, nullptr, e, dense, e_out, dtype, stream),
+          "fill kernel launch");
+  if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");
+  GateArgs a{e, dense, r, 0, (long long)B * K, Wv, Wg, dense ? nullptr : ge, B, K, d, rows, e_out};
+  const bool tc = tc_supported(dtype, d) && aligned16(e) && aligned16(r) && aligned16(Wv) &&
+                  aligned16(Wg) && aligned16(e_out);
+  RT_CUDA(tc ? launch_gate_tc(a, status_word(ws), stream) : launch_gate_simt(a, dtype, stream),
+          "gate kernel launch");
+  return RETRACE_OK;
+}
+
+retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
+                             int64_t logits_batch_stride, const int32_t* draft, const void* hD,
+                             const void* hT, const void* e, int64_t e_batch_stride,
+                             int64_t e_pos_stride, const void* Wc, const void* Wv, const void* Wg,
+                             float beta, retrace_dtype dtype, int B, int K, int V, int d,
+                             int32_t* accept_len, int32_t* committed, int32_t* bonus,
+                             int32_t* target_argmax, int32_t* n_out, void* e_out, void* ws,
+                             size_t ws_bytes, const cudaEvent_t* phase_events,
+                             cudaStream_t stream) {
+  g_err[0] = '\0';
+  retrace_status st = check_verify_args(logits, dtype, B, K, V, logits_row_stride,
+                                        logits_batch_stride, draft, accept_len, committed, bonus);
+  if (st != RETRACE_OK) return st;
+  if ((st = check_cond_shape(dtype, B, K, d)) != RETRACE_OK) return st;
+  if (B == 0) return RETRACE_OK;
+  if (!hD || !hT || !e || !Wc || !Wv || !Wg || !e_out)
+    return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
+  int dense = 0;
+  if ((st = e_mode(e_batch_stride, e_pos_stride, K, d, &dense)) != RETRACE_OK) return st;
+  const WsLayout L = ws_layout(B, K, d, elem_size(dtype));
+  if ((st = check_ws(ws, ws_bytes, L.total)) != RETRACE_OK) return st;
+  char* w = reinterpret_cast<char*>(ws);
+  float* ge = reinterpret_cast<float*>(w + L.ge);
+  void* r_ws = w + L.r;
+
+  if (phase_events) RT_CUDA(cudaEventRecord(phase_events[0], stream), "cudaEventRecord");
+  VerifyArgs va{};
+  va.logits = logits;
+  va.B = B;
+  va.K = K;
+  va.V = V;
+  va.row_stride = logits_row_stride;
+  va.batch_stride = logits_batch_stride;
+  va.draft = draft;
+  va.accept_len = accept_len;
+  va.committed = committed;
+  va.bonus = bonus;
+  va.target_argmax = target_argmax;
+  va.n_out = n_out;
+  va.keys = reinterpret_cast<unsigned long long*>(w + L.keys);
+  va.tickets = reinterpret_cast<uint32_t*>(w + L.tickets);
+  va.e = e;
+  va.e_batch_stride = e_batch_stride;
+  va.e_pos_stride = e_pos_stride;
+  va.e_out = e_out;
+  va.d = d;
+  RT_CUDA(launch_verify(va, dtype, stream), "verify kernel launch");
+  if (phase_events) RT_CUDA(cudaEventRecord(phase_events[1], stream), "cudaEventRecord");
+
+  const RowSource rows{accept_len, 1};
+  const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) &&
+                  aligned16(Wv) && aligned16(Wg) && aligned16(e) && aligned16(e_out);
+  CorrectArgs ca{hD, hT, Wc, beta, B, K, d, rows, r_ws, 1};
+  RT_CUDA(tc ? launch_correct_tc(ca, status_word(ws), stream) : launch_correct_simt(ca, dtype, stream),
+          "correction kernel launch");
+  if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
+
+  if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");
+  long long rmax = (long long)B * (K - 1);
+  GateArgs ga{e, dense, r_ws, 1, rmax > 0 ? rmax : 1, Wv, Wg, dense ? nullptr : ge, B, K, d, rows, e_out};
+  RT_CUDA(tc ? launch_gate_tc(ga, status_word(ws), stream) : launch_gate_simt(ga, dtype, stream),
+          "gate kernel launch");
+  if (phase_events) RT_CUDA(cudaEventRecord(phase_events[3], stream), "cudaEventRecord");
+  return RETRACE_OK;
+}
+
+}  // extern "C"

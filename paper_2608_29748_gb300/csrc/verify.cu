@@ -1,0 +1,319 @@
+// Greedy verification of a draft block (ReTrace Algorithm 1, Verify and
+// commit steps; greedy decoding = top_k 1).
+//
+// The [B, K+1, V] logits are one flat stream of B*(K+1) rows.  The rows are
+// cut into "slots" (16-byte vectors: 8 bf16 or 4 fp32; single elements on the
+// unaligned path) and the slot range is split evenly over the grid, so every
+// CTA streams the same number of bytes whatever B, K and V are.  A CTA reduces
+// each row segment it owns to one 64-bit (value, ~index) key and folds it into
+// the row's key with atomicMax.  The last CTA to finish a sequence (per-
+// sequence arrival ticket; nothing ever waits) decodes its K+1 argmaxes,
+// finds the first mismatch with a warp ballot and writes the accepted length,
+// committed tokens and bonus, resets the keys and ticket to zero for the next
+// call and, inside a fused round, copies the unconditioned drafter inputs.
+#include "common.cuh"
+#include "internal.h"
+
+namespace retrace {
+namespace {
+
+constexpr int kThreads = 512;
+constexpr int kUnroll = 4;
+
+struct VerifyParams {
+  const void* logits;
+  int B, K, V;
+  long long row_stride, batch_stride;
+  const int32_t* draft;
+  int32_t* accept_len;
+  int32_t* committed;
+  int32_t* bonus;
+  int32_t* target_argmax;
+  int32_t* n_out;
+  unsigned long long* keys;
+  uint32_t* tickets;
+  int slots_per_row;
+  long long total_slots;
+  const void* e;
+  long long e_batch_stride, e_pos_stride;
+  void* e_out;
+  int d;
+};
+
+// 16-byte vector helpers: the maximum of the vector's elements and element q.
+template <typename T>
+struct Vec;
+template <>
+struct Vec<__nv_bfloat16> {
+  static constexpr int E = 8;
+  __device__ static __forceinline__ float vmax(const uint4& v) {
+    const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&v.x);
+    const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&v.y);
+    const __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&v.z);
+    const __nv_bfloat162 d = *reinterpret_cast<const __nv_bfloat162*>(&v.w);
+    const __nv_bfloat162 m = __hmax2(__hmax2(a, b), __hmax2(c, d));
+    return fmaxf(__low2float(m), __high2float(m));
+  }
+  __device__ static __forceinline__ float elem(const uint4& v, int q) {
+    const uint32_t w = (q < 2) ? v.x : (q < 4) ? v.y : (q < 6) ? v.z : v.w;
+    return (q & 1) ? bf16_hi(w) : bf16_lo(w);
+  }
+};
+template <>
+struct Vec<float> {
+  static constexpr int E = 4;
+  __device__ static __forceinline__ float vmax(const uint4& v) {
+    return fmaxf(fmaxf(__uint_as_float(v.x), __uint_as_float(v.y)),
+                 fmaxf(__uint_as_float(v.z), __uint_as_float(v.w)));
+  }
+  __device__ static __forceinline__ float elem(const uint4& v, int q) {
+    const uint32_t w = (q == 0) ? v.x : (q == 1) ? v.y : (q == 2) ? v.z : v.w;
+    return __uint_as_float(w);
+  }
+};
+
+// Key of this thread's share of row slots [v0, v1).
+template <typename T, bool VEC>
+__device__ __forceinline__ unsigned long long segment_key(const T* __restrict__ rowp, int v0,
+                                                          int v1, int V) {
+  unsigned long long key = 0ull;
+  if constexpr (VEC) {
+    constexpr int E = Vec<T>::E;
+    const int full = V / E;  // complete 16-byte slots in the row
+    const int hi = v1 < full ? v1 : full;
+    const uint4* __restrict__ vp = reinterpret_cast<const uint4*>(rowp);
+    float best = -INFINITY;
+    int best_slot = -1;
+    uint4 best_vec = make_uint4(0, 0, 0, 0);
+    for (int s = v0 + (int)threadIdx.x; s < hi; s += kUnroll * kThreads) {
+      uint4 x[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int q = s + u * kThreads;
+        if (q < hi) x[u] = __ldcs(vp + q);
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int q = s + u * kThreads;
+        if (q < hi) {
+          const float m = Vec<T>::vmax(x[u]);
+          // strictly greater keeps the earliest slot among equal maxima
+          if (m > best || best_slot < 0) {
+            best = m;
+            best_slot = q;
+            best_vec = x[u];
+          }
+        }
+      }
+    }
+    if (best_slot >= 0) {
+#pragma unroll
+      for (int q = 0; q < E; ++q) {
+        if (Vec<T>::elem(best_vec, q) == best) {
+          key = make_key(best, (uint32_t)(best_slot * E + q));
+          break;
+        }
+      }
+    }
+    // Trailing partial slot (V not a multiple of E), read element by element.
+    if (v1 > full && threadIdx.x == 0) {
+      for (int v = full * E; v < V; ++v) key = umax64(key, make_key(to_f32<T>(rowp[v]), (uint32_t)v));
+    }
+  } else {
+    for (int v = v0 + (int)threadIdx.x; v < v1; v += kThreads)
+      key = umax64(key, make_key(to_f32<T>(rowp[v]), (uint32_t)v));
+  }
+  return key;
+}
+
+__device__ __forceinline__ unsigned long long block_max_key(unsigned long long key,
+                                                            unsigned long long* s_red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  key = warp_max_key(key);
+  if (lane == 0) s_red[warp] = key;
+  __syncthreads();
+  if (warp == 0) {
+    unsigned long long k = (lane < kThreads / 32) ? s_red[lane] : 0ull;
+    k = warp_max_key(k);
+    if (lane == 0) s_red[0] = k;
+  }
+  __syncthreads();
+  return s_red[0];
+}
+
+// Copy of drafter-input rows j in [nb, K) of sequence b into e_out.
+template <typename T>
+__device__ void copy_unconditioned_rows(const VerifyParams& p, int b, int nb) {
+  const int K = p.K, d = p.d;
+  const long long rows = K - nb;
+  if (rows <= 0) return;
+  T* dst = reinterpret_cast<T*>(p.e_out) + ((long long)b * K + nb) * d;
+  const T* src_b = reinterpret_cast<const T*>(p.e) + (long long)b * p.e_batch_stride;
+  const bool vec = ((d * (int)sizeof(T)) % 16 == 0) && ((uintptr_t)dst % 16 == 0) &&
+                   ((uintptr_t)src_b % 16 == 0) && ((p.e_pos_stride * (long long)sizeof(T)) % 16 == 0);
+  if (vec) {
+    const int vpr = d * (int)sizeof(T) / 16;
+    for (long long i = threadIdx.x; i < rows * vpr; i += kThreads) {
+      const long long jj = i / vpr, q = i % vpr;
+      const uint4* s = reinterpret_cast<const uint4*>(src_b + (nb + jj) * p.e_pos_stride);
+      reinterpret_cast<uint4*>(dst)[i] = s[q];
+    }
+  } else {
+    for (long long i = threadIdx.x; i < rows * d; i += kThreads) {
+      const long long jj = i / d, q = i % d;
+      dst[i] = src_b[(nb + jj) * p.e_pos_stride + q];
+    }
+  }
+}
+
+template <typename T>
+__device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s_A) {
+  const int K = p.K, K1 = K + 1;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int i = threadIdx.x; i < K1; i += kThreads)
+    s_t[i] = (int)key_index(__ldcg(&p.keys[(long long)b * K1 + i]));
+  __syncthreads();
+  if (warp == 0) {
+    int A = K;
+    for (int base = 0; base < K; base += 32) {
+      const int i = base + lane;
+      const bool mismatch = (i < K) && (s_t[i] != p.draft[(long long)b * K + i]);
+      const unsigned bal = __ballot_sync(0xFFFFFFFFu, mismatch);
+      if (bal) {
+        A = base + __ffs(bal) - 1;
+        break;
+      }
+    }
+    if (lane == 0) *s_A = A;
+  }
+  __syncthreads();
+  const int A = *s_A;
+  for (int i = threadIdx.x; i < K1; i += kThreads) {
+    const long long o = (long long)b * K1 + i;
+    p.committed[o] = (i <= A) ? s_t[i] : -1;
+    if (p.target_argmax) p.target_argmax[o] = s_t[i];
+    p.keys[o] = 0ull;
+  }
+  const int nb = (K - 1 - A) > 0 ? (K - 1 - A) : 0;
+  if (threadIdx.x == 0) {
+    p.accept_len[b] = A;
+    p.bonus[b] = s_t[A];
+    if (p.n_out) p.n_out[b] = nb;
+    p.tickets[b] = 0u;
+  }
+  if (p.e_out) copy_unconditioned_rows<T>(p, b, nb);
+}
+
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kThreads) verify_kernel(const VerifyParams p) {
+  __shared__ unsigned long long s_red[kThreads / 32];
+  __shared__ int s_t[kMaxK + 1];
+  __shared__ int s_A;
+  __shared__ int s_last;
+
+  const long long T_ = p.total_slots;
+  const long long G = gridDim.x;
+  const long long c = blockIdx.x;
+  const long long s_begin = c * T_ / G, s_end = (c + 1) * T_ / G;
+  const long long VV = p.slots_per_row;
+  const int K1 = p.K + 1;
+  const long long per_seq = (long long)K1 * VV;
+
+  long long s = s_begin;
+  while (s < s_end) {
+    const long long row = s / VV;
+    const int b = (int)(row / K1);
+    const int i = (int)(row - (long long)b * K1);
+    const long long seg_end = min(s_end, (row + 1) * VV);
+    const int v0 = (int)(s - row * VV), v1 = (int)(seg_end - row * VV);
+    const T* rowp = reinterpret_cast<const T*>(p.logits) + (long long)b * p.batch_stride +
+                    (long long)i * p.row_stride;
+
+    unsigned long long key = segment_key<T, VEC>(rowp, v0, v1, p.V);
+    key = block_max_key(key, s_red);
+    if (threadIdx.x == 0) atomicMax(&p.keys[row], key);
+    s = seg_end;
+
+    if (s == s_end || s % per_seq == 0) {
+      // This CTA has folded in all of its rows of sequence b.  The CTAs that
+      // own slots of b are those from the owner of its first slot to the
+      // owner of its last (every CTA range is non-empty: G <= total slots).
+      const long long first = (long long)b * per_seq, last = first + per_seq - 1;
+      const long long c_first = ((first + 1) * G - 1) / T_;
+      const long long c_last = ((last + 1) * G - 1) / T_;
+      const uint32_t count = (uint32_t)(c_last - c_first + 1);
+      if (threadIdx.x == 0) {
+        __threadfence();
+        const uint32_t prev = atomicAdd(&p.tickets[b], 1u);
+        s_last = (prev == count - 1u);
+      }
+      __syncthreads();
+      if (s_last) {
+        __threadfence();
+        finalize_sequence<T>(p, b, s_t, &s_A);
+      }
+      __syncthreads();
+    }
+  }
+}
+
+template <typename T, bool VEC>
+cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
+  DeviceInfo info;
+  cudaError_t err = device_info(&info);
+  if (err != cudaSuccess) return err;
+  static int occ_cache[64] = {0};
+  int& occ = occ_cache[info.device & 63];
+  if (occ == 0) {
+    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, verify_kernel<T, VEC>, kThreads, 0);
+    if (err != cudaSuccess) return err;
+    if (occ < 1) occ = 1;
+  }
+  VerifyParams p;
+  p.logits = a.logits;
+  p.B = a.B;
+  p.K = a.K;
+  p.V = a.V;
+  p.row_stride = a.row_stride;
+  p.batch_stride = a.batch_stride;
+  p.draft = a.draft;
+  p.accept_len = a.accept_len;
+  p.committed = a.committed;
+  p.bonus = a.bonus;
+  p.target_argmax = a.target_argmax;
+  p.n_out = a.n_out;
+  p.keys = a.keys;
+  p.tickets = a.tickets;
+  const int E = VEC ? 16 / (int)sizeof(T) : 1;
+  p.slots_per_row = (a.V + E - 1) / E;
+  p.total_slots = (long long)a.B * (a.K + 1) * p.slots_per_row;
+  p.e = a.e;
+  p.e_batch_stride = a.e_batch_stride;
+  p.e_pos_stride = a.e_pos_stride;
+  p.e_out = a.e_out;
+  p.d = a.d;
+  // Enough CTAs to fill every SM at full occupancy, but at least ~32 KB of
+  // logits per CTA so that small batches do not pay for idle CTAs.
+  const long long bytes = (long long)a.B * (a.K + 1) * a.V * (long long)sizeof(T);
+  long long grid = (long long)info.sm_count * occ;
+  const long long by_bytes = (bytes + 32767) / 32768;
+  if (by_bytes < grid) grid = by_bytes;
+  if (grid > p.total_slots) grid = p.total_slots;
+  if (grid < 1) grid = 1;
+  verify_kernel<T, VEC><<<(unsigned)grid, kThreads, 0, stream>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_verify(const VerifyArgs& a, retrace_dtype dtype, cudaStream_t stream) {
+  const size_t es = dtype == RETRACE_BF16 ? 2 : 4;
+  const bool vec = ((uintptr_t)a.logits % 16 == 0) && ((a.row_stride * (long long)es) % 16 == 0) &&
+                   ((a.batch_stride * (long long)es) % 16 == 0);
+  if (dtype == RETRACE_BF16)
+    return vec ? launch_typed<__nv_bfloat16, true>(a, stream)
+               : launch_typed<__nv_bfloat16, false>(a, stream);
+  return vec ? launch_typed<float, true>(a, stream) : launch_typed<float, false>(a, stream);
+}
+
+}  // namespace retrace

@@ -1,0 +1,75 @@
+"""Shared helpers of the GPU parity tests: host copies, oracle calls, tolerances.
+
+Tolerances (fixed by the arithmetic of the two sides):
+* integers (argmax, accepted length, committed and bonus tokens, n): bit-exact;
+* fp32 outputs: |gpu - oracle_f64| <= 1e-5;
+* bf16 outputs: the GPU rounds an fp32 result once to bf16, the oracle rounds
+  its float64 result at the same points.  The two roundings can land on
+  neighbouring bf16 values, so: |gpu - oracle_rounded| <= 2e-2, or <= 1 bf16
+  ulp of the reference where |reference| >= 4 (1 ulp there is >= 2^-5).
+  Rows the method leaves unconditioned must equal e bit-for-bit.
+"""
+
+import numpy as np
+import torch
+
+import oracle
+from paper_2608_29748_gb300.workloads import as_bits_numpy
+
+BF16_ABS_TOL = 2e-2
+F32_ABS_TOL = 1e-5
+
+
+def host_f64(t: torch.Tensor) -> np.ndarray:
+    """Exact float64 host copy of a bf16/fp32 tensor."""
+    if t.dtype == torch.bfloat16:
+        return oracle.bf16_bits_to_f64(as_bits_numpy(t))
+    return t.detach().cpu().double().numpy()
+
+
+def host_int(t: torch.Tensor) -> np.ndarray:
+    return t.detach().cpu().numpy().astype(np.int64)
+
+
+def oracle_round(x: dict) -> dict:
+    dtype = "bf16" if x["logits"].dtype == torch.bfloat16 else "f32"
+    return oracle.retrace_round(
+        host_f64(x["logits"]),
+        host_int(x["draft"]),
+        host_f64(x["hD"]),
+        host_f64(x["hT"]),
+        host_f64(x["e"]),
+        host_f64(x["Wc"]),
+        host_f64(x["Wv"]),
+        host_f64(x["Wg"]),
+        x["beta"],
+        dtype,
+    )
+
+
+def bf16_tolerance(ref_rounded: np.ndarray) -> np.ndarray:
+    return np.where(np.abs(ref_rounded) >= 4.0, np.maximum(BF16_ABS_TOL, oracle.bf16_ulp(ref_rounded)), BF16_ABS_TOL)
+
+
+def assert_close(gpu: torch.Tensor, ref64: np.ndarray, what: str = "") -> float:
+    """Checks gpu (bf16 or fp32) against the float64 oracle; returns max |gpu - ref64|."""
+    got = host_f64(gpu)
+    assert got.shape == ref64.shape, (got.shape, ref64.shape)
+    if gpu.dtype == torch.bfloat16:
+        ref_r = oracle.round_to_bf16(ref64)
+        err = np.abs(got - ref_r)
+        tol = bf16_tolerance(ref_r)
+        bad = err > tol
+        assert not bad.any(), f"{what}: {bad.sum()} elements out of tolerance; worst err {err.max():.4g}"
+    else:
+        err = np.abs(got - ref64)
+        assert err.max(initial=0.0) <= F32_ABS_TOL, f"{what}: max abs err {err.max():.3g} > {F32_ABS_TOL}"
+    return float(np.abs(got - ref64).max(initial=0.0))
+
+
+def assert_verify_exact(out: dict, accept_len, committed, bonus, target_argmax=None) -> None:
+    np.testing.assert_array_equal(host_int(accept_len), out["accept_len"])
+    np.testing.assert_array_equal(host_int(committed), out["committed"])
+    np.testing.assert_array_equal(host_int(bonus), out["bonus"])
+    if target_argmax is not None:
+        np.testing.assert_array_equal(host_int(target_argmax), out["target_argmax"])

@@ -1,0 +1,108 @@
+"""Host-side checks of the C ABI (no GPU needed).
+
+The library must load and export every entry point include/retrace.h
+declares; workspace sizing is pure host arithmetic; invalid arguments come back
+as status codes before anything touches CUDA.
+"""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_29748_gb300 import build as libbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "retrace.h")
+
+OK, INVALID, UNSUPPORTED, WORKSPACE = 0, 1, 2, 3
+F32, BF16 = 0, 1
+
+
+@pytest.fixture(scope="module")
+def lib():
+    path = libbuild.build()
+    L = ctypes.CDLL(path)
+    L.retrace_workspace_bytes.restype = ctypes.c_size_t
+    L.retrace_workspace_bytes.argtypes = [ctypes.c_int] * 5
+    L.retrace_last_error.restype = ctypes.c_char_p
+    L.retrace_version.restype = ctypes.c_char_p
+    return L
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(retrace_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_round_entry_points():
+    names = declared_functions()
+    for n in ("retrace_verify", "retrace_align_refine", "retrace_gate_fuse", "retrace_round",
+              "retrace_workspace_bytes", "retrace_last_error"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_version_string(lib):
+    assert b"sm_103a" in lib.retrace_version()
+
+
+def test_workspace_bytes(lib):
+    ws = lib.retrace_workspace_bytes
+    assert ws(-1, 16, 10, 8, BF16) == 0
+    assert ws(1, 16, 0, 8, BF16) == 0
+    assert ws(1, 16, 10, 8, 7) == 0
+    small = ws(1, 16, 151936, 2560, BF16)
+    big = ws(256, 16, 151936, 4096, BF16)
+    assert 0 < small < big
+    assert big % 256 == 0
+    # keys (8 B per row of K+1) + tickets + gate vector + compact r in bf16
+    assert big >= 256 * 17 * 8 + 256 * 4 + 4096 * 4 + 256 * 15 * 4096 * 2
+    assert ws(256, 16, 151936, 4096, F32) > big  # r stored in fp32 for fp32 workloads
+    assert ws(0, 16, 10, 8, BF16) > 0  # empty batch: still a valid (tiny) workspace
+
+
+def _verify(lib, logits=16, dtype=BF16, B=2, K=4, V=10, rs=10, bs=50, ws=None, ws_bytes=1 << 20, draft=16):
+    P = ctypes.c_void_p
+    return lib.retrace_verify(P(logits), dtype, B, K, V, ctypes.c_int64(rs), ctypes.c_int64(bs), P(draft),
+                              P(16), P(16), P(16), None, P(ws) if ws else None, ctypes.c_size_t(ws_bytes), None)
+
+
+def test_verify_argument_errors(lib):
+    assert _verify(lib, logits=0) == INVALID
+    assert _verify(lib, draft=0) == INVALID
+    assert _verify(lib, dtype=9) == INVALID
+    assert _verify(lib, V=0) == INVALID
+    assert _verify(lib, rs=9) == INVALID  # row stride below V
+    assert _verify(lib, bs=49) == INVALID  # batch stride below (K+1)*row_stride
+    assert _verify(lib, K=5000, bs=10 ** 6) == UNSUPPORTED
+    assert _verify(lib, ws=None) == WORKSPACE
+    assert _verify(lib, ws=256 * 3, ws_bytes=8) == WORKSPACE
+    assert _verify(lib, ws=256 * 3 + 8) == WORKSPACE  # misaligned workspace
+    assert b"workspace" in lib.retrace_last_error()
+    assert _verify(lib, B=0, logits=0, draft=0) == OK  # empty batch is a no-op
+
+
+def test_conditioning_argument_errors(lib):
+    P = ctypes.c_void_p
+    f = ctypes.c_float(1.0)
+    sz = ctypes.c_size_t(1 << 20)
+    # K must be >= 1 for conditioning
+    assert lib.retrace_align_refine(P(16), P(16), BF16, 2, 0, 8, P(16), P(16), f, P(16), P(16), P(256), sz, None) == INVALID
+    assert lib.retrace_align_refine(None, P(16), BF16, 2, 4, 8, P(16), P(16), f, P(16), P(16), P(256), sz, None) == INVALID
+    # e strides other than broadcast (0, 0) or dense (K*d, d)
+    st = lib.retrace_gate_fuse(P(16), ctypes.c_int64(8), ctypes.c_int64(8), P(16), P(16), P(16), P(16), BF16,
+                               2, 4, 8, P(16), P(256), sz, None)
+    assert st == UNSUPPORTED
+    assert b"strides" in lib.retrace_last_error()
+
+
+def test_workspace_init_rejects_null(lib):
+    lib.retrace_workspace_init.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
+    assert lib.retrace_workspace_init(None, 128, None) == INVALID

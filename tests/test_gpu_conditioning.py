@@ -1,0 +1,154 @@
+"""GPU parity of alignment/correction (Eq. 4-7) and gated fusion (Eq. 8) vs the oracle.
+
+Covers both kernel families: the tcgen05 tensor-core path (bf16, d a multiple
+of 256) and the FFMA path (fp32, and bf16 at other hidden sizes).
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from parity import assert_close, host_f64, host_int
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def rt():
+    from paper_2608_29748_gb300 import binding
+
+    return binding
+
+
+def make_inputs(B, K, d, dtype, seed, accept=None):
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    hD = torch.randn((B, K, d), generator=g, device="cuda").to(dtype)
+    hT = torch.randn((B, K, d), generator=g, device="cuda").to(dtype)
+    a = math.sqrt(2.0 / d)
+    Wc = ((torch.rand((d, 2 * d), generator=g, device="cuda") * 2 - 1) * a).to(dtype)
+    Wv = ((torch.rand((d, d), generator=g, device="cuda") * 2 - 1) * math.sqrt(3.0 / d)).to(dtype)
+    Wg = ((torch.rand((d, 2 * d), generator=g, device="cuda") * 2 - 1) * a).to(dtype)
+    e_vec = (torch.randn((d,), generator=g, device="cuda") * 0.02).to(dtype)
+    e_dense = (torch.randn((B, K, d), generator=g, device="cuda") * 0.02).to(dtype)
+    if accept is None:
+        edge = torch.tensor([0, K - 2, K - 1, K], device="cuda").clamp(min=0)
+        accept = torch.randint(0, K + 1, (B,), generator=g, device="cuda")
+        accept[: min(B, 4)] = edge[: min(B, 4)]
+    return dict(hD=hD, hT=hT, Wc=Wc, Wv=Wv, Wg=Wg, e_vec=e_vec, e_dense=e_dense,
+                accept=accept.to(torch.int32))
+
+
+SHAPES = [
+    # (B, K, d, dtype)  -- tensor-core path
+    (1, 16, 256, torch.bfloat16),
+    (5, 4, 512, torch.bfloat16),
+    (19, 16, 256, torch.bfloat16),  # 19 * 15 = 285 rows: 3 M tiles, ragged last tile
+    (3, 16, 2560, torch.bfloat16),
+    # FFMA path
+    (4, 8, 192, torch.bfloat16),
+    (3, 5, 100, torch.bfloat16),
+    (2, 8, 256, torch.float32),
+    (6, 16, 96, torch.float32),
+]
+
+
+@pytest.mark.parametrize("B,K,d,dtype", SHAPES)
+def test_align_refine(rt, B, K, d, dtype):
+    x = make_inputs(B, K, d, dtype, seed=B * 7 + K + d)
+    beta = 0.75
+    r = torch.full((B, K, d), 9.0, dtype=dtype, device="cuda")
+    n = torch.full((B,), -1, dtype=torch.int32, device="cuda")
+    ws = rt.Workspace(B, K, 8, d, dtype)
+    rt.retrace_align_refine(x["hD"], x["hT"], x["accept"], x["Wc"], beta, r, n, ws)
+    torch.cuda.synchronize()
+    assert ws.check() == 0
+    A = host_int(x["accept"])
+    np.testing.assert_array_equal(host_int(n), oracle.carried_rows(A, K))
+    m, u = oracle.align(host_f64(x["hD"]), host_f64(x["hT"]), A)
+    want = oracle.correct(m, u, host_f64(x["Wc"]), beta, round_r_bf16=False)
+    assert_close(r, want, "r")
+    # rows that carry nothing are exactly zero (Eq. 4-5 zero padding)
+    got = host_f64(r)
+    for b in range(B):
+        assert not got[b, oracle.carried_rows(A, K)[b]:].any()
+
+
+def test_align_refine_clamps_out_of_range_accept(rt):
+    B, K, d = 4, 6, 256
+    acc = torch.tensor([-3, 0, K + 5, 2], dtype=torch.int32, device="cuda")
+    x = make_inputs(B, K, d, torch.bfloat16, seed=5, accept=acc)
+    r = torch.empty((B, K, d), dtype=torch.bfloat16, device="cuda")
+    n = torch.empty((B,), dtype=torch.int32, device="cuda")
+    ws = rt.Workspace(B, K, 8, d, torch.bfloat16)
+    rt.retrace_align_refine(x["hD"], x["hT"], acc, x["Wc"], 1.0, r, n, ws)
+    torch.cuda.synchronize()
+    clamped = np.clip(host_int(acc), 0, K)
+    np.testing.assert_array_equal(host_int(n), oracle.carried_rows(clamped, K))
+    m, u = oracle.align(host_f64(x["hD"]), host_f64(x["hT"]), clamped)
+    assert_close(r, oracle.correct(m, u, host_f64(x["Wc"]), 1.0, False), "r")
+
+
+@pytest.mark.parametrize("dense_e", [False, True])
+@pytest.mark.parametrize("B,K,d,dtype", SHAPES)
+def test_gate_fuse(rt, B, K, d, dtype, dense_e):
+    x = make_inputs(B, K, d, dtype, seed=B + K * 3 + d + int(dense_e))
+    g = torch.Generator(device="cuda")
+    g.manual_seed(d)
+    r = torch.randn((B, K, d), generator=g, device="cuda").to(dtype)
+    n = torch.from_numpy(oracle.carried_rows(host_int(x["accept"]), K).astype(np.int32)).cuda()
+    e = x["e_dense"] if dense_e else x["e_vec"]
+    out = torch.full((B, K, d), 7.0, dtype=dtype, device="cuda")
+    ws = rt.Workspace(B, K, 8, d, dtype)
+    rt.retrace_gate_fuse(e, r, n, x["Wv"], x["Wg"], out, ws)
+    torch.cuda.synchronize()
+    assert ws.check() == 0
+    e_full = np.broadcast_to(host_f64(e), (B, K, d))
+    want = oracle.gate_fuse(e_full, host_f64(r), host_int(n), host_f64(x["Wv"]), host_f64(x["Wg"]))
+    assert_close(out, want, "e_tilde")
+    got = host_f64(out)
+    for b in range(B):
+        nb = int(n[b])
+        assert np.array_equal(got[b, nb:], e_full[b, nb:])  # unconditioned rows keep e exactly
+
+
+@pytest.mark.parametrize("d,dtype", [(256, torch.bfloat16), (512, torch.bfloat16), (192, torch.bfloat16), (256, torch.float32)])
+def test_closed_gate_reproduces_e_exactly(rt, d, dtype):
+    """W_v = 0 (the paper's initialisation): e~ == e bit-for-bit on every row."""
+    B, K = 7, 16
+    x = make_inputs(B, K, d, dtype, seed=3)
+    r = torch.randn((B, K, d), device="cuda").to(dtype)
+    n = torch.full((B,), K - 1, dtype=torch.int32, device="cuda")
+    out = torch.empty((B, K, d), dtype=dtype, device="cuda")
+    ws = rt.Workspace(B, K, 8, d, dtype)
+    rt.retrace_gate_fuse(x["e_vec"], r, n, torch.zeros_like(x["Wv"]), x["Wg"], out, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(out, x["e_vec"].expand(B, K, d))
+
+
+@pytest.mark.parametrize("d,dtype", [(256, torch.bfloat16), (192, torch.bfloat16), (256, torch.float32)])
+def test_half_gate_identity_value_is_exact(rt, d, dtype):
+    """W_g = 0, W_v = I, beta = 0: e~ = e + m/2 (Eq. 7-8 closed form), rows without signal keep e."""
+    B, K = 5, 8
+    x = make_inputs(B, K, d, dtype, seed=11)
+    eye = torch.eye(d, device="cuda").to(dtype)
+    r = torch.empty((B, K, d), dtype=dtype, device="cuda")
+    n = torch.empty((B,), dtype=torch.int32, device="cuda")
+    out = torch.empty((B, K, d), dtype=dtype, device="cuda")
+    ws = rt.Workspace(B, K, 8, d, dtype)
+    rt.retrace_align_refine(x["hD"], x["hT"], x["accept"], x["Wc"], 0.0, r, n, ws)
+    rt.retrace_gate_fuse(x["e_vec"], r, n, eye, torch.zeros_like(x["Wg"]), out, ws)
+    torch.cuda.synchronize()
+    A = host_int(x["accept"])
+    m, _ = oracle.align(host_f64(x["hD"]), host_f64(x["hT"]), A)
+    e_full = np.broadcast_to(host_f64(x["e_vec"]), (B, K, d))
+    # v = r = m and sigmoid(0) = 1/2 are exact on both sides; the only rounding
+    # left is the fp32 addition (then bf16 for bf16 outputs), mirrored here.
+    want = (e_full.astype(np.float32) + (0.5 * m).astype(np.float32)).astype(np.float64)
+    got = host_f64(out)
+    if dtype == torch.bfloat16:
+        want = oracle.round_to_bf16(want)
+    assert np.array_equal(got, want)

@@ -1,0 +1,123 @@
+"""GPU parity of the fused round (retrace_round) on the five workloads vs the oracle.
+
+Configs 1-4 are checked in full.  Config 5 (B = 256, 1.3 GB of logits) is
+checked in the launch configuration the benchmark times: verification outputs
+in full, the unconditioned rows in full (bit-exact copies of e), and a seeded
+sample of conditioned rows computed one by one by the oracle.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from parity import assert_close, assert_verify_exact, host_f64, host_int, oracle_round
+from paper_2608_29748_gb300.workloads import CONFIGS, make_round_inputs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def rt():
+    from paper_2608_29748_gb300 import binding
+
+    return binding
+
+
+def run(rt, x, ws=None, **kw):
+    cfg = x["cfg"]
+    if ws is None:
+        ws = rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype)
+    targ = torch.empty((cfg.B, cfg.K + 1), dtype=torch.int32, device="cuda")
+    out = rt.run_round(x, ws, target_argmax=targ, **kw)
+    torch.cuda.synchronize()
+    return out, targ, ws
+
+
+@pytest.mark.parametrize("cfg_id", [1, 2, 3, 4])
+def test_round_workloads_full(rt, cfg_id):
+    x = make_round_inputs(CONFIGS[cfg_id], device="cuda")
+    out, targ, ws = run(rt, x)
+    assert ws.check() == 0
+    want = oracle_round(x)
+    assert_verify_exact(want, out.accept_len, out.committed, out.bonus, targ)
+    np.testing.assert_array_equal(host_int(out.n), want["n"])
+    assert_close(out.e_out, want["e_tilde"], f"config {cfg_id} e_tilde")
+    # rows without an aligned signal keep the mask embedding bit-for-bit
+    got = host_f64(out.e_out)
+    e = host_f64(x["e"])
+    for b in range(x["cfg"].B):
+        assert np.array_equal(got[b, want["n"][b]:], np.broadcast_to(e, got[b, want["n"][b]:].shape))
+
+
+def test_round_serving_batch_sampled(rt):
+    """Config 5 at full size: B=256, K=16, V=151936, d=4096."""
+    cfg = CONFIGS[5]
+    x = make_round_inputs(cfg, device="cuda")
+    out, targ, ws = run(rt, x)
+    assert ws.check() == 0
+    want = oracle.verify(host_f64(x["logits"]), host_int(x["draft"]))
+    assert_verify_exact(want, out.accept_len, out.committed, out.bonus, targ)
+    A = want["accept_len"]
+    n = oracle.carried_rows(A, cfg.K)
+    np.testing.assert_array_equal(host_int(out.n), n)
+    # unconditioned rows: exact copies of e (checked on the device, all of them)
+    pos = torch.arange(cfg.K, device="cuda")[None, :]
+    mask = pos >= out.n.long()[:, None]
+    assert torch.equal(out.e_out[mask], x["e"].expand(int(mask.sum()), cfg.d))
+    # conditioned rows: a seeded sample, including the first and last rows of the plan
+    rng = np.random.default_rng(42)
+    cond = [(b, j) for b in range(cfg.B) for j in range(int(n[b]))]
+    pick = sorted({0, len(cond) - 1, *rng.choice(len(cond), size=40, replace=False).tolist()})
+    rows = [cond[i] for i in pick]
+    ref = oracle.conditioned_rows(rows, A, host_f64(x["hD"]), host_f64(x["hT"]), host_f64(x["e"]),
+                                  host_f64(x["Wc"]), host_f64(x["Wv"]), host_f64(x["Wg"]), x["beta"], "f32")
+    got = torch.stack([out.e_out[b, j] for b, j in rows])
+    assert_close(got, ref, "config 5 sampled rows")
+
+
+def test_round_dense_e_and_short_blocks(rt):
+    """Per-position e ([B, K, d]) and blocks of 1 and 2 drafts."""
+    for K in (1, 2, 16):
+        cfg = CONFIGS[2].__class__("t", 9, K, 3001, 512, "bf16", 1.0, "uniform", seed_offset=7)
+        x = make_round_inputs(cfg, device="cuda")
+        x["e"] = (torch.randn((cfg.B, K, cfg.d), device="cuda") * 0.02).to(torch.bfloat16)
+        out, targ, ws = run(rt, x)
+        want = oracle_round(x)
+        assert_verify_exact(want, out.accept_len, out.committed, out.bonus, targ)
+        assert_close(out.e_out, want["e_tilde"], f"K={K}")
+        if K == 1:  # a one-token block never carries anything: e~ == e
+            assert torch.equal(out.e_out, x["e"])
+
+
+def test_round_in_cuda_graph(rt):
+    """The round captures into a CUDA graph (no host sync, no allocation) and replays exactly."""
+    x = make_round_inputs(CONFIGS[4], device="cuda")
+    eager, targ, ws = run(rt, x)
+    out = rt.RoundBuffers(64, 16, 2560, torch.bfloat16)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        rt.run_round(x, ws, out=out, stream=s)  # warm-up on the capture stream
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        rt.run_round(x, ws, out=out, stream=s)
+    for _ in range(3):
+        out.e_out.zero_()
+        g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(out.e_out, eager.e_out)
+    assert torch.equal(out.committed, eager.committed)
+    assert ws.check() == 0
+
+
+def test_round_phase_events(rt):
+    x = make_round_inputs(CONFIGS[3], device="cuda")
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    for e in ev:
+        e.record()  # creates the underlying CUDA events
+    run(rt, x, phase_events=ev)
+    t = [ev[i].elapsed_time(ev[i + 1]) for i in range(3)]
+    assert all(v >= 0 for v in t)
