@@ -119,7 +119,7 @@ retrace_status retrace_workspace_check(const void* ws, size_t ws_bytes,
  *                 b*logits_batch_stride + i*logits_row_stride + v (elements).
  *                 Requires logits_row_stride >= V and
  *                 logits_batch_stride >= (K+1)*logits_row_stride.
- *   draft         [B, K] int32 draft tokens.
+ *   draft         [B, K] int32 draft tokens (may be NULL when K = 0).
  *   accept_len    [B] int32 out: A_b = first i < K with argmax(logits[b,i]) !=
  *                 draft[b,i], else K.
  *   committed     [B, K+1] int32 out: draft[b, 0..A_b-1], then the correction

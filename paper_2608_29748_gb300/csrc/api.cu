@@ -105,7 +105,7 @@ retrace_status check_verify_args(const void* logits, retrace_dtype dtype, int B,
   if (B < 0 || K < 0 || V < 1) return fail(RETRACE_ERR_INVALID_ARG, "bad shape B=%d K=%d V=%d", B, K, V);
   if (K > kMaxK) return fail(RETRACE_ERR_UNSUPPORTED, "K=%d exceeds the supported maximum %d", K, kMaxK);
   if (B == 0) return RETRACE_OK;
-  if (!logits || !draft || !accept_len || !committed || !bonus)
+  if (!logits || (!draft && K > 0) || !accept_len || !committed || !bonus)
     return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
   if (rs < V) return fail(RETRACE_ERR_INVALID_ARG, "logits_row_stride %lld < V %d", (long long)rs, V);
   if (bs < (int64_t)(K + 1) * rs)
