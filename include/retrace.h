@@ -187,6 +187,40 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
                              size_t ws_bytes, const cudaEvent_t* phase_events,
                              cudaStream_t stream);
 
+/* Size in bytes of the fixed device scratch used by retrace_verify_noalloc. */
+#define RETRACE_NOALLOC_SCRATCH_BYTES 65536
+
+/* Greedy verification for callers that cannot allocate device memory.
+ *
+ * The paper has no counterpart to this entry point; it exists for callers that
+ * are handed only their input and output buffers and have no way to obtain
+ * scratch memory (for example a custom operator whose host framework owns all
+ * device allocations and passes none through, or a serving loop that reserved
+ * its whole memory budget up front and must not call cudaMalloc while it runs).
+ * It computes exactly what retrace_verify computes, with the same arguments
+ * minus the workspace: the per-row argmax keys and per-sequence counters live
+ * in a fixed array of RETRACE_NOALLOC_SCRATCH_BYTES bytes inside the library,
+ * which every GPU that uses the library keeps until the process exits.
+ *
+ *   Limit      8 * B * (K+1) bytes (rounded up to a multiple of 256) plus
+ *              4 * B bytes must not exceed RETRACE_NOALLOC_SCRATCH_BYTES
+ *              (B = 256, K = 16 needs 35,840 bytes); a larger batch returns
+ *              RETRACE_ERR_UNSUPPORTED and enqueues nothing.
+ *   Set-up     the first call on each device looks up the array's device
+ *              address (cudaGetSymbolAddress) with that device current; make
+ *              that first call before any stream capture on the device.
+ *   Sharing    every call on a device uses the same array and clears the part
+ *              it needs (cudaMemsetAsync on `stream`) before its kernel runs.
+ *              Calls whose work may overlap on the GPU (different streams with
+ *              no ordering between them) race on the array and give wrong
+ *              results: order them on one stream.
+ *   Memory     calls no cudaMalloc, cudaFree or other allocating routine. */
+retrace_status retrace_verify_noalloc(const void* logits, retrace_dtype dtype, int B, int K, int V,
+                                      int64_t logits_row_stride, int64_t logits_batch_stride,
+                                      const int32_t* draft, int32_t* accept_len,
+                                      int32_t* committed, int32_t* bonus,
+                                      int32_t* target_argmax, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -141,6 +141,8 @@ uint32_t* status_word(void* ws) { return reinterpret_cast<uint32_t*>(ws); }
 
 }  // namespace
 
+void retrace::set_last_error(const char* msg) { snprintf(g_err, sizeof(g_err), "%s", msg); }
+
 extern "C" {
 
 const char* retrace_last_error(void) { return g_err; }

@@ -114,6 +114,9 @@ cudaError_t launch_fill_rows(int B, int K, int d, RowSource rows, int32_t* n_out
 // Whether the tensor-core path handles this conditioning shape.
 bool tc_supported(retrace_dtype dtype, int d);
 
+// Sets the thread-local message returned by retrace_last_error().
+void set_last_error(const char* msg);
+
 // cuTensorMapEncodeTiled through the runtime's driver entry point.
 CUresult encode_tensor_map_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows,
                               uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows);
