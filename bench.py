@@ -43,11 +43,11 @@ if ROOT not in sys.path:
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
-from paper_2608_29748_gb300.workloads import CONFIGS, RoundConfig, make_round_inputs  # noqa: E402
+from paper_2608_29748_gb300.workloads import CONFIGS, PROFILE_CONFIG, RoundConfig, make_round_inputs  # noqa: E402
 
 METRIC = "verify+ReTrace rounds/sec at 1 GB300; logits HBM GB/s and % of roofline"
 UNIT = "rounds/s"
-KERNELS_PER_ROUND = 4  # verify, correction GEMM, gate-bias GEMV, gate GEMM
+KERNELS_PER_ROUND = 5  # verify, row pack, correction GEMM, gate-bias GEMV, gate GEMM
 L2_FLUSH_BYTES = 256 << 20
 
 
@@ -105,7 +105,7 @@ def load_peaks() -> dict:
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 200 ms while running."""
+    """nvidia-smi clocks and throttle reasons sampled every 20 ms while running."""
 
     QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -122,7 +122,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+                 "-lms", "20"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
         return self
@@ -227,7 +227,7 @@ def run_gpu(args) -> dict | None:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    cfg = CONFIGS[args.config]
+    cfg = workload(args.config)
     peaks = load_peaks()
 
     x = make_round_inputs(cfg, device=dev, seed=shard_seed(42 + 1000 * cfg.seed_offset, rank))
@@ -276,7 +276,7 @@ def run_gpu(args) -> dict | None:
     flags = ws.check()
 
     # ---- end to end through the public API with host buffers ----
-    e2e = run_e2e(rt, cfg, x, ws, dev, min(steps, args.e2e_steps), world)
+    e2e = run_e2e(rt, cfg, x, ws, dev, min(steps, args.e2e_steps), world) if args.e2e_steps > 0 else None
 
     line = {
         "metric": METRIC,
@@ -312,7 +312,7 @@ def run_gpu(args) -> dict | None:
             "traffic": None,
         },
         "roofline_conditioning": {
-            "kernels": "tc_cond_kernel<0> + gate_bias_kernel + tc_cond_kernel<1>",
+            "kernels": "pack_rows_kernel + tc_gemm_kernel<0> + gate_bias_kernel + tc_gemm_kernel<1>",
             "bound": "tensor",
             "achieved": round(c_tflops, 2),
             "peak": peaks["bf16_tflops_sustained"],
@@ -388,7 +388,7 @@ def run_reference(args) -> dict | None:
     rank, _, world = dist_env()
     if rank != 0:
         return None
-    cfg = CONFIGS[args.config]
+    cfg = workload(args.config)
     host = prepare_oracle_sample(cfg, args.ref_sample, seed=500)
     for _ in range(min(args.warmup, 1)):
         time_oracle(host)
@@ -408,13 +408,18 @@ def run_reference(args) -> dict | None:
     }
 
 
+def workload(name: str) -> RoundConfig:
+    return PROFILE_CONFIG if name == "profile" else CONFIGS[int(name)]
+
+
 def parse_args(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", type=int, default=5, choices=sorted(CONFIGS))
+    ap.add_argument("--config", default="5", choices=[str(k) for k in sorted(CONFIGS)] + ["profile"],
+                    help="workload 1-5, or 'profile' (B=128 half batch for profiler captures)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--cpu-sample", type=int, default=32, help="sequences in the CPU-baseline sample")
     ap.add_argument("--ref-sample", type=int, default=2, help="sequences per step in the reference arm")

@@ -7,11 +7,6 @@
 
 namespace retrace {
 
-cudaError_t launch_correct_simt(const CorrectArgs& a, retrace_dtype dtype, cudaStream_t stream);
-cudaError_t launch_gate_simt(const GateArgs& a, retrace_dtype dtype, cudaStream_t stream);
-cudaError_t launch_correct_tc(const CorrectArgs& a, uint32_t* status, cudaStream_t stream);
-cudaError_t launch_gate_tc(const GateArgs& a, uint32_t* status, cudaStream_t stream);
-
 cudaError_t device_info(DeviceInfo* out) {
   static int sm_cache[64] = {0};
   int dev = 0;
@@ -210,14 +205,23 @@ retrace_status retrace_align_refine(const void* hD, const void* hT, retrace_dtyp
   if (!hD || !hT || !accept_len || !Wc || !r_out || !n_out)
     return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
   const WsLayout L = ws_layout(B, K, d, elem_size(dtype));
-  if ((st = check_ws(ws, ws_bytes, L.keys)) != RETRACE_OK) return st;
+  if ((st = check_ws(ws, ws_bytes, L.total)) != RETRACE_OK) return st;
   const RowSource rows{accept_len, 1};
   RT_CUDA(launch_fill_rows(B, K, d, rows, n_out, r_out, nullptr, 0, nullptr, dtype, stream),
           "fill kernel launch");
-  CorrectArgs a{hD, hT, Wc, beta, B, K, d, rows, r_out, 0};
   const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) && aligned16(r_out);
-  RT_CUDA(tc ? launch_correct_tc(a, status_word(ws), stream) : launch_correct_simt(a, dtype, stream),
-          "correction kernel launch");
+  if (tc) {
+    char* w = reinterpret_cast<char*>(ws);
+    int32_t* R = reinterpret_cast<int32_t*>(w + L.status) + kRowCountSlot;
+    int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
+    PackArgs pk{B, K, d, rows, 0, hD, hT, nullptr, 0, w + L.apack, nullptr, rowmap, R};
+    RT_CUDA(launch_pack(pk, stream), "pack kernel launch");
+    TcCorrectArgs a{B, K, d, w + L.apack, Wc, beta, R, rowmap, r_out, 0, status_word(ws)};
+    RT_CUDA(launch_correct_tc(a, stream), "correction kernel launch");
+  } else {
+    CorrectArgs a{hD, hT, Wc, beta, B, K, d, rows, r_out, 0};
+    RT_CUDA(launch_correct_simt(a, dtype, stream), "correction kernel launch");
+  }
   return RETRACE_OK;
 }
 
@@ -232,17 +236,27 @@ retrace_status retrace_gate_fuse(const void* e, int64_t e_batch_stride, int64_t 
   int dense = 0;
   if ((st = e_mode(e_batch_stride, e_pos_stride, K, d, &dense)) != RETRACE_OK) return st;
   const WsLayout L = ws_layout(B, K, d, elem_size(dtype));
-  if ((st = check_ws(ws, ws_bytes, L.r)) != RETRACE_OK) return st;
-  float* ge = reinterpret_cast<float*>((char*)ws + L.ge);
+  if ((st = check_ws(ws, ws_bytes, L.total)) != RETRACE_OK) return st;
+  char* w = reinterpret_cast<char*>(ws);
+  float* ge = reinterpret_cast<float*>(w + L.ge);
   const RowSource rows{n, 0};
   RT_CUDA(launch_fill_rows(B, K, d, rows, nullptr, nullptr, e, dense, e_out, dtype, stream),
           "fill kernel launch");
   if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");
-  GateArgs a{e, dense, r, 0, (long long)B * K, Wv, Wg, dense ? nullptr : ge, B, K, d, rows, e_out};
   const bool tc = tc_supported(dtype, d) && aligned16(e) && aligned16(r) && aligned16(Wv) &&
                   aligned16(Wg) && aligned16(e_out);
-  RT_CUDA(tc ? launch_gate_tc(a, status_word(ws), stream) : launch_gate_simt(a, dtype, stream),
-          "gate kernel launch");
+  if (tc) {
+    int32_t* R = reinterpret_cast<int32_t*>(w + L.status) + kRowCountSlot;
+    int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
+    PackArgs pk{B, K, d, rows, 1, r, nullptr, e, dense, w + L.r, w + L.epack, rowmap, R};
+    RT_CUDA(launch_pack(pk, stream), "pack kernel launch");
+    TcGateArgs a{B, K, d, w + L.r, e, w + L.epack, dense, dense ? nullptr : ge, Wv, Wg, R, rowmap, e_out,
+                 status_word(ws)};
+    RT_CUDA(launch_gate_tc(a, stream), "gate kernel launch");
+  } else {
+    GateArgs a{e, dense, r, 0, Wv, Wg, dense ? nullptr : ge, B, K, d, rows, e_out};
+    RT_CUDA(launch_gate_simt(a, dtype, stream), "gate kernel launch");
+  }
   return RETRACE_OK;
 }
 
@@ -298,16 +312,28 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   const RowSource rows{accept_len, 1};
   const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) &&
                   aligned16(Wv) && aligned16(Wg) && aligned16(e) && aligned16(e_out);
-  CorrectArgs ca{hD, hT, Wc, beta, B, K, d, rows, r_ws, 1};
-  RT_CUDA(tc ? launch_correct_tc(ca, status_word(ws), stream) : launch_correct_simt(ca, dtype, stream),
-          "correction kernel launch");
+  int32_t* R = reinterpret_cast<int32_t*>(w + L.status) + kRowCountSlot;
+  int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
+  if (tc) {
+    PackArgs pk{B, K, d, rows, 0, hD, hT, e, dense, w + L.apack, w + L.epack, rowmap, R};
+    RT_CUDA(launch_pack(pk, stream), "pack kernel launch");
+    TcCorrectArgs ca{B, K, d, w + L.apack, Wc, beta, R, rowmap, r_ws, 1, status_word(ws)};
+    RT_CUDA(launch_correct_tc(ca, stream), "correction kernel launch");
+  } else {
+    CorrectArgs ca{hD, hT, Wc, beta, B, K, d, rows, r_ws, 1};
+    RT_CUDA(launch_correct_simt(ca, dtype, stream), "correction kernel launch");
+  }
   if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
 
   if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");
-  long long rmax = (long long)B * (K - 1);
-  GateArgs ga{e, dense, r_ws, 1, rmax > 0 ? rmax : 1, Wv, Wg, dense ? nullptr : ge, B, K, d, rows, e_out};
-  RT_CUDA(tc ? launch_gate_tc(ga, status_word(ws), stream) : launch_gate_simt(ga, dtype, stream),
-          "gate kernel launch");
+  if (tc) {
+    TcGateArgs ga{B, K, d, r_ws, e, w + L.epack, dense, dense ? nullptr : ge, Wv, Wg, R, rowmap, e_out,
+                  status_word(ws)};
+    RT_CUDA(launch_gate_tc(ga, stream), "gate kernel launch");
+  } else {
+    GateArgs ga{e, dense, r_ws, 1, Wv, Wg, dense ? nullptr : ge, B, K, d, rows, e_out};
+    RT_CUDA(launch_gate_simt(ga, dtype, stream), "gate kernel launch");
+  }
   if (phase_events) RT_CUDA(cudaEventRecord(phase_events[3], stream), "cudaEventRecord");
   return RETRACE_OK;
 }

@@ -15,17 +15,25 @@ constexpr int kMaxK = 1024;  // largest draft block the kernels accept
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Workspace layout (all offsets 256-byte aligned):
-//   status   uint32 [64]        device status word (+ spare)
+//   status   uint32 [64]        [0] device status word, [kRowCountSlot] R of the last pack
 //   keys     uint64 [B*(K+1)]   per-row argmax keys, zero between calls
 //   tickets  uint32 [B]         per-sequence CTA arrival counters, zero between calls
 //   ge       fp32   [d]         W_g[:, :d] e for a broadcast e
 //   r        elem   [R_max, d]  compacted corrected signal, R_max = B*(K-1)
+//   apack    elem   [R_max, 2d] packed [m; u] rows (tensor-core path)
+//   epack    elem   [R_max, d]  packed per-position e rows (tensor-core path, dense e)
+//   rowmap   int32  [R_max]     packed row g -> position b*K + j
+constexpr int kRowCountSlot = 16;
+
 struct WsLayout {
-  size_t status, keys, tickets, ge, r, total;
+  size_t status, keys, tickets, ge, r, apack, epack, rowmap, total;
 };
 
 inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   WsLayout L;
+  const long long rmax0 = B * (K > 1 ? K - 1 : 0);
+  const size_t rmax = (size_t)(rmax0 > 0 ? rmax0 : 1);
+  const size_t dd = (size_t)(d > 0 ? d : 1);
   size_t off = 0;
   L.status = off;
   off = align_up(off + 64 * 4, 256);
@@ -34,10 +42,15 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   L.tickets = off;
   off = align_up(off + (size_t)B * 4, 256);
   L.ge = off;
-  off = align_up(off + (size_t)(d > 0 ? d : 1) * 4, 256);
+  off = align_up(off + dd * 4, 256);
   L.r = off;
-  long long rmax = B * (K > 1 ? K - 1 : 0);
-  off = align_up(off + (size_t)(rmax > 0 ? rmax : 1) * (size_t)(d > 0 ? d : 1) * elem, 256);
+  off = align_up(off + rmax * dd * elem, 256);
+  L.apack = off;
+  off = align_up(off + rmax * 2 * dd * elem, 256);
+  L.epack = off;
+  off = align_up(off + rmax * dd * elem, 256);
+  L.rowmap = off;
+  off = align_up(off + rmax * 4, 256);
   L.total = off;
   return L;
 }
@@ -77,6 +90,7 @@ struct RowSource {
   int n_from_accept;
 };
 
+// FFMA path (fp32, and bf16 shapes the tensor-core path does not take).
 struct CorrectArgs {
   const void* hD;
   const void* hT;
@@ -87,14 +101,13 @@ struct CorrectArgs {
   void* r_out;        // compact [R, d] (compact_out) or [B, K, d]
   int compact_out;
 };
-cudaError_t launch_correct(const CorrectArgs& a, retrace_dtype dtype, cudaStream_t stream);
+cudaError_t launch_correct_simt(const CorrectArgs& a, retrace_dtype dtype, cudaStream_t stream);
 
 struct GateArgs {
   const void* e;
   int e_dense;  // 0: broadcast vector [d]; 1: dense [B, K, d]
   const void* r;
   int r_compact;  // r rows are compact [R, d] (1) or [B, K, d] (0)
-  long long r_rows;  // rows of the r buffer (for the tensor map)
   const void* Wv;
   const void* Wg;
   const float* ge;  // W_g[:, :d] e for broadcast e (device, fp32), else null
@@ -102,9 +115,54 @@ struct GateArgs {
   RowSource rows;
   void* e_out;  // [B, K, d]
 };
-cudaError_t launch_gate(const GateArgs& a, retrace_dtype dtype, cudaStream_t stream);
+cudaError_t launch_gate_simt(const GateArgs& a, retrace_dtype dtype, cudaStream_t stream);
 cudaError_t launch_gate_bias(const void* Wg, const void* e, int d, float* ge, retrace_dtype dtype,
                              cudaStream_t stream);
+
+// Tensor-core path (bf16, d a multiple of 256).
+struct PackArgs {
+  int B, K, d;
+  RowSource rows;
+  int mode;          // 0: [m; u] rows from hD (src0) / hT (src1); 1: r rows from src0 [B, K, d]
+  const void* src0;
+  const void* src1;
+  const void* e;     // dense e [B, K, d] to pack (if e_dense)
+  int e_dense;
+  void* apack;       // mode 0: [R_max, 2d]; mode 1: [R_max, d]
+  void* epack;       // [R_max, d]
+  int32_t* rowmap;   // [R_max]
+  int32_t* R;        // row count out
+};
+cudaError_t launch_pack(const PackArgs& a, cudaStream_t stream);
+
+struct TcCorrectArgs {
+  int B, K, d;
+  const void* apack;
+  const void* Wc;
+  float beta;
+  const int32_t* R;
+  const int32_t* rowmap;
+  void* r_out;
+  int compact_out;  // 1: r_out is compact [R_max, d]; 0: r_out is [B, K, d] (rows via rowmap)
+  uint32_t* status;
+};
+cudaError_t launch_correct_tc(const TcCorrectArgs& a, cudaStream_t stream);
+
+struct TcGateArgs {
+  int B, K, d;
+  const void* rpack;  // compact r [R_max, d]
+  const void* e;      // broadcast vector [d] (when !e_dense)
+  const void* epack;  // packed e rows [R_max, d] (when e_dense)
+  int e_dense;
+  const float* ge;
+  const void* Wv;
+  const void* Wg;
+  const int32_t* R;
+  const int32_t* rowmap;
+  void* e_out;
+  uint32_t* status;
+};
+cudaError_t launch_gate_tc(const TcGateArgs& a, cudaStream_t stream);
 
 // Writes n_out and the rows j >= n_b (zeros for r, a copy of e for e_out).
 cudaError_t launch_fill_rows(int B, int K, int d, RowSource rows, int32_t* n_out, void* zero_dst,

@@ -74,6 +74,11 @@ CONFIGS = {
     5: RoundConfig("qwen3-8b-B256-K16", 256, 16, 151936, 4096, "bf16", 1.0, "geometric", 0.2, seed_offset=5),
 }
 
+# A half-size serving batch with config 5's per-sequence distributions, for
+# multi-pass profiler captures (inputs still larger than L2, under 1 GB held).
+PROFILE_CONFIG = RoundConfig("profile-qwen3-8b-B128-K16", 128, 16, 151936, 4096, "bf16", 1.0, "geometric", 0.2,
+                             seed_offset=6)
+
 # Offsets (in elements) at which copies of the row maximum are planted when
 # ``ties`` is set: same 16-byte vector, next vector, a few KB away, far away.
 TIE_DELTAS = (1, 3, 7, 8, 9, 61, 1024, 4093, 65537)
@@ -151,30 +156,38 @@ def plant_prefix(logits: torch.Tensor, draft: torch.Tensor, a: torch.Tensor, tie
     """
     B, K1, V = logits.shape
     K = K1 - 1
-    rowmax = logits.float().amax(dim=-1)  # [B, K+1]
-    rowmin = logits.float().amin(dim=-1)
-    a_host = a.tolist()
-    draft_host = draft.tolist()
-    for b in range(B):
-        ab = int(a_host[b])
-        for i in range(ab):
-            tok = draft_host[b][i]
-            top = rowmax[b, i] + 1.0
-            logits[b, i, tok] = top.to(logits.dtype)
-            if ties:
-                for k, delta in enumerate(TIE_DELTAS):
-                    if (i + k) % 3 == 0 and tok + delta < V:
-                        logits[b, i, tok + delta] = logits[b, i, tok]
-        if ab < K:
-            tok = draft_host[b][ab]
-            if ties and tok > 0:
-                delta = TIE_DELTAS[(b + ab) % len(TIE_DELTAS)]
-                lower = max(0, tok - delta)
-                top = (rowmax[b, ab] + 1.0).to(logits.dtype)
-                logits[b, ab, tok] = top
-                logits[b, ab, lower] = top
-            elif V > 1:
-                logits[b, ab, tok] = (rowmin[b, ab] - 1.0).to(logits.dtype)
+    dev = logits.device
+    draft = draft.to(dev).long()
+    a = a.to(dev).long()
+    rowmax = logits.amax(dim=-1).float()  # [B, K+1]; max is exact in any dtype
+    rowmin = logits.amin(dim=-1).float()
+    slot = torch.arange(K, device=dev)[None, :].expand(B, K)
+    bidx = torch.arange(B, device=dev)[:, None].expand(B, K)
+    acc = slot < a[:, None]  # accepted rows
+    bi, ii, tok = bidx[acc], slot[acc], draft[:, :K][acc]
+    logits[bi, ii, tok] = (rowmax[bi, ii] + 1.0).to(logits.dtype)
+    if ties:
+        for k, delta in enumerate(TIE_DELTAS):
+            sel = ((ii + k) % 3 == 0) & (tok + delta < V)
+            logits[bi[sel], ii[sel], tok[sel] + delta] = logits[bi[sel], ii[sel], tok[sel]]
+    mis = a < K  # sequences with a mismatch row a_b
+    mb = torch.nonzero(mis).flatten()
+    if mb.numel() == 0:
+        return
+    ma = a[mb]
+    mtok = draft[mb, ma.clamp(max=K - 1)]
+    if ties:
+        deltas = torch.tensor(TIE_DELTAS, device=dev)[(mb + ma) % len(TIE_DELTAS)]
+        lower_ok = mtok > 0
+        top = (rowmax[mb, ma] + 1.0).to(logits.dtype)
+        lb, la, lt = mb[lower_ok], ma[lower_ok], mtok[lower_ok]
+        lower = (lt - deltas[lower_ok]).clamp(min=0)
+        logits[lb, la, lt] = top[lower_ok]
+        logits[lb, la, lower] = top[lower_ok]
+        rest = ~lower_ok
+        mb, ma, mtok = mb[rest], ma[rest], mtok[rest]
+    if V > 1 and mb.numel() > 0:
+        logits[mb, ma, mtok] = (rowmin[mb, ma] - 1.0).to(logits.dtype)
 
 
 def as_bits_numpy(t: torch.Tensor):
