@@ -49,6 +49,13 @@ METRIC = "verify+ReTrace rounds/sec at 1 GB300; logits HBM GB/s and % of rooflin
 UNIT = "rounds/s"
 KERNELS_PER_ROUND = 5  # verify, row pack, correction GEMM, gate-bias GEMV, gate GEMM
 L2_FLUSH_BYTES = 256 << 20
+# DRAM traffic of one verify_kernel launch per sequence of the serving shapes
+# (K=16, V=151936, bf16), measured with ncu (dram__bytes_read.sum +
+# dram__bytes_write.sum) on the 128-sequence profiling workload: 661.34 MB read
+# + 3.25 MB written.  Traffic grows in proportion to the sequences (the logits
+# dominate).  Must be re-measured whenever verify_kernel changes.
+VERIFY_TRAFFIC_PER_SEQUENCE = (661.34e6 + 3.25e6) / 128
+VERIFY_TRAFFIC_SHAPE = (16, 151936, 4096, "bf16")
 
 
 # ---------------------------------------------------------------------------
@@ -309,7 +316,9 @@ def run_gpu(args) -> dict | None:
             "peak_source": peaks["source"] + " HBM copy bandwidth",
             "algorithmic_bytes": vbytes,
             "avg_launch_us": round(v_avg_s * 1e6, 2),
-            "traffic": None,
+            "traffic": (round(VERIFY_TRAFFIC_PER_SEQUENCE * cfg.B) if (cfg.K, cfg.V, cfg.d, cfg.dtype) == VERIFY_TRAFFIC_SHAPE
+                        else None),
+            "traffic_source": "ncu dram read+write on B=128 profiling workload, scaled by B/128",
         },
         "roofline_conditioning": {
             "kernels": "pack_rows_kernel + tc_gemm_kernel<0> + gate_bias_kernel + tc_gemm_kernel<1>",
