@@ -47,14 +47,15 @@ from paper_2608_29748_gb300.workloads import CONFIGS, PROFILE_CONFIG, RoundConfi
 
 METRIC = "verify+ReTrace rounds/sec at 1 GB300; logits HBM GB/s and % of roofline"
 UNIT = "rounds/s"
-KERNELS_PER_ROUND = 5  # verify, row pack, correction GEMM, gate-bias GEMV, gate GEMM
+KERNELS_PER_ROUND = 3  # verify (+ row packing), correction GEMM (+ gate-bias GEMV), gate GEMM
 L2_FLUSH_BYTES = 256 << 20
 # DRAM traffic of one verify_kernel launch per sequence of the serving shapes
-# (K=16, V=151936, bf16), measured with ncu (dram__bytes_read.sum +
-# dram__bytes_write.sum) on the 128-sequence profiling workload: 661.34 MB read
-# + 3.25 MB written.  Traffic grows in proportion to the sequences (the logits
-# dominate).  Must be re-measured whenever verify_kernel changes.
-VERIFY_TRAFFIC_PER_SEQUENCE = (661.34e6 + 3.25e6) / 128
+# (K=16, V=151936, d=4096, bf16), measured with ncu (dram__bytes_read.sum +
+# dram__bytes_write.sum) on the 128-sequence profiling workload: 685.63 MB read
+# + 3.00 MB written (the packed rows it writes stay in L2 during the launch).
+# Traffic grows in proportion to the sequences (the logits dominate).  Must be
+# re-measured whenever verify_kernel changes.
+VERIFY_TRAFFIC_PER_SEQUENCE = (685630208 + 3001344) / 128
 VERIFY_TRAFFIC_SHAPE = (16, 151936, 4096, "bf16")
 
 
@@ -205,7 +206,7 @@ def time_oracle(host: dict) -> float:
 # ---------------------------------------------------------------------------
 
 
-def verify_bytes(cfg: RoundConfig, n: np.ndarray) -> int:
+def verify_bytes(cfg: RoundConfig, n: np.ndarray, packs_rows: bool) -> int:
     """Algorithmic bytes of one verification launch in a fused round."""
     es = cfg.elem_bytes
     B, K, V, d = cfg.B, cfg.K, cfg.V, cfg.d
@@ -213,7 +214,9 @@ def verify_bytes(cfg: RoundConfig, n: np.ndarray) -> int:
     tokens_in = B * K * 4
     tokens_out = B * (K + 1) * 4 + 3 * B * 4  # committed; accept_len, bonus, n
     copies = int(np.sum(K - n)) * d * es  # unconditioned rows of e~ written
-    return logits + tokens_in + tokens_out + copies
+    R = int(np.sum(n))
+    packing = (2 * R * 2 * d * es + R * 4) if packs_rows else 0  # [m; u] rows read + written, row map
+    return logits + tokens_in + tokens_out + copies + packing
 
 
 def conditioning_flops(cfg: RoundConfig, R: int, dense_e: bool) -> int:
@@ -274,7 +277,8 @@ def run_gpu(args) -> dict | None:
 
     n = out.n.cpu().numpy().astype(np.int64)
     R = int(n.sum())
-    vbytes = verify_bytes(cfg, n)
+    packs_rows = cfg.dtype == "bf16" and cfg.d % 256 == 0  # tensor-core path: verify packs the rows
+    vbytes = verify_bytes(cfg, n, packs_rows)
     v_avg_s = statistics.mean(verify_ms) / 1e3
     v_gbs = vbytes / v_avg_s / 1e9
     cflops = conditioning_flops(cfg, R, dense_e=False)
@@ -307,7 +311,7 @@ def run_gpu(args) -> dict | None:
             "parallelism": f"replicas x{world} (batch-sharded, no collective)",
         },
         "roofline": {
-            "kernel": "verify_kernel (argmax/compare/commit + copy of unconditioned rows)",
+            "kernel": "verify_kernel (argmax/compare/commit + copy of unconditioned rows + row packing)",
             "bound": "hbm",
             "achieved": round(v_gbs, 1),
             "peak": peaks["hbm_gbs"],
@@ -316,12 +320,13 @@ def run_gpu(args) -> dict | None:
             "peak_source": peaks["source"] + " HBM copy bandwidth",
             "algorithmic_bytes": vbytes,
             "avg_launch_us": round(v_avg_s * 1e6, 2),
-            "traffic": (round(VERIFY_TRAFFIC_PER_SEQUENCE * cfg.B) if (cfg.K, cfg.V, cfg.d, cfg.dtype) == VERIFY_TRAFFIC_SHAPE
+            "traffic": (round(VERIFY_TRAFFIC_PER_SEQUENCE * cfg.B)
+                        if VERIFY_TRAFFIC_PER_SEQUENCE and (cfg.K, cfg.V, cfg.d, cfg.dtype) == VERIFY_TRAFFIC_SHAPE
                         else None),
             "traffic_source": "ncu dram read+write on B=128 profiling workload, scaled by B/128",
         },
         "roofline_conditioning": {
-            "kernels": "pack_rows_kernel + tc_gemm_kernel<0> + gate_bias_kernel + tc_gemm_kernel<1>",
+            "kernels": "tc_gemm_kernel<0> (+ gate-bias GEMV in idle warps) + tc_gemm_kernel<1>",
             "bound": "tensor",
             "achieved": round(c_tflops, 2),
             "peak": peaks["bf16_tflops_sustained"],

@@ -216,7 +216,7 @@ retrace_status retrace_align_refine(const void* hD, const void* hT, retrace_dtyp
     int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
     PackArgs pk{B, K, d, rows, 0, hD, hT, nullptr, 0, w + L.apack, nullptr, rowmap, R};
     RT_CUDA(launch_pack(pk, stream), "pack kernel launch");
-    TcCorrectArgs a{B, K, d, w + L.apack, Wc, beta, R, rowmap, r_out, 0, status_word(ws)};
+    TcCorrectArgs a{B, K, d, w + L.apack, Wc, beta, R, rowmap, r_out, 0, status_word(ws), nullptr, nullptr, nullptr};
     RT_CUDA(launch_correct_tc(a, stream), "correction kernel launch");
   } else {
     CorrectArgs a{hD, hT, Wc, beta, B, K, d, rows, r_out, 0};
@@ -285,7 +285,16 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   float* ge = reinterpret_cast<float*>(w + L.ge);
   void* r_ws = w + L.r;
 
+  const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) &&
+                  aligned16(Wv) && aligned16(Wg) && aligned16(e) && aligned16(e_out);
+  int32_t* R = reinterpret_cast<int32_t*>(w + L.status) + kRowCountSlot;
+  int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
+  const RowSource rows{accept_len, 1};
+
   if (phase_events) RT_CUDA(cudaEventRecord(phase_events[0], stream), "cudaEventRecord");
+  // The verification kernel packs the conditioned rows as sequences finish;
+  // they claim packed rows from a counter that starts at zero.
+  if (tc) RT_CUDA(cudaMemsetAsync(R, 0, sizeof(int32_t), stream), "cudaMemsetAsync(row count)");
   VerifyArgs va{};
   va.logits = logits;
   va.B = B;
@@ -306,18 +315,21 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   va.e_pos_stride = e_pos_stride;
   va.e_out = e_out;
   va.d = d;
+  if (tc) {
+    va.hD = hD;
+    va.hT = hT;
+    va.e_dense = dense;
+    va.apack = w + L.apack;
+    va.epack = w + L.epack;
+    va.rowmap = rowmap;
+    va.R_count = R;
+  }
   RT_CUDA(launch_verify(va, dtype, stream), "verify kernel launch");
   if (phase_events) RT_CUDA(cudaEventRecord(phase_events[1], stream), "cudaEventRecord");
 
-  const RowSource rows{accept_len, 1};
-  const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) &&
-                  aligned16(Wv) && aligned16(Wg) && aligned16(e) && aligned16(e_out);
-  int32_t* R = reinterpret_cast<int32_t*>(w + L.status) + kRowCountSlot;
-  int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
   if (tc) {
-    PackArgs pk{B, K, d, rows, 0, hD, hT, e, dense, w + L.apack, w + L.epack, rowmap, R};
-    RT_CUDA(launch_pack(pk, stream), "pack kernel launch");
-    TcCorrectArgs ca{B, K, d, w + L.apack, Wc, beta, R, rowmap, r_ws, 1, status_word(ws)};
+    TcCorrectArgs ca{B, K, d, w + L.apack, Wc, beta, R, rowmap, r_ws, 1, status_word(ws),
+                     Wg, e, dense ? nullptr : ge};
     RT_CUDA(launch_correct_tc(ca, stream), "correction kernel launch");
   } else {
     CorrectArgs ca{hD, hT, Wc, beta, B, K, d, rows, r_ws, 1};
@@ -325,12 +337,12 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   }
   if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
 
-  if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");
   if (tc) {
     TcGateArgs ga{B, K, d, r_ws, e, w + L.epack, dense, dense ? nullptr : ge, Wv, Wg, R, rowmap, e_out,
                   status_word(ws)};
     RT_CUDA(launch_gate_tc(ga, stream), "gate kernel launch");
   } else {
+    if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");
     GateArgs ga{e, dense, r_ws, 1, Wv, Wg, dense ? nullptr : ge, B, K, d, rows, e_out};
     RT_CUDA(launch_gate_simt(ga, dtype, stream), "gate kernel launch");
   }

@@ -134,6 +134,12 @@ struct TcParams {
   __nv_bfloat16* out;
   int compact_out;  // MODE 0: write row g (1) or row rowmap[g] (0)
   uint32_t* status;
+  // MODE 0 only, optional: ge_out[i] = sum_k W_g[i, k] e[k] over the e half
+  // (k < d) for a broadcast e, computed by the otherwise idle warps 2-3 while
+  // the tensor cores run, so the gated-fusion kernel finds it ready.
+  const __nv_bfloat16* Wg;
+  const __nv_bfloat16* e_vec;
+  float* ge_out;
 };
 
 __device__ __forceinline__ void raise_abort(volatile int* s_abort, uint32_t* status) {
@@ -286,6 +292,29 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (!ok) raise_abort(&s_abort, p.status);
     }
     __syncwarp();
+  } else if (MODE == 0 && (warp == 2 || warp == 3)) {
+    // ---------------- gate bias W_g[:, :d] e (broadcast e) ----------------
+    if (p.ge_out) {
+      const int active = tiles < (int)gridDim.x ? tiles : (int)gridDim.x;
+      const int vpr = d / 8;
+      const uint4* ev = reinterpret_cast<const uint4*>(p.e_vec);
+      for (int i = (int)blockIdx.x * 2 + (warp - 2); i < d; i += 2 * active) {
+        const uint4* wr = reinterpret_cast<const uint4*>(p.Wg + (long long)i * 2 * d);
+        float acc = 0.f;
+        for (int v = lane; v < vpr; v += 32) {
+          const uint4 w = __ldcs(wr + v), x = __ldg(ev + v);
+          const uint32_t ww[4] = {w.x, w.y, w.z, w.w}, xx[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            acc = fmaf(bf16_lo(ww[t]), bf16_lo(xx[t]), acc);
+            acc = fmaf(bf16_hi(ww[t]), bf16_hi(xx[t]), acc);
+          }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
+        if (lane == 0) p.ge_out[i] = acc;
+      }
+    }
   } else if (warp >= 4) {
     // ---------------- epilogue ----------------
     const int q = (warp - 4) * 32 + lane;  // tile row = TMEM lane
@@ -446,6 +475,9 @@ cudaError_t launch_correct_tc(const TcCorrectArgs& a, cudaStream_t stream) {
   p.out = reinterpret_cast<__nv_bfloat16*>(a.r_out);
   p.compact_out = a.compact_out;
   p.status = a.status;
+  p.Wg = reinterpret_cast<const __nv_bfloat16*>(a.Wg);
+  p.e_vec = reinterpret_cast<const __nv_bfloat16*>(a.e_vec);
+  p.ge_out = a.ge_out;
   const long long tiles_max = (rmax + BM - 1) / BM * p.tiles_n;
   tc_gemm_kernel<0><<<persistent_grid(tiles_max), THREADS, SMEM_BYTES, stream>>>(mA, mA, mB, mB, p);
   return cudaGetLastError();

@@ -79,6 +79,16 @@ struct VerifyArgs {
   long long e_batch_stride, e_pos_stride;
   void* e_out;
   int d;
+  // Optional fused packing of the conditioned rows for the tensor-core GEMMs
+  // (bf16, 16-byte aligned rows): each finalised sequence claims n_b rows of
+  // the packed buffers with an atomic on *R_count (zero before the launch).
+  const void* hD;
+  const void* hT;
+  int e_dense;
+  void* apack;     // [R_max, 2d]: [m; u] rows
+  void* epack;     // [R_max, d]: e rows (dense e only)
+  int32_t* rowmap; // [R_max]: packed row -> b*K + j
+  int32_t* R_count;
 };
 cudaError_t launch_verify(const VerifyArgs& a, retrace_dtype dtype, cudaStream_t stream);
 
@@ -145,6 +155,10 @@ struct TcCorrectArgs {
   void* r_out;
   int compact_out;  // 1: r_out is compact [R_max, d]; 0: r_out is [B, K, d] (rows via rowmap)
   uint32_t* status;
+  // Optional: also compute ge_out = W_g[:, :d] e_vec for a broadcast e.
+  const void* Wg;
+  const void* e_vec;
+  float* ge_out;
 };
 cudaError_t launch_correct_tc(const TcCorrectArgs& a, cudaStream_t stream);
 

@@ -38,6 +38,13 @@ struct VerifyParams {
   long long e_batch_stride, e_pos_stride;
   void* e_out;
   int d;
+  const void* hD;
+  const void* hT;
+  int e_dense;
+  void* apack;
+  void* epack;
+  int32_t* rowmap;
+  int32_t* R_count;
 };
 
 // 16-byte vector helpers: the maximum of the vector's elements and element q.
@@ -166,6 +173,37 @@ __device__ void copy_unconditioned_rows(const VerifyParams& p, int b, int nb) {
   }
 }
 
+// Packs sequence b's conditioned rows for the tensor-core projections: the
+// shifted draft states and target states [m_j; u_j] = [hD[b, A+1+j]; hT[b, A+j]]
+// (Eq. 4-5) and, for per-position e, e[b, j]; rows land at a block of n_b rows
+// claimed with one atomic (row order across sequences does not matter: every
+// packed row carries its position in rowmap).
+__device__ void pack_sequence_rows(const VerifyParams& p, int b, int A, int nb, int* s_off) {
+  const int K = p.K, d = p.d;
+  if (threadIdx.x == 0) *s_off = atomicAdd(p.R_count, nb);
+  __syncthreads();
+  const int off = *s_off;
+  for (int j = threadIdx.x; j < nb; j += kThreads) p.rowmap[off + j] = b * K + j;
+  const int vpr = d / 8;  // 16-byte vectors per bf16 row
+  const long long base = (long long)b * K;
+  const uint4* hD = reinterpret_cast<const uint4*>(p.hD);
+  const uint4* hT = reinterpret_cast<const uint4*>(p.hT);
+  uint4* out = reinterpret_cast<uint4*>(p.apack);
+  for (int i = threadIdx.x; i < nb * 2 * vpr; i += kThreads) {
+    const int j = i / (2 * vpr), c = i - j * 2 * vpr;
+    const uint4 v = (c < vpr) ? __ldg(hD + (base + A + 1 + j) * vpr + c) : __ldg(hT + (base + A + j) * vpr + c - vpr);
+    out[(long long)(off + j) * 2 * vpr + c] = v;
+  }
+  if (p.e_dense) {
+    const uint4* e = reinterpret_cast<const uint4*>(p.e);
+    uint4* eo = reinterpret_cast<uint4*>(p.epack);
+    for (int i = threadIdx.x; i < nb * vpr; i += kThreads) {
+      const int j = i / vpr, c = i - j * vpr;
+      eo[(long long)(off + j) * vpr + c] = __ldg(e + (base + j) * vpr + c);
+    }
+  }
+}
+
 template <typename T>
 __device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s_A) {
   const int K = p.K, K1 = K + 1;
@@ -202,13 +240,14 @@ __device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s
     p.tickets[b] = 0u;
   }
   if (p.e_out) copy_unconditioned_rows<T>(p, b, nb);
+  if (p.R_count && nb > 0) pack_sequence_rows(p, b, A, nb, s_A + 1);
 }
 
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads) verify_kernel(const VerifyParams p) {
   __shared__ unsigned long long s_red[kThreads / 32];
   __shared__ int s_t[kMaxK + 1];
-  __shared__ int s_A;
+  __shared__ int s_A[2];  // accepted length, packed-row offset
   __shared__ int s_last;
 
   const long long T_ = p.total_slots;
@@ -250,7 +289,7 @@ __global__ void __launch_bounds__(kThreads) verify_kernel(const VerifyParams p) 
       __syncthreads();
       if (s_last) {
         __threadfence();
-        finalize_sequence<T>(p, b, s_t, &s_A);
+        finalize_sequence<T>(p, b, s_t, s_A);
       }
       __syncthreads();
     }
@@ -292,6 +331,13 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
   p.e_pos_stride = a.e_pos_stride;
   p.e_out = a.e_out;
   p.d = a.d;
+  p.hD = a.hD;
+  p.hT = a.hT;
+  p.e_dense = a.e_dense;
+  p.apack = a.apack;
+  p.epack = a.epack;
+  p.rowmap = a.rowmap;
+  p.R_count = a.R_count;
   // Enough CTAs to fill every SM at full occupancy, but at least ~32 KB of
   // logits per CTA so that small batches do not pay for idle CTAs.
   const long long bytes = (long long)a.B * (a.K + 1) * a.V * (long long)sizeof(T);
