@@ -47,7 +47,7 @@ from paper_2608_29748_gb300.workloads import CONFIGS, PROFILE_CONFIG, RoundConfi
 
 METRIC = "verify+ReTrace rounds/sec at 1 GB300; logits HBM GB/s and % of roofline"
 UNIT = "rounds/s"
-KERNELS_PER_ROUND = 3  # verify (+ row packing), correction GEMM (+ gate-bias GEMV), gate GEMM
+KERNELS_PER_ROUND = 2  # verify_kernel (+ row packing), cond_kernel (both projections + gate-bias GEMV)
 L2_FLUSH_BYTES = 256 << 20
 # DRAM traffic of one verify_kernel launch per sequence of the serving shapes
 # (K=16, V=151936, d=4096, bf16), measured with ncu (dram__bytes_read.sum +
@@ -326,7 +326,7 @@ def run_gpu(args) -> dict | None:
             "traffic_source": "ncu dram read+write on B=128 profiling workload, scaled by B/128",
         },
         "roofline_conditioning": {
-            "kernels": "tc_gemm_kernel<0> (+ gate-bias GEMV in idle warps) + tc_gemm_kernel<1>",
+            "kernels": "cond_kernel: correction + gated-fusion projections (+ gate-bias GEMV), one persistent launch",
             "bound": "tensor",
             "achieved": round(c_tflops, 2),
             "peak": peaks["bf16_tflops_sustained"],

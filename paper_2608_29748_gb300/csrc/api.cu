@@ -212,12 +212,27 @@ retrace_status retrace_align_refine(const void* hD, const void* hT, retrace_dtyp
   const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) && aligned16(r_out);
   if (tc) {
     char* w = reinterpret_cast<char*>(ws);
-    int32_t* R = reinterpret_cast<int32_t*>(w + L.status) + kRowCountSlot;
+    uint32_t* sync = reinterpret_cast<uint32_t*>(w + L.sync);
+    int32_t* R = reinterpret_cast<int32_t*>(sync + kSyncRowCount);
     int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
+    RT_CUDA(cudaMemsetAsync(sync, 0, L.sync_bytes, stream), "cudaMemsetAsync(sync)");
     PackArgs pk{B, K, d, rows, 0, hD, hT, nullptr, 0, w + L.apack, nullptr, rowmap, R};
     RT_CUDA(launch_pack(pk, stream), "pack kernel launch");
-    TcCorrectArgs a{B, K, d, w + L.apack, Wc, beta, R, rowmap, r_out, 0, status_word(ws), nullptr, nullptr, nullptr};
-    RT_CUDA(launch_correct_tc(a, stream), "correction kernel launch");
+    TcCondArgs a{};
+    a.B = B;
+    a.K = K;
+    a.d = d;
+    a.do_correct = 1;
+    a.apack = w + L.apack;
+    a.Wc = Wc;
+    a.beta = beta;
+    a.r_out = r_out;
+    a.compact_out = 0;
+    a.R = R;
+    a.rowmap = rowmap;
+    a.sync = sync;
+    a.status = status_word(ws);
+    RT_CUDA(launch_cond_tc(a, stream), "correction kernel launch");
   } else {
     CorrectArgs a{hD, hT, Wc, beta, B, K, d, rows, r_out, 0};
     RT_CUDA(launch_correct_simt(a, dtype, stream), "correction kernel launch");
@@ -242,18 +257,35 @@ retrace_status retrace_gate_fuse(const void* e, int64_t e_batch_stride, int64_t 
   const RowSource rows{n, 0};
   RT_CUDA(launch_fill_rows(B, K, d, rows, nullptr, nullptr, e, dense, e_out, dtype, stream),
           "fill kernel launch");
-  if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");
   const bool tc = tc_supported(dtype, d) && aligned16(e) && aligned16(r) && aligned16(Wv) &&
                   aligned16(Wg) && aligned16(e_out);
   if (tc) {
-    int32_t* R = reinterpret_cast<int32_t*>(w + L.status) + kRowCountSlot;
+    uint32_t* sync = reinterpret_cast<uint32_t*>(w + L.sync);
+    int32_t* R = reinterpret_cast<int32_t*>(sync + kSyncRowCount);
     int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
+    RT_CUDA(cudaMemsetAsync(sync, 0, L.sync_bytes, stream), "cudaMemsetAsync(sync)");
     PackArgs pk{B, K, d, rows, 1, r, nullptr, e, dense, w + L.r, w + L.epack, rowmap, R};
     RT_CUDA(launch_pack(pk, stream), "pack kernel launch");
-    TcGateArgs a{B, K, d, w + L.r, e, w + L.epack, dense, dense ? nullptr : ge, Wv, Wg, R, rowmap, e_out,
-                 status_word(ws)};
-    RT_CUDA(launch_gate_tc(a, stream), "gate kernel launch");
+    TcCondArgs a{};
+    a.B = B;
+    a.K = K;
+    a.d = d;
+    a.do_gate = 1;
+    a.rpack = w + L.r;
+    a.e = e;
+    a.epack = w + L.epack;
+    a.e_dense = dense;
+    a.Wv = Wv;
+    a.Wg = Wg;
+    a.ge = ge;
+    a.e_out = e_out;
+    a.R = R;
+    a.rowmap = rowmap;
+    a.sync = sync;
+    a.status = status_word(ws);
+    RT_CUDA(launch_cond_tc(a, stream), "gate kernel launch");
   } else {
+    if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");
     GateArgs a{e, dense, r, 0, Wv, Wg, dense ? nullptr : ge, B, K, d, rows, e_out};
     RT_CUDA(launch_gate_simt(a, dtype, stream), "gate kernel launch");
   }
@@ -287,14 +319,15 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
 
   const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) &&
                   aligned16(Wv) && aligned16(Wg) && aligned16(e) && aligned16(e_out);
-  int32_t* R = reinterpret_cast<int32_t*>(w + L.status) + kRowCountSlot;
+  uint32_t* sync = reinterpret_cast<uint32_t*>(w + L.sync);
+  int32_t* R = reinterpret_cast<int32_t*>(sync + kSyncRowCount);
   int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
   const RowSource rows{accept_len, 1};
 
   if (phase_events) RT_CUDA(cudaEventRecord(phase_events[0], stream), "cudaEventRecord");
   // The verification kernel packs the conditioned rows as sequences finish;
   // they claim packed rows from a counter that starts at zero.
-  if (tc) RT_CUDA(cudaMemsetAsync(R, 0, sizeof(int32_t), stream), "cudaMemsetAsync(row count)");
+  if (tc) RT_CUDA(cudaMemsetAsync(sync, 0, L.sync_bytes, stream), "cudaMemsetAsync(sync)");
   VerifyArgs va{};
   va.logits = logits;
   va.B = B;
@@ -328,20 +361,38 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   if (phase_events) RT_CUDA(cudaEventRecord(phase_events[1], stream), "cudaEventRecord");
 
   if (tc) {
-    TcCorrectArgs ca{B, K, d, w + L.apack, Wc, beta, R, rowmap, r_ws, 1, status_word(ws),
-                     Wg, e, dense ? nullptr : ge};
-    RT_CUDA(launch_correct_tc(ca, stream), "correction kernel launch");
+    // Both projections in one persistent launch; its phase events bracket
+    // the whole conditioning (the correction/gate split point is not a
+    // stream position any more).
+    TcCondArgs a{};
+    a.B = B;
+    a.K = K;
+    a.d = d;
+    a.do_correct = 1;
+    a.do_gate = 1;
+    a.apack = w + L.apack;
+    a.Wc = Wc;
+    a.beta = beta;
+    a.r_out = r_ws;
+    a.compact_out = 1;
+    a.rpack = r_ws;
+    a.e = e;
+    a.epack = w + L.epack;
+    a.e_dense = dense;
+    a.Wv = Wv;
+    a.Wg = Wg;
+    a.ge = ge;
+    a.e_out = e_out;
+    a.R = R;
+    a.rowmap = rowmap;
+    a.sync = sync;
+    a.status = status_word(ws);
+    RT_CUDA(launch_cond_tc(a, stream), "conditioning kernel launch");
+    if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
   } else {
     CorrectArgs ca{hD, hT, Wc, beta, B, K, d, rows, r_ws, 1};
     RT_CUDA(launch_correct_simt(ca, dtype, stream), "correction kernel launch");
-  }
-  if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
-
-  if (tc) {
-    TcGateArgs ga{B, K, d, r_ws, e, w + L.epack, dense, dense ? nullptr : ge, Wv, Wg, R, rowmap, e_out,
-                  status_word(ws)};
-    RT_CUDA(launch_gate_tc(ga, stream), "gate kernel launch");
-  } else {
+    if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
     if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");
     GateArgs ga{e, dense, r_ws, 1, Wv, Wg, dense ? nullptr : ge, B, K, d, rows, e_out};
     RT_CUDA(launch_gate_simt(ga, dtype, stream), "gate kernel launch");

@@ -119,27 +119,26 @@ __global__ void __launch_bounds__(256) pack_rows_kernel(const PackParams p) {
 }
 
 // ---------------------------------------------------------------------------
-// Persistent GEMM
+// Persistent, dynamically scheduled projections
 // ---------------------------------------------------------------------------
-struct TcParams {
+struct CondParams {
   int d;
-  int tiles_n;       // N tiles (d/256 for MODE 0, d/128 for MODE 1)
-  const int32_t* R;  // conditioned rows (written by the pack kernel)
+  int do_correct, do_gate;
+  const int32_t* R;
   const int32_t* rowmap;
-  const __nv_bfloat16* apack;  // MODE 0: [R, 2d], the m half is re-read by the epilogue
+  // correction
+  const __nv_bfloat16* apack;  // [R, 2d]; the m half is re-read by the epilogue
   float beta;
-  const __nv_bfloat16* e;  // MODE 1: broadcast vector [d] or Epack [R, d]
+  __nv_bfloat16* r_out;
+  int compact_out;
+  // gate
+  const __nv_bfloat16* e;  // broadcast vector [d], or packed e rows [R, d] (e_dense)
   int e_dense;
-  const float* ge;
-  __nv_bfloat16* out;
-  int compact_out;  // MODE 0: write row g (1) or row rowmap[g] (0)
-  uint32_t* status;
-  // MODE 0 only, optional: ge_out[i] = sum_k W_g[i, k] e[k] over the e half
-  // (k < d) for a broadcast e, computed by the otherwise idle warps 2-3 while
-  // the tensor cores run, so the gated-fusion kernel finds it ready.
   const __nv_bfloat16* Wg;
-  const __nv_bfloat16* e_vec;
-  float* ge_out;
+  float* ge;  // [d] = W_g[:, :d] e, computed here for a broadcast e
+  __nv_bfloat16* e_out;
+  uint32_t* sync;
+  uint32_t* status;
 };
 
 __device__ __forceinline__ void raise_abort(volatile int* s_abort, uint32_t* status) {
@@ -158,16 +157,51 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
-template <int MODE>
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Waits until *counter >= target (written by other CTAs of this grid).
+// Bounded like every other wait: false after kWaitLimitNs or on abort.
+__device__ __forceinline__ bool wait_counter(const uint32_t* counter, uint32_t target,
+                                             volatile int* abort) {
+  if (ld_acquire(counter) >= target) return true;
+  const unsigned long long t0 = global_ns();
+  for (uint32_t it = 1;; ++it) {
+    __nanosleep(64);
+    if (ld_acquire(counter) >= target) return true;
+    if ((it & 63u) == 0u) {
+      if (*abort) return false;
+      if (global_ns() - t0 > kWaitLimitNs) return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+constexpr int TILE_SLOTS = 2;
+
+// Tile t < T0: correction tile (row block t / nt0, 256 output columns t % nt0);
+// T0 <= t < T0 + T1: gate tile (row block (t-T0) / nt1, 128 features).  Tiles
+// are handed out in this order by a global counter, so every gate tile's row
+// block was handed out (to a running CTA) before it.
 __global__ void __launch_bounds__(THREADS, 1)
-    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
-                   const __grid_constant__ CUtensorMap tmB0, const __grid_constant__ CUtensorMap tmB1,
-                   const TcParams p) {
+    cond_kernel(const __grid_constant__ CUtensorMap tmApack, const __grid_constant__ CUtensorMap tmWc,
+                const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmE,
+                const __grid_constant__ CUtensorMap tmWv, const __grid_constant__ CUtensorMap tmWg,
+                const CondParams p) {
   extern __shared__ uint8_t dsmem[];
   __shared__ __align__(8) uint64_t bar_full[STAGES];
   __shared__ __align__(8) uint64_t bar_empty[STAGES];
   __shared__ __align__(8) uint64_t bar_tfull[2];
   __shared__ __align__(8) uint64_t bar_tempty[2];
+  __shared__ __align__(8) uint64_t bar_tile_full[TILE_SLOTS];
+  __shared__ __align__(8) uint64_t bar_tile_empty[TILE_SLOTS];
+  __shared__ int s_tile[TILE_SLOTS];
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
 
@@ -175,8 +209,15 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int d = p.d;
   const int R = *(volatile const int32_t*)p.R;
   const int tiles_m = (R + BM - 1) / BM;
-  const int tiles = tiles_m * p.tiles_n;
-  if ((int)blockIdx.x >= tiles) return;  // uniform: no tile for this CTA
+  const int nt0 = d / 256, nt1 = d / 128;
+  const int T0 = p.do_correct ? tiles_m * nt0 : 0;
+  const int T = T0 + (p.do_gate ? tiles_m * nt1 : 0);
+  if (T == 0) return;  // nothing to condition
+  uint32_t* tile_queue = p.sync + kSyncTileQueue;
+  uint32_t* gemv_next = p.sync + kSyncGemvNext;
+  uint32_t* gemv_done = p.sync + kSyncGemvDone;
+  uint32_t* block_done = p.sync + kSyncBlockDone;
+  const bool need_ge = p.do_gate && !p.e_dense;
 
   if (tid == 0) {
     s_abort = 0;
@@ -188,14 +229,22 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_init(smem_u32(&bar_tfull[a]), 1);
       mbar_init(smem_u32(&bar_tempty[a]), 4);  // one arrival per epilogue warp
     }
+    for (int a = 0; a < TILE_SLOTS; ++a) {
+      mbar_init(smem_u32(&bar_tile_full[a]), 1);
+      mbar_init(smem_u32(&bar_tile_empty[a]), 5);  // MMA thread + four epilogue warps
+    }
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tmA0);
-    tma_prefetch_desc(&tmB0);
-    if (MODE == 1) {
-      tma_prefetch_desc(&tmA1);
-      tma_prefetch_desc(&tmB1);
+    if (p.do_correct) {
+      tma_prefetch_desc(&tmApack);
+      tma_prefetch_desc(&tmWc);
+    }
+    if (p.do_gate) {
+      tma_prefetch_desc(&tmR);
+      tma_prefetch_desc(&tmWv);
+      tma_prefetch_desc(&tmWg);
+      if (p.e_dense) tma_prefetch_desc(&tmE);
     }
   }
   if (warp == 2) {
@@ -207,17 +256,36 @@ __global__ void __launch_bounds__(THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = s_tmem;
   const uint32_t base = (smem_u32(dsmem) + 1023u) & ~1023u;
-  const int kb_half = d / BK;  // K blocks of one d-wide operand half
-  const int nkb = (MODE == 0) ? 2 * kb_half : kb_half + (p.e_dense ? kb_half : 0);
-  const int n_width = (MODE == 0) ? 256 : 128;
+  const int kb_half = d / BK;
 
   if (warp == 0) {
-    // ---------------- TMA producer ----------------
+    // ---------------- tile scheduler + TMA producer ----------------
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-        const int m0 = (t % tiles_m) * BM, n0 = (t / tiles_m) * n_width;
+      for (uint32_t lt = 0;; ++lt) {
+        const uint32_t slot = lt % TILE_SLOTS, sph = (lt / TILE_SLOTS) & 1u;
+        const int t = (int)atomicAdd(tile_queue, 1u);
+        if (!mbar_wait_bounded(smem_u32(&bar_tile_empty[slot]), sph ^ 1u, &s_abort)) {
+          ok = false;
+          break;
+        }
+        s_tile[slot] = t < T ? t : -1;
+        mbar_arrive(smem_u32(&bar_tile_full[slot]));
+        if (t >= T) break;
+        const bool corr = t < T0;
+        const int tt = corr ? t : t - T0;
+        const int m0 = (corr ? tt / nt0 : tt / nt1) * BM;
+        const int n0 = corr ? (tt % nt0) * 256 : (tt % nt1) * 128;
+        const int nkb = corr ? 2 * kb_half : kb_half + (p.e_dense ? kb_half : 0);
+        if (!corr && p.do_correct) {
+          // the r rows of this block are written by the correction epilogues
+          if (!wait_counter(block_done + m0 / BM, (uint32_t)(4 * nt0), &s_abort)) {
+            ok = false;
+            break;
+          }
+          fence_proxy_async_global();
+        }
         for (int kb = 0; kb < nkb; ++kb, ++it) {
           const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
           if (!mbar_wait_bounded(smem_u32(&bar_empty[s]), ph ^ 1u, &s_abort)) {
@@ -226,26 +294,26 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           const uint32_t a_dst = base + s * STAGE_BYTES, b_dst = a_dst + A_BYTES;
           const uint32_t full = smem_u32(&bar_full[s]);
-          if (MODE == 0) {
+          if (corr) {
             mbar_arrive_expect_tx(full, A_BYTES + B_BYTES);
-            tma_load_2d(a_dst, &tmA0, kb * BK, m0, full);  // [m; u] rows, K block kb
-            tma_load_2d(b_dst, &tmB0, kb * BK, n0, full);  // W_c rows n0..n0+255
+            tma_load_2d(a_dst, &tmApack, kb * BK, m0, full);  // [m; u] rows
+            tma_load_2d(b_dst, &tmWc, kb * BK, n0, full);     // W_c rows n0..n0+255
           } else if (kb < kb_half) {
             mbar_arrive_expect_tx(full, A_BYTES + B_BYTES);
-            tma_load_2d(a_dst, &tmA0, kb * BK, m0, full);                    // r rows
-            tma_load_2d(b_dst, &tmB0, kb * BK, n0, full);                    // W_v rows
-            tma_load_2d(b_dst + B_BYTES / 2, &tmB1, d + kb * BK, n0, full);  // W_g[:, d:2d] rows
+            tma_load_2d(a_dst, &tmR, kb * BK, m0, full);                     // r rows
+            tma_load_2d(b_dst, &tmWv, kb * BK, n0, full);                    // W_v rows
+            tma_load_2d(b_dst + B_BYTES / 2, &tmWg, d + kb * BK, n0, full);  // W_g[:, d:2d] rows
           } else {
             mbar_arrive_expect_tx(full, A_BYTES + B_BYTES / 2);
-            tma_load_2d(a_dst, &tmA1, (kb - kb_half) * BK, m0, full);                    // e rows
-            tma_load_2d(b_dst + B_BYTES / 2, &tmB1, (kb - kb_half) * BK, n0, full);  // W_g[:, :d]
+            tma_load_2d(a_dst, &tmE, (kb - kb_half) * BK, m0, full);                     // e rows
+            tma_load_2d(b_dst + B_BYTES / 2, &tmWg, (kb - kb_half) * BK, n0, full);  // W_g[:, :d]
           }
         }
+        if (!ok) break;
       }
       if (!ok) {
         raise_abort(&s_abort, p.status);
-        // Drain this CTA's own copies still in flight before the CTA may exit.
-        volatile int never = 0;
+        volatile int never = 0;  // drain this CTA's own copies still in flight
         const uint32_t first = it > STAGES ? it - STAGES : 0;
         for (uint32_t k = first; k < it; ++k)
           mbar_wait_bounded(smem_u32(&bar_full[k % STAGES]), (k / STAGES) & 1u, &never);
@@ -255,9 +323,19 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
-      uint32_t it = 0, lt = 0;
+      uint32_t it = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++lt) {
+      for (uint32_t lt = 0;; ++lt) {
+        const uint32_t slot = lt % TILE_SLOTS, sph = (lt / TILE_SLOTS) & 1u;
+        if (!mbar_wait_bounded(smem_u32(&bar_tile_full[slot]), sph, &s_abort)) {
+          ok = false;
+          break;
+        }
+        const int t = s_tile[slot];
+        mbar_arrive(smem_u32(&bar_tile_empty[slot]));
+        if (t < 0) break;
+        const bool corr = t < T0;
+        const int nkb = corr ? 2 * kb_half : kb_half + (p.e_dense ? kb_half : 0);
         const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
         if (!mbar_wait_bounded(smem_u32(&bar_tempty[acc]), aph ^ 1u, &s_abort)) {
           ok = false;
@@ -273,7 +351,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           tc_fence_after();
           const uint32_t a_base = base + s * STAGE_BYTES, b_base = a_base + A_BYTES;
-          const bool e_part = (MODE == 1) && kb >= kb_half;
+          const bool e_part = !corr && kb >= kb_half;
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             const uint64_t adesc = sw128_kmajor_desc(a_base + (uint32_t)k * 32u);
@@ -285,56 +363,88 @@ __global__ void __launch_bounds__(THREADS, 1)
               tc_mma_bf16(d_tmem + 128u, adesc, bdesc, IDESC_N128, 1u);
             }
           }
-          tc_commit(smem_u32(&bar_empty[s]));  // stage reusable once these MMAs finish
+          tc_commit(smem_u32(&bar_empty[s]));
         }
         tc_commit(smem_u32(&bar_tfull[acc]));  // accumulator ready (also after a failure)
+        if (!ok) break;
       }
       if (!ok) raise_abort(&s_abort, p.status);
     }
     __syncwarp();
-  } else if (MODE == 0 && (warp == 2 || warp == 3)) {
-    // ---------------- gate bias W_g[:, :d] e (broadcast e) ----------------
-    if (p.ge_out) {
-      const int active = tiles < (int)gridDim.x ? tiles : (int)gridDim.x;
+  } else if (warp == 2 || warp == 3) {
+    // ---------------- W_g[:, :d] e for a broadcast e (idle warps) ----------------
+    if (need_ge) {
       const int vpr = d / 8;
-      const uint4* ev = reinterpret_cast<const uint4*>(p.e_vec);
-      for (int i = (int)blockIdx.x * 2 + (warp - 2); i < d; i += 2 * active) {
+      const uint4* ev = reinterpret_cast<const uint4*>(p.e);
+      for (;;) {
+        int i = 0;
+        if (lane == 0) i = (int)atomicAdd(gemv_next, 1u);
+        i = __shfl_sync(0xFFFFFFFFu, i, 0);
+        if (i >= d) break;
         const uint4* wr = reinterpret_cast<const uint4*>(p.Wg + (long long)i * 2 * d);
         float acc = 0.f;
         for (int v = lane; v < vpr; v += 32) {
           const uint4 w = __ldcs(wr + v), x = __ldg(ev + v);
           const uint32_t ww[4] = {w.x, w.y, w.z, w.w}, xx[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            acc = fmaf(bf16_lo(ww[t]), bf16_lo(xx[t]), acc);
-            acc = fmaf(bf16_hi(ww[t]), bf16_hi(xx[t]), acc);
+          for (int q = 0; q < 4; ++q) {
+            acc = fmaf(bf16_lo(ww[q]), bf16_lo(xx[q]), acc);
+            acc = fmaf(bf16_hi(ww[q]), bf16_hi(xx[q]), acc);
           }
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
-        if (lane == 0) p.ge_out[i] = acc;
+        if (lane == 0) {
+          p.ge[i] = acc;
+          __threadfence();
+          atomicAdd(gemv_done, 1u);
+        }
       }
     }
   } else if (warp >= 4) {
     // ---------------- epilogue ----------------
     const int q = (warp - 4) * 32 + lane;  // tile row = TMEM lane
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-    uint32_t lt = 0;
-    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
+    bool have_ge = !need_ge;
+    for (uint32_t lt = 0;; ++lt) {
+      const uint32_t slot = lt % TILE_SLOTS, sph = (lt / TILE_SLOTS) & 1u;
+      bool ok = warp_wait(smem_u32(&bar_tile_full[slot]), sph, &s_abort);
+      if (!ok) {
+        if (lane == 0) raise_abort(&s_abort, p.status);
+        break;
+      }
+      const int t = s_tile[slot];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&bar_tile_empty[slot]));
+      if (t < 0) break;
+      const bool corr = t < T0;
+      const int tt = corr ? t : t - T0;
+      const int m0 = (corr ? tt / nt0 : tt / nt1) * BM;
+      const int n0 = corr ? (tt % nt0) * 256 : (tt % nt1) * 128;
       const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
-      const bool ok = warp_wait(smem_u32(&bar_tfull[acc]), aph, &s_abort);
+      ok = warp_wait(smem_u32(&bar_tfull[acc]), aph, &s_abort);
       tc_fence_after();
       if (!ok) {
         if (lane == 0) raise_abort(&s_abort, p.status);
         break;
       }
       if (s_abort) break;
-      const int m0 = (t % tiles_m) * BM, n0 = (t / tiles_m) * n_width;
+      if (!corr && !have_ge) {
+        int got = 1;
+        if (lane == 0) got = wait_counter(gemv_done, (uint32_t)d, &s_abort) ? 1 : 0;
+        got = __shfl_sync(0xFFFFFFFFu, got, 0);
+        if (!got) {
+          if (lane == 0) raise_abort(&s_abort, p.status);
+          break;
+        }
+        have_ge = true;
+      }
       const int g = m0 + q;
       const bool valid = g < R;
       const uint32_t taddr = tmem + acc * ACC_COLS + lane_base;
-      if (MODE == 0) {
-        const __nv_bfloat16* mrow = p.apack + (long long)g * 2 * d;  // m = first d columns
+      if (corr) {
+        // r = m + beta * c   (Eq. 7), m = first d columns of the packed row
+        const __nv_bfloat16* mrow = p.apack + (long long)g * 2 * d;
         const long long orow = valid ? (p.compact_out ? g : p.rowmap[g]) : 0;
         for (int cc = 0; cc < 8; ++cc) {
           float c[32];
@@ -342,7 +452,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           if (valid) {
             const int n = n0 + cc * 32;
             const uint4* mv = reinterpret_cast<const uint4*>(mrow + n);
-            uint4* ov = reinterpret_cast<uint4*>(p.out + orow * d + n);
+            uint4* ov = reinterpret_cast<uint4*>(p.r_out + orow * d + n);
 #pragma unroll
             for (int v = 0; v < 4; ++v) {
               const uint4 mw = __ldg(mv + v);
@@ -358,7 +468,16 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
           }
         }
+        if (p.do_gate) {
+          // Publish this warp's 32 rows of the (row block, column block) of r
+          // to the gate tiles: one count per epilogue warp, no wait.
+          __threadfence();
+          fence_proxy_async_global();
+          __syncwarp();
+          if (lane == 0) atomicAdd(block_done + m0 / BM, 1u);
+        }
       } else {
+        // e~ = e + v * sigmoid(g)   (Eq. 8)
         const long long orow = valid ? p.rowmap[g] : 0;
         const __nv_bfloat16* erow = p.e + (p.e_dense ? (long long)g * d : 0);
         for (int cc = 0; cc < 4; ++cc) {
@@ -368,7 +487,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           if (valid) {
             const int n = n0 + cc * 32;
             const uint4* ev = reinterpret_cast<const uint4*>(erow + n);
-            uint4* ov = reinterpret_cast<uint4*>(p.out + orow * d + n);
+            uint4* ov = reinterpret_cast<uint4*>(p.e_out + orow * d + n);
 #pragma unroll
             for (int x = 0; x < 4; ++x) {
               const uint4 ew = __ldg(ev + x);
@@ -379,8 +498,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int c0 = x * 8 + 2 * w;
                 float g0 = gt[c0], g1 = gt[c0 + 1];
                 if (!p.e_dense) {
-                  g0 += __ldg(p.ge + n + c0);
-                  g1 += __ldg(p.ge + n + c0 + 1);
+                  g0 += __ldcg(p.ge + n + c0);
+                  g1 += __ldcg(p.ge + n + c0 + 1);
                 }
                 const float s0 = 1.f / (1.f + expf(-g0));
                 const float s1 = 1.f / (1.f + expf(-g1));
@@ -391,7 +510,6 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
         }
       }
-      // hand the accumulator back to the MMA warp
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&bar_tempty[acc]));
@@ -406,27 +524,17 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
-template <int MODE>
 cudaError_t ensure_smem_attr() {
   static int done[64] = {0};
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
   if (!done[dev & 63]) {
-    err = cudaFuncSetAttribute(tc_gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               SMEM_BYTES);
+    err = cudaFuncSetAttribute(cond_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (err != cudaSuccess) return err;
     done[dev & 63] = 1;
   }
   return cudaSuccess;
-}
-
-unsigned persistent_grid(long long tiles_max) {
-  DeviceInfo info{0, 148};
-  device_info(&info);
-  long long g = info.sm_count;
-  if (tiles_max < g) g = tiles_max;
-  return (unsigned)(g > 0 ? g : 1);
 }
 
 }  // namespace
@@ -455,61 +563,50 @@ cudaError_t launch_pack(const PackArgs& a, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_correct_tc(const TcCorrectArgs& a, cudaStream_t stream) {
+cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream) {
   const long long rmax = (long long)a.B * (a.K - 1);
-  if (rmax <= 0) return cudaSuccess;
-  cudaError_t err = ensure_smem_attr<0>();
+  if (rmax <= 0 || (!a.do_correct && !a.do_gate)) return cudaSuccess;
+  cudaError_t err = ensure_smem_attr();
   if (err != cudaSuccess) return err;
-  CUtensorMap mA, mB;
-  if (encode_tensor_map_2d(&mA, a.apack, (uint64_t)2 * a.d, (uint64_t)rmax, (uint64_t)a.d * 4, BK, BM) !=
-          CUDA_SUCCESS ||
-      encode_tensor_map_2d(&mB, a.Wc, (uint64_t)2 * a.d, (uint64_t)a.d, (uint64_t)a.d * 4, BK, 256) != CUDA_SUCCESS)
+  const uint64_t d = (uint64_t)a.d;
+  CUtensorMap mApack, mWc, mR, mE, mWv, mWg;
+  // Maps of operands a call does not use point at a used buffer (never read).
+  const void* apack = a.do_correct ? a.apack : a.rpack;
+  const void* wc = a.do_correct ? a.Wc : a.Wv;
+  const void* rp = a.do_gate ? a.rpack : a.apack;
+  const void* erows = (a.do_gate && a.e_dense) ? a.epack : rp;
+  const void* wv = a.do_gate ? a.Wv : a.Wc;
+  const void* wg = a.do_gate ? a.Wg : a.Wc;
+  if (encode_tensor_map_2d(&mApack, apack, a.do_correct ? 2 * d : d, (uint64_t)rmax, (a.do_correct ? 4 : 2) * d, BK, BM) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWc, wc, a.do_correct ? 2 * d : d, d, (a.do_correct ? 4 : 2) * d, BK, 256) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mR, rp, d, (uint64_t)rmax, 2 * d, BK, BM) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mE, erows, d, (uint64_t)rmax, 2 * d, BK, BM) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWv, wv, a.do_gate ? d : 2 * d, d, (a.do_gate ? 2 : 4) * d, BK, 128) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWg, wg, 2 * d, d, 4 * d, BK, 128) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  TcParams p{};
+  CondParams p{};
   p.d = a.d;
-  p.tiles_n = a.d / 256;
+  p.do_correct = a.do_correct;
+  p.do_gate = a.do_gate;
   p.R = a.R;
   p.rowmap = a.rowmap;
   p.apack = reinterpret_cast<const __nv_bfloat16*>(a.apack);
   p.beta = a.beta;
-  p.out = reinterpret_cast<__nv_bfloat16*>(a.r_out);
+  p.r_out = reinterpret_cast<__nv_bfloat16*>(a.r_out);
   p.compact_out = a.compact_out;
-  p.status = a.status;
-  p.Wg = reinterpret_cast<const __nv_bfloat16*>(a.Wg);
-  p.e_vec = reinterpret_cast<const __nv_bfloat16*>(a.e_vec);
-  p.ge_out = a.ge_out;
-  const long long tiles_max = (rmax + BM - 1) / BM * p.tiles_n;
-  tc_gemm_kernel<0><<<persistent_grid(tiles_max), THREADS, SMEM_BYTES, stream>>>(mA, mA, mB, mB, p);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_gate_tc(const TcGateArgs& a, cudaStream_t stream) {
-  const long long rmax = (long long)a.B * (a.K - 1);
-  if (rmax <= 0) return cudaSuccess;
-  cudaError_t err = ensure_smem_attr<1>();
-  if (err != cudaSuccess) return err;
-  CUtensorMap mA0, mA1, mB0, mB1;
-  const void* e_rows = a.e_dense ? a.epack : a.rpack;
-  if (encode_tensor_map_2d(&mA0, a.rpack, (uint64_t)a.d, (uint64_t)rmax, (uint64_t)a.d * 2, BK, BM) !=
-          CUDA_SUCCESS ||
-      encode_tensor_map_2d(&mA1, e_rows, (uint64_t)a.d, (uint64_t)rmax, (uint64_t)a.d * 2, BK, BM) !=
-          CUDA_SUCCESS ||
-      encode_tensor_map_2d(&mB0, a.Wv, (uint64_t)a.d, (uint64_t)a.d, (uint64_t)a.d * 2, BK, 128) != CUDA_SUCCESS ||
-      encode_tensor_map_2d(&mB1, a.Wg, (uint64_t)2 * a.d, (uint64_t)a.d, (uint64_t)a.d * 4, BK, 128) !=
-          CUDA_SUCCESS)
-    return cudaErrorInvalidValue;
-  TcParams p{};
-  p.d = a.d;
-  p.tiles_n = a.d / 128;
-  p.R = a.R;
-  p.rowmap = a.rowmap;
   p.e = reinterpret_cast<const __nv_bfloat16*>(a.e_dense ? a.epack : a.e);
   p.e_dense = a.e_dense;
+  p.Wg = reinterpret_cast<const __nv_bfloat16*>(a.Wg);
   p.ge = a.ge;
-  p.out = reinterpret_cast<__nv_bfloat16*>(a.e_out);
+  p.e_out = reinterpret_cast<__nv_bfloat16*>(a.e_out);
+  p.sync = a.sync;
   p.status = a.status;
-  const long long tiles_max = (rmax + BM - 1) / BM * p.tiles_n;
-  tc_gemm_kernel<1><<<persistent_grid(tiles_max), THREADS, SMEM_BYTES, stream>>>(mA0, mA1, mB0, mB1, p);
+  DeviceInfo info{0, 148};
+  err = device_info(&info);
+  if (err != cudaSuccess) return err;
+  const long long tiles_max = (rmax + BM - 1) / BM * ((a.do_correct ? a.d / 256 : 0) + (a.do_gate ? a.d / 128 : 0));
+  const unsigned grid = (unsigned)(tiles_max < info.sm_count ? tiles_max : info.sm_count);
+  cond_kernel<<<grid, THREADS, SMEM_BYTES, stream>>>(mApack, mWc, mR, mE, mWv, mWg, p);
   return cudaGetLastError();
 }
 

@@ -15,7 +15,9 @@ constexpr int kMaxK = 1024;  // largest draft block the kernels accept
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Workspace layout (all offsets 256-byte aligned):
-//   status   uint32 [64]        [0] device status word, [kRowCountSlot] R of the last pack
+//   status   uint32 [64]        [0] device status word
+//   sync     uint32 [32+blocks] counters of a conditioning pass (row count, tile queue,
+//                               gate-bias progress, per-128-row-block progress)
 //   keys     uint64 [B*(K+1)]   per-row argmax keys, zero between calls
 //   tickets  uint32 [B]         per-sequence CTA arrival counters, zero between calls
 //   ge       fp32   [d]         W_g[:, :d] e for a broadcast e
@@ -23,10 +25,8 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 //   apack    elem   [R_max, 2d] packed [m; u] rows (tensor-core path)
 //   epack    elem   [R_max, d]  packed per-position e rows (tensor-core path, dense e)
 //   rowmap   int32  [R_max]     packed row g -> position b*K + j
-constexpr int kRowCountSlot = 16;
-
 struct WsLayout {
-  size_t status, keys, tickets, ge, r, apack, epack, rowmap, total;
+  size_t status, sync, sync_bytes, keys, tickets, ge, r, apack, epack, rowmap, total;
 };
 
 inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
@@ -37,6 +37,9 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   size_t off = 0;
   L.status = off;
   off = align_up(off + 64 * 4, 256);
+  L.sync = off;
+  L.sync_bytes = align_up((32 + (rmax + 127) / 128) * 4, 256);
+  off += L.sync_bytes;
   L.keys = off;
   off = align_up(off + (size_t)(B * (K + 1)) * 8, 256);
   L.tickets = off;
@@ -145,38 +148,37 @@ struct PackArgs {
 };
 cudaError_t launch_pack(const PackArgs& a, cudaStream_t stream);
 
-struct TcCorrectArgs {
+// Counters of one conditioning pass (uint32, zeroed before each pass).
+constexpr int kSyncRowCount = 0;    // packed rows claimed / R
+constexpr int kSyncTileQueue = 1;   // next tile of the dynamic schedule
+constexpr int kSyncGemvNext = 2;    // next row of W_g[:, :d] e
+constexpr int kSyncGemvDone = 3;    // rows of W_g[:, :d] e written
+constexpr int kSyncBlockDone = 32;  // per 128-row block: correction epilogue warps done
+
+struct TcCondArgs {
   int B, K, d;
+  int do_correct, do_gate;
+  // correction: r = m + beta * W_c [m; u] over the packed [m; u] rows
   const void* apack;
   const void* Wc;
   float beta;
-  const int32_t* R;
-  const int32_t* rowmap;
   void* r_out;
   int compact_out;  // 1: r_out is compact [R_max, d]; 0: r_out is [B, K, d] (rows via rowmap)
-  uint32_t* status;
-  // Optional: also compute ge_out = W_g[:, :d] e_vec for a broadcast e.
-  const void* Wg;
-  const void* e_vec;
-  float* ge_out;
-};
-cudaError_t launch_correct_tc(const TcCorrectArgs& a, cudaStream_t stream);
-
-struct TcGateArgs {
-  int B, K, d;
-  const void* rpack;  // compact r [R_max, d]
-  const void* e;      // broadcast vector [d] (when !e_dense)
-  const void* epack;  // packed e rows [R_max, d] (when e_dense)
+  // gate: e~ = e + (W_v r) .* sigmoid(W_g [e; r]) over the compact r rows
+  const void* rpack;
+  const void* e;
+  const void* epack;
   int e_dense;
-  const float* ge;
   const void* Wv;
   const void* Wg;
+  float* ge;  // [d] scratch for W_g[:, :d] e (broadcast e)
+  void* e_out;
   const int32_t* R;
   const int32_t* rowmap;
-  void* e_out;
+  uint32_t* sync;
   uint32_t* status;
 };
-cudaError_t launch_gate_tc(const TcGateArgs& a, cudaStream_t stream);
+cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream);
 
 // Writes n_out and the rows j >= n_b (zeros for r, a copy of e for e_out).
 cudaError_t launch_fill_rows(int B, int K, int d, RowSource rows, int32_t* n_out, void* zero_dst,
