@@ -10,7 +10,9 @@ from .retrace_oracle import (  # noqa: F401
     bf16_bits_to_f64,
     bf16_ulp,
     carried_rows,
+    VARIANTS,
     commit,
+    condition,
     conditioned_rows,
     correct,
     f64_to_bf16_bits,

@@ -240,11 +240,45 @@ def gate_fuse(e: np.ndarray, r: np.ndarray, n: np.ndarray, Wv: np.ndarray, Wg: n
     return np.where(rows[..., None], fused, e)
 
 
-def retrace_round(logits, draft, hD, hT, e, Wc, Wv, Wg, beta, dtype: str) -> dict:
+VARIANTS = ("corrected", "raw", "overwrite", "none")
+
+
+def condition(e_full, m, u, n, Wc, Wv, Wg, beta, variant: str, round_r_bf16: bool):
+    """How the aligned signal enters the next block; returns (r, e~).
+
+    The component ablation (Sec. "Component Ablation", Table 3; Appendix
+    "Ablation Settings") compares variants that build the same aligned
+    signal m (Eq. 4) and differ only in how it is used:
+
+    * ``corrected``: the method, r = m + beta W_c [m; u] (Eq. 6-7), then the
+      gated fusion of Eq. 8;
+    * ``raw``: the gated fusion of Eq. 8 without correction, r = m;
+    * ``overwrite``: the aligned states replace the mask inputs, e~_j = m_j;
+    * ``none``: no conditioning (the DFlash row of Table 3), e~ = e.
+
+    In every variant positions j >= n_b keep e.  r is None where a variant
+    has none.
+    """
+    if variant == "corrected":
+        r = correct(m, u, Wc, beta, round_r_bf16)
+        return r, gate_fuse(e_full, r, n, Wv, Wg)
+    if variant == "raw":
+        return m, gate_fuse(e_full, m, n, Wv, Wg)
+    K = m.shape[1]
+    rows = np.arange(K)[None, :] < np.asarray(n)[:, None]  # [B, K]
+    if variant == "overwrite":
+        return None, np.where(rows[..., None], m, e_full)
+    if variant == "none":
+        return None, np.array(e_full, dtype=np.float64, copy=True)
+    raise ValueError(f"unknown variant {variant!r}")
+
+
+def retrace_round(logits, draft, hD, hT, e, Wc, Wv, Wg, beta, dtype: str, variant: str = "corrected") -> dict:
     """One round: verify, then condition the next block (Algorithm 1).
 
     ``dtype`` is "bf16" or "f32", the precision of the GPU path being checked;
     it decides only whether r and the output are rounded to bfloat16.
+    ``variant`` is one of ``VARIANTS`` (see :func:`condition`).
     Returns the verification outputs plus ``n``, ``r`` and ``e_tilde``
     (float64) and, for bf16, ``e_tilde_rounded``.
     """
@@ -253,9 +287,8 @@ def retrace_round(logits, draft, hD, hT, e, Wc, Wv, Wg, beta, dtype: str) -> dic
     K = np.asarray(draft).shape[1]
     n = carried_rows(A, K)
     m, u = align(hD, hT, A)
-    r = correct(m, u, Wc, beta, round_r_bf16=(dtype == "bf16"))
     e_full = np.broadcast_to(np.asarray(e, dtype=np.float64), np.asarray(hD).shape)
-    e_tilde = gate_fuse(e_full, r, n, Wv, Wg)
+    r, e_tilde = condition(e_full, m, u, n, Wc, Wv, Wg, beta, variant, round_r_bf16=(dtype == "bf16"))
     out.update({"n": n, "r": r, "e_tilde": e_tilde})
     if dtype == "bf16":
         out["e_tilde_rounded"] = round_to_bf16(e_tilde)

@@ -313,6 +313,71 @@ def test_conditioned_rows_agree_with_full_round():
 
 
 # ---------------------------------------------------------------------------
+# Ablation variants (Sec. "Component Ablation", Table 3; Appendix "Ablation
+# Settings"): the same aligned signal, used three other ways
+# ---------------------------------------------------------------------------
+
+
+def test_fig3_overwrite_carries_the_rejected_suffix():
+    """Overwrite: the next block starts with the drafter states of "but he"
+    (Fig. 3) in place of the mask inputs; the other positions keep e."""
+    fx, vocab, tok = _fig3()
+    K, V, d = len(fx["draft"]), len(vocab), 3
+    draft = np.array([[tok[w] for w in fx["draft"]]])
+    logits = np.zeros((1, K + 1, V))
+    for i, w in enumerate(fx["target_choice_per_slot"]):
+        logits[0, i, tok["<unstated>" if w == "<unstated>" else w]] = 1.0
+    hD = np.zeros((1, K, d))
+    for k in range(K):
+        hD[0, k] = [draft[0, k], 10.0 + k, -0.5 * k]  # label, slot, a third distinct value
+    hT = np.full((1, K, d), 7.0)
+    e_vec = np.array([-1.0, -2.0, -3.0])
+    out = oracle.retrace_round(logits, draft, hD, hT, e_vec, None, None, None, 1.0, "f32", variant="overwrite")
+    n = fx["expected"]["carried_rows"]
+    assert int(out["n"][0]) == n
+    assert [vocab[int(out["e_tilde"][0, j, 0])] for j in range(n)] == fx["expected"]["carried_draft_tokens"]
+    A = fx["expected"]["accept_len"]
+    for j in range(n):  # the whole state row of slot A+1+j, bit for bit
+        assert np.array_equal(out["e_tilde"][0, j], hD[0, A + 1 + j])
+    assert np.array_equal(out["e_tilde"][0, n:], np.broadcast_to(e_vec, (K - n, d)))
+
+
+def _brute_rows(x, b, beta):
+    return bf.round_brute(x["logits"][b].tolist(), x["draft"][b].tolist(), x["hD"][b].tolist(), x["hT"][b].tolist(),
+                          x["e"][b].tolist(), x["Wc"].tolist(), x["Wv"].tolist(), x["Wg"].tolist(), beta)
+
+
+def test_raw_is_the_gated_fusion_of_the_aligned_draft_states():
+    """Raw conditioning, gated: Eq. 8 with r = m, which is the brute-force
+    round at beta = 0 (there r = m + 0 * c = m exactly).  The oracle is given
+    a non-zero beta, which the raw variant must ignore."""
+    rng = np.random.default_rng(21)
+    for B, K, V, d in [(3, 5, 11, 4), (2, 8, 7, 3), (4, 2, 5, 2)]:
+        x = _tiny(rng, B, K, V, d)
+        out = oracle.retrace_round(x["logits"], x["draft"], x["hD"], x["hT"], x["e"], x["Wc"], x["Wv"], x["Wg"],
+                                   x["beta"], "f32", variant="raw")
+        for b in range(B):
+            want = _brute_rows(x, b, 0.0)
+            assert int(out["n"][b]) == want["n"]
+            np.testing.assert_allclose(out["e_tilde"][b], np.array(want["e_tilde"]), rtol=1e-12, atol=1e-12)
+        corrected = oracle.retrace_round(x["logits"], x["draft"], x["hD"], x["hT"], x["e"], x["Wc"], x["Wv"],
+                                         x["Wg"], x["beta"], "f32")
+        if int(out["n"].sum()) > 0:  # the correction changes something where rows are carried
+            assert not np.allclose(out["e_tilde"], corrected["e_tilde"])
+
+
+def test_none_keeps_every_input_and_still_reports_n():
+    """No conditioning (the DFlash row): e~ = e everywhere; n_b is still the
+    carried-row count of the verification."""
+    rng = np.random.default_rng(22)
+    x = _tiny(rng, 4, 6, 9, 3)
+    out = oracle.retrace_round(x["logits"], x["draft"], x["hD"], x["hT"], x["e"], None, None, None, x["beta"],
+                               "bf16", variant="none")
+    assert np.array_equal(out["e_tilde"], x["e"])
+    assert [int(v) for v in out["n"]] == [_brute_rows(x, b, x["beta"])["n"] for b in range(4)]
+
+
+# ---------------------------------------------------------------------------
 # Planted mistakes: every one must make at least one pin above fail
 # ---------------------------------------------------------------------------
 
@@ -329,6 +394,9 @@ def _pins():
         test_half_open_gate_and_identity_value_projection,
         test_zero_correction_keeps_the_aligned_draft_state,
         test_sigmoid_reference_values,
+        test_fig3_overwrite_carries_the_rejected_suffix,
+        test_raw_is_the_gated_fusion_of_the_aligned_draft_states,
+        test_none_keeps_every_input_and_still_reports_n,
     ]
 
 
@@ -365,7 +433,26 @@ def _mut_align_keep_rejected(hD, hT, A):
     return m, u
 
 
+def _mut_condition(change):
+    def f(e_full, m, u, n, Wc, Wv, Wg, beta, variant, rr):
+        return orc.__dict__["_orig_condition"](e_full, m, u, n, Wc, Wv, Wg, beta, change.get(variant, variant), rr)
+    return f
+
+
+def _mut_overwrite_unshifted(e_full, m, u, n, Wc, Wv, Wg, beta, variant, rr):
+    if variant != "overwrite":
+        return orc.__dict__["_orig_condition"](e_full, m, u, n, Wc, Wv, Wg, beta, variant, rr)
+    K = m.shape[1]
+    rows = np.arange(K)[None, :] < np.asarray(n)[:, None]
+    shifted = np.concatenate([m[:, -1:], m[:, :-1]], axis=1)  # rows land one position late
+    return None, np.where(rows[..., None], shifted, e_full)
+
+
 MUTATIONS = {
+    "overwrite keeps the mask inputs": ("condition", _mut_condition({"overwrite": "none"})),
+    "raw applies the correction": ("condition", _mut_condition({"raw": "corrected"})),
+    "no conditioning runs the gate": ("condition", _mut_condition({"none": "raw"})),
+    "overwrite rows one position late": ("condition", _mut_overwrite_unshifted),
     "argmax picks the last maximum": ("target_argmax", _mut_argmax_last),
     "accept length counts all matches": (
         "accepted_length",
@@ -395,6 +482,7 @@ MUTATIONS = {
 def test_planted_mistakes_are_caught(name, monkeypatch):
     attr, fn = MUTATIONS[name]
     monkeypatch.setitem(orc.__dict__, "_orig_gate_fuse", orc.gate_fuse)
+    monkeypatch.setitem(orc.__dict__, "_orig_condition", orc.condition)
     monkeypatch.setattr(orc, attr, fn)
     monkeypatch.setattr(oracle, attr, fn, raising=False)
     caught = 0
