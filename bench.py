@@ -47,6 +47,7 @@ from paper_2608_29748_gb300.workloads import CONFIGS, PROFILE_CONFIG, RoundConfi
 
 METRIC = "verify+ReTrace rounds/sec at 1 GB300; logits HBM GB/s and % of roofline"
 UNIT = "rounds/s"
+KERNELS_PER_ROUND_FUSED = 1  # cond_kernel<FUSED>: the whole round
 KERNELS_PER_ROUND = 2  # verify_kernel (+ row packing), cond_kernel (both projections + gate-bias GEMV)
 L2_FLUSH_BYTES = 256 << 20
 # DRAM traffic of one verify_kernel launch per sequence of the serving shapes
@@ -57,6 +58,9 @@ L2_FLUSH_BYTES = 256 << 20
 # re-measured whenever verify_kernel changes.
 VERIFY_TRAFFIC_PER_SEQUENCE = (685630208 + 3001344) / 128
 VERIFY_TRAFFIC_SHAPE = (16, 151936, 4096, "bf16")
+# DRAM traffic of the single-kernel round per sequence (same shapes, same
+# profiling workload and method); None until measured for the current kernel.
+ROUND_TRAFFIC_PER_SEQUENCE = None
 
 
 # ---------------------------------------------------------------------------
@@ -191,13 +195,13 @@ def prepare_oracle_sample(cfg: RoundConfig, sample_B: int, seed: int) -> dict:
     return host
 
 
-def time_oracle(host: dict) -> float:
+def time_oracle(host: dict, variant: str = "corrected") -> float:
     """Seconds the CPU oracle takes for one round over the prepared sample."""
     from oracle import retrace_round as oracle_round_fn  # test infrastructure: CPU-baseline legs only
 
     t0 = time.perf_counter()
     oracle_round_fn(host["logits"], host["draft"], host["hD"], host["hT"], host["e"], host["Wc"], host["Wv"],
-                    host["Wg"], host["beta"], host["dtype"])
+                    host["Wg"], host["beta"], host["dtype"], variant=variant)
     return time.perf_counter() - t0
 
 
@@ -206,25 +210,52 @@ def time_oracle(host: dict) -> float:
 # ---------------------------------------------------------------------------
 
 
-def verify_bytes(cfg: RoundConfig, n: np.ndarray, packs_rows: bool) -> int:
-    """Algorithmic bytes of one verification launch in a fused round."""
+VARIANT_FLAGS = {"corrected": 0, "raw": 0x2, "overwrite": 0x4, "none": 0x8}  # include/retrace.h
+ROUND_OVERLAP_FLAG = 0x1
+
+
+def verify_bytes(cfg: RoundConfig, n: np.ndarray, packs_rows: bool, variant: str = "corrected") -> int:
+    """Algorithmic bytes of one verification launch of a round."""
     es = cfg.elem_bytes
     B, K, V, d = cfg.B, cfg.K, cfg.V, cfg.d
     logits = B * (K + 1) * V * es
     tokens_in = B * K * 4
     tokens_out = B * (K + 1) * 4 + 3 * B * 4  # committed; accept_len, bonus, n
-    copies = int(np.sum(K - n)) * d * es  # unconditioned rows of e~ written
     R = int(np.sum(n))
+    if variant in ("overwrite", "none"):  # verification writes every row of e~
+        copies = B * K * d * es + (R * d * es if variant == "overwrite" else 0)  # + the m rows read
+        return logits + tokens_in + tokens_out + copies
+    copies = int(np.sum(K - n)) * d * es  # unconditioned rows of e~ written
     packing = (2 * R * 2 * d * es + R * 4) if packs_rows else 0  # [m; u] rows read + written, row map
     return logits + tokens_in + tokens_out + copies + packing
 
 
-def conditioning_flops(cfg: RoundConfig, R: int, dense_e: bool) -> int:
+def conditioning_flops(cfg: RoundConfig, R: int, dense_e: bool, variant: str = "corrected") -> int:
     d = cfg.d
-    f = 2 * R * (2 * d) * d  # c = W_c [m; u]
+    if variant in ("overwrite", "none"):
+        return 0
+    f = 2 * R * (2 * d) * d if variant == "corrected" else 0  # c = W_c [m; u]
     f += 2 * R * d * (2 * d)  # [v; g_r] = [W_v; W_g,r] r
     f += 2 * R * d * d if dense_e else 2 * d * d  # W_g,e e (per row, or once for a broadcast e)
     return f
+
+
+def round_hbm_bytes(cfg: RoundConfig, R: int) -> int:
+    """Algorithmic HBM bytes of one round: what must cross HBM at least once.
+
+    Logits, draft tokens and outputs, the 2R conditioned hidden-state rows,
+    the three weight matrices (5 d^2 elements), the mask embedding and e~.
+    Packed intermediates are not counted (they can live in L2)."""
+    es = cfg.elem_bytes
+    B, K, V, d = cfg.B, cfg.K, cfg.V, cfg.d
+    return (B * (K + 1) * V * es + B * K * 4 + B * (K + 1) * 4 + 3 * B * 4
+            + 2 * R * d * es + 5 * d * d * es + d * es + B * K * d * es)
+
+
+def round_is_fused(cfg: RoundConfig) -> bool:
+    """Whether retrace_round takes the single-kernel path for this workload
+    (bf16, d a multiple of 256, 16-byte aligned logits rows, K >= 2)."""
+    return cfg.dtype == "bf16" and cfg.d % 256 == 0 and cfg.V % 8 == 0 and cfg.K >= 2
 
 
 def run_gpu(args) -> dict | None:
@@ -246,8 +277,12 @@ def run_gpu(args) -> dict | None:
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
 
+    fused = args.overlap and round_is_fused(cfg)
+    if args.overlap and not fused:
+        raise SystemExit("--overlap: the overlapped kernel does not cover this workload")
+    flags = VARIANT_FLAGS[args.variant] | (ROUND_OVERLAP_FLAG if fused else 0)
     for _ in range(args.warmup):
-        rt.run_round(x, ws, out=out)
+        rt.run_round(x, ws, out=out, flags=flags)
     torch.cuda.synchronize(dev)
 
     steps = args.steps
@@ -263,7 +298,7 @@ def run_gpu(args) -> dict | None:
         t_wall0 = time.perf_counter()
         for i in range(steps):
             flush.fill_(i & 0xFF)  # L2 flush: a 256 MB write between timed steps
-            rt.run_round(x, ws, out=out, phase_events=phase[i])
+            rt.run_round(x, ws, out=out, flags=flags, phase_events=phase[i])
         torch.cuda.synchronize(dev)
         t_wall = time.perf_counter() - t_wall0
     barrier(world)
@@ -277,17 +312,77 @@ def run_gpu(args) -> dict | None:
 
     n = out.n.cpu().numpy().astype(np.int64)
     R = int(n.sum())
-    packs_rows = cfg.dtype == "bf16" and cfg.d % 256 == 0  # tensor-core path: verify packs the rows
-    vbytes = verify_bytes(cfg, n, packs_rows)
-    v_avg_s = statistics.mean(verify_ms) / 1e3
-    v_gbs = vbytes / v_avg_s / 1e9
-    cflops = conditioning_flops(cfg, R, dense_e=False)
-    c_avg_s = statistics.mean(cond_ms) / 1e3
-    c_tflops = cflops / c_avg_s / 1e12
-    flags = ws.check()
+    step_avg_s = statistics.mean(step_ms) / 1e3
+    cflops = conditioning_flops(cfg, R, dense_e=False, variant=args.variant)
+    status_flags = ws.check()
+    if fused:
+        # One kernel does the whole round: its floor is the larger of the HBM
+        # time of its algorithmic bytes and the tensor time of its flops.
+        hbytes = round_hbm_bytes(cfg, R)
+        t_hbm = hbytes / (peaks["hbm_gbs"] * 1e9)
+        t_tc = cflops / (peaks["bf16_tflops_sustained"] * 1e12)
+        hbm_bound = t_hbm >= t_tc
+        roofline = {
+            "kernel": "cond_kernel<FUSED> (verification + both projections, one persistent launch per round)",
+            "bound": "hbm" if hbm_bound else "tensor",
+            "achieved": round(hbytes / step_avg_s / 1e9, 1) if hbm_bound else round(cflops / step_avg_s / 1e12, 2),
+            "peak": peaks["hbm_gbs"] if hbm_bound else peaks["bf16_tflops_sustained"],
+            "unit": "GB/s" if hbm_bound else "TFLOP/s",
+            "frac": round(max(t_hbm, t_tc) / step_avg_s, 4),
+            "peak_source": peaks["source"] + (" HBM copy bandwidth" if hbm_bound else " sustained bf16 (cuBLAS)"),
+            "algorithmic_bytes": hbytes,
+            "algorithmic_flops": cflops,
+            "floor_us": {"hbm": round(t_hbm * 1e6, 1), "tensor": round(t_tc * 1e6, 1)},
+            "avg_launch_us": round(step_avg_s * 1e6, 2),
+            "traffic": (round(ROUND_TRAFFIC_PER_SEQUENCE * cfg.B)
+                        if ROUND_TRAFFIC_PER_SEQUENCE and (cfg.K, cfg.V, cfg.d, cfg.dtype) == VERIFY_TRAFFIC_SHAPE
+                        else None),
+            "traffic_source": "ncu dram read+write on B=128 profiling workload, scaled by B/128",
+        }
+        line_extra = {"hbm_view": {"achieved_gbs": round(hbytes / step_avg_s / 1e9, 1),
+                                   "frac": round(t_hbm / step_avg_s, 4)},
+                      "tensor_view": {"achieved_tflops": round(cflops / step_avg_s / 1e12, 2),
+                                      "frac": round(t_tc / step_avg_s, 4)}}
+        logits_gbs = cfg.logits_bytes() / step_avg_s / 1e9
+    else:
+        packs_rows = cfg.dtype == "bf16" and cfg.d % 256 == 0  # tensor-core path: verify packs the rows
+        vbytes = verify_bytes(cfg, n, packs_rows and args.variant in ("corrected", "raw"), args.variant)
+        v_avg_s = statistics.mean(verify_ms) / 1e3
+        v_gbs = vbytes / v_avg_s / 1e9
+        c_avg_s = statistics.mean(cond_ms) / 1e3
+        c_tflops = cflops / c_avg_s / 1e12
+        roofline = {
+            "kernel": "verify_kernel (argmax/compare/commit + copy of unconditioned rows + row packing)",
+            "bound": "hbm",
+            "achieved": round(v_gbs, 1),
+            "peak": peaks["hbm_gbs"],
+            "unit": "GB/s",
+            "frac": round(v_gbs / peaks["hbm_gbs"], 4),
+            "peak_source": peaks["source"] + " HBM copy bandwidth",
+            "algorithmic_bytes": vbytes,
+            "avg_launch_us": round(v_avg_s * 1e6, 2),
+            "traffic": (round(VERIFY_TRAFFIC_PER_SEQUENCE * cfg.B)
+                        if VERIFY_TRAFFIC_PER_SEQUENCE and (cfg.K, cfg.V, cfg.d, cfg.dtype) == VERIFY_TRAFFIC_SHAPE
+                        else None),
+            "traffic_source": "ncu dram read+write on B=128 profiling workload, scaled by B/128",
+        }
+        line_extra = {} if cflops == 0 else {"roofline_conditioning": {
+            "kernels": "cond_kernel: correction + gated-fusion projections (+ gate-bias GEMV), one persistent launch",
+            "bound": "tensor",
+            "achieved": round(c_tflops, 2),
+            "peak": peaks["bf16_tflops_sustained"],
+            "unit": "TFLOP/s",
+            "frac": round(c_tflops / peaks["bf16_tflops_sustained"], 4),
+            "peak_source": peaks["source"] + " sustained bf16 (cuBLAS)",
+            "algorithmic_flops": cflops,
+            "avg_us": round(c_avg_s * 1e6, 2),
+        }}
+        if args.variant in ("overwrite", "none"):
+            roofline["kernel"] = "verify_kernel (argmax/compare/commit + every row of e~ copied)"
+        logits_gbs = cfg.logits_bytes() / v_avg_s / 1e9
 
     # ---- end to end through the public API with host buffers ----
-    e2e = run_e2e(rt, cfg, x, ws, dev, min(steps, args.e2e_steps), world) if args.e2e_steps > 0 else None
+    e2e = run_e2e(rt, cfg, x, ws, dev, min(steps, args.e2e_steps), world, flags) if args.e2e_steps > 0 else None
 
     line = {
         "metric": METRIC,
@@ -309,38 +404,17 @@ def run_gpu(args) -> dict | None:
             "conditioned_rows_R": R,
             "l2": "flushed before every timed step (256 MB write, outside the per-step events)",
             "parallelism": f"replicas x{world} (batch-sharded, no collective)",
+            "variant": args.variant,
+            "round_kernel": "overlapped (one persistent launch)" if fused else "two launches (verify, projections)",
         },
-        "roofline": {
-            "kernel": "verify_kernel (argmax/compare/commit + copy of unconditioned rows + row packing)",
-            "bound": "hbm",
-            "achieved": round(v_gbs, 1),
-            "peak": peaks["hbm_gbs"],
-            "unit": "GB/s",
-            "frac": round(v_gbs / peaks["hbm_gbs"], 4),
-            "peak_source": peaks["source"] + " HBM copy bandwidth",
-            "algorithmic_bytes": vbytes,
-            "avg_launch_us": round(v_avg_s * 1e6, 2),
-            "traffic": (round(VERIFY_TRAFFIC_PER_SEQUENCE * cfg.B)
-                        if VERIFY_TRAFFIC_PER_SEQUENCE and (cfg.K, cfg.V, cfg.d, cfg.dtype) == VERIFY_TRAFFIC_SHAPE
-                        else None),
-            "traffic_source": "ncu dram read+write on B=128 profiling workload, scaled by B/128",
-        },
-        "roofline_conditioning": {
-            "kernels": "cond_kernel: correction + gated-fusion projections (+ gate-bias GEMV), one persistent launch",
-            "bound": "tensor",
-            "achieved": round(c_tflops, 2),
-            "peak": peaks["bf16_tflops_sustained"],
-            "unit": "TFLOP/s",
-            "frac": round(c_tflops / peaks["bf16_tflops_sustained"], 4),
-            "peak_source": peaks["source"] + " sustained bf16 (cuBLAS)",
-            "algorithmic_flops": cflops,
-            "avg_us": round(c_avg_s * 1e6, 2),
-        },
-        "logits_gbs": round(cfg.logits_bytes() / v_avg_s / 1e9, 1),
+        "roofline": roofline,
+        **line_extra,
+        "logits_gbs": round(logits_gbs, 1),
         "e2e": e2e,
-        "gpu_launches": KERNELS_PER_ROUND * steps,
+        "gpu_launches": (KERNELS_PER_ROUND_FUSED if fused
+                         else KERNELS_PER_ROUND if cflops else 1) * steps,
         "wall_s_timed_region": round(t_wall, 4),
-        "device_status_flags": flags,
+        "device_status_flags": status_flags,
         "impl": "ours",
     }
     cs = clocks.summary()
@@ -350,7 +424,7 @@ def run_gpu(args) -> dict | None:
     return line if rank == 0 else None
 
 
-def run_e2e(rt, cfg, x, ws, dev, steps, world) -> dict:
+def run_e2e(rt, cfg, x, ws, dev, steps, world, flags=0) -> dict:
     """Rounds/s with the step's inputs in pinned host memory and the outputs read back."""
     names = ["logits", "draft", "hD", "hT"]
     host = {k: x[k].cpu().pin_memory() for k in names}
@@ -364,7 +438,7 @@ def run_e2e(rt, cfg, x, ws, dev, steps, world) -> dict:
     def step():
         for k in names:
             dev_in[k].copy_(host[k], non_blocking=True)
-        rt.run_round({**dev_in, **rest}, ws, out=out)
+        rt.run_round({**dev_in, **rest}, ws, out=out, flags=flags)
         for k, h in out_host.items():
             h.copy_(getattr(out, k), non_blocking=True)
 
@@ -386,7 +460,7 @@ def run_e2e(rt, cfg, x, ws, dev, steps, world) -> dict:
 
 def cpu_baseline(cfg: RoundConfig, args) -> dict:
     host = prepare_oracle_sample(cfg, args.cpu_sample, seed=1234)
-    secs = time_oracle(host)
+    secs = time_oracle(host, args.variant)
     rounds = host["B"] / cfg.B
     return {"value": round(rounds / secs, 6), "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
             "sample": f"{host['B']} of {cfg.B} sequences of {cfg.name}, full-size weights; one round of the "
@@ -405,15 +479,16 @@ def run_reference(args) -> dict | None:
     cfg = workload(args.config)
     host = prepare_oracle_sample(cfg, args.ref_sample, seed=500)
     for _ in range(min(args.warmup, 1)):
-        time_oracle(host)
-    total = sum(time_oracle(host) for _ in range(args.steps))
+        time_oracle(host, args.variant)
+    total = sum(time_oracle(host, args.variant) for _ in range(args.steps))
     value = args.steps * (host["B"] / cfg.B) / total
     return {
         "metric": METRIC, "value": round(value, 6), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(1e3 * total / args.steps, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": f"{cfg.name}: B={cfg.B} K={cfg.K} V={cfg.V} d={cfg.d} {cfg.dtype}",
-                   "sample_per_step": f"{args.ref_sample} of {cfg.B} sequences (full-size weights)"},
+                   "sample_per_step": f"{args.ref_sample} of {cfg.B} sequences (full-size weights)",
+                   "variant": args.variant},
         "impl": "reference",
         "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
                          "sample": f"{args.ref_sample} of {cfg.B} sequences per step, {args.steps} steps, "
@@ -438,6 +513,10 @@ def parse_args(argv=None):
     ap.add_argument("--cpu-sample", type=int, default=32, help="sequences in the CPU-baseline sample")
     ap.add_argument("--ref-sample", type=int, default=2, help="sequences per step in the reference arm")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--overlap", action="store_true",
+                    help="time the overlapped single-kernel round (RETRACE_ROUND_OVERLAP)")
+    ap.add_argument("--variant", choices=sorted(VARIANT_FLAGS), default="corrected",
+                    help="conditioning variant of the component ablation (default: the method)")
     return ap.parse_args(argv)
 
 

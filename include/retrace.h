@@ -167,12 +167,41 @@ retrace_status retrace_gate_fuse(const void* e, int64_t e_batch_stride, int64_t 
                                  retrace_dtype dtype, int B, int K, int d, void* e_out,
                                  void* ws, size_t ws_bytes, cudaStream_t stream);
 
+/* Flags of retrace_round.  With none set the round computes the method as
+ * written (corrected conditioning, gated).  The three conditioning variants of
+ * the component ablation (Sec. "Component Ablation", Table 3; Appendix
+ * "Ablation Settings") build the same aligned signal m_j = hD[b, A_b+1+j] and
+ * differ in how it enters the next block; at most one of them may be set:
+ *   RETRACE_COND_RAW        raw conditioning, gated: no correction, r = m
+ *                           (Eq. 8 applied to the aligned drafter states).
+ *   RETRACE_COND_OVERWRITE  raw conditioning, overwrite: e~_j = m_j for
+ *                           j < n_b (the mask inputs are replaced).
+ *   RETRACE_COND_NONE       no conditioning (the DFlash row): e~ = e.
+ * Rows j >= n_b keep e bit-exactly in every variant, and n_out still reports
+ * n_b.  Wc, Wv and Wg are not read where the variant does not use them (they
+ * may be NULL then).
+ *   RETRACE_ROUND_OVERLAP   run verification and both projections in one
+ *                           persistent launch whose warps overlap the logits
+ *                           stream with the tensor-core work (the corrected
+ *                           method only: bf16, d a multiple of 256, 16-byte
+ *                           aligned contiguous [B, K+1, V] logits with V a
+ *                           multiple of 8 and V >= 4096, K >= 2, 4d <= 16384).
+ *                           Same results bit for bit; other shapes or an
+ *                           ablation flag return RETRACE_ERR_UNSUPPORTED.
+ * Unknown bits, or two ablation flags together, return
+ * RETRACE_ERR_INVALID_ARG. */
+#define RETRACE_ROUND_OVERLAP 0x1u
+#define RETRACE_COND_RAW 0x2u
+#define RETRACE_COND_OVERWRITE 0x4u
+#define RETRACE_COND_NONE 0x8u
+
 /* One full round on one stream: verify, then align/refine and gated fusion of
  * the rejected suffix into the next block's inputs (Algorithm 1).  Arguments
  * have the meaning given above; r stays inside `ws` (compacted to the R =
  * sum_b n_b conditioned rows) and is not returned.  No host synchronisation.
  *   n_out          [B] int32 out, optional (NULL to skip).
  *   target_argmax  [B, K+1] int32 out, optional.
+ *   flags          0, or the RETRACE_ROUND_* / RETRACE_COND_* bits above.
  *   phase_events   optional array of 4 cudaEvent_t recorded on `stream`
  *                  before verification, after it, after the correction
  *                  projection and after the gated fusion (NULL to skip).
@@ -184,7 +213,7 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
                              float beta, retrace_dtype dtype, int B, int K, int V, int d,
                              int32_t* accept_len, int32_t* committed, int32_t* bonus,
                              int32_t* target_argmax, int32_t* n_out, void* e_out, void* ws,
-                             size_t ws_bytes, const cudaEvent_t* phase_events,
+                             size_t ws_bytes, uint32_t flags, const cudaEvent_t* phase_events,
                              cudaStream_t stream);
 
 /* Size in bytes of the fixed device scratch used by retrace_verify_noalloc. */

@@ -53,7 +53,7 @@ def _load() -> ctypes.CDLL:
     lib.retrace_align_refine.argtypes = [P, P, I, I, I, I, P, P, F, P, P, P, SZ, P]
     lib.retrace_gate_fuse.argtypes = [P, I64, I64, P, P, P, P, I, I, I, I, P, P, SZ, P]
     lib.retrace_round.argtypes = [P, I64, I64, P, P, P, P, I64, I64, P, P, P, F, I, I, I, I, I,
-                                  P, P, P, P, P, P, P, SZ, P, P]
+                                  P, P, P, P, P, P, P, SZ, ctypes.c_uint32, P, P]
     for name in ("retrace_workspace_init", "retrace_workspace_check", "retrace_verify",
                  "retrace_align_refine", "retrace_gate_fuse", "retrace_round"):
         getattr(lib, name).restype = I
@@ -167,9 +167,17 @@ def retrace_gate_fuse(e, r, n, Wv, Wg, e_out, ws, stream=None):
                                  _stream(stream)))
 
 
+# retrace_round flags (include/retrace.h)
+ROUND_OVERLAP = 0x1
+COND_RAW = 0x2
+COND_OVERWRITE = 0x4
+COND_NONE = 0x8
+
+
 def retrace_round(logits, draft, hD, hT, e, Wc, Wv, Wg, beta, accept_len, committed, bonus, e_out,
-                  ws, n_out=None, target_argmax=None, phase_events=None, stream=None):
-    """One fused round on one stream (see include/retrace.h)."""
+                  ws, n_out=None, target_argmax=None, flags=0, phase_events=None, stream=None):
+    """One round on one stream (see include/retrace.h); `flags` selects the
+    overlapped kernel or an ablation variant."""
     B, K1, V = logits.shape
     K = K1 - 1
     d = hD.shape[2]
@@ -183,7 +191,8 @@ def retrace_round(logits, draft, hD, hT, e, Wc, Wv, Wg, beta, accept_len, commit
                              _ptr(hT), _ptr(e), ebs, eps, _ptr(Wc), _ptr(Wv), _ptr(Wg), float(beta),
                              _dtype_code(logits), B, K, V, d, _ptr(accept_len), _ptr(committed),
                              _ptr(bonus), _ptr(target_argmax), _ptr(n_out), _ptr(e_out), ws.ptr,
-                             ws.nbytes, ctypes.cast(ev, ctypes.c_void_p) if ev is not None else None,
+                             ws.nbytes, int(flags),
+                             ctypes.cast(ev, ctypes.c_void_p) if ev is not None else None,
                              _stream(stream)))
 
 
@@ -199,7 +208,7 @@ class RoundBuffers:
 
 
 def run_round(x: dict, ws: Workspace, out: RoundBuffers | None = None, target_argmax=None,
-              phase_events=None, stream=None) -> RoundBuffers:
+              flags=0, phase_events=None, stream=None) -> RoundBuffers:
     """retrace_round over a dict of device tensors (keys as in workloads.make_round_inputs)."""
     logits = x["logits"]
     B, K1, _ = logits.shape
@@ -208,7 +217,7 @@ def run_round(x: dict, ws: Workspace, out: RoundBuffers | None = None, target_ar
         out = RoundBuffers(B, K1 - 1, d, logits.dtype, logits.device)
     retrace_round(logits, x["draft"], x["hD"], x["hT"], x["e"], x["Wc"], x["Wv"], x["Wg"], x["beta"],
                   out.accept_len, out.committed, out.bonus, out.e_out, ws, n_out=out.n,
-                  target_argmax=target_argmax, phase_events=phase_events, stream=stream)
+                  target_argmax=target_argmax, flags=flags, phase_events=phase_events, stream=stream)
     return out
 
 

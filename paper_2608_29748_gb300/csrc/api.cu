@@ -299,15 +299,24 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
                              float beta, retrace_dtype dtype, int B, int K, int V, int d,
                              int32_t* accept_len, int32_t* committed, int32_t* bonus,
                              int32_t* target_argmax, int32_t* n_out, void* e_out, void* ws,
-                             size_t ws_bytes, const cudaEvent_t* phase_events,
+                             size_t ws_bytes, uint32_t flags, const cudaEvent_t* phase_events,
                              cudaStream_t stream) {
   g_err[0] = '\0';
+  const uint32_t kAblations = RETRACE_COND_RAW | RETRACE_COND_OVERWRITE | RETRACE_COND_NONE;
+  if (flags & ~(RETRACE_ROUND_OVERLAP | kAblations)) return fail(RETRACE_ERR_INVALID_ARG, "unknown flag bits");
+  const uint32_t ablation = flags & kAblations;
+  if (ablation & (ablation - 1)) return fail(RETRACE_ERR_INVALID_ARG, "at most one RETRACE_COND_* flag");
+  if ((flags & RETRACE_ROUND_OVERLAP) && ablation)
+    return fail(RETRACE_ERR_UNSUPPORTED, "RETRACE_ROUND_OVERLAP runs the corrected method only");
   retrace_status st = check_verify_args(logits, dtype, B, K, V, logits_row_stride,
                                         logits_batch_stride, draft, accept_len, committed, bonus);
   if (st != RETRACE_OK) return st;
   if ((st = check_cond_shape(dtype, B, K, d)) != RETRACE_OK) return st;
   if (B == 0) return RETRACE_OK;
-  if (!hD || !hT || !e || !Wc || !Wv || !Wg || !e_out)
+  // the tensors each variant reads
+  const bool need_gate = ablation == 0 || ablation == RETRACE_COND_RAW;
+  const bool need_wc = ablation == 0;
+  if (!hD || !hT || !e || !e_out || (need_wc && !Wc) || (need_gate && (!Wv || !Wg)))
     return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
   int dense = 0;
   if ((st = e_mode(e_batch_stride, e_pos_stride, K, d, &dense)) != RETRACE_OK) return st;
@@ -317,8 +326,10 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   float* ge = reinterpret_cast<float*>(w + L.ge);
   void* r_ws = w + L.r;
 
-  const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) &&
-                  aligned16(Wv) && aligned16(Wg) && aligned16(e) && aligned16(e_out);
+  const bool tc = need_gate && tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) &&
+                  aligned16(Wc) && aligned16(Wv) && aligned16(Wg) && aligned16(e) && aligned16(e_out);
+  if ((flags & RETRACE_ROUND_OVERLAP) && !tc)
+    return fail(RETRACE_ERR_UNSUPPORTED, "RETRACE_ROUND_OVERLAP: bf16 with d a multiple of 256 and 16-byte aligned tensors only");
   uint32_t* sync = reinterpret_cast<uint32_t*>(w + L.sync);
   int32_t* R = reinterpret_cast<int32_t*>(sync + kSyncRowCount);
   int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
@@ -328,6 +339,52 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   // The verification kernel packs the conditioned rows as sequences finish;
   // they claim packed rows from a counter that starts at zero.
   if (tc) RT_CUDA(cudaMemsetAsync(sync, 0, L.sync_bytes, stream), "cudaMemsetAsync(sync)");
+  if (tc) {
+    TcRoundArgs ra{};
+    ra.logits = logits;
+    ra.B = B;
+    ra.K = K;
+    ra.V = V;
+    ra.d = d;
+    ra.row_stride = logits_row_stride;
+    ra.batch_stride = logits_batch_stride;
+    ra.draft = draft;
+    ra.accept_len = accept_len;
+    ra.committed = committed;
+    ra.bonus = bonus;
+    ra.target_argmax = target_argmax;
+    ra.n_out = n_out;
+    ra.keys = reinterpret_cast<unsigned long long*>(w + L.keys);
+    ra.tickets = reinterpret_cast<uint32_t*>(w + L.tickets);
+    ra.hD = hD;
+    ra.hT = hT;
+    ra.e = e;
+    ra.e_dense = dense;
+    ra.e_batch_stride = e_batch_stride;
+    ra.e_pos_stride = e_pos_stride;
+    ra.Wc = Wc;
+    ra.Wv = Wv;
+    ra.Wg = Wg;
+    ra.beta = beta;
+    ra.e_out = e_out;
+    ra.apack = w + L.apack;
+    ra.epack = w + L.epack;
+    ra.rpack = r_ws;
+    ra.ge = ge;
+    ra.rowmap = rowmap;
+    ra.sync = sync;
+    ra.status = status_word(ws);
+    if (flags & RETRACE_ROUND_OVERLAP) {
+      if (!round_fused_supported(ra))
+        return fail(RETRACE_ERR_UNSUPPORTED, "RETRACE_ROUND_OVERLAP: shape or layout outside the overlapped kernel");
+      // verification and both projections overlap inside one launch
+      RT_CUDA(launch_round_tc(ra, stream), "round kernel launch");
+      if (phase_events) {
+        for (int k = 1; k < 4; ++k) RT_CUDA(cudaEventRecord(phase_events[k], stream), "cudaEventRecord");
+      }
+      return RETRACE_OK;
+    }
+  }
   VerifyArgs va{};
   va.logits = logits;
   va.B = B;
@@ -348,8 +405,11 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   va.e_pos_stride = e_pos_stride;
   va.e_out = e_out;
   va.d = d;
+  va.hD = hD;
+  va.cond_copy = ablation == RETRACE_COND_NONE ? kCondCopyE
+                 : ablation == RETRACE_COND_OVERWRITE ? kCondCopyM
+                                                      : kCondCopyKeep;
   if (tc) {
-    va.hD = hD;
     va.hT = hT;
     va.e_dense = dense;
     va.apack = w + L.apack;
@@ -360,6 +420,14 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   RT_CUDA(launch_verify(va, dtype, stream), "verify kernel launch");
   if (phase_events) RT_CUDA(cudaEventRecord(phase_events[1], stream), "cudaEventRecord");
 
+  if (!need_gate) {
+    // overwrite / no conditioning: verification already wrote every row of e_out
+    if (phase_events) {
+      for (int k = 2; k < 4; ++k) RT_CUDA(cudaEventRecord(phase_events[k], stream), "cudaEventRecord");
+    }
+    return RETRACE_OK;
+  }
+  const bool raw = ablation == RETRACE_COND_RAW;
   if (tc) {
     // Both projections in one persistent launch; its phase events bracket
     // the whole conditioning (the correction/gate split point is not a
@@ -368,14 +436,16 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
     a.B = B;
     a.K = K;
     a.d = d;
-    a.do_correct = 1;
+    a.do_correct = raw ? 0 : 1;
     a.do_gate = 1;
     a.apack = w + L.apack;
     a.Wc = Wc;
     a.beta = beta;
     a.r_out = r_ws;
     a.compact_out = 1;
-    a.rpack = r_ws;
+    // raw: r = m is the first half of each packed [m; u] row
+    a.rpack = raw ? w + L.apack : r_ws;
+    a.r_row_stride = raw ? 2LL * d : 0;
     a.e = e;
     a.epack = w + L.epack;
     a.e_dense = dense;
@@ -390,7 +460,7 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
     RT_CUDA(launch_cond_tc(a, stream), "conditioning kernel launch");
     if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
   } else {
-    CorrectArgs ca{hD, hT, Wc, beta, B, K, d, rows, r_ws, 1};
+    CorrectArgs ca{hD, hT, Wc, beta, B, K, d, rows, r_ws, 1, raw ? 1 : 0};
     RT_CUDA(launch_correct_simt(ca, dtype, stream), "correction kernel launch");
     if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
     if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");

@@ -100,6 +100,9 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                : "memory");
 }
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -113,15 +116,39 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 }
 // Waits for the phase with `parity` to complete.  Gives up (returns false)
 // when *abort becomes non-zero or after kWaitLimitNs; never spins forever.
+// The clock is read only every 256 polls, so a short wait costs no clock read.
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
                                                   volatile int* abort) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const unsigned long long t0 = global_ns();
+  unsigned long long t0 = 0ull;
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 255u) == 0u) {
       if (*abort) return false;
-      if (global_ns() - t0 > kWaitLimitNs) return false;
+      const unsigned long long now = global_ns();
+      if (t0 == 0ull)
+        t0 = now;
+      else if (now - t0 > kWaitLimitNs)
+        return false;
+    }
+  }
+}
+
+// Spins until ready() holds (true), or until *abort becomes non-zero or about
+// kWaitLimitNs have passed (false), sleeping `sleep_ns` between polls; the
+// clock is read every 64 polls only.
+template <typename Ready>
+__device__ __forceinline__ bool spin_until(Ready&& ready, volatile int* abort, unsigned sleep_ns) {
+  unsigned long long t0 = 0ull;
+  for (uint32_t it = 1;; ++it) {
+    if (ready()) return true;
+    if (sleep_ns) __nanosleep(sleep_ns);
+    if ((it & 63u) == 0u) {
+      if (*abort) return false;
+      const unsigned long long now = global_ns();
+      if (t0 == 0ull)
+        t0 = now;
+      else if (now - t0 > kWaitLimitNs)
+        return false;
     }
   }
 }

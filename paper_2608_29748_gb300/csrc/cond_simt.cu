@@ -25,6 +25,7 @@ struct SimtCorrectParams {
   RowSource rows;
   void* out;
   int compact_out;
+  int raw;  // r = m: no accumulation, W_c not read
 };
 
 struct SimtGateParams {
@@ -72,7 +73,7 @@ __global__ void __launch_bounds__(kNT) simt_correct_kernel(const SimtCorrectPara
   const int ty = tid / 16, tx = tid % 16;
   float acc[2][4] = {};
   const int K2 = 2 * d;
-  for (int k0 = 0; k0 < K2; k0 += TK) {
+  for (int k0 = 0; k0 < (p.raw ? 0 : K2); k0 += TK) {
     for (int idx = tid; idx < TM * TK; idx += kNT) {
       const int r = idx / TK, kk = idx % TK, k = k0 + kk;
       float v = 0.f;
@@ -107,8 +108,8 @@ __global__ void __launch_bounds__(kNT) simt_correct_kernel(const SimtCorrectPara
     for (int q = 0; q < 4; ++q) {
       const int n = n0 + 4 * tx + q;
       if (n >= d) continue;
-      const float m = to_f32(hD[s_m[r] + n]);
-      out[orow * d + n] = from_f32<T>(m + p.beta * acc[rr][q]);
+      const T m = hD[s_m[r] + n];
+      out[orow * d + n] = p.raw ? m : from_f32<T>(to_f32(m) + p.beta * acc[rr][q]);
     }
   }
 }
@@ -251,7 +252,7 @@ __global__ void __launch_bounds__(256) fill_rows_kernel(int B, int K, int d, Row
 
 template <typename T>
 cudaError_t correct_typed(const CorrectArgs& a, cudaStream_t stream) {
-  SimtCorrectParams p{a.hD, a.hT, a.Wc, a.beta, a.B, a.K, a.d, a.rows, a.r_out, a.compact_out};
+  SimtCorrectParams p{a.hD, a.hT, a.Wc, a.beta, a.B, a.K, a.d, a.rows, a.r_out, a.compact_out, a.raw};
   const long long rmax = (long long)a.B * (a.K - 1);
   if (rmax <= 0) return cudaSuccess;
   dim3 grid((unsigned)((rmax + TM - 1) / TM), (unsigned)((a.d + TN - 1) / TN));

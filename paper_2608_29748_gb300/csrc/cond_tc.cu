@@ -35,6 +35,7 @@
 #include "common.cuh"
 #include "internal.h"
 #include "plan.cuh"
+#include "verify_stream.cuh"
 
 namespace retrace {
 namespace {
@@ -43,10 +44,15 @@ constexpr int BM = 128;
 constexpr int BK = 64;  // 64 bf16 = 128 bytes = one swizzle row
 constexpr int STAGES = 4;
 constexpr int THREADS = 256;
+constexpr int THREADS_FUSED = 2 * THREADS + 32;  // + consumer warps 8-15 and the bookkeeper warp 16
 constexpr int A_BYTES = BM * BK * 2;   // 16 KB
 constexpr int B_BYTES = 256 * BK * 2;  // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024;  // + slack for 1024-B alignment
+// The fused round kernel keeps three operand stages and gives the rest of the
+// shared memory to the ring that streams the logits.
+constexpr int STAGES_FUSED = 3;
+constexpr int SMEM_BYTES_FUSED = STAGES_FUSED * STAGE_BYTES + kRingBufs * kChunkBytes + kStageBytes + 1024;
 constexpr uint32_t ACC_COLS = 256;
 constexpr uint32_t TMEM_COLS = 2 * ACC_COLS;
 constexpr uint32_t IDESC_N256 = idesc_bf16_f32(128, 256);
@@ -138,6 +144,9 @@ struct CondParams {
   float* ge;  // [d] = W_g[:, :d] e, computed here for a broadcast e
   __nv_bfloat16* e_out;
   uint32_t* sync;
+  uint32_t* block_done;   // per 128-row block: correction epilogue warps finished
+  uint32_t* block_ready;  // per 128-row block: packed rows published (FUSED)
+  int max_blocks;         // 128-row blocks of the largest possible R
   uint32_t* status;
 };
 
@@ -146,15 +155,16 @@ __device__ __forceinline__ void raise_abort(volatile int* s_abort, uint32_t* sta
   atomicOr(status, kFlagWaitTimeout);
 }
 
-// Lane 0 waits, the warp agrees on the outcome.
+// Lane 0 waits, the warp agrees on the outcome.  The __syncwarp orders the
+// other lanes' later reads after lane 0's acquire: without it the compiler may
+// schedule their loads of what the arrive published (a tile index, a row
+// count) before lane 0 has seen the phase complete.
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
   int ok = 1;
   if ((threadIdx.x & 31) == 0) ok = mbar_wait_bounded(bar, parity, abort) ? 1 : 0;
-  return __shfl_sync(0xFFFFFFFFu, ok, 0) != 0;
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+  ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+  __syncwarp();
+  return ok != 0;
 }
 
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
@@ -185,15 +195,56 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 
 constexpr int TILE_SLOTS = 2;
 
+// One warp: rows i of ge = W_g[:, :d] e (broadcast e), claimed from a global
+// counter until all d rows are taken; each finished row is counted.
+__device__ void gate_bias_rows(const CondParams& p, int d, int lane, uint32_t* next, uint32_t* done) {
+  const int vpr = d / 8;
+  const uint4* ev = reinterpret_cast<const uint4*>(p.e);
+  for (;;) {
+    int i = 0;
+    if (lane == 0) i = (int)atomicAdd(next, 1u);
+    i = __shfl_sync(0xFFFFFFFFu, i, 0);
+    if (i >= d) break;
+    const uint4* wr = reinterpret_cast<const uint4*>(p.Wg + (long long)i * 2 * d);
+    float acc = 0.f;
+    for (int v = lane; v < vpr; v += 32) {
+      const uint4 w = __ldcs(wr + v), x = __ldg(ev + v);
+      const uint32_t ww[4] = {w.x, w.y, w.z, w.w}, xx[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        acc = fmaf(bf16_lo(ww[q]), bf16_lo(xx[q]), acc);
+        acc = fmaf(bf16_hi(ww[q]), bf16_hi(xx[q]), acc);
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
+    if (lane == 0) {
+      p.ge[i] = acc;
+      __threadfence();
+      atomicAdd(done, 1u);
+    }
+  }
+}
+
 // Tile t < T0: correction tile (row block t / nt0, 256 output columns t % nt0);
 // T0 <= t < T0 + T1: gate tile (row block (t-T0) / nt1, 128 features).  Tiles
 // are handed out in this order by a global counter, so every gate tile's row
 // block was handed out (to a running CTA) before it.
-__global__ void __launch_bounds__(THREADS, 1)
+// FUSED: the same kernel also runs verification (verify_stream.cuh): warp 3
+// streams the logits into a shared-memory ring, warps 8-15 reduce it, warp 16 folds the keys.  Packed rows then become available while the
+// kernel runs, so the tile queue is decoded in phases -- phase q holds the
+// correction tiles of row block q followed by the gate tiles of row block
+// q - kGateLag -- and the producer resolves each tile against the published
+// per-block row counts before loading it.  R (and the last partial block) is
+// known once every sequence is finalised.
+constexpr int kGateLag = 4;
+
+template <bool FUSED>
+__global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
     cond_kernel(const __grid_constant__ CUtensorMap tmApack, const __grid_constant__ CUtensorMap tmWc,
                 const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmE,
                 const __grid_constant__ CUtensorMap tmWv, const __grid_constant__ CUtensorMap tmWg,
-                const CondParams p) {
+                const CondParams p, const VerifyStreamParams vp) {
   extern __shared__ uint8_t dsmem[];
   __shared__ __align__(8) uint64_t bar_full[STAGES];
   __shared__ __align__(8) uint64_t bar_empty[STAGES];
@@ -202,26 +253,29 @@ __global__ void __launch_bounds__(THREADS, 1)
   __shared__ __align__(8) uint64_t bar_tile_full[TILE_SLOTS];
   __shared__ __align__(8) uint64_t bar_tile_empty[TILE_SLOTS];
   __shared__ int s_tile[TILE_SLOTS];
+  __shared__ int s_rows[TILE_SLOTS];  // valid rows of the tile (FUSED)
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
+  __shared__ VerifyStreamSmem vsm;
 
+  constexpr int NST = FUSED ? STAGES_FUSED : STAGES;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int d = p.d;
-  const int R = *(volatile const int32_t*)p.R;
-  const int tiles_m = (R + BM - 1) / BM;
   const int nt0 = d / 256, nt1 = d / 128;
-  const int T0 = p.do_correct ? tiles_m * nt0 : 0;
-  const int T = T0 + (p.do_gate ? tiles_m * nt1 : 0);
-  if (T == 0) return;  // nothing to condition
+  const int R = FUSED ? 0 : *(volatile const int32_t*)p.R;
+  const int tiles_m = (R + BM - 1) / BM;
+  const int T0 = FUSED ? 0 : (p.do_correct ? tiles_m * nt0 : 0);
+  const int T = FUSED ? 0 : T0 + (p.do_gate ? tiles_m * nt1 : 0);
+  if (!FUSED && T == 0) return;  // nothing to condition
   uint32_t* tile_queue = p.sync + kSyncTileQueue;
   uint32_t* gemv_next = p.sync + kSyncGemvNext;
   uint32_t* gemv_done = p.sync + kSyncGemvDone;
-  uint32_t* block_done = p.sync + kSyncBlockDone;
+  uint32_t* block_done = p.block_done;
   const bool need_ge = p.do_gate && !p.e_dense;
 
   if (tid == 0) {
     s_abort = 0;
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < NST; ++s) {
       mbar_init(smem_u32(&bar_full[s]), 1);
       mbar_init(smem_u32(&bar_empty[s]), 1);
     }
@@ -233,6 +287,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_init(smem_u32(&bar_tile_full[a]), 1);
       mbar_init(smem_u32(&bar_tile_empty[a]), 5);  // MMA thread + four epilogue warps
     }
+    if constexpr (FUSED) vs_init(vsm);
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
@@ -265,18 +320,76 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       for (uint32_t lt = 0;; ++lt) {
         const uint32_t slot = lt % TILE_SLOTS, sph = (lt / TILE_SLOTS) & 1u;
-        const int t = (int)atomicAdd(tile_queue, 1u);
+        int t, rows = BM, m0, n0;
+        bool corr, done = false;
+        if (!FUSED) {
+          t = (int)atomicAdd(tile_queue, 1u);
+          done = t >= T;
+          corr = t < T0;
+          const int tt = corr ? t : t - T0;
+          m0 = (corr ? tt / nt0 : tt / nt1) * BM;
+          n0 = corr ? (tt % nt0) * 256 : (tt % nt1) * 128;
+        } else {
+          // next valid tile of the phased queue
+          for (;;) {
+            t = (int)atomicAdd(tile_queue, 1u);
+            const int q = t / (nt0 + nt1), r = t % (nt0 + nt1);
+            corr = r < nt0;
+            const int m = corr ? q : q - kGateLag;
+            n0 = corr ? r * 256 : (r - nt0) * 128;
+            m0 = m * BM;
+            if (m < 0) continue;  // gate slots of the first phases
+            if (m >= p.max_blocks) {  // beyond any possible packed row
+              if (!corr) {
+                done = true;
+                break;
+              }
+              continue;
+            }
+            // wait until block m is complete, or verification is over
+            int state = 0;  // 1 valid, 2 past the last block
+            const unsigned long long t_start = global_ns();
+            for (uint32_t it2 = 0; state == 0; ++it2) {
+              const uint32_t ready = ld_acquire(p.block_ready + m);
+              if (ready >= (uint32_t)BM) {
+                state = 1;
+              } else if (ld_acquire(p.sync + kSyncSeqDone) >= (uint32_t)vp.B) {
+                const int Rf = (int)ld_acquire(p.sync + kSyncRowCount);
+                if (m0 >= Rf) state = 2;
+                else if (ready >= (uint32_t)(Rf - m0)) { state = 1; rows = Rf - m0; }
+              }
+              if (state == 0) {
+                __nanosleep(128);
+                if ((it2 & 63u) == 63u && (s_abort || global_ns() - t_start > kWaitLimitNs)) break;
+              }
+            }
+            if (state == 0) {
+              ok = false;
+              break;
+            }
+            if (state == 2) {
+              // Block m is past the last packed row.  Gate tiles come in
+              // increasing block order, so a gate tile past the end means
+              // nothing valid is left; a correction tile past the end may
+              // still be followed by valid gate tiles of earlier blocks.
+              if (!corr) {
+                done = true;
+                break;
+              }
+              continue;
+            }
+            break;
+          }
+          if (!ok) break;
+        }
         if (!mbar_wait_bounded(smem_u32(&bar_tile_empty[slot]), sph ^ 1u, &s_abort)) {
           ok = false;
           break;
         }
-        s_tile[slot] = t < T ? t : -1;
+        s_tile[slot] = done ? -1 : t;
+        s_rows[slot] = rows;
         mbar_arrive(smem_u32(&bar_tile_full[slot]));
-        if (t >= T) break;
-        const bool corr = t < T0;
-        const int tt = corr ? t : t - T0;
-        const int m0 = (corr ? tt / nt0 : tt / nt1) * BM;
-        const int n0 = corr ? (tt % nt0) * 256 : (tt % nt1) * 128;
+        if (done) break;
         const int nkb = corr ? 2 * kb_half : kb_half + (p.e_dense ? kb_half : 0);
         if (!corr && p.do_correct) {
           // the r rows of this block are written by the correction epilogues
@@ -287,7 +400,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           fence_proxy_async_global();
         }
         for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
+          const uint32_t s = it % NST, ph = (it / NST) & 1u;
           if (!mbar_wait_bounded(smem_u32(&bar_empty[s]), ph ^ 1u, &s_abort)) {
             ok = false;
             break;
@@ -314,9 +427,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (!ok) {
         raise_abort(&s_abort, p.status);
         volatile int never = 0;  // drain this CTA's own copies still in flight
-        const uint32_t first = it > STAGES ? it - STAGES : 0;
+        const uint32_t first = it > NST ? it - NST : 0;
         for (uint32_t k = first; k < it; ++k)
-          mbar_wait_bounded(smem_u32(&bar_full[k % STAGES]), (k / STAGES) & 1u, &never);
+          mbar_wait_bounded(smem_u32(&bar_full[k % NST]), (k / NST) & 1u, &never);
       }
     }
     __syncwarp();
@@ -334,7 +447,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int t = s_tile[slot];
         mbar_arrive(smem_u32(&bar_tile_empty[slot]));
         if (t < 0) break;
-        const bool corr = t < T0;
+        const bool corr = FUSED ? (t % (nt0 + nt1)) < nt0 : t < T0;
         const int nkb = corr ? 2 * kb_half : kb_half + (p.e_dense ? kb_half : 0);
         const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
         if (!mbar_wait_bounded(smem_u32(&bar_tempty[acc]), aph ^ 1u, &s_abort)) {
@@ -344,7 +457,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         tc_fence_after();
         const uint32_t d_tmem = tmem + acc * ACC_COLS;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const uint32_t s = it % STAGES, ph = (it / STAGES) & 1u;
+          const uint32_t s = it % NST, ph = (it / NST) & 1u;
           if (!mbar_wait_bounded(smem_u32(&bar_full[s]), ph, &s_abort)) {
             ok = false;
             break;
@@ -371,40 +484,33 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (!ok) raise_abort(&s_abort, p.status);
     }
     __syncwarp();
+  } else if (FUSED && warp == 3) {
+    // ---------------- logits stream into the verification ring ----------------
+    if (lane == 0) vs_producer(vp, vsm, base + NST * STAGE_BYTES, &s_abort);
+    __syncwarp();
+  } else if (FUSED && warp == 2) {
+    // ---------------- sequence finaliser (bulk copies through staging) ----------------
+    vs_finalizer(vp, vsm, base + NST * STAGE_BYTES + kRingBufs * kChunkBytes, blockIdx.x, gridDim.x, lane, &s_abort);
   } else if (warp == 2 || warp == 3) {
     // ---------------- W_g[:, :d] e for a broadcast e (idle warps) ----------------
-    if (need_ge) {
-      const int vpr = d / 8;
-      const uint4* ev = reinterpret_cast<const uint4*>(p.e);
-      for (;;) {
-        int i = 0;
-        if (lane == 0) i = (int)atomicAdd(gemv_next, 1u);
-        i = __shfl_sync(0xFFFFFFFFu, i, 0);
-        if (i >= d) break;
-        const uint4* wr = reinterpret_cast<const uint4*>(p.Wg + (long long)i * 2 * d);
-        float acc = 0.f;
-        for (int v = lane; v < vpr; v += 32) {
-          const uint4 w = __ldcs(wr + v), x = __ldg(ev + v);
-          const uint32_t ww[4] = {w.x, w.y, w.z, w.w}, xx[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            acc = fmaf(bf16_lo(ww[q]), bf16_lo(xx[q]), acc);
-            acc = fmaf(bf16_hi(ww[q]), bf16_hi(xx[q]), acc);
-          }
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
-        if (lane == 0) {
-          p.ge[i] = acc;
-          __threadfence();
-          atomicAdd(gemv_done, 1u);
-        }
-      }
-    }
+    if (need_ge) gate_bias_rows(p, d, lane, gemv_next, gemv_done);
+  } else if (warp >= 16) {
+    // ---------------- verification bookkeeping (FUSED only) ----------------
+    if constexpr (FUSED)
+      if (lane == 0) vs_bookkeeper(vp, vsm, &s_abort);
+    __syncwarp();
+  } else if (warp >= 8) {
+    // ---------------- verification (FUSED only: warps 8-15) ----------------
+    if constexpr (FUSED)
+      vs_consumer(vp, vsm, reinterpret_cast<const uint4*>(dsmem + (base + NST * STAGE_BYTES - smem_u32(dsmem))),
+                  warp - 8, lane, &s_abort);
   } else if (warp >= 4) {
     // ---------------- epilogue ----------------
     const int q = (warp - 4) * 32 + lane;  // tile row = TMEM lane
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    // In the fused kernel the epilogue warps have nothing to do until the
+    // first rows are packed: they compute W_g[:, :d] e meanwhile.
+    if (FUSED && need_ge) gate_bias_rows(p, d, lane, gemv_next, gemv_done);
     bool have_ge = !need_ge;
     for (uint32_t lt = 0;; ++lt) {
       const uint32_t slot = lt % TILE_SLOTS, sph = (lt / TILE_SLOTS) & 1u;
@@ -414,13 +520,23 @@ __global__ void __launch_bounds__(THREADS, 1)
         break;
       }
       const int t = s_tile[slot];
+      const int tile_rows = s_rows[slot];
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&bar_tile_empty[slot]));
       if (t < 0) break;
-      const bool corr = t < T0;
-      const int tt = corr ? t : t - T0;
-      const int m0 = (corr ? tt / nt0 : tt / nt1) * BM;
-      const int n0 = corr ? (tt % nt0) * 256 : (tt % nt1) * 128;
+      bool corr;
+      int m0, n0;
+      if (FUSED) {
+        const int q2 = t / (nt0 + nt1), r = t % (nt0 + nt1);
+        corr = r < nt0;
+        m0 = (corr ? q2 : q2 - kGateLag) * BM;
+        n0 = corr ? r * 256 : (r - nt0) * 128;
+      } else {
+        corr = t < T0;
+        const int tt = corr ? t : t - T0;
+        m0 = (corr ? tt / nt0 : tt / nt1) * BM;
+        n0 = corr ? (tt % nt0) * 256 : (tt % nt1) * 128;
+      }
       const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
       ok = warp_wait(smem_u32(&bar_tfull[acc]), aph, &s_abort);
       tc_fence_after();
@@ -440,12 +556,12 @@ __global__ void __launch_bounds__(THREADS, 1)
         have_ge = true;
       }
       const int g = m0 + q;
-      const bool valid = g < R;
+      const bool valid = FUSED ? q < tile_rows : g < R;
       const uint32_t taddr = tmem + acc * ACC_COLS + lane_base;
       if (corr) {
         // r = m + beta * c   (Eq. 7), m = first d columns of the packed row
         const __nv_bfloat16* mrow = p.apack + (long long)g * 2 * d;
-        const long long orow = valid ? (p.compact_out ? g : p.rowmap[g]) : 0;
+        const long long orow = valid ? (p.compact_out ? g : __ldcg(p.rowmap + g)) : 0;
         for (int cc = 0; cc < 8; ++cc) {
           float c[32];
           tmem_ld_32cols(taddr + (uint32_t)(cc * 32), c);
@@ -455,7 +571,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             uint4* ov = reinterpret_cast<uint4*>(p.r_out + orow * d + n);
 #pragma unroll
             for (int v = 0; v < 4; ++v) {
-              const uint4 mw = __ldg(mv + v);
+              const uint4 mw = __ldcg(mv + v);
               const uint32_t mwords[4] = {mw.x, mw.y, mw.z, mw.w};
               uint32_t o[4];
 #pragma unroll
@@ -478,7 +594,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
       } else {
         // e~ = e + v * sigmoid(g)   (Eq. 8)
-        const long long orow = valid ? p.rowmap[g] : 0;
+        const long long orow = valid ? __ldcg(p.rowmap + g) : 0;
         const __nv_bfloat16* erow = p.e + (p.e_dense ? (long long)g * d : 0);
         for (int cc = 0; cc < 4; ++cc) {
           float v[32], gt[32];
@@ -490,7 +606,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             uint4* ov = reinterpret_cast<uint4*>(p.e_out + orow * d + n);
 #pragma unroll
             for (int x = 0; x < 4; ++x) {
-              const uint4 ew = __ldg(ev + x);
+              const uint4 ew = __ldcg(ev + x);
               const uint32_t ewords[4] = {ew.x, ew.y, ew.z, ew.w};
               uint32_t o[4];
 #pragma unroll
@@ -524,13 +640,15 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+template <bool FUSED>
 cudaError_t ensure_smem_attr() {
   static int done[64] = {0};
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
   if (!done[dev & 63]) {
-    err = cudaFuncSetAttribute(cond_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    err = cudaFuncSetAttribute(cond_kernel<FUSED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               FUSED ? SMEM_BYTES_FUSED : SMEM_BYTES);
     if (err != cudaSuccess) return err;
     done[dev & 63] = 1;
   }
@@ -566,7 +684,7 @@ cudaError_t launch_pack(const PackArgs& a, cudaStream_t stream) {
 cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream) {
   const long long rmax = (long long)a.B * (a.K - 1);
   if (rmax <= 0 || (!a.do_correct && !a.do_gate)) return cudaSuccess;
-  cudaError_t err = ensure_smem_attr();
+  cudaError_t err = ensure_smem_attr<false>();
   if (err != cudaSuccess) return err;
   const uint64_t d = (uint64_t)a.d;
   CUtensorMap mApack, mWc, mR, mE, mWv, mWg;
@@ -579,7 +697,7 @@ cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream) {
   const void* wg = a.do_gate ? a.Wg : a.Wc;
   if (encode_tensor_map_2d(&mApack, apack, a.do_correct ? 2 * d : d, (uint64_t)rmax, (a.do_correct ? 4 : 2) * d, BK, BM) != CUDA_SUCCESS ||
       encode_tensor_map_2d(&mWc, wc, a.do_correct ? 2 * d : d, d, (a.do_correct ? 4 : 2) * d, BK, 256) != CUDA_SUCCESS ||
-      encode_tensor_map_2d(&mR, rp, d, (uint64_t)rmax, 2 * d, BK, BM) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mR, rp, d, (uint64_t)rmax, 2 * (a.r_row_stride ? (uint64_t)a.r_row_stride : d), BK, BM) != CUDA_SUCCESS ||
       encode_tensor_map_2d(&mE, erows, d, (uint64_t)rmax, 2 * d, BK, BM) != CUDA_SUCCESS ||
       encode_tensor_map_2d(&mWv, wv, a.do_gate ? d : 2 * d, d, (a.do_gate ? 2 : 4) * d, BK, 128) != CUDA_SUCCESS ||
       encode_tensor_map_2d(&mWg, wg, 2 * d, d, 4 * d, BK, 128) != CUDA_SUCCESS)
@@ -600,14 +718,117 @@ cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream) {
   p.ge = a.ge;
   p.e_out = reinterpret_cast<__nv_bfloat16*>(a.e_out);
   p.sync = a.sync;
+  p.block_done = a.sync + kSyncBlocks;
+  p.block_ready = a.sync + kSyncBlocks + blocks_max(a.B, a.K);
   p.status = a.status;
   DeviceInfo info{0, 148};
   err = device_info(&info);
   if (err != cudaSuccess) return err;
   const long long tiles_max = (rmax + BM - 1) / BM * ((a.do_correct ? a.d / 256 : 0) + (a.do_gate ? a.d / 128 : 0));
   const unsigned grid = (unsigned)(tiles_max < info.sm_count ? tiles_max : info.sm_count);
-  cond_kernel<<<grid, THREADS, SMEM_BYTES, stream>>>(mApack, mWc, mR, mE, mWv, mWg, p);
+  VerifyStreamParams vp{};
+  cond_kernel<false><<<grid, THREADS, SMEM_BYTES, stream>>>(mApack, mWc, mR, mE, mWv, mWg, p, vp);
   return cudaGetLastError();
+}
+
+}  // namespace retrace
+
+namespace retrace {
+
+bool round_fused_supported(const TcRoundArgs& a) {
+  // contiguous logits with rows of at least one stream chunk, so that a chunk
+  // is one contiguous copy and spans at most two rows
+  return tc_supported(RETRACE_BF16, a.d) && 4 * a.d <= kStageBytes && ((uintptr_t)a.logits % 16 == 0) && a.V % 8 == 0 &&
+         a.V >= 8 * kChunkSlots && a.row_stride == a.V && a.batch_stride == (long long)(a.K + 1) * a.V &&
+         a.K >= 2 && (long long)a.B * (a.K + 1) * (a.V / 8) < (1ll << 32) - kChunkSlots;
+}
+
+cudaError_t launch_round_tc(const TcRoundArgs& a, cudaStream_t stream) {
+  cudaError_t err = ensure_smem_attr<true>();
+  if (err != cudaSuccess) return err;
+  const uint64_t d = (uint64_t)a.d;
+  const long long rmax = (long long)a.B * (a.K - 1);
+  CUtensorMap mApack, mWc, mR, mE, mWv, mWg;
+  if (encode_tensor_map_2d(&mApack, a.apack, 2 * d, (uint64_t)rmax, 4 * d, BK, BM) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWc, a.Wc, 2 * d, d, 4 * d, BK, 256) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mR, a.rpack, d, (uint64_t)rmax, 2 * d, BK, BM) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mE, a.e_dense ? a.epack : a.rpack, d, (uint64_t)rmax, 2 * d, BK, BM) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWv, a.Wv, d, d, 2 * d, BK, 128) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWg, a.Wg, 2 * d, d, 4 * d, BK, 128) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  const long long blocks = blocks_max(a.B, a.K);
+  CondParams p{};
+  p.d = a.d;
+  p.do_correct = 1;
+  p.do_gate = 1;
+  p.R = reinterpret_cast<const int32_t*>(a.sync + kSyncRowCount);
+  p.rowmap = a.rowmap;
+  p.apack = reinterpret_cast<const __nv_bfloat16*>(a.apack);
+  p.beta = a.beta;
+  p.r_out = reinterpret_cast<__nv_bfloat16*>(a.rpack);
+  p.compact_out = 1;
+  p.e = reinterpret_cast<const __nv_bfloat16*>(a.e_dense ? a.epack : a.e);
+  p.e_dense = a.e_dense;
+  p.Wg = reinterpret_cast<const __nv_bfloat16*>(a.Wg);
+  p.ge = a.ge;
+  p.e_out = reinterpret_cast<__nv_bfloat16*>(a.e_out);
+  p.sync = a.sync;
+  p.block_done = a.sync + kSyncBlocks;
+  p.block_ready = a.sync + kSyncBlocks + blocks;
+  p.max_blocks = (int)blocks;
+  p.status = a.status;
+
+  VerifyStreamParams vp{};
+  vp.logits = reinterpret_cast<const __nv_bfloat16*>(a.logits);
+  vp.B = a.B;
+  vp.K = a.K;
+  vp.V = a.V;
+  vp.draft = a.draft;
+  vp.accept_len = a.accept_len;
+  vp.committed = a.committed;
+  vp.bonus = a.bonus;
+  vp.target_argmax = a.target_argmax;
+  vp.n_out = a.n_out;
+  vp.keys = a.keys;
+  vp.tickets = a.tickets;
+  vp.e = reinterpret_cast<const __nv_bfloat16*>(a.e);
+  vp.e_batch_stride = a.e_batch_stride;
+  vp.e_pos_stride = a.e_pos_stride;
+  vp.e_out = reinterpret_cast<__nv_bfloat16*>(a.e_out);
+  vp.d = a.d;
+  vp.hD = reinterpret_cast<const __nv_bfloat16*>(a.hD);
+  vp.hT = reinterpret_cast<const __nv_bfloat16*>(a.hT);
+  vp.e_dense = a.e_dense;
+  vp.apack = reinterpret_cast<__nv_bfloat16*>(a.apack);
+  vp.epack = reinterpret_cast<__nv_bfloat16*>(a.epack);
+  vp.rowmap = a.rowmap;
+  vp.R_count = a.sync + kSyncRowCount;
+  vp.rows_ready = a.sync + kSyncBlocks + blocks;
+  vp.seq_done = a.sync + kSyncSeqDone;
+  vp.slots_per_row = a.V / 8;
+  vp.total_slots = (long long)a.B * (a.K + 1) * vp.slots_per_row;
+  vp.total_chunks = (uint32_t)((vp.total_slots + kChunkSlots - 1) / kChunkSlots);
+  vp.chunk_next = a.sync + kSyncChunkNext;
+  vp.status = a.status;
+
+  DeviceInfo info{0, 148};
+  err = device_info(&info);
+  if (err != cudaSuccess) return err;
+  const long long grid = info.sm_count;
+  // Cooperative: every CTA's share of the logits feeds other CTAs' tiles, so
+  // all CTAs must be resident together (one per SM); the launch fails
+  // instead of starting if they cannot be.
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(THREADS_FUSED);
+  cfg.dynamicSmemBytes = SMEM_BYTES_FUSED;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, cond_kernel<true>, mApack, mWc, mR, mE, mWv, mWg, p, vp);
 }
 
 }  // namespace retrace

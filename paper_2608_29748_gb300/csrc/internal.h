@@ -38,7 +38,7 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   L.status = off;
   off = align_up(off + 64 * 4, 256);
   L.sync = off;
-  L.sync_bytes = align_up((32 + (rmax + 127) / 128) * 4, 256);
+  L.sync_bytes = align_up((size_t)(32 + 2 * ((rmax + 127) / 128)) * 4, 256);
   off += L.sync_bytes;
   L.keys = off;
   off = align_up(off + (size_t)(B * (K + 1)) * 8, 256);
@@ -92,7 +92,14 @@ struct VerifyArgs {
   void* epack;     // [R_max, d]: e rows (dense e only)
   int32_t* rowmap; // [R_max]: packed row -> b*K + j
   int32_t* R_count;
+  // Rows j < n_b of e_out in the copy above (no packing then): kCondCopyKeep
+  // leaves them to the conditioning kernels, kCondCopyE writes e (no
+  // conditioning), kCondCopyM writes m_j = hD[b, A_b+1+j] (overwrite).
+  int cond_copy;
 };
+constexpr int kCondCopyKeep = 0;
+constexpr int kCondCopyE = 1;
+constexpr int kCondCopyM = 2;
 cudaError_t launch_verify(const VerifyArgs& a, retrace_dtype dtype, cudaStream_t stream);
 
 // ---- conditioning -----------------------------------------------------------
@@ -113,6 +120,7 @@ struct CorrectArgs {
   RowSource rows;
   void* r_out;        // compact [R, d] (compact_out) or [B, K, d]
   int compact_out;
+  int raw;            // 1: r = m (no correction; W_c is not read)
 };
 cudaError_t launch_correct_simt(const CorrectArgs& a, retrace_dtype dtype, cudaStream_t stream);
 
@@ -148,12 +156,26 @@ struct PackArgs {
 };
 cudaError_t launch_pack(const PackArgs& a, cudaStream_t stream);
 
-// Counters of one conditioning pass (uint32, zeroed before each pass).
-constexpr int kSyncRowCount = 0;    // packed rows claimed / R
-constexpr int kSyncTileQueue = 1;   // next tile of the dynamic schedule
-constexpr int kSyncGemvNext = 2;    // next row of W_g[:, :d] e
-constexpr int kSyncGemvDone = 3;    // rows of W_g[:, :d] e written
-constexpr int kSyncBlockDone = 32;  // per 128-row block: correction epilogue warps done
+// Counters of one conditioning pass (uint32, zeroed before each pass):
+//   [kSyncRowCount]   packed rows claimed / R
+//   [kSyncTileQueue]  next tile of the dynamic schedule
+//   [kSyncGemvNext]   next row of W_g[:, :d] e;  [kSyncGemvDone] rows written
+//   [kSyncSeqDone]    sequences finalised (fused round)
+//   [kSyncChunkNext]  next group of logits chunks to stream (fused round)
+//   [kSyncBlocks ...]            per 128-row block: correction epilogue warps done
+//   [kSyncBlocks + blocks ...]   per 128-row block: packed rows published (fused round)
+constexpr int kSyncRowCount = 0;
+constexpr int kSyncTileQueue = 1;
+constexpr int kSyncGemvNext = 2;
+constexpr int kSyncGemvDone = 3;
+constexpr int kSyncSeqDone = 4;
+constexpr int kSyncChunkNext = 5;
+constexpr int kSyncBlocks = 32;
+
+inline long long blocks_max(long long B, long long K) {
+  const long long rmax = B * (K > 1 ? K - 1 : 0);
+  return (rmax + 127) / 128;
+}
 
 struct TcCondArgs {
   int B, K, d;
@@ -166,6 +188,7 @@ struct TcCondArgs {
   int compact_out;  // 1: r_out is compact [R_max, d]; 0: r_out is [B, K, d] (rows via rowmap)
   // gate: e~ = e + (W_v r) .* sigmoid(W_g [e; r]) over the compact r rows
   const void* rpack;
+  long long r_row_stride;  // elements between rpack rows (0: d)
   const void* e;
   const void* epack;
   int e_dense;
@@ -179,6 +202,42 @@ struct TcCondArgs {
   uint32_t* status;
 };
 cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream);
+
+// The whole round in one persistent launch: verification warps and
+// tensor-core warps share every SM (bf16, d a multiple of 256, 16-byte
+// aligned logits rows, K >= 2).
+struct TcRoundArgs {
+  const void* logits;
+  int B, K, V, d;
+  long long row_stride, batch_stride;
+  const int32_t* draft;
+  int32_t* accept_len;
+  int32_t* committed;
+  int32_t* bonus;
+  int32_t* target_argmax;
+  int32_t* n_out;
+  unsigned long long* keys;
+  uint32_t* tickets;
+  const void* hD;
+  const void* hT;
+  const void* e;
+  int e_dense;
+  long long e_batch_stride, e_pos_stride;
+  const void* Wc;
+  const void* Wv;
+  const void* Wg;
+  float beta;
+  void* e_out;
+  void* apack;
+  void* epack;
+  void* rpack;
+  float* ge;
+  int32_t* rowmap;
+  uint32_t* sync;
+  uint32_t* status;
+};
+bool round_fused_supported(const TcRoundArgs& a);
+cudaError_t launch_round_tc(const TcRoundArgs& a, cudaStream_t stream);
 
 // Writes n_out and the rows j >= n_b (zeros for r, a copy of e for e_out).
 cudaError_t launch_fill_rows(int B, int K, int d, RowSource rows, int32_t* n_out, void* zero_dst,

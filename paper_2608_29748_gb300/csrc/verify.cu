@@ -45,6 +45,7 @@ struct VerifyParams {
   void* epack;
   int32_t* rowmap;
   int32_t* R_count;
+  int cond_copy;
 };
 
 // 16-byte vector helpers: the maximum of the vector's elements and element q.
@@ -148,27 +149,31 @@ __device__ __forceinline__ unsigned long long block_max_key(unsigned long long k
   return s_red[0];
 }
 
-// Copy of drafter-input rows j in [nb, K) of sequence b into e_out.
+// Copy of rows [j0, K) of sequence b into e_out: rows j < j_m from the
+// aligned drafter states m_j = hD[b, A+1+j] (the overwrite ablation), the
+// others from the drafter inputs e.
 template <typename T>
-__device__ void copy_unconditioned_rows(const VerifyParams& p, int b, int nb) {
+__device__ void copy_rows(const VerifyParams& p, int b, int A, int j0, int j_m) {
   const int K = p.K, d = p.d;
-  const long long rows = K - nb;
+  const long long rows = K - j0;
   if (rows <= 0) return;
-  T* dst = reinterpret_cast<T*>(p.e_out) + ((long long)b * K + nb) * d;
+  T* dst = reinterpret_cast<T*>(p.e_out) + ((long long)b * K + j0) * d;
   const T* src_b = reinterpret_cast<const T*>(p.e) + (long long)b * p.e_batch_stride;
+  const T* m_b = reinterpret_cast<const T*>(p.hD) + ((long long)b * K + A + 1) * d;  // row j: m_b + j*d
   const bool vec = ((d * (int)sizeof(T)) % 16 == 0) && ((uintptr_t)dst % 16 == 0) &&
-                   ((uintptr_t)src_b % 16 == 0) && ((p.e_pos_stride * (long long)sizeof(T)) % 16 == 0);
+                   ((uintptr_t)src_b % 16 == 0) && ((p.e_pos_stride * (long long)sizeof(T)) % 16 == 0) &&
+                   (j_m <= j0 || (uintptr_t)p.hD % 16 == 0);
   if (vec) {
     const int vpr = d * (int)sizeof(T) / 16;
     for (long long i = threadIdx.x; i < rows * vpr; i += kThreads) {
-      const long long jj = i / vpr, q = i % vpr;
-      const uint4* s = reinterpret_cast<const uint4*>(src_b + (nb + jj) * p.e_pos_stride);
-      reinterpret_cast<uint4*>(dst)[i] = s[q];
+      const long long j = j0 + i / vpr, q = i % vpr;
+      const T* row = (j < j_m) ? m_b + j * d : src_b + j * p.e_pos_stride;
+      reinterpret_cast<uint4*>(dst)[i] = reinterpret_cast<const uint4*>(row)[q];
     }
   } else {
     for (long long i = threadIdx.x; i < rows * d; i += kThreads) {
-      const long long jj = i / d, q = i % d;
-      dst[i] = src_b[(nb + jj) * p.e_pos_stride + q];
+      const long long j = j0 + i / d, q = i % d;
+      dst[i] = (j < j_m) ? m_b[j * d + q] : src_b[j * p.e_pos_stride + q];
     }
   }
 }
@@ -239,7 +244,11 @@ __device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s
     if (p.n_out) p.n_out[b] = nb;
     p.tickets[b] = 0u;
   }
-  if (p.e_out) copy_unconditioned_rows<T>(p, b, nb);
+  if (p.e_out) {
+    if (p.cond_copy == kCondCopyKeep) copy_rows<T>(p, b, A, nb, 0);
+    else if (p.cond_copy == kCondCopyE) copy_rows<T>(p, b, A, 0, 0);
+    else copy_rows<T>(p, b, A, 0, nb);
+  }
   if (p.R_count && nb > 0) pack_sequence_rows(p, b, A, nb, s_A + 1);
 }
 
@@ -338,6 +347,7 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
   p.epack = a.epack;
   p.rowmap = a.rowmap;
   p.R_count = a.R_count;
+  p.cond_copy = a.cond_copy;
   // Enough CTAs to fill every SM at full occupancy, but at least ~32 KB of
   // logits per CTA so that small batches do not pay for idle CTAs.
   const long long bytes = (long long)a.B * (a.K + 1) * a.V * (long long)sizeof(T);

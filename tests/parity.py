@@ -31,19 +31,21 @@ def host_int(t: torch.Tensor) -> np.ndarray:
     return t.detach().cpu().numpy().astype(np.int64)
 
 
-def oracle_round(x: dict) -> dict:
+def oracle_round(x: dict, variant: str = "corrected") -> dict:
     dtype = "bf16" if x["logits"].dtype == torch.bfloat16 else "f32"
+    weight = lambda k: None if x.get(k) is None else host_f64(x[k])  # noqa: E731
     return oracle.retrace_round(
         host_f64(x["logits"]),
         host_int(x["draft"]),
         host_f64(x["hD"]),
         host_f64(x["hT"]),
         host_f64(x["e"]),
-        host_f64(x["Wc"]),
-        host_f64(x["Wv"]),
-        host_f64(x["Wg"]),
+        weight("Wc"),
+        weight("Wv"),
+        weight("Wg"),
         x["beta"],
         dtype,
+        variant=variant,
     )
 
 

@@ -106,3 +106,32 @@ def test_conditioning_argument_errors(lib):
 def test_workspace_init_rejects_null(lib):
     lib.retrace_workspace_init.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
     assert lib.retrace_workspace_init(None, 128, None) == INVALID
+
+
+def _round(lib, flags, Wc=16, Wv=16, Wg=16, B=0):
+    """retrace_round with fake pointers; every case here returns before any
+    CUDA call (argument checks, or B = 0)."""
+    P, I64 = ctypes.c_void_p, ctypes.c_int64
+    return lib.retrace_round(P(16), I64(10), I64(50), P(16), P(16), P(16), P(16), I64(0), I64(0),
+                             P(Wc) if Wc else None, P(Wv) if Wv else None, P(Wg) if Wg else None,
+                             ctypes.c_float(1.0), BF16, B, 4, 10, 8, P(16), P(16), P(16), None, None, P(16),
+                             P(256), ctypes.c_size_t(1 << 20), ctypes.c_uint32(flags), None, None)
+
+
+def test_round_flag_errors(lib):
+    RAW, OVERWRITE, NONE, OVERLAP = 0x2, 0x4, 0x8, 0x1
+    assert _round(lib, 0x100) == INVALID  # unknown bit
+    assert b"flag" in lib.retrace_last_error()
+    assert _round(lib, RAW | NONE) == INVALID  # two ablation variants
+    assert _round(lib, OVERWRITE | RAW) == INVALID
+    assert _round(lib, OVERLAP | RAW) == UNSUPPORTED  # the overlapped kernel runs the method only
+    for flags in (0, RAW, OVERWRITE, NONE, OVERLAP):
+        assert _round(lib, flags) == OK  # B = 0: nothing to do
+
+
+def test_round_header_documents_the_flags():
+    text = open(HEADER).read()
+    for name, value in (("RETRACE_ROUND_OVERLAP", 0x1), ("RETRACE_COND_RAW", 0x2),
+                        ("RETRACE_COND_OVERWRITE", 0x4), ("RETRACE_COND_NONE", 0x8)):
+        m = re.search(r"#define\s+%s\s+(0x[0-9a-fA-F]+)u" % name, text)
+        assert m and int(m.group(1), 16) == value, name

@@ -135,3 +135,112 @@ def test_round_repeatable_bitwise(rt):
         assert torch.equal(again.committed, first.committed)
         assert torch.equal(again.accept_len, first.accept_len)
     assert ws.check() == 0
+
+
+@pytest.mark.parametrize("cfg_id", [3, 4])
+def test_overlapped_round_equals_separate_entry_points(rt, cfg_id):
+    """retrace_round with RETRACE_ROUND_OVERLAP (verification and both
+    projections overlapped in one persistent kernel) against retrace_verify +
+    retrace_align_refine + retrace_gate_fuse on the same inputs: identical
+    bits, since every output element is computed by the same arithmetic in
+    the same order."""
+    x = make_round_inputs(CONFIGS[cfg_id], device="cuda")
+    cfg = x["cfg"]
+    fused, targ, ws = run(rt, x, flags=rt.ROUND_OVERLAP)
+    B, K, d = cfg.B, cfg.K, cfg.d
+    acc = torch.empty(B, dtype=torch.int32, device="cuda")
+    com = torch.empty(B, K + 1, dtype=torch.int32, device="cuda")
+    bon = torch.empty(B, dtype=torch.int32, device="cuda")
+    r = torch.empty(B, K, d, dtype=torch.bfloat16, device="cuda")
+    n = torch.empty(B, dtype=torch.int32, device="cuda")
+    e_out = torch.empty(B, K, d, dtype=torch.bfloat16, device="cuda")
+    rt.retrace_verify(x["logits"], x["draft"], acc, com, bon, ws)
+    rt.retrace_align_refine(x["hD"], x["hT"], acc, x["Wc"], x["beta"], r, n, ws)
+    rt.retrace_gate_fuse(x["e"], r, n, x["Wv"], x["Wg"], e_out, ws)
+    torch.cuda.synchronize()
+    assert ws.check() == 0
+    assert torch.equal(acc, fused.accept_len)
+    assert torch.equal(com, fused.committed)
+    assert torch.equal(bon, fused.bonus)
+    assert torch.equal(n, fused.n)
+    assert torch.equal(e_out, fused.e_out)
+
+
+def test_overlapped_round_matches_the_oracle_and_the_default_path(rt):
+    """The overlapped kernel on the serving shape's sibling (B = 64): oracle
+    parity, and the same bits as the default two-launch round."""
+    x = make_round_inputs(CONFIGS[4], device="cuda")
+    over, targ, ws = run(rt, x, flags=rt.ROUND_OVERLAP)
+    assert ws.check() == 0
+    want = oracle_round(x)
+    assert_verify_exact(want, over.accept_len, over.committed, over.bonus, targ)
+    assert_close(over.e_out, want["e_tilde"], "overlapped round")
+    plain, _, _ = run(rt, x, ws=ws)
+    assert torch.equal(plain.e_out, over.e_out)
+    assert torch.equal(plain.n, over.n)
+
+
+def test_overlap_flag_rejects_what_the_kernel_does_not_cover(rt):
+    """RETRACE_ROUND_OVERLAP on an fp32 round or with an ablation flag is
+    refused with UNSUPPORTED before anything is enqueued."""
+    x = make_round_inputs(CONFIGS[1], device="cuda")  # fp32
+    with pytest.raises(rt.RetraceError) as ei:
+        run(rt, x, flags=rt.ROUND_OVERLAP)
+    assert ei.value.status == 2
+    x = make_round_inputs(CONFIGS[3], device="cuda")
+    with pytest.raises(rt.RetraceError) as ei:
+        run(rt, x, flags=rt.ROUND_OVERLAP | rt.COND_RAW)
+    assert ei.value.status == 2
+
+
+# Ablation variants (component ablation, Table 3): raw conditioning gated,
+# raw conditioning overwrite, no conditioning.
+SMALL_SIMT_BF16 = CONFIGS[2].__class__("bf16 d=320 (FFMA path)", 6, 16, 5003, 320, "bf16", 1.0, "uniform", seed_offset=9)
+
+
+def _flag(rt, variant):
+    return {"raw": rt.COND_RAW, "overwrite": rt.COND_OVERWRITE, "none": rt.COND_NONE}[variant]
+
+
+@pytest.mark.parametrize("variant", ["raw", "overwrite", "none"])
+@pytest.mark.parametrize("cfg_id", [1, 3, 4, "simt-bf16"])
+def test_ablation_variants(rt, cfg_id, variant):
+    cfg = SMALL_SIMT_BF16 if cfg_id == "simt-bf16" else CONFIGS[cfg_id]
+    x = make_round_inputs(cfg, device="cuda")
+    if variant != "raw":  # weights the variant does not use may be absent
+        x = {**x, "Wc": None, "Wv": None, "Wg": None}
+    else:
+        x = {**x, "Wc": None}
+    out, targ, ws = run(rt, x, flags=_flag(rt, variant))
+    assert ws.check() == 0
+    want = oracle_round(x, variant)
+    assert_verify_exact(want, out.accept_len, out.committed, out.bonus, targ)
+    np.testing.assert_array_equal(host_int(out.n), want["n"])
+    if variant == "raw":
+        assert_close(out.e_out, want["e_tilde"], f"config {cfg_id} raw")
+    else:  # pure copies: bit-exact
+        assert np.array_equal(host_f64(out.e_out), want["e_tilde"]), f"config {cfg_id} {variant}"
+
+
+@pytest.mark.parametrize("variant", ["raw", "overwrite", "none"])
+def test_ablation_variants_dense_e_and_short_blocks(rt, variant):
+    for K in (1, 2, 16):
+        cfg = CONFIGS[2].__class__("t", 9, K, 3001, 512, "bf16", 1.0, "uniform", seed_offset=11)
+        x = make_round_inputs(cfg, device="cuda")
+        x["e"] = (torch.randn((cfg.B, K, cfg.d), device="cuda") * 0.02).to(torch.bfloat16)
+        out, targ, ws = run(rt, x, flags=_flag(rt, variant))
+        want = oracle_round(x, variant)
+        assert_verify_exact(want, out.accept_len, out.committed, out.bonus, targ)
+        if variant == "raw":
+            assert_close(out.e_out, want["e_tilde"], f"K={K} raw")
+        else:
+            assert np.array_equal(host_f64(out.e_out), want["e_tilde"]), f"K={K} {variant}"
+
+
+def test_raw_variant_equals_zero_beta_on_the_default_path(rt):
+    """Raw conditioning skips the correction GEMM; beta = 0 runs it and adds
+    0 * c: both give r = m, so the outputs agree bit for bit."""
+    x = make_round_inputs(CONFIGS[4], device="cuda")
+    raw, _, ws = run(rt, x, flags=rt.COND_RAW)
+    zero, _, _ = run(rt, {**x, "beta": 0.0}, ws=ws)
+    assert torch.equal(raw.e_out, zero.e_out)
