@@ -17,6 +17,10 @@ from .retrace_oracle import (  # noqa: F401
     correct,
     f64_to_bf16_bits,
     gate_fuse,
+    LOWRANK_CORRECTION,
+    LOWRANK_LATENT,
+    lowrank_condition,
+    retrace_round_lowrank,
     retrace_round,
     round_to_bf16,
     sigmoid,

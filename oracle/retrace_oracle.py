@@ -325,3 +325,64 @@ def conditioned_rows(rows, A, hD, hT, e, Wc, Wv, Wg, beta, dtype: str) -> np.nda
         out.append(e_bj + v * sigmoid(g))
     res = np.stack(out) if out else np.zeros((0, np.asarray(hD).shape[2]))
     return round_to_bf16(res) if dtype == "bf16" else res
+
+
+# ---------------------------------------------------------------------------
+# Low-rank realisation of the conditioning (Appendix "Concurrent-Serving
+# Experiment"): rank-64 rejected-suffix latents, a rank-32 target-aware
+# correction, and input-side latent residual fusion, for one round.
+# ---------------------------------------------------------------------------
+
+LOWRANK_LATENT = 64
+LOWRANK_CORRECTION = 32
+
+
+def lowrank_condition(e_full, m, u, n, P, Bc, Ac, Wv, Wg, beta, round_bf16: bool):
+    """The conditioning path with low-rank factors; returns (z, rho, e~).
+
+    The appendix names the parts without equations; this is the reading used
+    here, the method's Eq. 6-8 with every d-wide signal replaced by a rank-64
+    latent and the correction factored through rank 32:
+
+    * latent of the rejected drafter state:  z = P m            (P: [64, d])
+    * rank-32 target-aware correction:      rho = z + beta A_c (B_c [z; u])
+                                             (B_c: [32, 64 + d], A_c: [64, 32])
+    * input-side latent residual fusion:    e~ = e + (W_v rho) * sigmoid(W_g [e; rho])
+                                             (W_v: [d, 64], W_g: [d, d + 64])
+
+    Rows j >= n_b keep e.  With ``round_bf16`` the latent z and rho are
+    rounded to bfloat16 where the GPU stores them (z as the carried latent,
+    rho as the input of the up-projections).
+    """
+    P = np.asarray(P, dtype=np.float64)
+    Bc = np.asarray(Bc, dtype=np.float64)
+    Ac = np.asarray(Ac, dtype=np.float64)
+    z = np.asarray(m, dtype=np.float64) @ P.T  # [B, K, 64]
+    if round_bf16:
+        z = round_to_bf16(z)
+    t = np.concatenate([z, np.asarray(u, dtype=np.float64)], axis=-1) @ Bc.T  # [B, K, 32]
+    rho = z + float(beta) * (t @ Ac.T)
+    if round_bf16:
+        rho = round_to_bf16(rho)
+    e_full = np.asarray(e_full, dtype=np.float64)
+    v = rho @ np.asarray(Wv, dtype=np.float64).T
+    g = np.concatenate([e_full, rho], axis=-1) @ np.asarray(Wg, dtype=np.float64).T
+    fused = e_full + v * sigmoid(g)
+    K = e_full.shape[1]
+    rows = np.arange(K)[None, :] < np.asarray(n)[:, None]
+    return z, rho, np.where(rows[..., None], fused, e_full)
+
+
+def retrace_round_lowrank(logits, draft, hD, hT, e, P, Bc, Ac, Wv, Wg, beta, dtype: str) -> dict:
+    """One round with the low-rank conditioning path (see lowrank_condition)."""
+    out = verify(logits, draft)
+    A = out["accept_len"]
+    K = np.asarray(draft).shape[1]
+    n = carried_rows(A, K)
+    m, u = align(hD, hT, A)
+    e_full = np.broadcast_to(np.asarray(e, dtype=np.float64), np.asarray(hD).shape)
+    z, rho, e_tilde = lowrank_condition(e_full, m, u, n, P, Bc, Ac, Wv, Wg, beta, round_bf16=(dtype == "bf16"))
+    out.update({"n": n, "z": z, "rho": rho, "e_tilde": e_tilde})
+    if dtype == "bf16":
+        out["e_tilde_rounded"] = round_to_bf16(e_tilde)
+    return out

@@ -61,3 +61,40 @@ def round_brute(logits, draft, hD, hT, e, Wc, Wv, Wg, beta, rnd=None):
             row.append(e[j][i] + v * (1.0 / (1.0 + math.exp(-g))))
         out.append(row)
     return {"t": t, "A": A, "committed": committed, "bonus": t[A], "n": n, "e_tilde": out}
+
+
+def lowrank_brute(logits, draft, hD, hT, e, P, Bc, Ac, Wv, Wg, beta, rnd=None):
+    """One sequence's round with the low-rank conditioning, by explicit sums.
+
+    P [L][d], Bc [C][L + d] (columns 0..L-1 act on the latent), Ac [L][C],
+    Wv [d][L], Wg [d][d + L] (columns 0..d-1 act on e).  ``rnd`` (optional)
+    rounds the latent and the corrected latent.
+    """
+    K = len(draft)
+    d = len(Wv)
+    L = len(P)
+    C = len(Bc)
+    t = [argmax_by_sort(logits[i]) for i in range(K + 1)]
+    A = accept_len_by_search(t, draft)
+    n = sum(1 for j in range(K) if A + 1 + j <= K - 1)
+    out = []
+    for j in range(K):
+        if j >= n:
+            out.append(list(e[j]))
+            continue
+        m = hD[A + 1 + j]
+        u = hT[A + j]
+        z = [sum(P[i][k] * m[k] for k in range(d)) for i in range(L)]
+        if rnd is not None:
+            z = rnd(z)
+        tc = [sum(Bc[c][i] * z[i] for i in range(L)) + sum(Bc[c][L + k] * u[k] for k in range(d)) for c in range(C)]
+        rho = [z[i] + beta * sum(Ac[i][c] * tc[c] for c in range(C)) for i in range(L)]
+        if rnd is not None:
+            rho = rnd(rho)
+        row = []
+        for f in range(d):
+            v = sum(Wv[f][i] * rho[i] for i in range(L))
+            g = sum(Wg[f][k] * e[j][k] for k in range(d)) + sum(Wg[f][d + i] * rho[i] for i in range(L))
+            row.append(e[j][f] + v * (1.0 / (1.0 + math.exp(-g))))
+        out.append(row)
+    return {"t": t, "A": A, "n": n, "e_tilde": out}

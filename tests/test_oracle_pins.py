@@ -378,6 +378,73 @@ def test_none_keeps_every_input_and_still_reports_n():
 
 
 # ---------------------------------------------------------------------------
+# Low-rank realisation (Appendix "Concurrent-Serving Experiment")
+# ---------------------------------------------------------------------------
+
+
+def _tiny_lowrank(rng, B, K, V, d, L, C):
+    x = _tiny(rng, B, K, V, d)
+    x.update(
+        P=rng.standard_normal((L, d)) / math.sqrt(d),
+        Bc=rng.standard_normal((C, L + d)) / math.sqrt(L + d),
+        Ac=rng.standard_normal((L, C)) / math.sqrt(C),
+        Wv=rng.standard_normal((d, L)) / math.sqrt(L),
+        Wg=rng.standard_normal((d, d + L)) / math.sqrt(d + L),
+    )
+    return x
+
+
+def _check_lowrank_against_brute(x, dtype="f32"):
+    out = oracle.retrace_round_lowrank(x["logits"], x["draft"], x["hD"], x["hT"], x["e"], x["P"], x["Bc"], x["Ac"],
+                                       x["Wv"], x["Wg"], x["beta"], dtype)
+    rnd = (lambda r: list(oracle.round_to_bf16(np.array(r)))) if dtype == "bf16" else None
+    for b in range(x["draft"].shape[0]):
+        ref = bf.lowrank_brute(x["logits"][b].tolist(), x["draft"][b].tolist(), x["hD"][b].tolist(),
+                               x["hT"][b].tolist(), x["e"][b].tolist(), x["P"].tolist(), x["Bc"].tolist(),
+                               x["Ac"].tolist(), x["Wv"].tolist(), x["Wg"].tolist(), x["beta"], rnd=rnd)
+        assert out["accept_len"][b] == ref["A"] and out["n"][b] == ref["n"]
+        np.testing.assert_allclose(out["e_tilde"][b], np.array(ref["e_tilde"]), rtol=1e-12, atol=1e-12)
+
+
+def test_lowrank_brute_force_random_tiny_shapes():
+    rng = np.random.default_rng(31)
+    for _ in range(60):
+        B, K, V, d = int(rng.integers(1, 3)), int(rng.integers(1, 8)), int(rng.integers(2, 40)), int(rng.integers(1, 7))
+        L, C = int(rng.integers(1, 5)), int(rng.integers(1, 4))
+        _check_lowrank_against_brute(_tiny_lowrank(rng, B, K, V, d, L, C))
+
+
+def test_lowrank_brute_force_bf16_rounding_points():
+    rng = np.random.default_rng(32)
+    for _ in range(30):
+        _check_lowrank_against_brute(_tiny_lowrank(rng, 2, 6, 16, 5, 3, 2), dtype="bf16")
+
+
+def test_lowrank_with_a_full_width_latent_is_the_method():
+    """With the latent as wide as the state (L = d) and P = I, the low-rank
+    path is Eq. 6-8 with W_c = A_c B_c (a rank-C correction), the value and
+    gate projections unchanged: the brute-force method round must agree."""
+    rng = np.random.default_rng(33)
+    for _ in range(20):
+        d, C = int(rng.integers(2, 6)), int(rng.integers(1, 4))
+        x = _tiny_lowrank(rng, 2, 6, 12, d, d, C)
+        x["P"] = np.eye(d)
+        Wc = x["Ac"] @ x["Bc"]  # [d, 2d]
+        for dtype in ("f32", "bf16"):
+            # bf16: the latent z = m is then exact (m holds bf16 values), and
+            # both paths round the same corrected value once
+            hD = oracle.round_to_bf16(x["hD"]) if dtype == "bf16" else x["hD"]
+            out = oracle.retrace_round_lowrank(x["logits"], x["draft"], hD, x["hT"], x["e"], x["P"], x["Bc"],
+                                               x["Ac"], x["Wv"], x["Wg"], x["beta"], dtype)
+            rnd = (lambda r: list(oracle.round_to_bf16(np.array(r)))) if dtype == "bf16" else None
+            for b in range(2):
+                ref = bf.round_brute(x["logits"][b].tolist(), x["draft"][b].tolist(), hD[b].tolist(),
+                                     x["hT"][b].tolist(), x["e"][b].tolist(), Wc.tolist(), x["Wv"].tolist(),
+                                     x["Wg"].tolist(), x["beta"], rnd=rnd)
+                np.testing.assert_allclose(out["e_tilde"][b], np.array(ref["e_tilde"]), rtol=1e-11, atol=1e-11)
+
+
+# ---------------------------------------------------------------------------
 # Planted mistakes: every one must make at least one pin above fail
 # ---------------------------------------------------------------------------
 
@@ -397,6 +464,9 @@ def _pins():
         test_fig3_overwrite_carries_the_rejected_suffix,
         test_raw_is_the_gated_fusion_of_the_aligned_draft_states,
         test_none_keeps_every_input_and_still_reports_n,
+        test_lowrank_brute_force_random_tiny_shapes,
+        test_lowrank_brute_force_bf16_rounding_points,
+        test_lowrank_with_a_full_width_latent_is_the_method,
     ]
 
 
@@ -448,7 +518,33 @@ def _mut_overwrite_unshifted(e_full, m, u, n, Wc, Wv, Wg, beta, variant, rr):
     return None, np.where(rows[..., None], shifted, e_full)
 
 
+def _mut_lowrank(**change):
+    def f(e_full, m, u, n, P, Bc, Ac, Wv, Wg, beta, round_bf16):
+        args = dict(e_full=e_full, m=m, u=u, n=n, P=P, Bc=Bc, Ac=Ac, Wv=Wv, Wg=Wg, beta=beta, round_bf16=round_bf16)
+        for k, fn in change.items():
+            args[k] = fn(args)
+        return orc.__dict__["_orig_lowrank"](**args)
+    return f
+
+
+def _mut_lowrank_swapped_halves(e_full, m, u, n, P, Bc, Ac, Wv, Wg, beta, round_bf16):
+    L = np.asarray(P).shape[0]
+    d = np.asarray(m).shape[-1]
+    Bc = np.asarray(Bc)
+    # B_c applied to [u; z] instead of [z; u]: the first d columns act on u
+    swapped = np.concatenate([Bc[:, d:], Bc[:, :d]], axis=1) if Bc.shape[1] == L + d and L != d else Bc[:, ::-1]
+    return orc.__dict__["_orig_lowrank"](e_full, m, u, n, P, swapped, Ac, Wv, Wg, beta, round_bf16)
+
+
 MUTATIONS = {
+    "low-rank correction drops beta": ("lowrank_condition", _mut_lowrank(beta=lambda a: 1.0)),
+    "low-rank latent not rounded": ("lowrank_condition", _mut_lowrank(round_bf16=lambda a: False)),
+    "low-rank gate ignores e": (
+        "lowrank_condition",
+        _mut_lowrank(Wg=lambda a: np.concatenate([np.zeros_like(np.asarray(a["Wg"])[:, : np.asarray(a["m"]).shape[-1]]),
+                                                  np.asarray(a["Wg"])[:, np.asarray(a["m"]).shape[-1]:]], 1)),
+    ),
+    "low-rank B_c halves swapped": ("lowrank_condition", _mut_lowrank_swapped_halves),
     "overwrite keeps the mask inputs": ("condition", _mut_condition({"overwrite": "none"})),
     "raw applies the correction": ("condition", _mut_condition({"raw": "corrected"})),
     "no conditioning runs the gate": ("condition", _mut_condition({"none": "raw"})),
@@ -483,6 +579,7 @@ def test_planted_mistakes_are_caught(name, monkeypatch):
     attr, fn = MUTATIONS[name]
     monkeypatch.setitem(orc.__dict__, "_orig_gate_fuse", orc.gate_fuse)
     monkeypatch.setitem(orc.__dict__, "_orig_condition", orc.condition)
+    monkeypatch.setitem(orc.__dict__, "_orig_lowrank", orc.lowrank_condition)
     monkeypatch.setattr(orc, attr, fn)
     monkeypatch.setattr(oracle, attr, fn, raising=False)
     caught = 0
