@@ -185,7 +185,7 @@ def cpu_threads() -> int:
         return os.cpu_count() or 1
 
 
-def prepare_oracle_sample(cfg: RoundConfig, sample_B: int, seed: int) -> dict:
+def prepare_oracle_sample(cfg: RoundConfig, sample_B: int, seed: int, lowrank: bool = False) -> dict:
     """Host float64 inputs for `sample_B` sequences drawn like `cfg` (weights at full size)."""
     from oracle import bf16_bits_to_f64  # test infrastructure: CPU-baseline legs only
     from paper_2608_29748_gb300.workloads import as_bits_numpy
@@ -199,16 +199,26 @@ def prepare_oracle_sample(cfg: RoundConfig, sample_B: int, seed: int) -> dict:
 
     host = {k: f64(x[k]) for k in ("logits", "hD", "hT", "e", "Wc", "Wv", "Wg")}
     host.update(draft=x["draft"].numpy(), beta=x["beta"], dtype=cfg.dtype, B=sample_B)
+    if lowrank:
+        from paper_2608_29748_gb300.workloads import make_lowrank_weights
+
+        host["lowrank"] = {k: f64(v) for k, v in make_lowrank_weights(cfg, device="cpu").items()}
     return host
 
 
 def time_oracle(host: dict, variant: str = "corrected") -> float:
     """Seconds the CPU oracle takes for one round over the prepared sample."""
-    from oracle import retrace_round as oracle_round_fn  # test infrastructure: CPU-baseline legs only
+    # test infrastructure: CPU-baseline legs only
+    from oracle import retrace_round as oracle_round_fn, retrace_round_lowrank as oracle_lowrank_fn
 
     t0 = time.perf_counter()
-    oracle_round_fn(host["logits"], host["draft"], host["hD"], host["hT"], host["e"], host["Wc"], host["Wv"],
-                    host["Wg"], host["beta"], host["dtype"], variant=variant)
+    if "lowrank" in host:
+        w = host["lowrank"]
+        oracle_lowrank_fn(host["logits"], host["draft"], host["hD"], host["hT"], host["e"], w["P"], w["Bc"],
+                          w["Ac"], w["Wv_lr"], w["Wg_lr"], host["beta"], host["dtype"])
+    else:
+        oracle_round_fn(host["logits"], host["draft"], host["hD"], host["hT"], host["e"], host["Wc"], host["Wv"],
+                        host["Wg"], host["beta"], host["dtype"], variant=variant)
     return time.perf_counter() - t0
 
 
@@ -245,6 +255,27 @@ def conditioning_flops(cfg: RoundConfig, R: int, dense_e: bool, variant: str = "
     f += 2 * R * d * (2 * d)  # [v; g_r] = [W_v; W_g,r] r
     f += 2 * R * d * d if dense_e else 2 * d * d  # W_g,e e (per row, or once for a broadcast e)
     return f
+
+
+LOWRANK_L, LOWRANK_C = 64, 32
+KERNELS_PER_ROUND_LOWRANK = 4  # verify_kernel, gate-bias GEMV, latent projection, latent fusion (tensor cores)
+
+
+def lowrank_flops(cfg: RoundConfig, R: int) -> int:
+    """Flops of the low-rank conditioning: per conditioned row z = P m,
+    t = B_c [z; u], rho = z + beta A_c t, [v; g_rho] = [W_v; W_g,rho] rho,
+    plus W_g,e e once."""
+    d, Lr, Cr = cfg.d, LOWRANK_L, LOWRANK_C
+    per_row = 2 * (Lr * d + Cr * (Lr + d) + Lr * Cr + 2 * d * Lr)
+    return R * per_row + 2 * d * d
+
+
+def lowrank_bytes(cfg: RoundConfig, R: int) -> int:
+    """Algorithmic bytes of the low-rank conditioning phase: the weights once
+    (W_g's e columns dominate), the packed [m; u] rows read, e~ rows written."""
+    es, d, Lr, Cr = cfg.elem_bytes, cfg.d, LOWRANK_L, LOWRANK_C
+    weights = (Lr * d + Cr * (Lr + d) + Lr * Cr + d * Lr + d * (d + Lr)) * es
+    return weights + R * 2 * d * es + R * d * es + d * es
 
 
 def round_hbm_bytes(cfg: RoundConfig, R: int) -> int:
@@ -287,9 +318,21 @@ def run_gpu(args) -> dict | None:
     fused = args.overlap and round_is_fused(cfg)
     if args.overlap and not fused:
         raise SystemExit("--overlap: the overlapped kernel does not cover this workload")
+    if args.lowrank and (args.overlap or args.variant != "corrected"):
+        raise SystemExit("--lowrank runs the corrected low-rank path alone")
     flags = VARIANT_FLAGS[args.variant] | (ROUND_OVERLAP_FLAG if fused else 0)
+    if args.lowrank:
+        from paper_2608_29748_gb300.workloads import make_lowrank_weights
+
+        lw = make_lowrank_weights(cfg, device=dev, seed=shard_seed(77 + 1000 * cfg.seed_offset, rank))
+
+        def round_fn(inputs, **kw):
+            return rt.run_round_lowrank(inputs, lw, ws, out=out, **kw)
+    else:
+        def round_fn(inputs, **kw):
+            return rt.run_round(inputs, ws, out=out, flags=flags, **kw)
     for _ in range(args.warmup):
-        rt.run_round(x, ws, out=out, flags=flags)
+        round_fn(x)
     torch.cuda.synchronize(dev)
 
     steps = args.steps
@@ -305,7 +348,7 @@ def run_gpu(args) -> dict | None:
         t_wall0 = time.perf_counter()
         for i in range(steps):
             flush.fill_(i & 0xFF)  # L2 flush: a 256 MB write between timed steps
-            rt.run_round(x, ws, out=out, flags=flags, phase_events=phase[i])
+            round_fn(x, phase_events=phase[i])
         torch.cuda.synchronize(dev)
         t_wall = time.perf_counter() - t_wall0
     barrier(world)
@@ -320,7 +363,8 @@ def run_gpu(args) -> dict | None:
     n = out.n.cpu().numpy().astype(np.int64)
     R = int(n.sum())
     step_avg_s = statistics.mean(step_ms) / 1e3
-    cflops = conditioning_flops(cfg, R, dense_e=False, variant=args.variant)
+    cflops = (lowrank_flops(cfg, R) if args.lowrank
+              else conditioning_flops(cfg, R, dense_e=False, variant=args.variant))
     status_flags = ws.check()
     if fused:
         # One kernel does the whole round: its floor is the larger of the HBM
@@ -376,7 +420,23 @@ def run_gpu(args) -> dict | None:
         if args.variant in ("overwrite", "none"):
             v_roof["kernel"] = "verify_kernel (argmax/compare/commit + every row of e~ copied)"
         c_roof = None
-        if cflops:
+        if args.lowrank:
+            cbytes = lowrank_bytes(cfg, R)
+            c_roof = {
+                "kernel": "low-rank conditioning: gate-bias GEMV + latent projection (tcgen05, split-K) + latent "
+                          "fusion (tcgen05)",
+                "bound": "hbm",
+                "achieved": round(cbytes / c_avg_s / 1e9, 1),
+                "peak": peaks["hbm_gbs"],
+                "unit": "GB/s",
+                "frac": round(cbytes / c_avg_s / 1e9 / peaks["hbm_gbs"], 4),
+                "peak_source": peaks["source"] + " HBM copy bandwidth",
+                "algorithmic_bytes": cbytes,
+                "algorithmic_flops": cflops,
+                "avg_launch_us": round(c_avg_s * 1e6, 2),
+                "traffic": None,
+            }
+        elif cflops:
             c_roof = {
                 "kernel": "cond_kernel: correction + gated-fusion projections (+ gate-bias GEMV), one persistent launch",
                 "bound": "tensor",
@@ -397,7 +457,7 @@ def run_gpu(args) -> dict | None:
         logits_gbs = cfg.logits_bytes() / v_avg_s / 1e9
 
     # ---- end to end through the public API with host buffers ----
-    e2e = run_e2e(rt, cfg, x, ws, dev, min(steps, args.e2e_steps), world, flags) if args.e2e_steps > 0 else None
+    e2e = run_e2e(cfg, x, dev, min(steps, args.e2e_steps), world, round_fn) if args.e2e_steps > 0 else None
 
     line = {
         "metric": METRIC,
@@ -419,14 +479,17 @@ def run_gpu(args) -> dict | None:
             "conditioned_rows_R": R,
             "l2": "flushed before every timed step (256 MB write, outside the per-step events)",
             "parallelism": f"replicas x{world} (batch-sharded, no collective)",
-            "variant": args.variant,
-            "round_kernel": "overlapped (one persistent launch)" if fused else "two launches (verify, projections)",
+            "variant": "low-rank (rank-64 latents, rank-32 correction)" if args.lowrank else args.variant,
+            "round_kernel": ("overlapped (one persistent launch)" if fused
+                             else "verify, GEMV, latent projection, latent fusion" if args.lowrank
+                             else "two launches (verify, projections)"),
         },
         "roofline": roofline,
         **line_extra,
         "logits_gbs": round(logits_gbs, 1),
         "e2e": e2e,
         "gpu_launches": (KERNELS_PER_ROUND_FUSED if fused
+                         else KERNELS_PER_ROUND_LOWRANK if args.lowrank
                          else KERNELS_PER_ROUND if cflops else 1) * steps,
         "wall_s_timed_region": round(t_wall, 4),
         "device_status_flags": status_flags,
@@ -439,13 +502,13 @@ def run_gpu(args) -> dict | None:
     return line if rank == 0 else None
 
 
-def run_e2e(rt, cfg, x, ws, dev, steps, world, flags=0) -> dict:
+def run_e2e(cfg, x, dev, steps, world, round_fn) -> dict:
     """Rounds/s with the step's inputs in pinned host memory and the outputs read back."""
     names = ["logits", "draft", "hD", "hT"]
     host = {k: x[k].cpu().pin_memory() for k in names}
     dev_in = {k: torch.empty_like(x[k]) for k in names}
     rest = {k: x[k] for k in ("e", "Wc", "Wv", "Wg", "beta", "cfg")}  # model parameters stay resident
-    out = rt.RoundBuffers(cfg.B, cfg.K, cfg.d, cfg.torch_dtype, device=dev)
+    out = round_fn(x)  # the round's output buffers
     out_host = {k: torch.empty(getattr(out, k).shape, dtype=getattr(out, k).dtype).pin_memory()
                 for k in ("accept_len", "committed", "bonus", "n", "e_out")}
     stream = torch.cuda.current_stream(dev)
@@ -453,7 +516,7 @@ def run_e2e(rt, cfg, x, ws, dev, steps, world, flags=0) -> dict:
     def step():
         for k in names:
             dev_in[k].copy_(host[k], non_blocking=True)
-        rt.run_round({**dev_in, **rest}, ws, out=out, flags=flags)
+        round_fn({**dev_in, **rest})
         for k, h in out_host.items():
             h.copy_(getattr(out, k), non_blocking=True)
 
@@ -474,7 +537,7 @@ def run_e2e(rt, cfg, x, ws, dev, steps, world, flags=0) -> dict:
 
 
 def cpu_baseline(cfg: RoundConfig, args) -> dict:
-    host = prepare_oracle_sample(cfg, args.cpu_sample, seed=1234)
+    host = prepare_oracle_sample(cfg, args.cpu_sample, seed=1234, lowrank=args.lowrank)
     secs = time_oracle(host, args.variant)
     rounds = host["B"] / cfg.B
     return {"value": round(rounds / secs, 6), "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
@@ -492,7 +555,7 @@ def run_reference(args) -> dict | None:
     if rank != 0:
         return None
     cfg = workload(args.config)
-    host = prepare_oracle_sample(cfg, args.ref_sample, seed=500)
+    host = prepare_oracle_sample(cfg, args.ref_sample, seed=500, lowrank=args.lowrank)
     for _ in range(min(args.warmup, 1)):
         time_oracle(host, args.variant)
     total = sum(time_oracle(host, args.variant) for _ in range(args.steps))
@@ -530,6 +593,8 @@ def parse_args(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--overlap", action="store_true",
                     help="time the overlapped single-kernel round (RETRACE_ROUND_OVERLAP)")
+    ap.add_argument("--lowrank", action="store_true",
+                    help="time the low-rank conditioning path (retrace_round_lowrank)")
     ap.add_argument("--variant", choices=sorted(VARIANT_FLAGS), default="corrected",
                     help="conditioning variant of the component ablation (default: the method)")
     return ap.parse_args(argv)

@@ -216,6 +216,42 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
                              size_t ws_bytes, uint32_t flags, const cudaEvent_t* phase_events,
                              cudaStream_t stream);
 
+/* Ranks of the low-rank conditioning path (Appendix "Concurrent-Serving
+ * Experiment": rank-64 rejected-suffix latents, rank-32 correction). */
+#define RETRACE_LOWRANK_LATENT 64
+#define RETRACE_LOWRANK_CORRECTION 32
+
+/* One round with the low-rank realisation of the conditioning path
+ * (Appendix "Concurrent-Serving Experiment").  The paper names its parts
+ * (rank-64 rejected-suffix latents, input-side latent residual fusion, a
+ * rank-32 target-aware correction, a one-round lifetime) without equations;
+ * the reading implemented here is Eq. 6-8 with the d-wide signal replaced by
+ * a rank-64 latent.  For each conditioned row j < n_b, with
+ * m = hD[b, A_b+1+j] and u = hT[b, A_b+j] (Eq. 4-5):
+ *     z   = P m                                   (the latent)
+ *     rho = z + beta * A_c (B_c [z; u])           (rank-32 correction)
+ *     e~  = e + (W_v rho) .* sigmoid(W_g [e; rho])
+ * z and rho are rounded to bf16 (bf16 dtype); rows j >= n_b keep e exactly.
+ * Verification outputs are those of retrace_round.
+ *   e     [d], the broadcast drafter input (the DFlash mask embedding); a
+ *         per-position e is not supported by this form.
+ *   P     [64, d];  B_c [32, 64 + d] (columns 0..63 act on z);  A_c [64, 32];
+ *   W_v   [d, 64];  W_g [d, d + 64] (columns 0..d-1 act on e); all `dtype`,
+ *         row-major.
+ *   phase_events  optional 4 events: before verification, after it, after
+ *         the latent projections, after the fusion.
+ * Tensor cores for bf16 with d a multiple of 128 and 16-byte aligned tensors;
+ * an FFMA kernel otherwise.  K >= 1, V >= 1, d >= 1. */
+retrace_status retrace_round_lowrank(const void* logits, int64_t logits_row_stride,
+                                     int64_t logits_batch_stride, const int32_t* draft,
+                                     const void* hD, const void* hT, const void* e, const void* P,
+                                     const void* Bc, const void* Ac, const void* Wv, const void* Wg,
+                                     float beta, retrace_dtype dtype, int B, int K, int V, int d,
+                                     int32_t* accept_len, int32_t* committed, int32_t* bonus,
+                                     int32_t* target_argmax, int32_t* n_out, void* e_out, void* ws,
+                                     size_t ws_bytes, const cudaEvent_t* phase_events,
+                                     cudaStream_t stream);
+
 /* Size in bytes of the fixed device scratch used by retrace_verify_noalloc. */
 #define RETRACE_NOALLOC_SCRATCH_BYTES 65536
 

@@ -54,8 +54,10 @@ def _load() -> ctypes.CDLL:
     lib.retrace_gate_fuse.argtypes = [P, I64, I64, P, P, P, P, I, I, I, I, P, P, SZ, P]
     lib.retrace_round.argtypes = [P, I64, I64, P, P, P, P, I64, I64, P, P, P, F, I, I, I, I, I,
                                   P, P, P, P, P, P, P, SZ, ctypes.c_uint32, P, P]
+    lib.retrace_round_lowrank.argtypes = [P, I64, I64, P, P, P, P, P, P, P, P, P, F, I, I, I, I, I,
+                                          P, P, P, P, P, P, P, SZ, P, P]
     for name in ("retrace_workspace_init", "retrace_workspace_check", "retrace_verify",
-                 "retrace_align_refine", "retrace_gate_fuse", "retrace_round"):
+                 "retrace_align_refine", "retrace_gate_fuse", "retrace_round", "retrace_round_lowrank"):
         getattr(lib, name).restype = I
     return lib
 
@@ -196,6 +198,28 @@ def retrace_round(logits, draft, hD, hT, e, Wc, Wv, Wg, beta, accept_len, commit
                              _stream(stream)))
 
 
+def retrace_round_lowrank(logits, draft, hD, hT, e, P, Bc, Ac, Wv, Wg, beta, accept_len, committed, bonus,
+                          e_out, ws, n_out=None, target_argmax=None, phase_events=None, stream=None):
+    """One round with the low-rank conditioning path (see include/retrace.h)."""
+    B, K1, V = logits.shape
+    K = K1 - 1
+    d = hD.shape[2]
+    if logits.stride(2) != 1:
+        raise ValueError("logits: vocabulary dimension must be contiguous")
+    if e.dim() != 1:
+        raise ValueError("e: the low-rank path takes one broadcast vector [d]")
+    ev = None
+    if phase_events is not None:
+        ev = (ctypes.c_void_p * 4)(*[x._as_parameter_.value for x in phase_events])
+    _check(lib.retrace_round_lowrank(_ptr(logits), logits.stride(1), logits.stride(0), _ptr(draft), _ptr(hD),
+                                     _ptr(hT), _ptr(e), _ptr(P), _ptr(Bc), _ptr(Ac), _ptr(Wv), _ptr(Wg),
+                                     float(beta), _dtype_code(logits), B, K, V, d, _ptr(accept_len),
+                                     _ptr(committed), _ptr(bonus), _ptr(target_argmax), _ptr(n_out), _ptr(e_out),
+                                     ws.ptr, ws.nbytes,
+                                     ctypes.cast(ev, ctypes.c_void_p) if ev is not None else None,
+                                     _stream(stream)))
+
+
 class RoundBuffers:
     """Device outputs of one round for a (B, K, d) shape."""
 
@@ -223,3 +247,18 @@ def run_round(x: dict, ws: Workspace, out: RoundBuffers | None = None, target_ar
 
 def version() -> str:
     return lib.retrace_version().decode()
+
+
+def run_round_lowrank(x: dict, w: dict, ws: Workspace, out: RoundBuffers | None = None, target_argmax=None,
+                      phase_events=None, stream=None) -> RoundBuffers:
+    """retrace_round_lowrank over the round inputs ``x`` and low-rank weights ``w``
+    (keys as in workloads.make_round_inputs / make_lowrank_weights)."""
+    logits = x["logits"]
+    B, K1, _ = logits.shape
+    d = x["hD"].shape[2]
+    if out is None:
+        out = RoundBuffers(B, K1 - 1, d, logits.dtype, logits.device)
+    retrace_round_lowrank(logits, x["draft"], x["hD"], x["hT"], x["e"], w["P"], w["Bc"], w["Ac"], w["Wv_lr"],
+                          w["Wg_lr"], x["beta"], out.accept_len, out.committed, out.bonus, out.e_out, ws,
+                          n_out=out.n, target_argmax=target_argmax, phase_events=phase_events, stream=stream)
+    return out

@@ -471,4 +471,97 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   return RETRACE_OK;
 }
 
+retrace_status retrace_round_lowrank(const void* logits, int64_t logits_row_stride,
+                                     int64_t logits_batch_stride, const int32_t* draft,
+                                     const void* hD, const void* hT, const void* e, const void* P,
+                                     const void* Bc, const void* Ac, const void* Wv, const void* Wg,
+                                     float beta, retrace_dtype dtype, int B, int K, int V, int d,
+                                     int32_t* accept_len, int32_t* committed, int32_t* bonus,
+                                     int32_t* target_argmax, int32_t* n_out, void* e_out, void* ws,
+                                     size_t ws_bytes, const cudaEvent_t* phase_events,
+                                     cudaStream_t stream) {
+  g_err[0] = '\0';
+  retrace_status st = check_verify_args(logits, dtype, B, K, V, logits_row_stride,
+                                        logits_batch_stride, draft, accept_len, committed, bonus);
+  if (st != RETRACE_OK) return st;
+  if ((st = check_cond_shape(dtype, B, K, d)) != RETRACE_OK) return st;
+  if (B == 0) return RETRACE_OK;
+  if (!hD || !hT || !e || !P || !Bc || !Ac || !Wv || !Wg || !e_out)
+    return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
+  const WsLayout Lw = ws_layout(B, K, d, elem_size(dtype));
+  if ((st = check_ws(ws, ws_bytes, Lw.total)) != RETRACE_OK) return st;
+  char* w = reinterpret_cast<char*>(ws);
+  const bool tc = lowrank_tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(e) &&
+                  aligned16(P) && aligned16(Bc) && aligned16(Ac) && aligned16(Wv) && aligned16(Wg) &&
+                  aligned16(e_out);
+  uint32_t* sync = reinterpret_cast<uint32_t*>(w + Lw.sync);
+  int32_t* R = reinterpret_cast<int32_t*>(sync + kSyncRowCount);
+  int32_t* rowmap = reinterpret_cast<int32_t*>(w + Lw.rowmap);
+
+  if (phase_events) RT_CUDA(cudaEventRecord(phase_events[0], stream), "cudaEventRecord");
+  if (tc) RT_CUDA(cudaMemsetAsync(sync, 0, Lw.sync_bytes, stream), "cudaMemsetAsync(sync)");
+  VerifyArgs va{};
+  va.logits = logits;
+  va.B = B;
+  va.K = K;
+  va.V = V;
+  va.row_stride = logits_row_stride;
+  va.batch_stride = logits_batch_stride;
+  va.draft = draft;
+  va.accept_len = accept_len;
+  va.committed = committed;
+  va.bonus = bonus;
+  va.target_argmax = target_argmax;
+  va.n_out = n_out;
+  va.keys = reinterpret_cast<unsigned long long*>(w + Lw.keys);
+  va.tickets = reinterpret_cast<uint32_t*>(w + Lw.tickets);
+  va.e = e;
+  va.e_batch_stride = 0;
+  va.e_pos_stride = 0;
+  va.e_out = e_out;
+  va.d = d;
+  va.hD = hD;
+  va.cond_copy = kCondCopyKeep;
+  if (tc) {  // the finalising CTA of each sequence packs its [m; u] rows
+    va.hT = hT;
+    va.apack = w + Lw.apack;
+    va.epack = w + Lw.epack;
+    va.rowmap = rowmap;
+    va.R_count = R;
+  }
+  RT_CUDA(launch_verify(va, dtype, stream), "verify kernel launch");
+  if (phase_events) RT_CUDA(cudaEventRecord(phase_events[1], stream), "cudaEventRecord");
+
+  LowRankArgs la{};
+  la.B = B;
+  la.K = K;
+  la.d = d;
+  la.dtype = dtype;
+  la.beta = beta;
+  la.hD = hD;
+  la.hT = hT;
+  la.e = e;
+  la.P = P;
+  la.Bc = Bc;
+  la.Ac = Ac;
+  la.Wv = Wv;
+  la.Wg = Wg;
+  la.accept_len = accept_len;
+  la.e_out = e_out;
+  la.ge = reinterpret_cast<float*>(w + Lw.ge);
+  la.apack = w + Lw.apack;
+  la.rowmap = rowmap;
+  la.R = R;
+  la.zpart = reinterpret_cast<float*>(w + Lw.lrz);
+  la.tpart = reinterpret_cast<float*>(w + Lw.lrt);
+  la.rho = w + Lw.lrrho;
+  la.tickets = reinterpret_cast<uint32_t*>(w + Lw.lrtk);
+  la.status = status_word(ws);
+  RT_CUDA(launch_lowrank(la, tc, stream), "low-rank conditioning launch");
+  if (phase_events) {
+    for (int k = 2; k < 4; ++k) RT_CUDA(cudaEventRecord(phase_events[k], stream), "cudaEventRecord");
+  }
+  return RETRACE_OK;
+}
+
 }  // extern "C"

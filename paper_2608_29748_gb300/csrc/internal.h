@@ -25,8 +25,15 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 //   apack    elem   [R_max, 2d] packed [m; u] rows (tensor-core path)
 //   epack    elem   [R_max, d]  packed per-position e rows (tensor-core path, dense e)
 //   rowmap   int32  [R_max]     packed row g -> position b*K + j
+//   lrz      fp32   [S, R_max, 64]  low-rank path: split partials of the latent P m
+//   lrt      fp32   [S, R_max, 32]  low-rank path: split partials of B_c[:, 64:] u
+//   lrrho    elem   [R_max, 64]     low-rank path: corrected latent rho
+//   lrtk     uint32 [4 * row blocks] low-rank path: split arrival counters, zero between calls
+constexpr int kLowRankLatent = 64;      // rank of the rejected-suffix latents
+constexpr int kLowRankCorrection = 32;  // rank of the target-aware correction
+constexpr int kLowRankSplits = 8;       // split-K parts per half of the [m; u] reduction
 struct WsLayout {
-  size_t status, sync, sync_bytes, keys, tickets, ge, r, apack, epack, rowmap, total;
+  size_t status, sync, sync_bytes, keys, tickets, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, lrtk, total;
 };
 
 inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
@@ -54,6 +61,14 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   off = align_up(off + rmax * dd * elem, 256);
   L.rowmap = off;
   off = align_up(off + rmax * 4, 256);
+  L.lrz = off;
+  off = align_up(off + (size_t)kLowRankSplits * rmax * kLowRankLatent * 4, 256);
+  L.lrt = off;
+  off = align_up(off + (size_t)kLowRankSplits * rmax * kLowRankCorrection * 4, 256);
+  L.lrrho = off;
+  off = align_up(off + rmax * kLowRankLatent * elem, 256);
+  L.lrtk = off;
+  off = align_up(off + 4 * ((rmax + 127) / 128) * 4, 256);
   L.total = off;
   return L;
 }
@@ -202,6 +217,35 @@ struct TcCondArgs {
   uint32_t* status;
 };
 cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream);
+
+// Low-rank conditioning (rank-64 latents, rank-32 correction; broadcast e).
+struct LowRankArgs {
+  int B, K, d;
+  retrace_dtype dtype;
+  float beta;
+  const void* hD;
+  const void* hT;
+  const void* e;   // [d]
+  const void* P;   // [64, d]
+  const void* Bc;  // [32, 64 + d]
+  const void* Ac;  // [64, 32]
+  const void* Wv;  // [d, 64]
+  const void* Wg;  // [d, d + 64]
+  const int32_t* accept_len;
+  void* e_out;
+  float* ge;  // [d]: W_g[:, :d] e
+  // tensor-core path: rows packed by the verification kernel
+  const void* apack;
+  const int32_t* rowmap;
+  const int32_t* R;
+  float* zpart;
+  float* tpart;
+  void* rho;
+  uint32_t* tickets;
+  uint32_t* status;
+};
+bool lowrank_tc_supported(retrace_dtype dtype, int d);
+cudaError_t launch_lowrank(const LowRankArgs& a, bool tc, cudaStream_t stream);
 
 // The whole round in one persistent launch: verification warps and
 // tensor-core warps share every SM (bf16, d a multiple of 256, 16-byte

@@ -140,6 +140,25 @@ def make_round_inputs(cfg: RoundConfig, device="cpu", seed: int | None = None) -
     }
 
 
+LOWRANK_LATENT = 64  # ranks of the low-rank conditioning weights (Appendix "Concurrent-Serving Experiment")
+LOWRANK_CORRECTION = 32
+
+
+def make_lowrank_weights(cfg: RoundConfig, device="cpu", seed: int | None = None) -> dict:
+    """Seeded Xavier-uniform weights of the low-rank conditioning path for ``cfg``:
+    P [64, d], B_c [32, 64 + d], A_c [64, 32], W_v [d, 64], W_g [d, d + 64]."""
+    seed = SEED + 1000 * cfg.seed_offset + 7 if seed is None else seed
+    g = _gen(device, seed)
+    d, Lr, Cr, dt = cfg.d, LOWRANK_LATENT, LOWRANK_CORRECTION, cfg.torch_dtype
+    return {
+        "P": xavier_uniform((Lr, d), g, device).to(dt),
+        "Bc": xavier_uniform((Cr, Lr + d), g, device).to(dt),
+        "Ac": xavier_uniform((Lr, Cr), g, device).to(dt),
+        "Wv_lr": xavier_uniform((d, Lr), g, device).to(dt),
+        "Wg_lr": xavier_uniform((d, d + Lr), g, device).to(dt),
+    }
+
+
 def xavier_uniform(shape, g, device) -> torch.Tensor:
     """U(-a, a) with a = sqrt(6 / (fan_in + fan_out)) for a [fan_out, fan_in] matrix."""
     fan_out, fan_in = shape
