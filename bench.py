@@ -258,7 +258,7 @@ def conditioning_flops(cfg: RoundConfig, R: int, dense_e: bool, variant: str = "
 
 
 LOWRANK_L, LOWRANK_C = 64, 32
-KERNELS_PER_ROUND_LOWRANK = 4  # verify_kernel, gate-bias GEMV, latent projection, latent fusion (tensor cores)
+KERNELS_PER_ROUND_LOWRANK = 4  # verify_kernel, latent projection, finish (+ GEMV), latent fusion (tensor cores)
 
 
 def lowrank_flops(cfg: RoundConfig, R: int) -> int:
@@ -423,8 +423,8 @@ def run_gpu(args) -> dict | None:
         if args.lowrank:
             cbytes = lowrank_bytes(cfg, R)
             c_roof = {
-                "kernel": "low-rank conditioning: gate-bias GEMV + latent projection (tcgen05, split-K) + latent "
-                          "fusion (tcgen05)",
+                "kernel": "low-rank conditioning: latent projection (tcgen05, split-K), finish (rho, + the "
+                          "gate-bias GEMV), latent fusion (tcgen05, persistent)",
                 "bound": "hbm",
                 "achieved": round(cbytes / c_avg_s / 1e9, 1),
                 "peak": peaks["hbm_gbs"],
@@ -481,7 +481,7 @@ def run_gpu(args) -> dict | None:
             "parallelism": f"replicas x{world} (batch-sharded, no collective)",
             "variant": "low-rank (rank-64 latents, rank-32 correction)" if args.lowrank else args.variant,
             "round_kernel": ("overlapped (one persistent launch)" if fused
-                             else "verify, GEMV, latent projection, latent fusion" if args.lowrank
+                             else "verify, latent projection, finish + GEMV, latent fusion" if args.lowrank
                              else "two launches (verify, projections)"),
         },
         "roofline": roofline,

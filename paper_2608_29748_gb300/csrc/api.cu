@@ -555,7 +555,7 @@ retrace_status retrace_round_lowrank(const void* logits, int64_t logits_row_stri
   la.zpart = reinterpret_cast<float*>(w + Lw.lrz);
   la.tpart = reinterpret_cast<float*>(w + Lw.lrt);
   la.rho = w + Lw.lrrho;
-  la.tickets = reinterpret_cast<uint32_t*>(w + Lw.lrtk);
+  la.gemv_next = sync + kSyncGemvNext;
   la.status = status_word(ws);
   RT_CUDA(launch_lowrank(la, tc, stream), "low-rank conditioning launch");
   if (phase_events) {

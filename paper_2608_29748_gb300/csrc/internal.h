@@ -28,12 +28,11 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 //   lrz      fp32   [S, R_max, 64]  low-rank path: split partials of the latent P m
 //   lrt      fp32   [S, R_max, 32]  low-rank path: split partials of B_c[:, 64:] u
 //   lrrho    elem   [R_max, 64]     low-rank path: corrected latent rho
-//   lrtk     uint32 [4 * row blocks] low-rank path: split arrival counters, zero between calls
 constexpr int kLowRankLatent = 64;      // rank of the rejected-suffix latents
 constexpr int kLowRankCorrection = 32;  // rank of the target-aware correction
 constexpr int kLowRankSplits = 8;       // split-K parts per half of the [m; u] reduction
 struct WsLayout {
-  size_t status, sync, sync_bytes, keys, tickets, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, lrtk, total;
+  size_t status, sync, sync_bytes, keys, tickets, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, total;
 };
 
 inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
@@ -67,8 +66,6 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   off = align_up(off + (size_t)kLowRankSplits * rmax * kLowRankCorrection * 4, 256);
   L.lrrho = off;
   off = align_up(off + rmax * kLowRankLatent * elem, 256);
-  L.lrtk = off;
-  off = align_up(off + 4 * ((rmax + 127) / 128) * 4, 256);
   L.total = off;
   return L;
 }
@@ -241,7 +238,7 @@ struct LowRankArgs {
   float* zpart;
   float* tpart;
   void* rho;
-  uint32_t* tickets;
+  uint32_t* gemv_next;  // zero before the call
   uint32_t* status;
 };
 bool lowrank_tc_supported(retrace_dtype dtype, int d);

@@ -10,15 +10,20 @@
 // z and rho are rounded to bf16 where they are stored (bf16 workloads); e is
 // the broadcast mask embedding, so W_g[:, :d] e is one GEMV per call.
 //
-// Tensor-core path (bf16, d a multiple of 128), two launches after the GEMV:
+// Tensor-core path (bf16, d a multiple of 128), three launches:
 //   lr_project_kernel  split-K over the packed [m; u] rows: the m half against
-//                      P (N = 64), the u half against B_c's u columns (N = 32);
-//                      fp32 partials per split, and the last CTA of each
-//                      (row block, warp quarter) sums them in a fixed order and
-//                      finishes z, t and rho for its 32 rows on CUDA cores;
-//   lr_fuse_kernel     one (128-row, 128-feature) tile per CTA: rho [128, 64]
-//                      against [W_v; W_g,rho] [256, 64] in four K16 MMAs, the
-//                      gate and residual in the epilogue.
+//                      P (N = 64), the u half against B_c's u columns (N = 32),
+//                      fp32 partials per split;
+//   lr_finish_kernel   one warp per row: sums the partials in a fixed order
+//                      (bitwise repeatable), rounds z, adds B_c[:, :64] z and
+//                      forms rho (lanes over the latent and correction ranks);
+//                      then every warp takes rows of the GEMV W_g[:, :d] e from
+//                      a counter (the grid has at least two CTAs per SM);
+//   lr_fuse_kernel     persistent over (128-row, 64-feature) tiles, two CTAs
+//                      per SM: rho [128, 64] against [W_v; W_g,rho] [128, 64]
+//                      in four K16 MMAs into one of two TMEM accumulators, the
+//                      gate and residual in an eight-warp epilogue (with K = 64
+//                      the epilogue, not the MMA, is the long pole).
 // FFMA path (fp32, other shapes): lr_simt_kernel, one CTA per conditioned row.
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -38,15 +43,22 @@ constexpr int A_BYTES = BM * BK * 2;          // 16 KB: 128 packed rows x 64
 constexpr int BP_BYTES = L * BK * 2;          // 8 KB: P tile (the 4 KB B_c tile uses the same slot)
 constexpr int STAGE_BYTES = A_BYTES + BP_BYTES;
 constexpr int SMEM_PROJECT = ST * STAGE_BYTES + 1024;
-// 48 KB of operands, padded so that at most two CTAs share an SM: each holds
-// 256 TMEM columns, and a third would wait in tcgen05.alloc.
+constexpr int kFuseThreads = 384;  // warps 0-3: TMA, MMA, TMEM; warps 4-11: epilogue
+constexpr int kFuseFeat = 64;      // features per fusion tile
+// Two stages of (rho tile 16 KB + B tile 16 KB), padded so that exactly two
+// CTAs share an SM: each holds 256 TMEM columns (two 128-column accumulators),
+// and a third CTA would only wait in tcgen05.alloc.
 constexpr int SMEM_FUSE = 80 * 1024;
+static_assert(SMEM_FUSE >= 2 * (BM * BK * 2 + 2 * kFuseFeat * BK * 2) + 1024, "fusion operands do not fit");
+static_assert(3 * SMEM_FUSE > 228 * 1024, "a third fusion CTA must not fit on an SM");
 constexpr uint32_t IDESC_P = idesc_bf16_f32(128, L);
 constexpr uint32_t IDESC_B = idesc_bf16_f32(128, C);
-constexpr uint32_t IDESC_F = idesc_bf16_f32(128, 256);
+constexpr uint32_t IDESC_F = idesc_bf16_f32(128, 128);
+
+constexpr int H = kLowRankSplits;  // split-K parts per half of the [m; u] reduction
 
 struct LrParams {
-  int d, H;  // H: splits per half of the [m; u] reduction
+  int d;
   const int32_t* R;
   float beta;
   const __nv_bfloat16* Bc;  // [32, 64 + d]
@@ -54,8 +66,12 @@ struct LrParams {
   float* zpart;             // [H, R_max, 64]
   float* tpart;             // [H, R_max, 32]
   __nv_bfloat16* rho;       // [R_max, 64]
-  uint32_t* tickets;        // [4 * row blocks]
   long long rmax;
+  // W_g[:, :d] e in the projection's idle warps
+  const __nv_bfloat16* Wg;  // [d, d + 64]
+  const __nv_bfloat16* e;   // [d]
+  float* ge;                // [d]
+  uint32_t* gemv_next;      // row counter, zero before the launch
   uint32_t* status;
 };
 
@@ -84,66 +100,12 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 
 __device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
-// z, t and rho of packed row g from the split partials (fixed summation order).
-__device__ void finish_row(const LrParams& p, long long g) {
-  const int d = p.d;
-  float z[L], t[C];
-#pragma unroll
-  for (int i = 0; i < L; ++i) z[i] = 0.f;
-#pragma unroll
-  for (int c = 0; c < C; ++c) t[c] = 0.f;
-  for (int s = 0; s < p.H; ++s) {
-    const float4* zp = reinterpret_cast<const float4*>(p.zpart + ((long long)s * p.rmax + g) * L);
-    const float4* tp = reinterpret_cast<const float4*>(p.tpart + ((long long)s * p.rmax + g) * C);
-#pragma unroll
-    for (int q = 0; q < L / 4; ++q) {
-      const float4 v = __ldcg(zp + q);
-      z[4 * q] += v.x;
-      z[4 * q + 1] += v.y;
-      z[4 * q + 2] += v.z;
-      z[4 * q + 3] += v.w;
-    }
-#pragma unroll
-    for (int q = 0; q < C / 4; ++q) {
-      const float4 v = __ldcg(tp + q);
-      t[4 * q] += v.x;
-      t[4 * q + 1] += v.y;
-      t[4 * q + 2] += v.z;
-      t[4 * q + 3] += v.w;
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < L; ++i) z[i] = bf16_round(z[i]);  // the stored latent
-  // t += B_c[:, :64] z   (the u part is already in t)
-#pragma unroll
-  for (int c = 0; c < C; ++c) {
-    const __nv_bfloat16* brow = p.Bc + (long long)c * (L + d);
-    float s = t[c];
-#pragma unroll
-    for (int i = 0; i < L; ++i) s = fmaf(__bfloat162float(brow[i]), z[i], s);
-    t[c] = s;
-  }
-  // rho = z + beta A_c t, rounded; 64 bf16 = 128 bytes
-  uint4* out = reinterpret_cast<uint4*>(p.rho + g * L);
-#pragma unroll
-  for (int q = 0; q < L / 8; ++q) {
-    uint32_t w[4];
-#pragma unroll
-    for (int h = 0; h < 4; ++h) {
-      float r2[2];
-#pragma unroll
-      for (int k = 0; k < 2; ++k) {
-        const int i = 8 * q + 2 * h + k;
-        const __nv_bfloat16* arow = p.Ac + i * C;
-        float s = 0.f;
-#pragma unroll
-        for (int c = 0; c < C; ++c) s = fmaf(__bfloat162float(arow[c]), t[c], s);
-        r2[k] = z[i] + p.beta * s;
-      }
-      w[h] = pack_bf16x2(r2[0], r2[1]);
-    }
-    out[q] = make_uint4(w[0], w[1], w[2], w[3]);
-  }
+// Logistic function from the fast exponential and division intrinsics: their
+// relative error (a few fp32 ulp) is far below the bf16 rounding of the
+// output.  The argument is clamped to [-80, 80], where the fp32 logistic is
+// already 0 or 1 to within its rounding.
+__device__ __forceinline__ float fast_sigmoid(float x) {
+  return __fdividef(1.f, 1.f + __expf(-fminf(fmaxf(x, -80.f), 80.f)));
 }
 
 // grid (row blocks, 2H): blockIdx.y < H reduces over the m half against P,
@@ -163,9 +125,9 @@ __global__ void __launch_bounds__(256, 1)
   const int m0 = blockIdx.x * BM;
   if (m0 >= R) return;
   const int d = p.d;
-  const int half = (int)blockIdx.y / p.H, part = (int)blockIdx.y % p.H;
+  const int half = (int)blockIdx.y / H, part = (int)blockIdx.y % H;
   const int KB = d / BK;  // k-blocks per half
-  const int kb0 = part * KB / p.H, kb1 = (part + 1) * KB / p.H;
+  const int kb0 = part * KB / H, kb1 = (part + 1) * KB / H;
   const int nkb = kb1 - kb0;
   const int N = half == 0 ? L : C;
 
@@ -256,20 +218,6 @@ __global__ void __launch_bounds__(256, 1)
             o[x] = nkb > 0 ? make_float4(v[4 * x], v[4 * x + 1], v[4 * x + 2], v[4 * x + 3]) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
       }
-      // The last of the 2H split CTAs to finish this warp's 32 rows finishes them.
-      __threadfence();
-      __syncwarp();
-      int last = 0;
-      if (lane == 0) {
-        uint32_t* tk = p.tickets + (long long)blockIdx.x * 4 + (warp - 4);
-        last = atomicAdd(tk, 1u) == (uint32_t)(2 * p.H - 1) ? 1 : 0;
-        if (last) *tk = 0u;  // ready for the next call
-      }
-      last = __shfl_sync(0xFFFFFFFFu, last, 0);
-      if (last) {
-        __threadfence();
-        if (g < R) finish_row(p, g);
-      }
     }
   }
   tc_fence_before();
@@ -280,25 +228,132 @@ __global__ void __launch_bounds__(256, 1)
   }
 }
 
-// grid (row blocks, d / 128): rows [m0, m0+128) x features [n0, n0+128).
-__global__ void __launch_bounds__(256, 1)
+// One warp per packed row g: z = sum of the split partials (fixed order),
+// rounded; t = the u partials + B_c[:, :64] z; rho = z + beta A_c t, rounded.
+// B_c[:, :64] and A_c are staged as fp32, transposed so lanes read
+// consecutive words.  Called by whole CTAs (it synchronises them).
+__device__ __forceinline__ void finish_rows(const LrParams& p, long long g, int R, int d, int lane) {
+  __shared__ float s_bct[L * C];  // B_c[c][i] at [i][c]
+  __shared__ float s_act[C * L];  // A_c[i][c] at [c][i]
+  for (int k = threadIdx.x; k < C * L; k += 256) {  // consecutive threads write consecutive words
+    const int i = k / C, c = k % C;
+    s_bct[k] = __bfloat162float(p.Bc[(long long)c * (L + d) + i]);
+    const int c2 = k / L, i2 = k % L;
+    s_act[k] = __bfloat162float(p.Ac[i2 * C + c2]);
+  }
+  __syncthreads();
+  if (g >= R) return;
+  float zs[H][2], ts[H];
+#pragma unroll
+  for (int s2 = 0; s2 < H; ++s2) {  // every load in flight at once
+    const float* zp = p.zpart + ((long long)s2 * p.rmax + g) * L;
+    zs[s2][0] = __ldcg(zp + lane);
+    zs[s2][1] = __ldcg(zp + 32 + lane);
+    ts[s2] = __ldcg(p.tpart + ((long long)s2 * p.rmax + g) * C + lane);
+  }
+  float z0 = 0.f, z1 = 0.f, t = 0.f;
+#pragma unroll
+  for (int s2 = 0; s2 < H; ++s2) {  // fixed order over the splits
+    z0 += zs[s2][0];
+    z1 += zs[s2][1];
+    t += ts[s2];
+  }
+  z0 = bf16_round(z0);  // the stored latent
+  z1 = bf16_round(z1);
+  const unsigned FULL = 0xFFFFFFFFu;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) t = fmaf(s_bct[i * C + lane], __shfl_sync(FULL, z0, i), t);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) t = fmaf(s_bct[(32 + i) * C + lane], __shfl_sync(FULL, z1, i), t);
+  float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    const float tc = __shfl_sync(FULL, t, c);
+    r0 = fmaf(s_act[c * L + lane], tc, r0);
+    r1 = fmaf(s_act[c * L + 32 + lane], tc, r1);
+  }
+  p.rho[g * L + lane] = __float2bfloat16_rn(z0 + p.beta * r0);
+  p.rho[g * L + 32 + lane] = __float2bfloat16_rn(z1 + p.beta * r1);
+}
+
+// W_g[:, :d] e, one row of W_g per claim from the counter; eight 16-byte loads
+// in flight per lane (d a multiple of 8).
+__device__ __forceinline__ void lr_gemv_rows(const LrParams& p, int d, int lane) {
+  const uint4* ev = reinterpret_cast<const uint4*>(p.e);
+  const int nv = d / 8;
+  for (;;) {
+    uint32_t i = 0;
+    if (lane == 0) i = atomicAdd(p.gemv_next, 1u);
+    i = __shfl_sync(0xFFFFFFFFu, i, 0);
+    if (i >= (uint32_t)d) return;
+    const uint4* wv = reinterpret_cast<const uint4*>(p.Wg + (long long)i * (d + L));
+    float acc = 0.f;
+    for (int k0 = 0; k0 < nv; k0 += 8 * 32) {
+      uint4 a[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int k = k0 + u * 32 + lane;
+        a[u] = k < nv ? __ldg(wv + k) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int k = k0 + u * 32 + lane;
+        if (k < nv) {
+          const uint4 b = __ldg(ev + k);
+          const uint32_t aw[4] = {a[u].x, a[u].y, a[u].z, a[u].w}, bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+          for (int x = 0; x < 4; ++x) {
+            acc = fmaf(bf16_lo(aw[x]), bf16_lo(bw[x]), acc);
+            acc = fmaf(bf16_hi(aw[x]), bf16_hi(bw[x]), acc);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, off);
+    if (lane == 0) p.ge[i] = acc;
+  }
+}
+
+// grid >= ceil(R_max / 8) and >= two CTAs per SM: rows first, then the GEMV.
+__global__ void __launch_bounds__(256) lr_finish_kernel(const LrParams p) {
+  const int R = *(volatile const int32_t*)p.R;
+  const long long g = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int d = p.d, lane = threadIdx.x & 31;
+  if ((long long)blockIdx.x * 8 < R) finish_rows(p, g, R, d, lane);  // uniform over the CTA
+  lr_gemv_rows(p, d, lane);
+}
+
+// Persistent: CTA c takes tiles c, c + G, ... of the (row block, 64-feature
+// block) grid, feature blocks fastest.  Two operand stages (rho tile + B tile)
+// and two TMEM accumulators, so a tile's loads and MMAs overlap the previous
+// tile's epilogue; two CTAs per SM interleave their epilogues.
+__global__ void __launch_bounds__(kFuseThreads, 2)
     lr_fuse_kernel(const __grid_constant__ CUtensorMap tmRho, const __grid_constant__ CUtensorMap tmWv,
                    const __grid_constant__ CUtensorMap tmWg, const LrFuseParams p) {
   extern __shared__ uint8_t dsmem[];
-  __shared__ __align__(8) uint64_t bar_full;
-  __shared__ __align__(8) uint64_t bar_acc;
+  __shared__ __align__(8) uint64_t bar_full[2];
+  __shared__ __align__(8) uint64_t bar_empty[2];
+  __shared__ __align__(8) uint64_t bar_acc[2];
+  __shared__ __align__(8) uint64_t bar_free[2];
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int R = *(volatile const int32_t*)p.R;
-  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * 128;
-  if (m0 >= R) return;
   const int d = p.d;
+  const int nb = d / kFuseFeat;
+  const int tiles = (R + BM - 1) / BM * nb;
+  if ((int)blockIdx.x >= tiles) return;
+  const int my_tiles = (tiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
   if (threadIdx.x == 0) {
     s_abort = 0;
-    mbar_init(smem_u32(&bar_full), 1);
-    mbar_init(smem_u32(&bar_acc), 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&bar_full[b]), 1);
+      mbar_init(smem_u32(&bar_empty[b]), 1);
+      mbar_init(smem_u32(&bar_acc[b]), 1);
+      mbar_init(smem_u32(&bar_free[b]), 8);  // one arrival per epilogue warp
+    }
     fence_mbar_init();
   }
   if (warp == 2) {
@@ -309,60 +364,105 @@ __global__ void __launch_bounds__(256, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = s_tmem;
-  const uint32_t a_base = (smem_u32(dsmem) + 1023u) & ~1023u;
-  const uint32_t b_base = a_base + BM * BK * 2;
+  const uint32_t base = (smem_u32(dsmem) + 1023u) & ~1023u;
+  constexpr uint32_t A_TILE = BM * BK * 2, B_TILE = 2 * kFuseFeat * BK * 2, STAGE = A_TILE + B_TILE;
 
   if (warp == 0) {
+    // ---- TMA: the rho tile and the B tile of each of this CTA's tiles ----
     if (lane == 0) {
-      // rho rows, then the B tile: 128 rows of W_v over the matching 128 rows
-      // of W_g[:, d:d+64], so v and the gate pre-activation share a TMEM lane
-      mbar_arrive_expect_tx(smem_u32(&bar_full), BM * BK * 2 + 256 * BK * 2);
-      tma_load_2d(a_base, &tmRho, 0, m0, smem_u32(&bar_full));
-      tma_load_2d(b_base, &tmWv, 0, n0, smem_u32(&bar_full));
-      tma_load_2d(b_base + 128 * BK * 2, &tmWg, d, n0, smem_u32(&bar_full));
-      const bool ok = mbar_wait_bounded(smem_u32(&bar_full), 0, &s_abort);
-      if (ok) {
-        tc_fence_after();
-#pragma unroll
-        for (int k = 0; k < BK / 16; ++k)
-          tc_mma_bf16(tmem, sw128_kmajor_desc(a_base + (uint32_t)k * 32u),
-                      sw128_kmajor_desc(b_base + (uint32_t)k * 32u), IDESC_F, k > 0 ? 1u : 0u);
-      } else {
-        raise_abort(&s_abort, p.status);
+      bool ok = true;
+      int k = 0;
+      for (; k < my_tiles; ++k) {
+        const int t = (int)blockIdx.x + k * (int)gridDim.x;
+        const int m0 = t / nb * BM, n0 = t % nb * kFuseFeat;
+        const uint32_t b = k & 1, ph = (k >> 1) & 1u;
+        if (!mbar_wait_bounded(smem_u32(&bar_empty[b]), ph ^ 1u, &s_abort)) {
+          ok = false;
+          break;
+        }
+        const uint32_t a_dst = base + b * STAGE, b_dst = a_dst + A_TILE;
+        // 64 rows of W_v over the matching 64 rows of W_g[:, d:d+64]: v and
+        // the gate pre-activation of a feature share a TMEM lane
+        mbar_arrive_expect_tx(smem_u32(&bar_full[b]), STAGE);
+        tma_load_2d(a_dst, &tmRho, 0, m0, smem_u32(&bar_full[b]));
+        tma_load_2d(b_dst, &tmWv, 0, n0, smem_u32(&bar_full[b]));
+        tma_load_2d(b_dst + kFuseFeat * BK * 2, &tmWg, d, n0, smem_u32(&bar_full[b]));
       }
-      tc_commit(smem_u32(&bar_acc));
+      if (!ok) {
+        raise_abort(&s_abort, p.status);
+        volatile int never = 0;  // drain this CTA's own copies in flight
+        for (int j = k > 2 ? k - 2 : 0; j < k; ++j) mbar_wait_bounded(smem_u32(&bar_full[j & 1]), (j >> 1) & 1u, &never);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---- MMA: tile k into accumulator k % 2 ----
+    if (lane == 0) {
+      bool ok = true;
+      for (int k = 0; k < my_tiles; ++k) {
+        const uint32_t b = k & 1, ph = (k >> 1) & 1u;
+        if (!mbar_wait_bounded(smem_u32(&bar_free[b]), ph ^ 1u, &s_abort) ||
+            !mbar_wait_bounded(smem_u32(&bar_full[b]), ph, &s_abort)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a_src = base + b * STAGE, b_src = a_src + A_TILE;
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk)
+          tc_mma_bf16(tmem + b * 128u, sw128_kmajor_desc(a_src + (uint32_t)kk * 32u),
+                      sw128_kmajor_desc(b_src + (uint32_t)kk * 32u), IDESC_F, kk > 0 ? 1u : 0u);
+        tc_commit(smem_u32(&bar_empty[b]));  // operand stage free once these MMAs complete
+        tc_commit(smem_u32(&bar_acc[b]));
+      }
+      if (!ok) {
+        raise_abort(&s_abort, p.status);
+        for (int b = 0; b < 2; ++b) tc_commit(smem_u32(&bar_acc[b]));  // release a waiting epilogue
+      }
     }
     __syncwarp();
   } else if (warp >= 4) {
-    const int q = (warp - 4) * 32 + lane;
-    const int g = m0 + q;
-    const uint32_t taddr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-    const bool ok = warp_wait(smem_u32(&bar_acc), 0, &s_abort);
-    tc_fence_after();
-    if (ok && !s_abort) {
+    // ---- epilogue: e~ = e + v * sigmoid(ge + g); warp w: rows 32 (w % 4) + lane
+    // (a warp reaches TMEM lanes 32 (w % 4) .. +31 only), features
+    // 32 ((w - 4) / 4) .. +31 of the tile ----
+    const int fh = (warp - 4) >> 2;
+    for (int k = 0; k < my_tiles; ++k) {
+      const int t = (int)blockIdx.x + k * (int)gridDim.x;
+      const int m0 = t / nb * BM, n = t % nb * kFuseFeat + fh * 32;
+      const int g = m0 + (warp & 3) * 32 + lane;
+      const uint32_t b = k & 1, ph = (k >> 1) & 1u;
+      const bool ok = warp_wait(smem_u32(&bar_acc[b]), ph, &s_abort);
+      tc_fence_after();
+      if (!ok || s_abort) {
+        if (!ok && lane == 0) raise_abort(&s_abort, p.status);
+        break;
+      }
       const long long orow = g < R ? __ldg(p.rowmap + g) : 0;
-      for (int cc = 0; cc < 4; ++cc) {
-        float v[32], gt[32];
-        tmem_ld_32cols(taddr + (uint32_t)(cc * 32), v);
-        tmem_ld_32cols(taddr + 128u + (uint32_t)(cc * 32), gt);
-        if (g < R) {
-          const int n = n0 + cc * 32;
-          const uint4* ev = reinterpret_cast<const uint4*>(p.e + n);
-          uint4* ov = reinterpret_cast<uint4*>(p.e_out + orow * d + n);
+      const uint32_t taddr = tmem + b * 128u + ((uint32_t)((warp & 3) * 32) << 16);
+      float v[32], gt[32];
+      tmem_ld_32cols(taddr + (uint32_t)(fh * 32), v);
+      tmem_ld_32cols(taddr + (uint32_t)(kFuseFeat + fh * 32), gt);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&bar_free[b]));  // accumulator read: the next tile may use it
+      if (g < R) {
+        const uint4* ev = reinterpret_cast<const uint4*>(p.e + n);
+        const float4* gv = reinterpret_cast<const float4*>(p.ge + n);
+        uint4* ov = reinterpret_cast<uint4*>(p.e_out + orow * d + n);
 #pragma unroll
-          for (int x = 0; x < 4; ++x) {
-            const uint4 ew = __ldg(ev + x);
-            const uint32_t ewords[4] = {ew.x, ew.y, ew.z, ew.w};
-            uint32_t o[4];
+        for (int x = 0; x < 4; ++x) {
+          const uint4 ew = __ldg(ev + x);
+          const float4 ga = __ldg(gv + 2 * x), gb = __ldg(gv + 2 * x + 1);
+          const float gw[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
+          const uint32_t ewords[4] = {ew.x, ew.y, ew.z, ew.w};
+          uint32_t o[4];
 #pragma unroll
-            for (int w = 0; w < 4; ++w) {
-              const int c0 = x * 8 + 2 * w;
-              const float g0 = gt[c0] + __ldg(p.ge + n + c0), g1 = gt[c0 + 1] + __ldg(p.ge + n + c0 + 1);
-              const float s0 = 1.f / (1.f + expf(-g0)), s1 = 1.f / (1.f + expf(-g1));
-              o[w] = pack_bf16x2(bf16_lo(ewords[w]) + v[c0] * s0, bf16_hi(ewords[w]) + v[c0 + 1] * s1);
-            }
-            ov[x] = make_uint4(o[0], o[1], o[2], o[3]);
+          for (int w = 0; w < 4; ++w) {
+            const int c0 = x * 8 + 2 * w;
+            const float s0 = fast_sigmoid(gt[c0] + gw[2 * w]), s1 = fast_sigmoid(gt[c0 + 1] + gw[2 * w + 1]);
+            o[w] = pack_bf16x2(bf16_lo(ewords[w]) + v[c0] * s0, bf16_hi(ewords[w]) + v[c0 + 1] * s1);
           }
+          ov[x] = make_uint4(o[0], o[1], o[2], o[3]);
         }
       }
     }
@@ -465,39 +565,39 @@ __global__ void __launch_bounds__(256) lr_simt_kernel(const LowRankArgs a) {
 
 }  // namespace
 
-bool lowrank_tc_supported(retrace_dtype dtype, int d) { return dtype == RETRACE_BF16 && d % 128 == 0; }
+bool lowrank_tc_supported(retrace_dtype dtype, int d) { return dtype == RETRACE_BF16 && d % kFuseFeat == 0; }
 
 cudaError_t launch_lowrank(const LowRankArgs& a, bool tc, cudaStream_t stream) {
   const long long rmax = (long long)a.B * (a.K > 1 ? a.K - 1 : 0);
   if (rmax <= 0) return cudaSuccess;
-  const unsigned gemv_grid = (unsigned)((a.d + 7) / 8);
-  if (a.dtype == RETRACE_BF16)
-    lr_gemv_kernel<__nv_bfloat16><<<gemv_grid, 256, 0, stream>>>(
-        reinterpret_cast<const __nv_bfloat16*>(a.Wg), (long long)a.d + L,
-        reinterpret_cast<const __nv_bfloat16*>(a.e), a.d, a.ge);
-  else
-    lr_gemv_kernel<float><<<gemv_grid, 256, 0, stream>>>(reinterpret_cast<const float*>(a.Wg), (long long)a.d + L,
-                                                         reinterpret_cast<const float*>(a.e), a.d, a.ge);
-  cudaError_t err = cudaGetLastError();
-  if (err != cudaSuccess) return err;
+  cudaError_t err;
   if (!tc) {
+    const unsigned gemv_grid = (unsigned)((a.d + 7) / 8);
+    if (a.dtype == RETRACE_BF16)
+      lr_gemv_kernel<__nv_bfloat16><<<gemv_grid, 256, 0, stream>>>(
+          reinterpret_cast<const __nv_bfloat16*>(a.Wg), (long long)a.d + L,
+          reinterpret_cast<const __nv_bfloat16*>(a.e), a.d, a.ge);
+    else
+      lr_gemv_kernel<float><<<gemv_grid, 256, 0, stream>>>(reinterpret_cast<const float*>(a.Wg), (long long)a.d + L,
+                                                           reinterpret_cast<const float*>(a.e), a.d, a.ge);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
     if (a.dtype == RETRACE_BF16)
       lr_simt_kernel<__nv_bfloat16><<<(unsigned)rmax, 256, 0, stream>>>(a);
     else
       lr_simt_kernel<float><<<(unsigned)rmax, 256, 0, stream>>>(a);
     return cudaGetLastError();
   }
+  DeviceInfo info{0, 148};
+  if ((err = device_info(&info)) != cudaSuccess) return err;
   static bool attr_done[64] = {false};
-  int dev = 0;
-  if ((err = cudaGetDevice(&dev)) != cudaSuccess) return err;
-  if (!attr_done[dev & 63]) {
+  if (!attr_done[info.device & 63]) {
     if ((err = cudaFuncSetAttribute(lr_project_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_PROJECT)) !=
         cudaSuccess)
       return err;
     if ((err = cudaFuncSetAttribute(lr_fuse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_FUSE)) !=
         cudaSuccess)
       return err;
-    attr_done[dev & 63] = true;
+    attr_done[info.device & 63] = true;
   }
   const uint64_t d = (uint64_t)a.d;
   CUtensorMap mA, mP, mBc, mRho, mWv, mWg;
@@ -505,13 +605,12 @@ cudaError_t launch_lowrank(const LowRankArgs& a, bool tc, cudaStream_t stream) {
       encode_tensor_map_2d(&mP, a.P, d, L, 2 * d, BK, L) != CUDA_SUCCESS ||
       encode_tensor_map_2d(&mBc, a.Bc, L + d, C, 2 * (L + d), BK, C) != CUDA_SUCCESS ||
       encode_tensor_map_2d(&mRho, a.rho, L, (uint64_t)rmax, 2 * L, BK, BM) != CUDA_SUCCESS ||
-      encode_tensor_map_2d(&mWv, a.Wv, L, d, 2 * L, BK, 128) != CUDA_SUCCESS ||
-      encode_tensor_map_2d(&mWg, a.Wg, d + L, d, 2 * (d + L), BK, 128) != CUDA_SUCCESS)
+      encode_tensor_map_2d(&mWv, a.Wv, L, d, 2 * L, BK, kFuseFeat) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWg, a.Wg, d + L, d, 2 * (d + L), BK, kFuseFeat) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
   const unsigned mt = (unsigned)((rmax + BM - 1) / BM);
   LrParams p{};
   p.d = a.d;
-  p.H = kLowRankSplits;
   p.R = a.R;
   p.beta = a.beta;
   p.Bc = reinterpret_cast<const __nv_bfloat16*>(a.Bc);
@@ -519,10 +618,16 @@ cudaError_t launch_lowrank(const LowRankArgs& a, bool tc, cudaStream_t stream) {
   p.zpart = a.zpart;
   p.tpart = a.tpart;
   p.rho = reinterpret_cast<__nv_bfloat16*>(a.rho);
-  p.tickets = a.tickets;
   p.rmax = rmax;
+  p.Wg = reinterpret_cast<const __nv_bfloat16*>(a.Wg);
+  p.e = reinterpret_cast<const __nv_bfloat16*>(a.e);
+  p.ge = a.ge;
+  p.gemv_next = a.gemv_next;
   p.status = a.status;
-  lr_project_kernel<<<dim3(mt, 2 * kLowRankSplits), 256, SMEM_PROJECT, stream>>>(mA, mP, mBc, p);
+  lr_project_kernel<<<dim3(mt, 2 * H), 256, SMEM_PROJECT, stream>>>(mA, mP, mBc, p);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  const long long fgrid = (rmax + 7) / 8 > 2LL * info.sm_count ? (rmax + 7) / 8 : 2LL * info.sm_count;
+  lr_finish_kernel<<<(unsigned)fgrid, 256, 0, stream>>>(p);
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
   LrFuseParams f{};
   f.d = a.d;
@@ -532,7 +637,10 @@ cudaError_t launch_lowrank(const LowRankArgs& a, bool tc, cudaStream_t stream) {
   f.ge = a.ge;
   f.e_out = reinterpret_cast<__nv_bfloat16*>(a.e_out);
   f.status = a.status;
-  lr_fuse_kernel<<<dim3(mt, (unsigned)(a.d / 128)), 256, SMEM_FUSE, stream>>>(mRho, mWv, mWg, f);
+  const long long tiles_max = (long long)mt * (a.d / kFuseFeat);
+  const long long slots = 2LL * info.sm_count;  // two CTAs per SM
+  const unsigned grid = (unsigned)(tiles_max < slots ? tiles_max : slots);
+  lr_fuse_kernel<<<grid, kFuseThreads, SMEM_FUSE, stream>>>(mRho, mWv, mWg, f);
   return cudaGetLastError();
 }
 
