@@ -16,6 +16,7 @@ from .retrace_oracle import (  # noqa: F401
     conditioned_rows,
     correct,
     f64_to_bf16_bits,
+    filtered_distribution,
     gate_fuse,
     LOWRANK_CORRECTION,
     LOWRANK_LATENT,
@@ -26,4 +27,5 @@ from .retrace_oracle import (  # noqa: F401
     sigmoid,
     target_argmax,
     verify,
+    verify_sampled,
 )

@@ -386,3 +386,90 @@ def retrace_round_lowrank(logits, draft, hD, hT, e, P, Bc, Ac, Wv, Wg, beta, dty
     if dtype == "bf16":
         out["e_tilde_rounded"] = round_to_bf16(e_tilde)
     return out
+
+
+# ---------------------------------------------------------------------------
+# Stochastic verification at temperature T (Appendix "Evaluation Protocol":
+# T = 1 with top_p = 0.95 and top_k = 20).  The paper keeps the underlying
+# speculative-decoding verification and does not state it; the reading used
+# here is standard speculative sampling on the filtered distributions, with
+# the random numbers passed in as inputs.
+# ---------------------------------------------------------------------------
+
+
+def filtered_distribution(logits_row, T: float, top_k: int, top_p: float):
+    """Tokens and probabilities of the sampling distribution of one row.
+
+    softmax(logits / T), restricted to the top_k largest logits (the lowest
+    index first among equal values), renormalised, then restricted to the
+    shortest prefix of those tokens, in that order, whose probability sums to
+    at least top_p, and renormalised again.  Returns (tokens, probs) in that
+    order (descending probability).
+    """
+    x = np.asarray(logits_row, dtype=np.float64)
+    idx = np.arange(x.shape[0])
+    order = np.lexsort((idx, -x))[:top_k]  # descending value, ascending index
+    w = np.exp((x[order] - x[order[0]]) / float(T))
+    p = w / w.sum()
+    keep = int(np.searchsorted(np.cumsum(p), top_p, side="left")) + 1  # first prefix reaching top_p
+    keep = min(keep, len(order))
+    w = w[:keep]
+    return order[:keep], w / w.sum()
+
+
+def _prob_of(tokens, probs, y):
+    hit = np.flatnonzero(tokens == y)
+    return float(probs[hit[0]]) if hit.size else 0.0
+
+
+def _sample(tokens, probs, u: float) -> int:
+    """Inverse-CDF draw in the given token order: the first token whose
+    cumulative probability exceeds u (u in [0, 1))."""
+    c = np.cumsum(probs)
+    j = int(np.searchsorted(c, u * c[-1], side="right"))
+    return int(tokens[min(j, len(tokens) - 1)])
+
+
+def verify_sampled(target_logits, draft_logits, draft, uniforms, T: float, top_k: int, top_p: float) -> dict:
+    """Speculative sampling of one block per sequence.
+
+    With p_i and q_i the filtered target and draft distributions of slot i,
+    draft token x_i is accepted iff u_i q_i(x_i) < p_i(x_i), i.e. with
+    probability min(1, p_i(x_i) / q_i(x_i)); verification stops at the first
+    rejection A.  The token appended after the accepted prefix is drawn with
+    u_K: from the residual max(0, p_A - q_A) (renormalised; from p_A if it is
+    zero everywhere) when A < K, from p_K when every draft was accepted.
+    A draft token outside [0, V) is rejected.
+    """
+    tl = np.asarray(target_logits)
+    dl = np.asarray(draft_logits)
+    draft = np.asarray(draft)
+    u = np.asarray(uniforms, dtype=np.float64)
+    B, K = draft.shape
+    V = tl.shape[2]
+    A = np.full(B, K, dtype=np.int64)
+    committed = np.full((B, K + 1), -1, dtype=np.int64)
+    bonus = np.empty(B, dtype=np.int64)
+    for b in range(B):
+        a = K
+        for i in range(K):
+            x = int(draft[b, i])
+            pt, pp = filtered_distribution(tl[b, i], T, top_k, top_p)
+            qt, qp = filtered_distribution(dl[b, i], T, top_k, top_p)
+            px = _prob_of(pt, pp, x) if 0 <= x < V else 0.0
+            qx = _prob_of(qt, qp, x) if 0 <= x < V else 0.0
+            if not (0 <= x < V and u[b, i] * qx < px):
+                a = i
+                break
+        pt, pp = filtered_distribution(tl[b, a], T, top_k, top_p)
+        if a < K:
+            qt, qp = filtered_distribution(dl[b, a], T, top_k, top_p)
+            res = np.array([max(0.0, pp[j] - _prob_of(qt, qp, int(pt[j]))) for j in range(len(pt))])
+            y = _sample(pt, res, u[b, K]) if res.sum() > 0 else _sample(pt, pp, u[b, K])
+        else:
+            y = _sample(pt, pp, u[b, K])
+        A[b] = a
+        committed[b, :a] = draft[b, :a]
+        committed[b, a] = y
+        bonus[b] = y
+    return {"accept_len": A, "committed": committed, "bonus": bonus}

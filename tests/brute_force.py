@@ -98,3 +98,59 @@ def lowrank_brute(logits, draft, hD, hT, e, P, Bc, Ac, Wv, Wg, beta, rnd=None):
             row.append(e[j][f] + v * (1.0 / (1.0 + math.exp(-g))))
         out.append(row)
     return {"t": t, "A": A, "n": n, "e_tilde": out}
+
+
+def filtered_brute(row, T, top_k, top_p):
+    """Sampling distribution of one row by explicit loops: a full sort by
+    (value descending, index ascending), the first top_k, softmax at T over
+    them, the shortest prefix reaching top_p, renormalised."""
+    order = sorted(range(len(row)), key=lambda v: (-row[v], v))[:top_k]
+    w = [math.exp((row[v] - row[order[0]]) / T) for v in order]
+    total = sum(w)
+    acc, keep = 0.0, len(order)
+    for j in range(len(order)):
+        acc += w[j] / total
+        if acc >= top_p:
+            keep = j + 1
+            break
+    z = sum(w[:keep])
+    return order[:keep], [x / z for x in w[:keep]]
+
+
+def sampled_brute(tlog, dlog, draft, u, T, top_k, top_p):
+    """One sequence of speculative sampling (accept iff u_i q(x) < p(x);
+    residual max(0, p - q) at the first rejection, else p at slot K;
+    inverse CDF in the filtered order)."""
+    K = len(draft)
+    V = len(tlog[0])
+
+    def prob(dist, y):
+        toks, ps = dist
+        return ps[toks.index(y)] if y in toks else 0.0
+
+    def draw(toks, ws, r):
+        total = sum(ws)
+        acc = 0.0
+        for t, w in zip(toks, ws):
+            acc += w
+            if acc > r * total:
+                return t
+        return toks[-1]
+
+    a = K
+    for i in range(K):
+        x = draft[i]
+        ok = False
+        if 0 <= x < V:
+            ok = u[i] * prob(filtered_brute(dlog[i], T, top_k, top_p), x) < prob(filtered_brute(tlog[i], T, top_k, top_p), x)
+        if not ok:
+            a = i
+            break
+    pd = filtered_brute(tlog[a], T, top_k, top_p)
+    if a < K:
+        qd = filtered_brute(dlog[a], T, top_k, top_p)
+        res = [max(0.0, pd[1][j] - prob(qd, pd[0][j])) for j in range(len(pd[0]))]
+        y = draw(pd[0], res, u[K]) if sum(res) > 0 else draw(pd[0], pd[1], u[K])
+    else:
+        y = draw(pd[0], pd[1], u[K])
+    return {"A": a, "committed": list(draft[:a]) + [y]}

@@ -445,6 +445,96 @@ def test_lowrank_with_a_full_width_latent_is_the_method():
 
 
 # ---------------------------------------------------------------------------
+# Stochastic verification (speculative sampling on filtered distributions)
+# ---------------------------------------------------------------------------
+
+
+def _sampled_case(rng, B, K, V, spread=1.5):
+    tl = rng.standard_normal((B, K + 1, V)) * spread
+    dl = tl[:, :K] + rng.standard_normal((B, K, V)) * 0.7  # a drafter close to the target
+    draft = np.argsort(-dl, axis=-1, kind="stable")[:, :, :3][np.arange(B)[:, None], np.arange(K)[None, :],
+                                                              rng.integers(0, 3, size=(B, K))]
+    return tl, dl, draft, rng.random((B, K + 1))
+
+
+def test_filtered_distribution_brute_force():
+    rng = np.random.default_rng(41)
+    for _ in range(200):
+        V = int(rng.integers(1, 30))
+        row = np.round(rng.standard_normal(V) * 2, 1)  # rounding plants equal logits
+        T, k, pth = float(rng.uniform(0.3, 2.0)), int(rng.integers(1, V + 1)), float(rng.uniform(0.05, 1.0))
+        toks, probs = oracle.filtered_distribution(row, T, k, pth)
+        bt, bp = bf.filtered_brute(row.tolist(), T, k, pth)
+        assert list(toks) == bt
+        np.testing.assert_allclose(probs, bp, rtol=1e-12, atol=1e-14)
+
+
+def test_sampled_verification_brute_force():
+    rng = np.random.default_rng(42)
+    for _ in range(40):
+        B, K, V = int(rng.integers(1, 4)), int(rng.integers(1, 7)), int(rng.integers(2, 25))
+        T, k, pth = float(rng.uniform(0.5, 1.5)), int(rng.integers(1, V + 1)), float(rng.uniform(0.5, 1.0))
+        tl, dl, draft, u = _sampled_case(rng, B, K, V)
+        out = oracle.verify_sampled(tl, dl, draft, u, T, k, pth)
+        for b in range(B):
+            ref = bf.sampled_brute(tl[b].tolist(), dl[b].tolist(), draft[b].tolist(), u[b].tolist(), T, k, pth)
+            assert out["accept_len"][b] == ref["A"]
+            assert list(out["committed"][b, : ref["A"] + 1]) == ref["committed"]
+
+
+def test_sampled_verification_is_lossless():
+    """The defining property: over the random numbers, the first committed
+    token is distributed as the filtered target distribution p_0, whatever the
+    draft token and the draft distribution (integrated over a fine grid of
+    (u_0, u_K) here, exact up to the grid)."""
+    rng = np.random.default_rng(43)
+    V, T, k, pth = 7, 1.0, 5, 0.9
+    N = 400
+    grid = (np.arange(N) + 0.5) / N
+    for _ in range(3):
+        tl = rng.standard_normal((1, 2, V)) * 1.5
+        dl = rng.standard_normal((1, 1, V)) * 1.5
+        qt, qp = oracle.filtered_distribution(dl[0, 0], T, k, pth)
+        pt, pp = oracle.filtered_distribution(tl[0, 0], T, k, pth)
+        want = np.zeros(V)
+        want[pt] = pp
+        got = np.zeros(V)
+        for x, qx in zip(qt, qp):  # the draft token is drawn from q
+            for u0 in grid:
+                for uk in grid[::8]:
+                    y = oracle.verify_sampled(tl, dl, np.array([[x]]), np.array([[u0, uk]]), T, k, pth)["committed"][0, 0]
+                    got[y] += qx / (N * len(grid[::8]))
+        np.testing.assert_allclose(got, want, atol=3e-2)
+
+
+def test_sampled_verification_with_top_k_one_is_greedy():
+    """top_k = 1 makes both distributions one-hot on the row argmax, so with
+    drafts equal to the drafter's argmax the block is verified exactly as by
+    greedy verification, for any random numbers."""
+    rng = np.random.default_rng(44)
+    for _ in range(20):
+        B, K, V = 3, 6, 17
+        tl = rng.standard_normal((B, K + 1, V))
+        dl = tl[:, :K] + rng.standard_normal((B, K, V)) * 0.6
+        draft = np.argmax(dl, axis=-1)
+        out = oracle.verify_sampled(tl, dl, draft, rng.random((B, K + 1)), 1.0, 1, 0.95)
+        ref = oracle.verify(tl, draft)
+        np.testing.assert_array_equal(out["accept_len"], ref["accept_len"])
+        np.testing.assert_array_equal(out["committed"], ref["committed"])
+
+
+def test_sampled_verification_accepts_everything_when_draft_equals_target():
+    """q = p and drafts drawn from it: u q(x) < p(x) = q(x) holds for every
+    u < 1, so the whole block is accepted and the bonus comes from p_K."""
+    rng = np.random.default_rng(45)
+    B, K, V = 4, 5, 11
+    tl = rng.standard_normal((B, K + 1, V))
+    draft = np.argsort(-tl[:, :K], axis=-1, kind="stable")[:, :, 0]
+    out = oracle.verify_sampled(tl, tl[:, :K].copy(), draft, rng.random((B, K + 1)), 1.0, 4, 0.9)
+    assert (out["accept_len"] == K).all()
+
+
+# ---------------------------------------------------------------------------
 # Planted mistakes: every one must make at least one pin above fail
 # ---------------------------------------------------------------------------
 
@@ -467,6 +557,10 @@ def _pins():
         test_lowrank_brute_force_random_tiny_shapes,
         test_lowrank_brute_force_bf16_rounding_points,
         test_lowrank_with_a_full_width_latent_is_the_method,
+        test_filtered_distribution_brute_force,
+        test_sampled_verification_brute_force,
+        test_sampled_verification_with_top_k_one_is_greedy,
+        test_sampled_verification_accepts_everything_when_draft_equals_target,
     ]
 
 
@@ -536,7 +630,23 @@ def _mut_lowrank_swapped_halves(e_full, m, u, n, P, Bc, Ac, Wv, Wg, beta, round_
     return orc.__dict__["_orig_lowrank"](e_full, m, u, n, P, swapped, Ac, Wv, Wg, beta, round_bf16)
 
 
+def _mut_filtered(kind):
+    def f(logits_row, T, top_k, top_p):
+        if kind == "no_temperature":
+            return orc.__dict__["_orig_filtered"](logits_row, 1.0, top_k, top_p)
+        toks, probs = orc.__dict__["_orig_filtered"](logits_row, T, top_k, 1.0)
+        if kind == "top_p_drops_crossing":  # keeps only the prefix strictly below top_p
+            keep = max(1, int(np.searchsorted(np.cumsum(probs), top_p, side="left")))
+        else:  # top-p ignored
+            keep = len(toks)
+        return toks[:keep], probs[:keep] / probs[:keep].sum()
+    return f
+
+
 MUTATIONS = {
+    "temperature ignored": ("filtered_distribution", _mut_filtered("no_temperature")),
+    "top-p drops the crossing token": ("filtered_distribution", _mut_filtered("top_p_drops_crossing")),
+    "top-p ignored": ("filtered_distribution", _mut_filtered("no_top_p")),
     "low-rank correction drops beta": ("lowrank_condition", _mut_lowrank(beta=lambda a: 1.0)),
     "low-rank latent not rounded": ("lowrank_condition", _mut_lowrank(round_bf16=lambda a: False)),
     "low-rank gate ignores e": (
@@ -580,6 +690,7 @@ def test_planted_mistakes_are_caught(name, monkeypatch):
     monkeypatch.setitem(orc.__dict__, "_orig_gate_fuse", orc.gate_fuse)
     monkeypatch.setitem(orc.__dict__, "_orig_condition", orc.condition)
     monkeypatch.setitem(orc.__dict__, "_orig_lowrank", orc.lowrank_condition)
+    monkeypatch.setitem(orc.__dict__, "_orig_filtered", orc.filtered_distribution)
     monkeypatch.setattr(orc, attr, fn)
     monkeypatch.setattr(oracle, attr, fn, raising=False)
     caught = 0
