@@ -185,7 +185,8 @@ def cpu_threads() -> int:
         return os.cpu_count() or 1
 
 
-def prepare_oracle_sample(cfg: RoundConfig, sample_B: int, seed: int, lowrank: bool = False) -> dict:
+def prepare_oracle_sample(cfg: RoundConfig, sample_B: int, seed: int, lowrank: bool = False,
+                          sampled: bool = False) -> dict:
     """Host float64 inputs for `sample_B` sequences drawn like `cfg` (weights at full size)."""
     from oracle import bf16_bits_to_f64  # test infrastructure: CPU-baseline legs only
     from paper_2608_29748_gb300.workloads import as_bits_numpy
@@ -203,6 +204,13 @@ def prepare_oracle_sample(cfg: RoundConfig, sample_B: int, seed: int, lowrank: b
         from paper_2608_29748_gb300.workloads import make_lowrank_weights
 
         host["lowrank"] = {k: f64(v) for k, v in make_lowrank_weights(cfg, device="cpu").items()}
+    if sampled:
+        from paper_2608_29748_gb300.workloads import make_sampled_inputs
+
+        sm = make_sampled_inputs(sub, x["logits"], device="cpu", seed=seed + 1)
+        host["sampled"] = {"draft_logits": f64(sm["draft_logits"]), "draft": sm["draft"].numpy(),
+                           "uniforms": sm["uniforms"].double().numpy(), "T": sm["temperature"], "k": sm["top_k"],
+                           "p": sm["top_p"]}
     return host
 
 
@@ -212,7 +220,18 @@ def time_oracle(host: dict, variant: str = "corrected") -> float:
     from oracle import retrace_round as oracle_round_fn, retrace_round_lowrank as oracle_lowrank_fn
 
     t0 = time.perf_counter()
-    if "lowrank" in host:
+    if "sampled" in host:
+        import oracle
+
+        sm = host["sampled"]
+        out = oracle.verify_sampled(host["logits"], sm["draft_logits"], sm["draft"], sm["uniforms"], sm["T"], sm["k"],
+                                    sm["p"])
+        K = sm["draft"].shape[1]
+        m, u = oracle.align(host["hD"], host["hT"], out["accept_len"])
+        e_full = np.broadcast_to(host["e"], host["hD"].shape)
+        oracle.condition(e_full, m, u, oracle.carried_rows(out["accept_len"], K), host["Wc"], host["Wv"], host["Wg"],
+                         host["beta"], "corrected", host["dtype"] == "bf16")
+    elif "lowrank" in host:
         w = host["lowrank"]
         oracle_lowrank_fn(host["logits"], host["draft"], host["hD"], host["hT"], host["e"], w["P"], w["Bc"],
                           w["Ac"], w["Wv_lr"], w["Wg_lr"], host["beta"], host["dtype"])
@@ -258,6 +277,7 @@ def conditioning_flops(cfg: RoundConfig, R: int, dense_e: bool, variant: str = "
 
 
 LOWRANK_L, LOWRANK_C = 64, 32
+KERNELS_PER_ROUND_SAMPLED = 6  # sampled top-k and finalize; pack + cond_kernel for each conditioning entry point
 KERNELS_PER_ROUND_LOWRANK = 4  # verify_kernel, latent projection, finish (+ GEMV), latent fusion (tensor cores)
 
 
@@ -318,8 +338,10 @@ def run_gpu(args) -> dict | None:
     fused = args.overlap and round_is_fused(cfg)
     if args.overlap and not fused:
         raise SystemExit("--overlap: the overlapped kernel does not cover this workload")
-    if args.lowrank and (args.overlap or args.variant != "corrected"):
-        raise SystemExit("--lowrank runs the corrected low-rank path alone")
+    if (args.lowrank or args.sampled) and (args.overlap or args.variant != "corrected"):
+        raise SystemExit("--lowrank / --sampled run the corrected path alone")
+    if args.lowrank and args.sampled:
+        raise SystemExit("--lowrank and --sampled are separate paths")
     flags = VARIANT_FLAGS[args.variant] | (ROUND_OVERLAP_FLAG if fused else 0)
     if args.lowrank:
         from paper_2608_29748_gb300.workloads import make_lowrank_weights
@@ -328,6 +350,30 @@ def run_gpu(args) -> dict | None:
 
         def round_fn(inputs, **kw):
             return rt.run_round_lowrank(inputs, lw, ws, out=out, **kw)
+    elif args.sampled:
+        from paper_2608_29748_gb300.workloads import make_sampled_inputs
+
+        x.update(make_sampled_inputs(cfg, x["logits"], device=dev, seed=shard_seed(99 + 1000 * cfg.seed_offset, rank)))
+        r_buf = torch.empty((cfg.B, cfg.K, cfg.d), dtype=cfg.torch_dtype, device=dev)
+
+        def round_fn(inputs, phase_events=None):
+            # a temperature-1 round: sampled verification, then the conditioning entry points
+            ev = phase_events or [None] * 4
+            st = torch.cuda.current_stream(dev)
+            if ev[0] is not None:
+                ev[0].record(st)
+            rt.retrace_verify_sampled(inputs["logits"], inputs["draft_logits"], inputs["draft"], inputs["uniforms"],
+                                      x["temperature"], x["top_k"], x["top_p"], out.accept_len, out.committed,
+                                      out.bonus, ws)
+            if ev[1] is not None:
+                ev[1].record(st)
+            rt.retrace_align_refine(inputs["hD"], inputs["hT"], out.accept_len, x["Wc"], x["beta"], r_buf, out.n, ws)
+            if ev[2] is not None:
+                ev[2].record(st)
+            rt.retrace_gate_fuse(x["e"], r_buf, out.n, x["Wv"], x["Wg"], out.e_out, ws)
+            if ev[3] is not None:
+                ev[3].record(st)
+            return out
     else:
         def round_fn(inputs, **kw):
             return rt.run_round(inputs, ws, out=out, flags=flags, **kw)
@@ -402,6 +448,10 @@ def run_gpu(args) -> dict | None:
         v_gbs = vbytes / v_avg_s / 1e9
         c_avg_s = statistics.mean(cond_ms) / 1e3
         c_tflops = cflops / c_avg_s / 1e12
+        if args.sampled:  # both logits tensors are read once
+            vbytes = (cfg.B * (2 * cfg.K + 1) * cfg.V * cfg.elem_bytes + cfg.B * (cfg.K + 1) * 4 * 2
+                      + cfg.B * cfg.K * 4 + 3 * cfg.B * 4)
+            v_gbs = vbytes / v_avg_s / 1e9
         v_roof = {
             "kernel": "verify_kernel (argmax/compare/commit + copy of unconditioned rows + row packing)",
             "bound": "hbm",
@@ -419,6 +469,10 @@ def run_gpu(args) -> dict | None:
         }
         if args.variant in ("overwrite", "none"):
             v_roof["kernel"] = "verify_kernel (argmax/compare/commit + every row of e~ copied)"
+        if args.sampled:
+            v_roof["kernel"] = ("sampled_topk_kernel + sampled_finalize_kernel (top-k of every target and drafter "
+                                "row, accept tests, draw)")
+            v_roof["traffic"] = None
         c_roof = None
         if args.lowrank:
             cbytes = lowrank_bytes(cfg, R)
@@ -457,7 +511,8 @@ def run_gpu(args) -> dict | None:
         logits_gbs = cfg.logits_bytes() / v_avg_s / 1e9
 
     # ---- end to end through the public API with host buffers ----
-    e2e = run_e2e(cfg, x, dev, min(steps, args.e2e_steps), world, round_fn) if args.e2e_steps > 0 else None
+    names = ["logits", "draft", "hD", "hT"] + (["draft_logits", "uniforms"] if args.sampled else [])
+    e2e = run_e2e(cfg, x, dev, min(steps, args.e2e_steps), world, round_fn, names) if args.e2e_steps > 0 else None
 
     line = {
         "metric": METRIC,
@@ -479,7 +534,9 @@ def run_gpu(args) -> dict | None:
             "conditioned_rows_R": R,
             "l2": "flushed before every timed step (256 MB write, outside the per-step events)",
             "parallelism": f"replicas x{world} (batch-sharded, no collective)",
-            "variant": "low-rank (rank-64 latents, rank-32 correction)" if args.lowrank else args.variant,
+            "variant": ("low-rank (rank-64 latents, rank-32 correction)" if args.lowrank
+                        else f"temperature {x['temperature']}, top_k {x['top_k']}, top_p {x['top_p']} "
+                             "(speculative sampling)" if args.sampled else args.variant),
             "round_kernel": ("overlapped (one persistent launch)" if fused
                              else "verify, latent projection, finish + GEMV, latent fusion" if args.lowrank
                              else "two launches (verify, projections)"),
@@ -490,6 +547,7 @@ def run_gpu(args) -> dict | None:
         "e2e": e2e,
         "gpu_launches": (KERNELS_PER_ROUND_FUSED if fused
                          else KERNELS_PER_ROUND_LOWRANK if args.lowrank
+                         else KERNELS_PER_ROUND_SAMPLED if args.sampled
                          else KERNELS_PER_ROUND if cflops else 1) * steps,
         "wall_s_timed_region": round(t_wall, 4),
         "device_status_flags": status_flags,
@@ -502,9 +560,8 @@ def run_gpu(args) -> dict | None:
     return line if rank == 0 else None
 
 
-def run_e2e(cfg, x, dev, steps, world, round_fn) -> dict:
+def run_e2e(cfg, x, dev, steps, world, round_fn, names) -> dict:
     """Rounds/s with the step's inputs in pinned host memory and the outputs read back."""
-    names = ["logits", "draft", "hD", "hT"]
     host = {k: x[k].cpu().pin_memory() for k in names}
     dev_in = {k: torch.empty_like(x[k]) for k in names}
     rest = {k: x[k] for k in ("e", "Wc", "Wv", "Wg", "beta", "cfg")}  # model parameters stay resident
@@ -537,7 +594,7 @@ def run_e2e(cfg, x, dev, steps, world, round_fn) -> dict:
 
 
 def cpu_baseline(cfg: RoundConfig, args) -> dict:
-    host = prepare_oracle_sample(cfg, args.cpu_sample, seed=1234, lowrank=args.lowrank)
+    host = prepare_oracle_sample(cfg, args.cpu_sample, seed=1234, lowrank=args.lowrank, sampled=args.sampled)
     secs = time_oracle(host, args.variant)
     rounds = host["B"] / cfg.B
     return {"value": round(rounds / secs, 6), "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
@@ -555,7 +612,7 @@ def run_reference(args) -> dict | None:
     if rank != 0:
         return None
     cfg = workload(args.config)
-    host = prepare_oracle_sample(cfg, args.ref_sample, seed=500, lowrank=args.lowrank)
+    host = prepare_oracle_sample(cfg, args.ref_sample, seed=500, lowrank=args.lowrank, sampled=args.sampled)
     for _ in range(min(args.warmup, 1)):
         time_oracle(host, args.variant)
     total = sum(time_oracle(host, args.variant) for _ in range(args.steps))
@@ -593,6 +650,8 @@ def parse_args(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--overlap", action="store_true",
                     help="time the overlapped single-kernel round (RETRACE_ROUND_OVERLAP)")
+    ap.add_argument("--sampled", action="store_true",
+                    help="time a temperature-1 round (retrace_verify_sampled + the conditioning entry points)")
     ap.add_argument("--lowrank", action="store_true",
                     help="time the low-rank conditioning path (retrace_round_lowrank)")
     ap.add_argument("--variant", choices=sorted(VARIANT_FLAGS), default="corrected",

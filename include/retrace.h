@@ -216,6 +216,36 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
                              size_t ws_bytes, uint32_t flags, const cudaEvent_t* phase_events,
                              cudaStream_t stream);
 
+/* Stochastic verification of a draft block at temperature T with top-k /
+ * top-p filtering (the paper samples at T = 1 with top_p = 0.95 and
+ * top_k = 20, Appendix "Evaluation Protocol", and keeps the underlying
+ * verification, which it does not state).  The rule implemented is standard
+ * speculative sampling on the filtered distributions:
+ *   p_i, q_i   softmax(logits / T) of target row i and drafter row i,
+ *              restricted to the top_k logits (the lower index first among
+ *              equal values), renormalised, then to the shortest prefix of
+ *              them whose probability reaches top_p, renormalised;
+ *   accept     draft token x_i iff uniforms[b, i] * q_i(x_i) < p_i(x_i) (a
+ *              token outside [0, V) is rejected); A_b = the first rejection;
+ *   draw       with uniforms[b, K], inverse CDF over the filtered list (in
+ *              descending probability): from max(0, p_A - q_A), renormalised
+ *              (from p_A if it is zero), when A_b < K, else from p_K.
+ * Outputs as in retrace_verify, with the drawn token as committed[b, A_b]
+ * and bonus[b].  Uniforms are the caller's random numbers, in [0, 1).
+ *   target_logits  [B, K+1, V]; draft_logits [B, K, V] (the drafter's logits
+ *                  of the proposals), both `dtype`, V contiguous, strides in
+ *                  elements.
+ *   temperature > 0, 1 <= top_k <= 64 and top_k <= V, 0 < top_p <= 1.
+ * The conditioning of the next block is unchanged: retrace_align_refine and
+ * retrace_gate_fuse take this call's accept_len. */
+retrace_status retrace_verify_sampled(const void* target_logits, int64_t target_row_stride,
+                                      int64_t target_batch_stride, const void* draft_logits,
+                                      int64_t draft_row_stride, int64_t draft_batch_stride,
+                                      retrace_dtype dtype, int B, int K, int V, const int32_t* draft,
+                                      const float* uniforms, float temperature, int top_k, float top_p,
+                                      int32_t* accept_len, int32_t* committed, int32_t* bonus, void* ws,
+                                      size_t ws_bytes, cudaStream_t stream);
+
 /* Ranks of the low-rank conditioning path (Appendix "Concurrent-Serving
  * Experiment": rank-64 rejected-suffix latents, rank-32 correction). */
 #define RETRACE_LOWRANK_LATENT 64

@@ -56,8 +56,10 @@ def _load() -> ctypes.CDLL:
                                   P, P, P, P, P, P, P, SZ, ctypes.c_uint32, P, P]
     lib.retrace_round_lowrank.argtypes = [P, I64, I64, P, P, P, P, P, P, P, P, P, F, I, I, I, I, I,
                                           P, P, P, P, P, P, P, SZ, P, P]
+    lib.retrace_verify_sampled.argtypes = [P, I64, I64, P, I64, I64, I, I, I, I, P, P, F, I, F, P, P, P, P, SZ, P]
     for name in ("retrace_workspace_init", "retrace_workspace_check", "retrace_verify",
-                 "retrace_align_refine", "retrace_gate_fuse", "retrace_round", "retrace_round_lowrank"):
+                 "retrace_align_refine", "retrace_gate_fuse", "retrace_round", "retrace_round_lowrank",
+                 "retrace_verify_sampled"):
         getattr(lib, name).restype = I
     return lib
 
@@ -196,6 +198,26 @@ def retrace_round(logits, draft, hD, hT, e, Wc, Wv, Wg, beta, accept_len, commit
                              ws.nbytes, int(flags),
                              ctypes.cast(ev, ctypes.c_void_p) if ev is not None else None,
                              _stream(stream)))
+
+
+def retrace_verify_sampled(target_logits, draft_logits, draft, uniforms, temperature, top_k, top_p, accept_len,
+                           committed, bonus, ws, stream=None):
+    """Speculative sampling of one block per sequence (see include/retrace.h)."""
+    B, K1, V = target_logits.shape
+    K = K1 - 1
+    if target_logits.stride(2) != 1 or draft_logits.stride(2) != 1:
+        raise ValueError("logits: vocabulary dimension must be contiguous")
+    if tuple(draft_logits.shape) != (B, K, V) or draft_logits.dtype != target_logits.dtype:
+        raise ValueError("draft_logits must be [B, K, V] of the target logits' dtype")
+    if uniforms.dtype != torch.float32 or tuple(uniforms.shape) != (B, K1) or not uniforms.is_contiguous():
+        raise ValueError("uniforms must be contiguous float32 [B, K+1]")
+    for t, name in ((draft, "draft"), (accept_len, "accept_len"), (committed, "committed"), (bonus, "bonus")):
+        _int32(t, name)
+    _check(lib.retrace_verify_sampled(_ptr(target_logits), target_logits.stride(1), target_logits.stride(0),
+                                      _ptr(draft_logits), draft_logits.stride(1), draft_logits.stride(0),
+                                      _dtype_code(target_logits), B, K, V, _ptr(draft), _ptr(uniforms),
+                                      float(temperature), int(top_k), float(top_p), _ptr(accept_len),
+                                      _ptr(committed), _ptr(bonus), ws.ptr, ws.nbytes, _stream(stream)))
 
 
 def retrace_round_lowrank(logits, draft, hD, hT, e, P, Bc, Ac, Wv, Wg, beta, accept_len, committed, bonus,

@@ -20,7 +20,7 @@ ROOT = os.path.dirname(PKG)
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB_PATH = os.path.join(PKG, "libretrace.so")
-SOURCES = ["api.cu", "verify.cu", "cond_simt.cu", "cond_tc.cu", "verify_noalloc.cu", "lowrank.cu"]
+SOURCES = ["api.cu", "verify.cu", "cond_simt.cu", "cond_tc.cu", "verify_noalloc.cu", "lowrank.cu", "verify_sampled.cu"]
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 NVCC_FLAGS = [
     "-O3",

@@ -471,6 +471,53 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   return RETRACE_OK;
 }
 
+retrace_status retrace_verify_sampled(const void* target_logits, int64_t target_row_stride,
+                                      int64_t target_batch_stride, const void* draft_logits,
+                                      int64_t draft_row_stride, int64_t draft_batch_stride,
+                                      retrace_dtype dtype, int B, int K, int V, const int32_t* draft,
+                                      const float* uniforms, float temperature, int top_k, float top_p,
+                                      int32_t* accept_len, int32_t* committed, int32_t* bonus, void* ws,
+                                      size_t ws_bytes, cudaStream_t stream) {
+  g_err[0] = '\0';
+  retrace_status st = check_verify_args(target_logits, dtype, B, K, V, target_row_stride,
+                                        target_batch_stride, draft, accept_len, committed, bonus);
+  if (st != RETRACE_OK) return st;
+  if (K < 1) return fail(RETRACE_ERR_INVALID_ARG, "K must be >= 1");
+  if (B > 0 && (!draft_logits || !uniforms)) return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
+  if (draft_row_stride < V || draft_batch_stride < (int64_t)K * draft_row_stride)
+    return fail(RETRACE_ERR_INVALID_ARG, "draft logits strides (%lld, %lld) below [B, K, V] packing",
+                (long long)draft_row_stride, (long long)draft_batch_stride);
+  if (!(temperature > 0.f) || temperature > 3.0e38f)
+    return fail(RETRACE_ERR_INVALID_ARG, "temperature must be positive and finite");
+  if (top_k < 1 || top_k > kMaxTopK || top_k > V)
+    return fail(RETRACE_ERR_INVALID_ARG, "top_k must be in [1, min(64, V)], got %d", top_k);
+  if (!(top_p > 0.f && top_p <= 1.f)) return fail(RETRACE_ERR_INVALID_ARG, "top_p must be in (0, 1]");
+  if (B == 0) return RETRACE_OK;
+  const WsLayout Lw = ws_layout(B, K, 1, elem_size(dtype));
+  if ((st = check_ws(ws, ws_bytes, Lw.total)) != RETRACE_OK) return st;
+  SampledArgs a{};
+  a.tlogits = target_logits;
+  a.t_row = target_row_stride;
+  a.t_batch = target_batch_stride;
+  a.dlogits = draft_logits;
+  a.d_row = draft_row_stride;
+  a.d_batch = draft_batch_stride;
+  a.B = B;
+  a.K = K;
+  a.V = V;
+  a.draft = draft;
+  a.uniforms = uniforms;
+  a.temperature = temperature;
+  a.top_k = top_k;
+  a.top_p = top_p;
+  a.accept_len = accept_len;
+  a.committed = committed;
+  a.bonus = bonus;
+  a.keys = reinterpret_cast<unsigned long long*>(reinterpret_cast<char*>(ws) + Lw.skeys);
+  RT_CUDA(launch_verify_sampled(a, dtype, stream), "sampled verification launch");
+  return RETRACE_OK;
+}
+
 retrace_status retrace_round_lowrank(const void* logits, int64_t logits_row_stride,
                                      int64_t logits_batch_stride, const int32_t* draft,
                                      const void* hD, const void* hT, const void* e, const void* P,

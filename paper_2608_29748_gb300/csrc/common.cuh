@@ -71,6 +71,11 @@ __device__ __forceinline__ unsigned long long make_key(float v, uint32_t idx) {
 __device__ __forceinline__ uint32_t key_index(unsigned long long key) {
   return 0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull);
 }
+// The value of a key (the inverse of ordered_bits; -0 comes back as +0).
+__device__ __forceinline__ float key_value(unsigned long long key) {
+  const uint32_t o = (uint32_t)(key >> 32);
+  return __uint_as_float((o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o);
+}
 __device__ __forceinline__ unsigned long long umax64(unsigned long long a, unsigned long long b) {
   return a > b ? a : b;
 }

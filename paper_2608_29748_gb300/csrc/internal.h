@@ -31,8 +31,10 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 constexpr int kLowRankLatent = 64;      // rank of the rejected-suffix latents
 constexpr int kLowRankCorrection = 32;  // rank of the target-aware correction
 constexpr int kLowRankSplits = 8;       // split-K parts per half of the [m; u] reduction
+//   skeys    uint64 [B*(2K+1), 64]  sampled verification: top-k keys per target and drafter row
+constexpr int kMaxTopK = 64;            // largest top_k of sampled verification
 struct WsLayout {
-  size_t status, sync, sync_bytes, keys, tickets, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, total;
+  size_t status, sync, sync_bytes, keys, tickets, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, skeys, total;
 };
 
 inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
@@ -66,6 +68,8 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   off = align_up(off + (size_t)kLowRankSplits * rmax * kLowRankCorrection * 4, 256);
   L.lrrho = off;
   off = align_up(off + rmax * kLowRankLatent * elem, 256);
+  L.skeys = off;
+  off = align_up(off + (size_t)(B * (2 * K + 1)) * kMaxTopK * 8, 256);
   L.total = off;
   return L;
 }
@@ -113,6 +117,25 @@ constexpr int kCondCopyKeep = 0;
 constexpr int kCondCopyE = 1;
 constexpr int kCondCopyM = 2;
 cudaError_t launch_verify(const VerifyArgs& a, retrace_dtype dtype, cudaStream_t stream);
+
+// Stochastic verification (speculative sampling on top-k / top-p filtered
+// distributions at temperature T).
+struct SampledArgs {
+  const void* tlogits;  // [B, K+1, V]
+  long long t_row, t_batch;
+  const void* dlogits;  // [B, K, V]
+  long long d_row, d_batch;
+  int B, K, V;
+  const int32_t* draft;
+  const float* uniforms;  // [B, K+1]
+  float temperature, top_p;
+  int top_k;
+  int32_t* accept_len;
+  int32_t* committed;
+  int32_t* bonus;
+  unsigned long long* keys;  // [B (2K+1), kMaxTopK]
+};
+cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cudaStream_t stream);
 
 // ---- conditioning -----------------------------------------------------------
 // Row plan used by every conditioning kernel: sequence b owns n_b rows, where

@@ -1,0 +1,466 @@
+// Stochastic verification of a draft block (speculative sampling) at
+// temperature T with top-k / top-p filtering (Appendix "Evaluation Protocol":
+// T = 1, top_p = 0.95, top_k = 20).  The paper keeps the underlying
+// verification unchanged; the rule implemented is standard speculative
+// sampling on the filtered distributions p (target) and q (drafter):
+// accept x_i iff u_i q_i(x_i) < p_i(x_i); at the first rejection A draw the
+// appended token from max(0, p_A - q_A) (renormalised; p_A if that is zero),
+// else the bonus from p_K; draws are inverse-CDF in the filtered order.
+//
+// Only the top_k logits of a row enter its filtered distribution, so the
+// row's full softmax is never formed:
+//   sampled_topk_kernel      one CTA per row (target rows, then drafter rows):
+//                            elements above a proven lower bound of the row's
+//                            k-th largest (a sample's k-th largest, then the
+//                            best warp's k-th largest candidate) go to per-warp
+//                            buffers; the CTA merges the warps' lists by rank;
+//   sampled_finalize_kernel  one warp per sequence: the filtered
+//                            probabilities from the sorted lists, the accept
+//                            tests in order, and the draw.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace retrace {
+namespace {
+
+constexpr int kThreads = 512;
+constexpr int kWarps = kThreads / 32;
+constexpr int kBuf = 384;  // candidate keys per warp: the compaction trigger (<= 128) + one chunk
+
+struct TopkParams {
+  const void* tlogits;
+  long long t_row, t_batch;
+  const void* dlogits;
+  long long d_row, d_batch;
+  int B, K, V, k;
+  unsigned long long* keys;  // [B (2K+1), kMaxTopK]: target rows b*(K+1)+i, then drafter rows
+};
+
+// The largest key whose value is below v: every element of value >= v beats it.
+__device__ __forceinline__ unsigned long long below_value(float v) {
+  return ((unsigned long long)ordered_bits(v) << 32) - 1ull;
+}
+
+template <typename T>
+struct Chunk;  // one lane's share of a chunk: raw bits, the lane maximum, element values
+template <>
+struct Chunk<__nv_bfloat16> {
+  static constexpr int E = 8;
+  uint4 w;
+  __device__ float lane_max() const {
+    const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&w.x);
+    const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&w.y);
+    const __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&w.z);
+    const __nv_bfloat162 d = *reinterpret_cast<const __nv_bfloat162*>(&w.w);
+    const __nv_bfloat162 m = __hmax2(__hmax2(a, b), __hmax2(c, d));
+    return fmaxf(__low2float(m), __high2float(m));
+  }
+  __device__ float value(int e) const {
+    const uint32_t x = e < 2 ? w.x : e < 4 ? w.y : e < 6 ? w.z : w.w;
+    return (e & 1) ? bf16_hi(x) : bf16_lo(x);
+  }
+  __device__ void load(const __nv_bfloat16* p) { w = __ldcs(reinterpret_cast<const uint4*>(p)); }
+  __device__ void fill() { w = make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u); }  // -inf
+};
+template <>
+struct Chunk<float> {
+  static constexpr int E = 4;
+  float4 w;
+  __device__ float lane_max() const { return fmaxf(fmaxf(w.x, w.y), fmaxf(w.z, w.w)); }
+  __device__ float value(int e) const { return e == 0 ? w.x : e == 1 ? w.y : e == 2 ? w.z : w.w; }
+  __device__ void load(const float* p) { w = __ldcs(reinterpret_cast<const float4*>(p)); }
+  __device__ void fill() { w = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY); }
+};
+
+// Ranks the warp's `n` buffered keys (distinct) and keeps the largest
+// min(n, k) in descending order at the front of the buffer; returns their
+// count.  Lane-parallel rank counting (every key's rank is the number of
+// larger keys); the thresholds keep n small.
+__device__ int warp_compact(unsigned long long* buf, unsigned long long* tmp, int n, int k, int lane) {
+  for (int a = lane; a < n; a += 32) {
+    const unsigned long long x = buf[a];
+    int rank = 0;
+    for (int c = 0; c < n; ++c) rank += buf[c] > x ? 1 : 0;
+    if (rank < k) tmp[rank] = x;
+  }
+  __syncwarp();
+  const int m = n < k ? n : k;
+  for (int a = lane; a < m; a += 32) buf[a] = tmp[a];
+  __syncwarp();
+  return m;
+}
+
+// One CTA per row; warp w scans a contiguous part of it.  Elements are kept
+// as candidates only above a proven lower bound of the row's k-th largest
+// key: first the k-th largest of a sample (the lane maxima of every warp's
+// first chunks: each is an element of the row), then any warp's k-th largest
+// candidate so far (shared through s_thr).  A warp appends its candidates to
+// its buffer with shared-memory atomics and keeps only its top k when the
+// buffer passes a trigger; the row's top k are merged from the warps' lists.
+template <typename T>
+__global__ void __launch_bounds__(kThreads) sampled_topk_kernel(const TopkParams p) {
+  using CT = Chunk<T>;
+  constexpr int E = CT::E;
+  constexpr int U = 4;  // chunks loaded ahead of their processing
+  __shared__ unsigned long long s_buf[kWarps][kBuf];
+  __shared__ unsigned long long s_tmp[kWarps][kMaxTopK];
+  __shared__ float s_sample[kThreads];
+  __shared__ int s_n[kWarps];
+  __shared__ unsigned long long s_thr;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long row = blockIdx.x;
+  const long long nt = (long long)p.B * (p.K + 1);
+  const T* x;
+  if (row < nt) {
+    const long long b = row / (p.K + 1), i = row % (p.K + 1);
+    x = reinterpret_cast<const T*>(p.tlogits) + b * p.t_batch + i * p.t_row;
+  } else {
+    const long long r = row - nt, b = r / p.K, i = r % p.K;
+    x = reinterpret_cast<const T*>(p.dlogits) + b * p.d_batch + i * p.d_row;
+  }
+  const int V = p.V, k = p.k;
+  unsigned long long* buf = s_buf[warp];
+  unsigned long long* tmp = s_tmp[warp];
+  if (lane == 0) s_n[warp] = 0;
+  const unsigned FULL = 0xFFFFFFFFu;
+  const bool vec = (V % E == 0) && ((uintptr_t)x % 16 == 0);
+  const long long per = vec ? E : 1;
+  const long long span = 32 * per;
+  const long long nchunks = (V + span - 1) / span;
+  const long long c0 = nchunks * warp / kWarps, c1 = nchunks * (warp + 1) / kWarps;
+  const int trigger = 2 * k > 64 ? 2 * k : 64;  // <= 128 = kBuf - 32 * 8
+  unsigned long long bound = 0ull;
+
+  auto load = [&](CT& ch, long long c) {
+    const long long base = c * span + lane * per;
+    ch.fill();
+    if (c < c1 && base < V) {
+      if (vec) {
+        ch.load(x + base);
+      } else {
+        Chunk<float> one;
+        one.fill();
+        one.w.x = to_f32(x[base]);
+        if constexpr (sizeof(T) == 4) ch.w = one.w;
+        else ch.w.x = pack_bf16x2(one.w.x, -INFINITY), ch.w.y = ch.w.z = ch.w.w = 0xFF80FF80u;
+      }
+    }
+  };
+  // U consecutive chunks: one vote decides whether any of their elements can
+  // beat the threshold (the common case: none), then chunk by chunk.
+  auto process = [&](const CT (&ch)[U], long long c) {
+    const unsigned long long shared_thr = *(volatile unsigned long long*)&s_thr;
+    const unsigned long long t = bound > shared_thr ? bound : shared_thr;
+    const float tv = t ? key_value(t) : -INFINITY;
+    float gmax = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < U; ++q)
+      if (c + q < c1 && (c + q) * span + lane * per < V) gmax = fmaxf(gmax, ch[q].lane_max());
+    if (!__any_sync(FULL, gmax >= tv)) return;
+#pragma unroll
+    for (int q = 0; q < U; ++q) {
+      const long long base = (c + q) * span + lane * per;
+      if (c + q < c1 && base < V && ch[q].lane_max() >= tv) {
+        for (int e = 0; e < per; ++e) {
+          const float v = ch[q].value(e);
+          if (v >= tv) {
+            const unsigned long long key = make_key(v, (uint32_t)(base + e));
+            if (key > t) buf[atomicAdd(&s_n[warp], 1)] = key;
+          }
+        }
+      }
+      __syncwarp();
+      int n = *(volatile int*)&s_n[warp];
+      if (n > trigger) {  // keep the top k so far (kBuf leaves room for one more chunk)
+        n = warp_compact(buf, tmp, n, k, lane);
+        if (lane == 0) s_n[warp] = n;
+        if (n >= k) {
+          bound = buf[k - 1];
+          if (lane == 0) atomicMax(&s_thr, bound);
+        }
+        __syncwarp();
+      }
+    }
+  };
+
+  // Sampling: the lane maxima of every warp's first U chunks (each an
+  // element of the row); their k-th largest value bounds the row's k-th
+  // largest from below.  A bitonic sort of the 512 maxima finds it.
+  CT first[U];
+#pragma unroll
+  for (int q = 0; q < U; ++q) load(first[q], c0 + q);
+  {
+    float smax = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < U; ++q)
+      if (c0 + q < c1 && (c0 + q) * span + lane * per < V) smax = fmaxf(smax, first[q].lane_max());
+    s_sample[threadIdx.x] = smax;
+    const int i = threadIdx.x;
+    for (int size = 2; size <= kThreads; size <<= 1) {
+      for (int stride = size >> 1; stride > 0; stride >>= 1) {
+        __syncthreads();
+        const int j = i ^ stride;
+        if (j > i) {
+          const float a = s_sample[i], b = s_sample[j];
+          const bool desc = (i & size) == 0;  // the final pass (size = 512) sorts descending
+          if (desc ? a < b : a > b) {
+            s_sample[i] = b;
+            s_sample[j] = a;
+          }
+        }
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      const float vk = s_sample[k - 1];
+      s_thr = vk > -INFINITY ? below_value(vk) : 0ull;
+    }
+    __syncthreads();
+  }
+  process(first, c0);
+  for (long long c = c0 + U; c < c1; c += U) {
+    CT ch[U];
+#pragma unroll
+    for (int q = 0; q < U; ++q) load(ch[q], c + q);
+    process(ch, c);
+  }
+  int n = warp_compact(buf, tmp, *(volatile int*)&s_n[warp], k, lane);
+  if (lane == 0) s_n[warp] = n;
+  __syncthreads();
+  // Merge the warps' sorted lists: lane w of warp 0 holds the head of list w;
+  // the largest head is the next key of the row.
+  if (warp == 0) {
+    unsigned long long* out = p.keys + row * kMaxTopK;
+    int pos = 0;
+    const int len = lane < kWarps ? s_n[lane] : 0;
+    for (int r = 0; r < k; ++r) {
+      const unsigned long long head = pos < len ? s_buf[lane][pos] : 0ull;
+      const unsigned long long best = warp_max_key(head);
+      if (lane == 0) out[r] = best;  // 0 once every list is exhausted (V < k)
+      if (head == best && best != 0ull) ++pos;
+    }
+  }
+}
+
+struct FinalizeParams {
+  const unsigned long long* keys;
+  int B, K, V, k;
+  float inv_T, top_p;
+  const int32_t* draft;
+  const float* uniforms;
+  int32_t* accept_len;
+  int32_t* committed;
+  int32_t* bonus;
+};
+
+// The filtered distribution of one row, lane j holding entries j and 32 + j
+// of the sorted list: weight (0 beyond the top-p cut) and token (-1 if none).
+struct RowDist {
+  float w[2];
+  int tok[2];
+  float total;  // sum of the kept weights
+};
+
+__device__ RowDist row_dist(const FinalizeParams& p, long long row, int lane) {
+  const unsigned FULL = 0xFFFFFFFFu;
+  const unsigned long long* keys = p.keys + row * kMaxTopK;
+  RowDist r;
+  const float v0 = key_value(keys[0]);
+  float w[2];
+  int tok[2];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int j = 32 * h + lane;
+    const unsigned long long key = j < p.k ? keys[j] : 0ull;
+    tok[h] = key ? (int)key_index(key) : -1;
+    w[h] = key ? expf((key_value(key) - v0) * p.inv_T) : 0.f;
+  }
+  // softmax over the top k, then the shortest prefix reaching top_p
+  float z = w[0] + w[1];
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(FULL, z, off);
+  float c0 = w[0];  // inclusive prefix over entries 0..31
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float t = __shfl_up_sync(FULL, c0, off);
+    if (lane >= off) c0 += t;
+  }
+  const float s0 = __shfl_sync(FULL, c0, 31);
+  float c1 = w[1];
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float t = __shfl_up_sync(FULL, c1, off);
+    if (lane >= off) c1 += t;
+  }
+  c1 += s0;
+  // entry j is kept iff the prefix before it is below top_p
+  const float before0 = c0 - w[0], before1 = c1 - w[1];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const float before = h == 0 ? before0 : before1;
+    const bool keep = tok[h] >= 0 && before < p.top_p * z;
+    r.w[h] = keep ? w[h] : 0.f;
+    r.tok[h] = keep ? tok[h] : -1;
+  }
+  float t = r.w[0] + r.w[1];
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) t += __shfl_xor_sync(FULL, t, off);
+  r.total = t;
+  return r;
+}
+
+// Probability of token y under the row distribution (same value on every lane).
+__device__ float dist_prob(const RowDist& r, int y) {
+  const unsigned FULL = 0xFFFFFFFFu;
+  float w = (r.tok[0] == y ? r.w[0] : 0.f) + (r.tok[1] == y ? r.w[1] : 0.f);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) w += __shfl_xor_sync(FULL, w, off);
+  return w / r.total;
+}
+
+// Inverse-CDF draw over entries in list order with weights wt (this lane's
+// two entries): the first entry whose inclusive cumulative weight exceeds
+// u * total; the last kept entry if rounding leaves none.
+__device__ int draw(const RowDist& r, const float wt[2], float u, int lane) {
+  const unsigned FULL = 0xFFFFFFFFu;
+  float c0 = wt[0];
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float t = __shfl_up_sync(FULL, c0, off);
+    if (lane >= off) c0 += t;
+  }
+  const float s0 = __shfl_sync(FULL, c0, 31);
+  float c1 = wt[1];
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float t = __shfl_up_sync(FULL, c1, off);
+    if (lane >= off) c1 += t;
+  }
+  c1 += s0;
+  const float total = __shfl_sync(FULL, c1, 31);
+  const float target = u * total;
+  const unsigned b0 = __ballot_sync(FULL, wt[0] > 0.f && c0 > target);
+  const unsigned b1 = __ballot_sync(FULL, wt[1] > 0.f && c1 > target);
+  int src, h;
+  if (b0) {
+    src = __ffs(b0) - 1;
+    h = 0;
+  } else if (b1) {
+    src = __ffs(b1) - 1;
+    h = 1;
+  } else {  // last entry with weight
+    const unsigned l0 = __ballot_sync(FULL, wt[0] > 0.f), l1 = __ballot_sync(FULL, wt[1] > 0.f);
+    if (l1) {
+      src = 31 - __clz(l1);
+      h = 1;
+    } else {
+      src = 31 - __clz(l0);
+      h = 0;
+    }
+  }
+  const int t0 = __shfl_sync(FULL, r.tok[0], src), t1 = __shfl_sync(FULL, r.tok[1], src);
+  return h == 0 ? t0 : t1;
+}
+
+__global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizeParams p) {
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (b >= p.B) return;
+  const int K = p.K, K1 = K + 1;
+  const long long tbase = (long long)b * K1, dbase = (long long)p.B * K1 + (long long)b * K;
+  const int32_t* dr = p.draft + (long long)b * K;
+  const float* u = p.uniforms + (long long)b * K1;
+  int A = K;
+  for (int i = 0; i < K; ++i) {
+    const int x = dr[i];
+    bool ok = false;
+    if (x >= 0 && x < p.V) {
+      const RowDist pt = row_dist(p, tbase + i, lane);
+      const RowDist qd = row_dist(p, dbase + i, lane);
+      ok = u[i] * dist_prob(qd, x) < dist_prob(pt, x);
+    }
+    if (!ok) {
+      A = i;
+      break;
+    }
+  }
+  const RowDist pt = row_dist(p, tbase + A, lane);
+  int y;
+  if (A < K) {
+    // residual max(0, p - q) over the target's kept tokens
+    const RowDist qd = row_dist(p, dbase + A, lane);
+    float res[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      // q of this lane's token: every lane looks it up in the drafter's list
+      float qw = 0.f;
+      for (int s = 0; s < 32; ++s) {
+        const int t0 = __shfl_sync(0xFFFFFFFFu, qd.tok[0], s), t1 = __shfl_sync(0xFFFFFFFFu, qd.tok[1], s);
+        const float w0 = __shfl_sync(0xFFFFFFFFu, qd.w[0], s), w1 = __shfl_sync(0xFFFFFFFFu, qd.w[1], s);
+        if (pt.tok[h] >= 0 && t0 == pt.tok[h]) qw = w0;
+        if (pt.tok[h] >= 0 && t1 == pt.tok[h]) qw = w1;
+      }
+      res[h] = pt.tok[h] >= 0 ? fmaxf(0.f, pt.w[h] / pt.total - qw / qd.total) : 0.f;
+    }
+    float rs = res[0] + res[1];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) rs += __shfl_xor_sync(0xFFFFFFFFu, rs, off);
+    y = rs > 0.f ? draw(pt, res, u[K], lane) : draw(pt, pt.w, u[K], lane);
+  } else {
+    y = draw(pt, pt.w, u[K], lane);
+  }
+  for (int i = lane; i < K1; i += 32) {
+    const long long o = (long long)b * K1 + i;
+    p.committed[o] = i < A ? dr[i] : (i == A ? y : -1);
+  }
+  if (lane == 0) {
+    p.accept_len[b] = A;
+    p.bonus[b] = y;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cudaStream_t stream) {
+  if (a.B <= 0) return cudaSuccess;
+  TopkParams tp{};
+  tp.tlogits = a.tlogits;
+  tp.t_row = a.t_row;
+  tp.t_batch = a.t_batch;
+  tp.dlogits = a.dlogits;
+  tp.d_row = a.d_row;
+  tp.d_batch = a.d_batch;
+  tp.B = a.B;
+  tp.K = a.K;
+  tp.V = a.V;
+  tp.k = a.top_k;
+  tp.keys = a.keys;
+  const long long rows = (long long)a.B * (2 * a.K + 1);
+  if (dtype == RETRACE_BF16)
+    sampled_topk_kernel<__nv_bfloat16><<<(unsigned)rows, kThreads, 0, stream>>>(tp);
+  else
+    sampled_topk_kernel<float><<<(unsigned)rows, kThreads, 0, stream>>>(tp);
+  cudaError_t err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  FinalizeParams fp{};
+  fp.keys = a.keys;
+  fp.B = a.B;
+  fp.K = a.K;
+  fp.V = a.V;
+  fp.k = a.top_k;
+  fp.inv_T = 1.f / a.temperature;
+  fp.top_p = a.top_p;
+  fp.draft = a.draft;
+  fp.uniforms = a.uniforms;
+  fp.accept_len = a.accept_len;
+  fp.committed = a.committed;
+  fp.bonus = a.bonus;
+  sampled_finalize_kernel<<<(unsigned)((a.B + 7) / 8), 256, 0, stream>>>(fp);
+  return cudaGetLastError();
+}
+
+}  // namespace retrace

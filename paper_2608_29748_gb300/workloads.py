@@ -159,6 +159,31 @@ def make_lowrank_weights(cfg: RoundConfig, device="cpu", seed: int | None = None
     }
 
 
+SAMPLING = {"temperature": 1.0, "top_k": 20, "top_p": 0.95}  # Appendix "Evaluation Protocol", temperature 1
+
+
+def make_sampled_inputs(cfg: RoundConfig, target_logits: torch.Tensor, device="cpu", seed: int | None = None,
+                        draft_noise: float = 0.7) -> dict:
+    """Drafter logits, draft tokens and uniforms for sampled verification of
+    ``target_logits`` [B, K+1, V]: the drafter's logits are the target's plus
+    N(0, (draft_noise * std)^2) noise, each draft token is one of its row's
+    eight largest drafter logits (uniformly), and the uniforms are U[0, 1)."""
+    seed = SEED + 1000 * cfg.seed_offset + 11 if seed is None else seed
+    g = _gen(device, seed)
+    B, K, V = cfg.B, cfg.K, cfg.V
+    dl = torch.empty((B, K, V), dtype=target_logits.dtype, device=device)
+    draft = torch.empty((B, K), dtype=torch.int32, device=device)
+    for b in range(B):  # one sequence at a time bounds the fp32 temporary
+        noise = torch.randn((K, V), generator=g, device=device) * (draft_noise * cfg.logits_std)
+        row = target_logits[b, :K].float() + noise
+        dl[b] = row.to(target_logits.dtype)
+        top8 = torch.topk(dl[b].float(), 8, dim=-1).indices
+        pick = torch.randint(0, 8, (K, 1), generator=g, device=device)
+        draft[b] = torch.gather(top8, 1, pick)[:, 0].to(torch.int32)
+    uniforms = torch.rand((B, K + 1), generator=g, device=device, dtype=torch.float32)
+    return {"draft_logits": dl, "draft": draft, "uniforms": uniforms, **SAMPLING}
+
+
 def xavier_uniform(shape, g, device) -> torch.Tensor:
     """U(-a, a) with a = sqrt(6 / (fan_in + fan_out)) for a [fan_out, fan_in] matrix."""
     fan_out, fan_in = shape
