@@ -135,3 +135,42 @@ def test_round_header_documents_the_flags():
                         ("RETRACE_COND_OVERWRITE", 0x4), ("RETRACE_COND_NONE", 0x8)):
         m = re.search(r"#define\s+%s\s+(0x[0-9a-fA-F]+)u" % name, text)
         assert m and int(m.group(1), 16) == value, name
+
+
+def _sampled(lib, T=1.0, k=20, p=0.95, B=2, K=4, V=100, dl=16, u=16, drs=100, dbs=400):
+    """retrace_verify_sampled with fake pointers; the cases here return
+    before any CUDA call."""
+    P, I64 = ctypes.c_void_p, ctypes.c_int64
+    return lib.retrace_verify_sampled(P(16), I64(V), I64((K + 1) * V), P(dl) if dl else None, I64(drs), I64(dbs),
+                                      BF16, B, K, V, P(16), P(u) if u else None, ctypes.c_float(T), k,
+                                      ctypes.c_float(p), P(16), P(16), P(16), P(256), ctypes.c_size_t(1 << 30), None)
+
+
+def test_sampled_verification_argument_errors(lib):
+    assert _sampled(lib, T=0.0) == INVALID
+    assert _sampled(lib, T=float("inf")) == INVALID
+    assert _sampled(lib, k=0) == INVALID
+    assert _sampled(lib, k=65) == INVALID  # above the supported maximum
+    assert _sampled(lib, k=20, V=10, drs=10, dbs=40) == INVALID  # top_k > V
+    assert _sampled(lib, p=0.0) == INVALID
+    assert _sampled(lib, p=1.5) == INVALID
+    assert _sampled(lib, dl=0) == INVALID
+    assert _sampled(lib, u=0) == INVALID
+    assert _sampled(lib, drs=99) == INVALID  # drafter row stride below V
+    assert _sampled(lib, dbs=399) == INVALID  # drafter batch stride below K * row stride
+    assert _sampled(lib, B=0) == OK
+
+
+def test_lowrank_round_argument_errors(lib):
+    P, I64 = ctypes.c_void_p, ctypes.c_int64
+
+    def call(B=2, P_=16, d=8, K=4):
+        return lib.retrace_round_lowrank(P(16), I64(10), I64(50), P(16), P(16), P(16), P(16), P(P_) if P_ else None,
+                                         P(16), P(16), P(16), P(16), ctypes.c_float(1.0), BF16, B, K, 10, d,
+                                         P(16), P(16), P(16), None, None, P(16), P(256), ctypes.c_size_t(1 << 20),
+                                         None, None)
+
+    assert call(P_=0) == INVALID  # a NULL weight
+    assert call(K=0) == INVALID
+    assert call(d=0) == INVALID
+    assert call(B=0) == OK
