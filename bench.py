@@ -277,7 +277,7 @@ def conditioning_flops(cfg: RoundConfig, R: int, dense_e: bool, variant: str = "
 
 
 LOWRANK_L, LOWRANK_C = 64, 32
-KERNELS_PER_ROUND_SAMPLED = 6  # sampled top-k and finalize; pack + cond_kernel for each conditioning entry point
+KERNELS_PER_ROUND_SAMPLED = 3  # sampled top-k, sampled finalize (copies + packing), cond_kernel
 KERNELS_PER_ROUND_LOWRANK = 4  # verify_kernel, latent projection, finish (+ GEMV), latent fusion (tensor cores)
 
 
@@ -354,26 +354,11 @@ def run_gpu(args) -> dict | None:
         from paper_2608_29748_gb300.workloads import make_sampled_inputs
 
         x.update(make_sampled_inputs(cfg, x["logits"], device=dev, seed=shard_seed(99 + 1000 * cfg.seed_offset, rank)))
-        r_buf = torch.empty((cfg.B, cfg.K, cfg.d), dtype=cfg.torch_dtype, device=dev)
 
-        def round_fn(inputs, phase_events=None):
-            # a temperature-1 round: sampled verification, then the conditioning entry points
-            ev = phase_events or [None] * 4
-            st = torch.cuda.current_stream(dev)
-            if ev[0] is not None:
-                ev[0].record(st)
-            rt.retrace_verify_sampled(inputs["logits"], inputs["draft_logits"], inputs["draft"], inputs["uniforms"],
-                                      x["temperature"], x["top_k"], x["top_p"], out.accept_len, out.committed,
-                                      out.bonus, ws)
-            if ev[1] is not None:
-                ev[1].record(st)
-            rt.retrace_align_refine(inputs["hD"], inputs["hT"], out.accept_len, x["Wc"], x["beta"], r_buf, out.n, ws)
-            if ev[2] is not None:
-                ev[2].record(st)
-            rt.retrace_gate_fuse(x["e"], r_buf, out.n, x["Wv"], x["Wg"], out.e_out, ws)
-            if ev[3] is not None:
-                ev[3].record(st)
-            return out
+        def round_fn(inputs, **kw):
+            # a temperature-1 round: sampled verification, then the corrected, gated conditioning
+            return rt.run_round_sampled(inputs, dict(inputs, temperature=x["temperature"], top_k=x["top_k"],
+                                                     top_p=x["top_p"]), ws, out=out, **kw)
     else:
         def round_fn(inputs, **kw):
             return rt.run_round(inputs, ws, out=out, flags=flags, **kw)
@@ -448,9 +433,8 @@ def run_gpu(args) -> dict | None:
         v_gbs = vbytes / v_avg_s / 1e9
         c_avg_s = statistics.mean(cond_ms) / 1e3
         c_tflops = cflops / c_avg_s / 1e12
-        if args.sampled:  # both logits tensors are read once
-            vbytes = (cfg.B * (2 * cfg.K + 1) * cfg.V * cfg.elem_bytes + cfg.B * (cfg.K + 1) * 4 * 2
-                      + cfg.B * cfg.K * 4 + 3 * cfg.B * 4)
+        if args.sampled:  # the drafter's logits and the uniforms are read too
+            vbytes += cfg.B * cfg.K * cfg.V * cfg.elem_bytes + cfg.B * (cfg.K + 1) * 4
             v_gbs = vbytes / v_avg_s / 1e9
         v_roof = {
             "kernel": "verify_kernel (argmax/compare/commit + copy of unconditioned rows + row packing)",
@@ -471,7 +455,7 @@ def run_gpu(args) -> dict | None:
             v_roof["kernel"] = "verify_kernel (argmax/compare/commit + every row of e~ copied)"
         if args.sampled:
             v_roof["kernel"] = ("sampled_topk_kernel + sampled_finalize_kernel (top-k of every target and drafter "
-                                "row, accept tests, draw)")
+                                "row, accept tests, draw, copy of unconditioned rows + row packing)")
             v_roof["traffic"] = None
         c_roof = None
         if args.lowrank:
@@ -539,6 +523,7 @@ def run_gpu(args) -> dict | None:
                              "(speculative sampling)" if args.sampled else args.variant),
             "round_kernel": ("overlapped (one persistent launch)" if fused
                              else "verify, latent projection, finish + GEMV, latent fusion" if args.lowrank
+                             else "three launches (sampled top-k, sampled finalize, projections)" if args.sampled
                              else "two launches (verify, projections)"),
         },
         "roofline": roofline,
@@ -651,7 +636,7 @@ def parse_args(argv=None):
     ap.add_argument("--overlap", action="store_true",
                     help="time the overlapped single-kernel round (RETRACE_ROUND_OVERLAP)")
     ap.add_argument("--sampled", action="store_true",
-                    help="time a temperature-1 round (retrace_verify_sampled + the conditioning entry points)")
+                    help="time a temperature-1 round (retrace_round_sampled)")
     ap.add_argument("--lowrank", action="store_true",
                     help="time the low-rank conditioning path (retrace_round_lowrank)")
     ap.add_argument("--variant", choices=sorted(VARIANT_FLAGS), default="corrected",

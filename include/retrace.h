@@ -237,7 +237,8 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
  *                  elements.
  *   temperature > 0, 1 <= top_k <= 64 and top_k <= V, 0 < top_p <= 1.
  * The conditioning of the next block is unchanged: retrace_align_refine and
- * retrace_gate_fuse take this call's accept_len. */
+ * retrace_gate_fuse take this call's accept_len (retrace_round_sampled runs
+ * both steps as one round). */
 retrace_status retrace_verify_sampled(const void* target_logits, int64_t target_row_stride,
                                       int64_t target_batch_stride, const void* draft_logits,
                                       int64_t draft_row_stride, int64_t draft_batch_stride,
@@ -245,6 +246,32 @@ retrace_status retrace_verify_sampled(const void* target_logits, int64_t target_
                                       const float* uniforms, float temperature, int top_k, float top_p,
                                       int32_t* accept_len, int32_t* committed, int32_t* bonus, void* ws,
                                       size_t ws_bytes, cudaStream_t stream);
+
+/* One round at temperature T: the stochastic verification of
+ * retrace_verify_sampled, then the corrected, gated conditioning of the
+ * rejected suffix (Eq. 4-8) exactly as retrace_round computes it, with A_b the
+ * sampled accepted length (Algorithm 1 with its acceptance test replaced by
+ * speculative sampling; the paper evaluates at T = 1).  Arguments are those of
+ * retrace_verify_sampled followed by those of retrace_round; there is no
+ * target_argmax output and no flags.  The finalize kernel writes the rows
+ * j >= n_b of e_out and, on the tensor-core path (bf16, d a multiple of 256,
+ * 16-byte aligned tensors), packs the conditioned rows for one persistent
+ * conditioning launch.
+ *   phase_events  optional 4 events: before verification, after it, after the
+ *                 correction (after both projections on the tensor-core
+ *                 path), after the gated fusion.
+ * temperature > 0, 1 <= top_k <= 64 and top_k <= V, 0 < top_p <= 1, K >= 1,
+ * V >= 1, d >= 1. */
+retrace_status retrace_round_sampled(const void* target_logits, int64_t target_row_stride,
+                                     int64_t target_batch_stride, const void* draft_logits,
+                                     int64_t draft_row_stride, int64_t draft_batch_stride,
+                                     const int32_t* draft, const float* uniforms, float temperature,
+                                     int top_k, float top_p, const void* hD, const void* hT, const void* e,
+                                     int64_t e_batch_stride, int64_t e_pos_stride, const void* Wc,
+                                     const void* Wv, const void* Wg, float beta, retrace_dtype dtype, int B,
+                                     int K, int V, int d, int32_t* accept_len, int32_t* committed,
+                                     int32_t* bonus, int32_t* n_out, void* e_out, void* ws, size_t ws_bytes,
+                                     const cudaEvent_t* phase_events, cudaStream_t stream);
 
 /* Ranks of the low-rank conditioning path (Appendix "Concurrent-Serving
  * Experiment": rank-64 rejected-suffix latents, rank-32 correction). */

@@ -57,9 +57,11 @@ def _load() -> ctypes.CDLL:
     lib.retrace_round_lowrank.argtypes = [P, I64, I64, P, P, P, P, P, P, P, P, P, F, I, I, I, I, I,
                                           P, P, P, P, P, P, P, SZ, P, P]
     lib.retrace_verify_sampled.argtypes = [P, I64, I64, P, I64, I64, I, I, I, I, P, P, F, I, F, P, P, P, P, SZ, P]
+    lib.retrace_round_sampled.argtypes = [P, I64, I64, P, I64, I64, P, P, F, I, F, P, P, P, I64, I64, P, P, P, F,
+                                          I, I, I, I, I, P, P, P, P, P, P, SZ, P, P]
     for name in ("retrace_workspace_init", "retrace_workspace_check", "retrace_verify",
                  "retrace_align_refine", "retrace_gate_fuse", "retrace_round", "retrace_round_lowrank",
-                 "retrace_verify_sampled"):
+                 "retrace_verify_sampled", "retrace_round_sampled"):
         getattr(lib, name).restype = I
     return lib
 
@@ -203,6 +205,19 @@ def retrace_round(logits, draft, hD, hT, e, Wc, Wv, Wg, beta, accept_len, commit
 def retrace_verify_sampled(target_logits, draft_logits, draft, uniforms, temperature, top_k, top_p, accept_len,
                            committed, bonus, ws, stream=None):
     """Speculative sampling of one block per sequence (see include/retrace.h)."""
+    _check_sampled(target_logits, draft_logits, uniforms)
+    B, K1, V = target_logits.shape
+    K = K1 - 1
+    for t, name in ((draft, "draft"), (accept_len, "accept_len"), (committed, "committed"), (bonus, "bonus")):
+        _int32(t, name)
+    _check(lib.retrace_verify_sampled(_ptr(target_logits), target_logits.stride(1), target_logits.stride(0),
+                                      _ptr(draft_logits), draft_logits.stride(1), draft_logits.stride(0),
+                                      _dtype_code(target_logits), B, K, V, _ptr(draft), _ptr(uniforms),
+                                      float(temperature), int(top_k), float(top_p), _ptr(accept_len),
+                                      _ptr(committed), _ptr(bonus), ws.ptr, ws.nbytes, _stream(stream)))
+
+
+def _check_sampled(target_logits, draft_logits, uniforms):
     B, K1, V = target_logits.shape
     K = K1 - 1
     if target_logits.stride(2) != 1 or draft_logits.stride(2) != 1:
@@ -211,13 +226,30 @@ def retrace_verify_sampled(target_logits, draft_logits, draft, uniforms, tempera
         raise ValueError("draft_logits must be [B, K, V] of the target logits' dtype")
     if uniforms.dtype != torch.float32 or tuple(uniforms.shape) != (B, K1) or not uniforms.is_contiguous():
         raise ValueError("uniforms must be contiguous float32 [B, K+1]")
+
+
+def retrace_round_sampled(target_logits, draft_logits, draft, uniforms, temperature, top_k, top_p, hD, hT, e, Wc,
+                          Wv, Wg, beta, accept_len, committed, bonus, e_out, ws, n_out=None, phase_events=None,
+                          stream=None):
+    """One round with sampled verification (see include/retrace.h)."""
+    _check_sampled(target_logits, draft_logits, uniforms)
+    B, K1, V = target_logits.shape
+    K = K1 - 1
+    d = hD.shape[2]
     for t, name in ((draft, "draft"), (accept_len, "accept_len"), (committed, "committed"), (bonus, "bonus")):
         _int32(t, name)
-    _check(lib.retrace_verify_sampled(_ptr(target_logits), target_logits.stride(1), target_logits.stride(0),
-                                      _ptr(draft_logits), draft_logits.stride(1), draft_logits.stride(0),
-                                      _dtype_code(target_logits), B, K, V, _ptr(draft), _ptr(uniforms),
-                                      float(temperature), int(top_k), float(top_p), _ptr(accept_len),
-                                      _ptr(committed), _ptr(bonus), ws.ptr, ws.nbytes, _stream(stream)))
+    ebs, eps = _e_strides(e, B, K, d)
+    ev = None
+    if phase_events is not None:
+        ev = (ctypes.c_void_p * 4)(*[x._as_parameter_.value for x in phase_events])
+    _check(lib.retrace_round_sampled(_ptr(target_logits), target_logits.stride(1), target_logits.stride(0),
+                                     _ptr(draft_logits), draft_logits.stride(1), draft_logits.stride(0), _ptr(draft),
+                                     _ptr(uniforms), float(temperature), int(top_k), float(top_p), _ptr(hD), _ptr(hT),
+                                     _ptr(e), ebs, eps, _ptr(Wc), _ptr(Wv), _ptr(Wg), float(beta),
+                                     _dtype_code(target_logits), B, K, V, d, _ptr(accept_len), _ptr(committed),
+                                     _ptr(bonus), _ptr(n_out), _ptr(e_out), ws.ptr, ws.nbytes,
+                                     ctypes.cast(ev, ctypes.c_void_p) if ev is not None else None,
+                                     _stream(stream)))
 
 
 def retrace_round_lowrank(logits, draft, hD, hT, e, P, Bc, Ac, Wv, Wg, beta, accept_len, committed, bonus,
@@ -283,4 +315,21 @@ def run_round_lowrank(x: dict, w: dict, ws: Workspace, out: RoundBuffers | None 
     retrace_round_lowrank(logits, x["draft"], x["hD"], x["hT"], x["e"], w["P"], w["Bc"], w["Ac"], w["Wv_lr"],
                           w["Wg_lr"], x["beta"], out.accept_len, out.committed, out.bonus, out.e_out, ws,
                           n_out=out.n, target_argmax=target_argmax, phase_events=phase_events, stream=stream)
+    return out
+
+
+def run_round_sampled(x: dict, s: dict, ws: Workspace, out: RoundBuffers | None = None, phase_events=None,
+                      stream=None) -> RoundBuffers:
+    """retrace_round_sampled over the round inputs ``x`` (its logits are the
+    target's) and the sampling inputs ``s`` (keys as in
+    workloads.make_sampled_inputs; its draft tokens replace x["draft"])."""
+    logits = x["logits"]
+    B, K1, _ = logits.shape
+    d = x["hD"].shape[2]
+    if out is None:
+        out = RoundBuffers(B, K1 - 1, d, logits.dtype, logits.device)
+    retrace_round_sampled(logits, s["draft_logits"], s["draft"], s["uniforms"], s["temperature"], s["top_k"],
+                          s["top_p"], x["hD"], x["hT"], x["e"], x["Wc"], x["Wv"], x["Wg"], x["beta"], out.accept_len,
+                          out.committed, out.bonus, out.e_out, ws, n_out=out.n, phase_events=phase_events,
+                          stream=stream)
     return out

@@ -134,6 +134,88 @@ retrace_status e_mode(int64_t ebs, int64_t eps, int K, int d, int* dense) {
 
 uint32_t* status_word(void* ws) { return reinterpret_cast<uint32_t*>(ws); }
 
+
+retrace_status check_sampling(int B, int K, int V, const void* draft_logits, int64_t draft_row_stride,
+                              int64_t draft_batch_stride, const float* uniforms, float temperature, int top_k,
+                              float top_p) {
+  if (K < 1) return fail(RETRACE_ERR_INVALID_ARG, "K must be >= 1");
+  if (B > 0 && (!draft_logits || !uniforms)) return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
+  if (draft_row_stride < V || draft_batch_stride < (int64_t)K * draft_row_stride)
+    return fail(RETRACE_ERR_INVALID_ARG, "draft logits strides (%lld, %lld) below [B, K, V] packing",
+                (long long)draft_row_stride, (long long)draft_batch_stride);
+  if (!(temperature > 0.f) || temperature > 3.0e38f)
+    return fail(RETRACE_ERR_INVALID_ARG, "temperature must be positive and finite");
+  if (top_k < 1 || top_k > kMaxTopK || top_k > V)
+    return fail(RETRACE_ERR_INVALID_ARG, "top_k must be in [1, min(64, V)], got %d", top_k);
+  if (!(top_p > 0.f && top_p <= 1.f)) return fail(RETRACE_ERR_INVALID_ARG, "top_p must be in (0, 1]");
+  return RETRACE_OK;
+}
+
+// Tensors of the conditioning step shared by the rounds.
+struct ConditioningArgs {
+  const void* hD;
+  const void* hT;
+  const void* e;
+  int64_t e_batch_stride, e_pos_stride;
+  int e_dense;
+  const void* Wc;
+  const void* Wv;
+  const void* Wg;
+  float beta;
+  void* e_out;
+};
+
+// Correction (Eq. 6-7) and gated fusion (Eq. 8) of the rows j < n_b, after a
+// verification kernel has written accept_len and the unconditioned rows of
+// e_out and, on the tensor-core path, packed the [m; u] rows.  Records
+// phase_events[2] after the correction (after both projections on the
+// tensor-core path, which runs them in one launch).
+retrace_status enqueue_conditioning(const ConditioningArgs& c, retrace_dtype dtype, int B, int K, int d,
+                                    bool tc, bool raw, const int32_t* accept_len, void* ws, const WsLayout& L,
+                                    const cudaEvent_t* phase_events, cudaStream_t stream) {
+  char* w = reinterpret_cast<char*>(ws);
+  float* ge = reinterpret_cast<float*>(w + L.ge);
+  void* r_ws = w + L.r;
+  const RowSource rows{accept_len, 1};
+  if (tc) {
+    uint32_t* sync = reinterpret_cast<uint32_t*>(w + L.sync);
+    TcCondArgs a{};
+    a.B = B;
+    a.K = K;
+    a.d = d;
+    a.do_correct = raw ? 0 : 1;
+    a.do_gate = 1;
+    a.apack = w + L.apack;
+    a.Wc = c.Wc;
+    a.beta = c.beta;
+    a.r_out = r_ws;
+    a.compact_out = 1;
+    // raw: r = m is the first half of each packed [m; u] row
+    a.rpack = raw ? w + L.apack : r_ws;
+    a.r_row_stride = raw ? 2LL * d : 0;
+    a.e = c.e;
+    a.epack = w + L.epack;
+    a.e_dense = c.e_dense;
+    a.Wv = c.Wv;
+    a.Wg = c.Wg;
+    a.ge = ge;
+    a.e_out = c.e_out;
+    a.R = reinterpret_cast<int32_t*>(sync + kSyncRowCount);
+    a.rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
+    a.sync = sync;
+    a.status = status_word(ws);
+    RT_CUDA(launch_cond_tc(a, stream), "conditioning kernel launch");
+    if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
+  } else {
+    CorrectArgs ca{c.hD, c.hT, c.Wc, c.beta, B, K, d, rows, r_ws, 1, raw ? 1 : 0};
+    RT_CUDA(launch_correct_simt(ca, dtype, stream), "correction kernel launch");
+    if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
+    if (!c.e_dense) RT_CUDA(launch_gate_bias(c.Wg, c.e, d, ge, dtype, stream), "gate bias kernel launch");
+    GateArgs ga{c.e, c.e_dense, r_ws, 1, c.Wv, c.Wg, c.e_dense ? nullptr : ge, B, K, d, rows, c.e_out};
+    RT_CUDA(launch_gate_simt(ga, dtype, stream), "gate kernel launch");
+  }
+  return RETRACE_OK;
+}
 }  // namespace
 
 void retrace::set_last_error(const char* msg) { snprintf(g_err, sizeof(g_err), "%s", msg); }
@@ -333,7 +415,6 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   uint32_t* sync = reinterpret_cast<uint32_t*>(w + L.sync);
   int32_t* R = reinterpret_cast<int32_t*>(sync + kSyncRowCount);
   int32_t* rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
-  const RowSource rows{accept_len, 1};
 
   if (phase_events) RT_CUDA(cudaEventRecord(phase_events[0], stream), "cudaEventRecord");
   // The verification kernel packs the conditioned rows as sequences finish;
@@ -427,46 +508,10 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
     }
     return RETRACE_OK;
   }
-  const bool raw = ablation == RETRACE_COND_RAW;
-  if (tc) {
-    // Both projections in one persistent launch; its phase events bracket
-    // the whole conditioning (the correction/gate split point is not a
-    // stream position any more).
-    TcCondArgs a{};
-    a.B = B;
-    a.K = K;
-    a.d = d;
-    a.do_correct = raw ? 0 : 1;
-    a.do_gate = 1;
-    a.apack = w + L.apack;
-    a.Wc = Wc;
-    a.beta = beta;
-    a.r_out = r_ws;
-    a.compact_out = 1;
-    // raw: r = m is the first half of each packed [m; u] row
-    a.rpack = raw ? w + L.apack : r_ws;
-    a.r_row_stride = raw ? 2LL * d : 0;
-    a.e = e;
-    a.epack = w + L.epack;
-    a.e_dense = dense;
-    a.Wv = Wv;
-    a.Wg = Wg;
-    a.ge = ge;
-    a.e_out = e_out;
-    a.R = R;
-    a.rowmap = rowmap;
-    a.sync = sync;
-    a.status = status_word(ws);
-    RT_CUDA(launch_cond_tc(a, stream), "conditioning kernel launch");
-    if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
-  } else {
-    CorrectArgs ca{hD, hT, Wc, beta, B, K, d, rows, r_ws, 1, raw ? 1 : 0};
-    RT_CUDA(launch_correct_simt(ca, dtype, stream), "correction kernel launch");
-    if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
-    if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");
-    GateArgs ga{e, dense, r_ws, 1, Wv, Wg, dense ? nullptr : ge, B, K, d, rows, e_out};
-    RT_CUDA(launch_gate_simt(ga, dtype, stream), "gate kernel launch");
-  }
+  ConditioningArgs c{hD, hT, e, e_batch_stride, e_pos_stride, dense, Wc, Wv, Wg, beta, e_out};
+  if ((st = enqueue_conditioning(c, dtype, B, K, d, tc, ablation == RETRACE_COND_RAW, accept_len, ws, L,
+                                 phase_events, stream)) != RETRACE_OK)
+    return st;
   if (phase_events) RT_CUDA(cudaEventRecord(phase_events[3], stream), "cudaEventRecord");
   return RETRACE_OK;
 }
@@ -482,16 +527,9 @@ retrace_status retrace_verify_sampled(const void* target_logits, int64_t target_
   retrace_status st = check_verify_args(target_logits, dtype, B, K, V, target_row_stride,
                                         target_batch_stride, draft, accept_len, committed, bonus);
   if (st != RETRACE_OK) return st;
-  if (K < 1) return fail(RETRACE_ERR_INVALID_ARG, "K must be >= 1");
-  if (B > 0 && (!draft_logits || !uniforms)) return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
-  if (draft_row_stride < V || draft_batch_stride < (int64_t)K * draft_row_stride)
-    return fail(RETRACE_ERR_INVALID_ARG, "draft logits strides (%lld, %lld) below [B, K, V] packing",
-                (long long)draft_row_stride, (long long)draft_batch_stride);
-  if (!(temperature > 0.f) || temperature > 3.0e38f)
-    return fail(RETRACE_ERR_INVALID_ARG, "temperature must be positive and finite");
-  if (top_k < 1 || top_k > kMaxTopK || top_k > V)
-    return fail(RETRACE_ERR_INVALID_ARG, "top_k must be in [1, min(64, V)], got %d", top_k);
-  if (!(top_p > 0.f && top_p <= 1.f)) return fail(RETRACE_ERR_INVALID_ARG, "top_p must be in (0, 1]");
+  if ((st = check_sampling(B, K, V, draft_logits, draft_row_stride, draft_batch_stride, uniforms, temperature,
+                           top_k, top_p)) != RETRACE_OK)
+    return st;
   if (B == 0) return RETRACE_OK;
   const WsLayout Lw = ws_layout(B, K, 1, elem_size(dtype));
   if ((st = check_ws(ws, ws_bytes, Lw.total)) != RETRACE_OK) return st;
@@ -515,6 +553,82 @@ retrace_status retrace_verify_sampled(const void* target_logits, int64_t target_
   a.bonus = bonus;
   a.keys = reinterpret_cast<unsigned long long*>(reinterpret_cast<char*>(ws) + Lw.skeys);
   RT_CUDA(launch_verify_sampled(a, dtype, stream), "sampled verification launch");
+  return RETRACE_OK;
+}
+
+retrace_status retrace_round_sampled(const void* target_logits, int64_t target_row_stride,
+                                     int64_t target_batch_stride, const void* draft_logits,
+                                     int64_t draft_row_stride, int64_t draft_batch_stride,
+                                     const int32_t* draft, const float* uniforms, float temperature,
+                                     int top_k, float top_p, const void* hD, const void* hT, const void* e,
+                                     int64_t e_batch_stride, int64_t e_pos_stride, const void* Wc,
+                                     const void* Wv, const void* Wg, float beta, retrace_dtype dtype, int B,
+                                     int K, int V, int d, int32_t* accept_len, int32_t* committed,
+                                     int32_t* bonus, int32_t* n_out, void* e_out, void* ws, size_t ws_bytes,
+                                     const cudaEvent_t* phase_events, cudaStream_t stream) {
+  g_err[0] = '\0';
+  retrace_status st = check_verify_args(target_logits, dtype, B, K, V, target_row_stride,
+                                        target_batch_stride, draft, accept_len, committed, bonus);
+  if (st != RETRACE_OK) return st;
+  if ((st = check_sampling(B, K, V, draft_logits, draft_row_stride, draft_batch_stride, uniforms, temperature,
+                           top_k, top_p)) != RETRACE_OK)
+    return st;
+  if ((st = check_cond_shape(dtype, B, K, d)) != RETRACE_OK) return st;
+  if (B == 0) return RETRACE_OK;
+  if (!hD || !hT || !e || !e_out || !Wc || !Wv || !Wg) return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
+  int dense = 0;
+  if ((st = e_mode(e_batch_stride, e_pos_stride, K, d, &dense)) != RETRACE_OK) return st;
+  const WsLayout L = ws_layout(B, K, d, elem_size(dtype));
+  if ((st = check_ws(ws, ws_bytes, L.total)) != RETRACE_OK) return st;
+  char* w = reinterpret_cast<char*>(ws);
+  const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) && aligned16(Wv) &&
+                  aligned16(Wg) && aligned16(e) && aligned16(e_out);
+  uint32_t* sync = reinterpret_cast<uint32_t*>(w + L.sync);
+
+  if (phase_events) RT_CUDA(cudaEventRecord(phase_events[0], stream), "cudaEventRecord");
+  // the finalize kernel packs the conditioned rows behind a counter at zero
+  if (tc) RT_CUDA(cudaMemsetAsync(sync, 0, L.sync_bytes, stream), "cudaMemsetAsync(sync)");
+  SampledArgs a{};
+  a.tlogits = target_logits;
+  a.t_row = target_row_stride;
+  a.t_batch = target_batch_stride;
+  a.dlogits = draft_logits;
+  a.d_row = draft_row_stride;
+  a.d_batch = draft_batch_stride;
+  a.B = B;
+  a.K = K;
+  a.V = V;
+  a.draft = draft;
+  a.uniforms = uniforms;
+  a.temperature = temperature;
+  a.top_k = top_k;
+  a.top_p = top_p;
+  a.accept_len = accept_len;
+  a.committed = committed;
+  a.bonus = bonus;
+  a.keys = reinterpret_cast<unsigned long long*>(w + L.skeys);
+  a.n_out = n_out;
+  a.e = e;
+  a.e_batch_stride = e_batch_stride;
+  a.e_pos_stride = e_pos_stride;
+  a.e_out = e_out;
+  a.d = d;
+  if (tc) {
+    a.hD = hD;
+    a.hT = hT;
+    a.e_dense = dense;
+    a.apack = w + L.apack;
+    a.epack = w + L.epack;
+    a.rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
+    a.R_count = reinterpret_cast<int32_t*>(sync + kSyncRowCount);
+  }
+  RT_CUDA(launch_verify_sampled(a, dtype, stream), "sampled verification launch");
+  if (phase_events) RT_CUDA(cudaEventRecord(phase_events[1], stream), "cudaEventRecord");
+  ConditioningArgs c{hD, hT, e, e_batch_stride, e_pos_stride, dense, Wc, Wv, Wg, beta, e_out};
+  if ((st = enqueue_conditioning(c, dtype, B, K, d, tc, false, accept_len, ws, L, phase_events, stream)) !=
+      RETRACE_OK)
+    return st;
+  if (phase_events) RT_CUDA(cudaEventRecord(phase_events[3], stream), "cudaEventRecord");
   return RETRACE_OK;
 }
 

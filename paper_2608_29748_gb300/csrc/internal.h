@@ -134,6 +134,21 @@ struct SampledArgs {
   int32_t* committed;
   int32_t* bonus;
   unsigned long long* keys;  // [B (2K+1), kMaxTopK]
+  // a whole round (optional, e_out != NULL): n, the unconditioned rows of e~
+  // copied from e (rows a multiple of 16 bytes, 16-byte aligned), and with
+  // R_count the packed rows of the tensor-core projections
+  int32_t* n_out;
+  const void* e;
+  long long e_batch_stride, e_pos_stride;  // elements
+  void* e_out;
+  int d;
+  const void* hD;
+  const void* hT;
+  int e_dense;
+  void* apack;
+  void* epack;
+  int32_t* rowmap;
+  int32_t* R_count;
 };
 cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cudaStream_t stream);
 

@@ -255,6 +255,20 @@ struct FinalizeParams {
   int32_t* accept_len;
   int32_t* committed;
   int32_t* bonus;
+  // a whole round (optional): n, copies of the unconditioned rows of e~, and
+  // the packed [m; u] rows of the tensor-core projections
+  int32_t* n_out;
+  const void* e;
+  long long e_batch_stride, e_pos_stride;
+  void* e_out;
+  int d, elem;
+  const void* hD;
+  const void* hT;
+  int e_dense;
+  void* apack;
+  void* epack;
+  int32_t* rowmap;
+  int32_t* R_count;
 };
 
 // The filtered distribution of one row, lane j holding entries j and 32 + j
@@ -366,60 +380,128 @@ __device__ int draw(const RowDist& r, const float wt[2], float u, int lane) {
   return h == 0 ? t0 : t1;
 }
 
+// One CTA per sequence: warp 0 takes the accept decisions and the draw; then
+// every thread writes the outputs and, for a round, copies and packs rows.
 __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizeParams p) {
-  const int lane = threadIdx.x & 31;
-  const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
-  if (b >= p.B) return;
+  __shared__ int s_A, s_y, s_off;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int b = blockIdx.x;
   const int K = p.K, K1 = K + 1;
-  const long long tbase = (long long)b * K1, dbase = (long long)p.B * K1 + (long long)b * K;
   const int32_t* dr = p.draft + (long long)b * K;
-  const float* u = p.uniforms + (long long)b * K1;
-  int A = K;
-  for (int i = 0; i < K; ++i) {
-    const int x = dr[i];
-    bool ok = false;
-    if (x >= 0 && x < p.V) {
-      const RowDist pt = row_dist(p, tbase + i, lane);
-      const RowDist qd = row_dist(p, dbase + i, lane);
-      ok = u[i] * dist_prob(qd, x) < dist_prob(pt, x);
-    }
-    if (!ok) {
-      A = i;
-      break;
-    }
-  }
-  const RowDist pt = row_dist(p, tbase + A, lane);
-  int y;
-  if (A < K) {
-    // residual max(0, p - q) over the target's kept tokens
-    const RowDist qd = row_dist(p, dbase + A, lane);
-    float res[2];
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      // q of this lane's token: every lane looks it up in the drafter's list
-      float qw = 0.f;
-      for (int s = 0; s < 32; ++s) {
-        const int t0 = __shfl_sync(0xFFFFFFFFu, qd.tok[0], s), t1 = __shfl_sync(0xFFFFFFFFu, qd.tok[1], s);
-        const float w0 = __shfl_sync(0xFFFFFFFFu, qd.w[0], s), w1 = __shfl_sync(0xFFFFFFFFu, qd.w[1], s);
-        if (pt.tok[h] >= 0 && t0 == pt.tok[h]) qw = w0;
-        if (pt.tok[h] >= 0 && t1 == pt.tok[h]) qw = w1;
+  if (warp == 0) {
+    const long long tbase = (long long)b * K1, dbase = (long long)p.B * K1 + (long long)b * K;
+    const float* u = p.uniforms + (long long)b * K1;
+    int A = K;
+    for (int i = 0; i < K; ++i) {
+      const int x = dr[i];
+      bool ok = false;
+      if (x >= 0 && x < p.V) {
+        const RowDist pt = row_dist(p, tbase + i, lane);
+        const RowDist qd = row_dist(p, dbase + i, lane);
+        ok = u[i] * dist_prob(qd, x) < dist_prob(pt, x);
       }
-      res[h] = pt.tok[h] >= 0 ? fmaxf(0.f, pt.w[h] / pt.total - qw / qd.total) : 0.f;
+      if (!ok) {
+        A = i;
+        break;
+      }
     }
-    float rs = res[0] + res[1];
+    const RowDist pt = row_dist(p, tbase + A, lane);
+    int y;
+    if (A < K) {
+      // residual max(0, p - q) over the target's kept tokens
+      const RowDist qd = row_dist(p, dbase + A, lane);
+      float res[2];
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) rs += __shfl_xor_sync(0xFFFFFFFFu, rs, off);
-    y = rs > 0.f ? draw(pt, res, u[K], lane) : draw(pt, pt.w, u[K], lane);
-  } else {
-    y = draw(pt, pt.w, u[K], lane);
+      for (int h = 0; h < 2; ++h) {
+        // q of this lane's token: every lane looks it up in the drafter's list
+        float qw = 0.f;
+        for (int s2 = 0; s2 < 32; ++s2) {
+          const int t0 = __shfl_sync(0xFFFFFFFFu, qd.tok[0], s2), t1 = __shfl_sync(0xFFFFFFFFu, qd.tok[1], s2);
+          const float w0 = __shfl_sync(0xFFFFFFFFu, qd.w[0], s2), w1 = __shfl_sync(0xFFFFFFFFu, qd.w[1], s2);
+          if (pt.tok[h] >= 0 && t0 == pt.tok[h]) qw = w0;
+          if (pt.tok[h] >= 0 && t1 == pt.tok[h]) qw = w1;
+        }
+        res[h] = pt.tok[h] >= 0 ? fmaxf(0.f, pt.w[h] / pt.total - qw / qd.total) : 0.f;
+      }
+      float rs = res[0] + res[1];
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) rs += __shfl_xor_sync(0xFFFFFFFFu, rs, off);
+      y = rs > 0.f ? draw(pt, res, u[K], lane) : draw(pt, pt.w, u[K], lane);
+    } else {
+      y = draw(pt, pt.w, u[K], lane);
+    }
+    if (lane == 0) {
+      s_A = A;
+      s_y = y;
+      const int nb = K - 1 - A > 0 ? K - 1 - A : 0;
+      s_off = (p.R_count && nb > 0) ? atomicAdd(p.R_count, nb) : 0;
+    }
   }
-  for (int i = lane; i < K1; i += 32) {
+  __syncthreads();
+  const int A = s_A, y = s_y;
+  for (int i = threadIdx.x; i < K1; i += blockDim.x) {
     const long long o = (long long)b * K1 + i;
     p.committed[o] = i < A ? dr[i] : (i == A ? y : -1);
   }
-  if (lane == 0) {
+  const int nb = K - 1 - A > 0 ? K - 1 - A : 0;
+  if (threadIdx.x == 0) {
     p.accept_len[b] = A;
     p.bonus[b] = y;
+    if (p.n_out) p.n_out[b] = nb;
+  }
+  if (!p.e_out) return;
+  // rows j >= n_b keep the drafter input, bit for bit
+  const long long base_row = (long long)b * K;
+  const char* e_b = static_cast<const char*>(p.e) + b * p.e_batch_stride * p.elem;
+  const long long rows = K - nb;
+  const bool vec = (p.d * p.elem) % 16 == 0 && (uintptr_t)e_b % 16 == 0 && (uintptr_t)p.e_out % 16 == 0 &&
+                   (p.e_pos_stride * p.elem) % 16 == 0;
+  if (vec) {
+    const int vpr = p.d * p.elem / 16;
+    const long long pos_vec = p.e_pos_stride * p.elem / 16;
+    const uint4* src = reinterpret_cast<const uint4*>(e_b);
+    uint4* dst = reinterpret_cast<uint4*>(p.e_out) + (base_row + nb) * vpr;
+    for (long long i = threadIdx.x; i < rows * vpr; i += blockDim.x) {
+      const long long j = nb + i / vpr, c = i % vpr;
+      dst[i] = __ldg(src + j * pos_vec + c);
+    }
+  } else if (p.elem == 2) {
+    const uint16_t* src = reinterpret_cast<const uint16_t*>(e_b);
+    uint16_t* dst = reinterpret_cast<uint16_t*>(p.e_out) + (base_row + nb) * p.d;
+    for (long long i = threadIdx.x; i < rows * p.d; i += blockDim.x) {
+      const long long j = nb + i / p.d, c = i % p.d;
+      dst[i] = src[j * p.e_pos_stride + c];
+    }
+  } else {
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(e_b);
+    uint32_t* dst = reinterpret_cast<uint32_t*>(p.e_out) + (base_row + nb) * p.d;
+    for (long long i = threadIdx.x; i < rows * p.d; i += blockDim.x) {
+      const long long j = nb + i / p.d, c = i % p.d;
+      dst[i] = src[j * p.e_pos_stride + c];
+    }
+  }
+  if (!p.R_count || nb == 0) return;
+  // packed rows [m_j; u_j] = [hD[b, A+1+j]; hT[b, A+j]] (Eq. 4-5), and e[b, j]
+  // for a per-position e; the tensor-core path is bf16 with 16-byte rows
+  const int off = s_off;
+  const int vpr = p.d / 8;
+  const uint4* e_v = reinterpret_cast<const uint4*>(e_b);
+  const long long pos_vec = p.e_pos_stride / 8;
+  for (int j = threadIdx.x; j < nb; j += blockDim.x) p.rowmap[off + j] = b * K + j;
+  const uint4* hD = reinterpret_cast<const uint4*>(p.hD);
+  const uint4* hT = reinterpret_cast<const uint4*>(p.hT);
+  uint4* ap = reinterpret_cast<uint4*>(p.apack);
+  for (long long i = threadIdx.x; i < (long long)nb * 2 * vpr; i += blockDim.x) {
+    const long long j = i / (2 * vpr), c = i % (2 * vpr);
+    ap[(off + j) * 2 * vpr + c] = c < vpr ? __ldg(hD + (base_row + A + 1 + j) * vpr + c)
+                                          : __ldg(hT + (base_row + A + j) * vpr + c - vpr);
+  }
+  if (p.e_dense) {
+    uint4* ep = reinterpret_cast<uint4*>(p.epack);
+    for (long long i = threadIdx.x; i < (long long)nb * vpr; i += blockDim.x) {
+      const long long j = i / vpr, c = i % vpr;
+      ep[(off + j) * vpr + c] = __ldg(e_v + j * pos_vec + c);
+    }
   }
 }
 
@@ -459,7 +541,21 @@ cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cud
   fp.accept_len = a.accept_len;
   fp.committed = a.committed;
   fp.bonus = a.bonus;
-  sampled_finalize_kernel<<<(unsigned)((a.B + 7) / 8), 256, 0, stream>>>(fp);
+  fp.n_out = a.n_out;
+  fp.e = a.e;
+  fp.e_batch_stride = a.e_batch_stride;
+  fp.e_pos_stride = a.e_pos_stride;
+  fp.e_out = a.e_out;
+  fp.d = a.d;
+  fp.elem = dtype == RETRACE_BF16 ? 2 : 4;
+  fp.hD = a.hD;
+  fp.hT = a.hT;
+  fp.e_dense = a.e_dense;
+  fp.apack = a.apack;
+  fp.epack = a.epack;
+  fp.rowmap = a.rowmap;
+  fp.R_count = a.R_count;
+  sampled_finalize_kernel<<<(unsigned)a.B, 256, 0, stream>>>(fp);
   return cudaGetLastError();
 }
 

@@ -161,6 +161,27 @@ def test_sampled_verification_argument_errors(lib):
     assert _sampled(lib, B=0) == OK
 
 
+def test_sampled_round_argument_errors(lib):
+    P, I64, F = ctypes.c_void_p, ctypes.c_int64, ctypes.c_float
+
+    def call(B=2, K=4, V=100, d=8, T=1.0, k=20, Wc=16, u=16, ebs=0, eps=0, ws_bytes=1 << 30):
+        return lib.retrace_round_sampled(P(16), I64(V), I64((K + 1) * V), P(16), I64(V), I64(K * V), P(16),
+                                         P(u) if u else None, F(T), k, F(0.95), P(16), P(16), P(16), I64(ebs),
+                                         I64(eps), P(Wc) if Wc else None, P(16), P(16), F(1.0), BF16, B, K, V, d,
+                                         P(16), P(16), P(16), None, P(16), P(256), ctypes.c_size_t(ws_bytes), None,
+                                         None)
+
+    assert call(Wc=0) == INVALID  # a NULL weight
+    assert call(u=0) == INVALID
+    assert call(T=-1.0) == INVALID
+    assert call(k=65) == INVALID
+    assert call(K=0) == INVALID
+    assert call(d=0) == INVALID
+    assert call(ebs=7, eps=3) == UNSUPPORTED  # e neither broadcast nor dense
+    assert call(ws_bytes=64) == WORKSPACE  # workspace too small
+    assert call(B=0) == OK
+
+
 def test_lowrank_round_argument_errors(lib):
     P, I64 = ctypes.c_void_p, ctypes.c_int64
 
