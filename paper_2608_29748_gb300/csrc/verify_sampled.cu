@@ -46,18 +46,32 @@ __device__ __forceinline__ unsigned long long below_value(float v) {
 }
 
 template <typename T>
-struct Chunk;  // one lane's share of a chunk: raw bits, the lane maximum, element values
+struct Chunk;  // one lane's share of a chunk (16 bytes): raw bits, partial maxima, candidate masks
 template <>
 struct Chunk<__nv_bfloat16> {
   static constexpr int E = 8;
+  using Part = __nv_bfloat162;  // two running maxima
   uint4 w;
-  __device__ float lane_max() const {
+  __device__ Part part() const {
     const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&w.x);
     const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&w.y);
     const __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&w.z);
     const __nv_bfloat162 d = *reinterpret_cast<const __nv_bfloat162*>(&w.w);
-    const __nv_bfloat162 m = __hmax2(__hmax2(a, b), __hmax2(c, d));
-    return fmaxf(__low2float(m), __high2float(m));
+    return __hmax2(__hmax2(a, b), __hmax2(c, d));
+  }
+  static __device__ Part combine(Part a, Part b) { return __hmax2(a, b); }
+  static __device__ float finish(Part m) { return fmaxf(__low2float(m), __high2float(m)); }
+  static __device__ Part lowest() { return __floats2bfloat162_rn(-INFINITY, -INFINITY); }
+  // bit e set iff element e >= tv
+  __device__ unsigned mask(float tv) const {
+    const uint32_t q[4] = {w.x, w.y, w.z, w.w};
+    unsigned m = 0;
+#pragma unroll
+    for (int h = 0; h < 4; ++h) {
+      m |= (bf16_lo(q[h]) >= tv ? 1u : 0u) << (2 * h);
+      m |= (bf16_hi(q[h]) >= tv ? 1u : 0u) << (2 * h + 1);
+    }
+    return m;
   }
   __device__ float value(int e) const {
     const uint32_t x = e < 2 ? w.x : e < 4 ? w.y : e < 6 ? w.z : w.w;
@@ -65,15 +79,24 @@ struct Chunk<__nv_bfloat16> {
   }
   __device__ void load(const __nv_bfloat16* p) { w = __ldcs(reinterpret_cast<const uint4*>(p)); }
   __device__ void fill() { w = make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u); }  // -inf
+  __device__ void set_single(float v) { w = make_uint4(pack_bf16x2(v, -INFINITY), 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u); }
 };
 template <>
 struct Chunk<float> {
   static constexpr int E = 4;
+  using Part = float;
   float4 w;
-  __device__ float lane_max() const { return fmaxf(fmaxf(w.x, w.y), fmaxf(w.z, w.w)); }
+  __device__ Part part() const { return fmaxf(fmaxf(w.x, w.y), fmaxf(w.z, w.w)); }
+  static __device__ Part combine(Part a, Part b) { return fmaxf(a, b); }
+  static __device__ float finish(Part m) { return m; }
+  static __device__ Part lowest() { return -INFINITY; }
+  __device__ unsigned mask(float tv) const {
+    return (w.x >= tv ? 1u : 0u) | (w.y >= tv ? 2u : 0u) | (w.z >= tv ? 4u : 0u) | (w.w >= tv ? 8u : 0u);
+  }
   __device__ float value(int e) const { return e == 0 ? w.x : e == 1 ? w.y : e == 2 ? w.z : w.w; }
   __device__ void load(const float* p) { w = __ldcs(reinterpret_cast<const float4*>(p)); }
   __device__ void fill() { w = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY); }
+  __device__ void set_single(float v) { w = make_float4(v, -INFINITY, -INFINITY, -INFINITY); }
 };
 
 // Ranks the warp's `n` buffered keys (distinct) and keeps the largest
@@ -94,18 +117,23 @@ __device__ int warp_compact(unsigned long long* buf, unsigned long long* tmp, in
   return m;
 }
 
-// One CTA per row; warp w scans a contiguous part of it.  Elements are kept
-// as candidates only above a proven lower bound of the row's k-th largest
-// key: first the k-th largest of a sample (the lane maxima of every warp's
-// first chunks: each is an element of the row), then any warp's k-th largest
-// candidate so far (shared through s_thr).  A warp appends its candidates to
-// its buffer with shared-memory atomics and keeps only its top k when the
-// buffer passes a trigger; the row's top k are merged from the warps' lists.
+// One CTA per row; warp w scans a contiguous part of it, U chunks (16 bytes
+// per lane each) per step.  Elements are kept as candidates only above a
+// proven lower bound of the row's k-th largest key: first the k-th largest
+// of a sample (every lane's maximum over its first U chunks: each is an
+// element of the row), then any warp's k-th largest candidate so far (shared
+// through s_thr).  One vote per step on the packed maxima decides whether
+// any element can pass (the common case: none); otherwise a ballot per chunk
+// skips the chunks without one, and the lanes that have some append them, by
+// bit mask, to the warp's buffer with shared-memory atomics.  A buffer that
+// passes a trigger is cut to its top k.  The row's top k are merged from the
+// warps' sorted lists.
 template <typename T>
-__global__ void __launch_bounds__(kThreads) sampled_topk_kernel(const TopkParams p) {
+__global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkParams p) {
   using CT = Chunk<T>;
+  using Part = typename CT::Part;
   constexpr int E = CT::E;
-  constexpr int U = 4;  // chunks loaded ahead of their processing
+  constexpr int U = 4;
   __shared__ unsigned long long s_buf[kWarps][kBuf];
   __shared__ unsigned long long s_tmp[kWarps][kMaxTopK];
   __shared__ float s_sample[kThreads];
@@ -128,50 +156,41 @@ __global__ void __launch_bounds__(kThreads) sampled_topk_kernel(const TopkParams
   if (lane == 0) s_n[warp] = 0;
   const unsigned FULL = 0xFFFFFFFFu;
   const bool vec = (V % E == 0) && ((uintptr_t)x % 16 == 0);
-  const long long per = vec ? E : 1;
-  const long long span = 32 * per;
-  const long long nchunks = (V + span - 1) / span;
-  const long long c0 = nchunks * warp / kWarps, c1 = nchunks * (warp + 1) / kWarps;
+  const int per = vec ? E : 1;  // elements of the row per lane per chunk
+  const int span = 32 * per;
+  const int nchunks = (V + span - 1) / span;
+  const int c0 = (int)((long long)nchunks * warp / kWarps), c1 = (int)((long long)nchunks * (warp + 1) / kWarps);
   const int trigger = 2 * k > 64 ? 2 * k : 64;  // <= 128 = kBuf - 32 * 8
+  const unsigned valid_bits = vec ? (1u << E) - 1u : 1u;  // the scalar path fills elements 1.. with -inf
   unsigned long long bound = 0ull;
 
-  auto load = [&](CT& ch, long long c) {
-    const long long base = c * span + lane * per;
+  // chunk c of this lane: valid iff c < c1 and its first element is in the row
+  auto load = [&](CT& ch, int c) {
+    const int base = c * span + lane * per;
     ch.fill();
     if (c < c1 && base < V) {
-      if (vec) {
-        ch.load(x + base);
-      } else {
-        Chunk<float> one;
-        one.fill();
-        one.w.x = to_f32(x[base]);
-        if constexpr (sizeof(T) == 4) ch.w = one.w;
-        else ch.w.x = pack_bf16x2(one.w.x, -INFINITY), ch.w.y = ch.w.z = ch.w.w = 0xFF80FF80u;
-      }
+      if (vec) ch.load(x + base);
+      else ch.set_single(to_f32(x[base]));
     }
   };
-  // U consecutive chunks: one vote decides whether any of their elements can
-  // beat the threshold (the common case: none), then chunk by chunk.
-  auto process = [&](const CT (&ch)[U], long long c) {
+  auto process = [&](const CT (&ch)[U], int c) {
     const unsigned long long shared_thr = *(volatile unsigned long long*)&s_thr;
     const unsigned long long t = bound > shared_thr ? bound : shared_thr;
     const float tv = t ? key_value(t) : -INFINITY;
-    float gmax = -INFINITY;
+    Part m = ch[0].part();
 #pragma unroll
-    for (int q = 0; q < U; ++q)
-      if (c + q < c1 && (c + q) * span + lane * per < V) gmax = fmaxf(gmax, ch[q].lane_max());
-    if (!__any_sync(FULL, gmax >= tv)) return;
+    for (int q = 1; q < U; ++q) m = CT::combine(m, ch[q].part());
+    // invalid chunks hold -inf; they can pass only with no bound at all
+    if (!__any_sync(FULL, CT::finish(m) >= tv)) return;
 #pragma unroll
     for (int q = 0; q < U; ++q) {
-      const long long base = (c + q) * span + lane * per;
-      if (c + q < c1 && base < V && ch[q].lane_max() >= tv) {
-        for (int e = 0; e < per; ++e) {
-          const float v = ch[q].value(e);
-          if (v >= tv) {
-            const unsigned long long key = make_key(v, (uint32_t)(base + e));
-            if (key > t) buf[atomicAdd(&s_n[warp], 1)] = key;
-          }
-        }
+      const int base = (c + q) * span + lane * per;
+      const unsigned bits = (c + q < c1 && base < V) ? ch[q].mask(tv) & valid_bits : 0u;
+      if (!__ballot_sync(FULL, bits != 0u)) continue;
+      for (unsigned r = bits; r; r &= r - 1) {
+        const int e = __ffs(r) - 1;
+        const unsigned long long key = make_key(ch[q].value(e), (uint32_t)(base + e));
+        if (key > t) buf[atomicAdd(&s_n[warp], 1)] = key;
       }
       __syncwarp();
       int n = *(volatile int*)&s_n[warp];
@@ -187,43 +206,50 @@ __global__ void __launch_bounds__(kThreads) sampled_topk_kernel(const TopkParams
     }
   };
 
-  // Sampling: the lane maxima of every warp's first U chunks (each an
-  // element of the row); their k-th largest value bounds the row's k-th
-  // largest from below.  A bitonic sort of the 512 maxima finds it.
-  CT first[U];
+  CT ch[U];
 #pragma unroll
-  for (int q = 0; q < U; ++q) load(first[q], c0 + q);
+  for (int q = 0; q < U; ++q) load(ch[q], c0 + q);
   {
-    float smax = -INFINITY;
+    // Sampling: each lane's maximum over its first U chunks, sorted within
+    // the warp (bitonic, by shuffles); warp 0 merges the 16 sorted lists up
+    // to the k-th largest, a lower bound of the row's k-th largest.
+    Part m = ch[0].part();
 #pragma unroll
-    for (int q = 0; q < U; ++q)
-      if (c0 + q < c1 && (c0 + q) * span + lane * per < V) smax = fmaxf(smax, first[q].lane_max());
-    s_sample[threadIdx.x] = smax;
-    const int i = threadIdx.x;
-    for (int size = 2; size <= kThreads; size <<= 1) {
+    for (int q = 1; q < U; ++q) m = CT::combine(m, ch[q].part());
+    float v = CT::finish(m);
+    if (v != v) v = -INFINITY;  // all-NaN lane: no sample
+#pragma unroll
+    for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
       for (int stride = size >> 1; stride > 0; stride >>= 1) {
-        __syncthreads();
-        const int j = i ^ stride;
-        if (j > i) {
-          const float a = s_sample[i], b = s_sample[j];
-          const bool desc = (i & size) == 0;  // the final pass (size = 512) sorts descending
-          if (desc ? a < b : a > b) {
-            s_sample[i] = b;
-            s_sample[j] = a;
-          }
-        }
+        const float o = __shfl_xor_sync(FULL, v, stride);
+        const bool keep_max = ((lane & size) == 0) == ((lane & stride) == 0);  // descending at size 32
+        v = keep_max ? fmaxf(v, o) : fminf(v, o);
       }
     }
+    s_sample[threadIdx.x] = v;
+    if (threadIdx.x == 0) s_thr = 0ull;
     __syncthreads();
-    if (threadIdx.x == 0) {
-      const float vk = s_sample[k - 1];
-      s_thr = vk > -INFINITY ? below_value(vk) : 0ull;
+    if (warp == 0) {
+      int pos = 0;
+      float head = lane < kWarps ? s_sample[lane * 32] : -INFINITY;
+      float best = -INFINITY;
+      for (int r = 0; r < k; ++r) {
+        best = head;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) best = fmaxf(best, __shfl_xor_sync(FULL, best, off));
+        const unsigned own = __ballot_sync(FULL, head == best);
+        if (lane == __ffs(own) - 1) {
+          ++pos;
+          head = pos < 32 ? s_sample[lane * 32 + pos] : -INFINITY;
+        }
+      }
+      if (lane == 0) s_thr = best > -INFINITY ? below_value(best) : 0ull;
     }
     __syncthreads();
   }
-  process(first, c0);
-  for (long long c = c0 + U; c < c1; c += U) {
-    CT ch[U];
+  process(ch, c0);
+  for (int c = c0 + U; c < c1; c += U) {
 #pragma unroll
     for (int q = 0; q < U; ++q) load(ch[q], c + q);
     process(ch, c);
