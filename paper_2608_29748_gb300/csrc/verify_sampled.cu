@@ -121,8 +121,8 @@ __device__ int warp_compact(unsigned long long* buf, unsigned long long* tmp, in
 // per lane each) per step.  Elements are kept as candidates only above a
 // proven lower bound of the row's k-th largest key: first the k-th largest
 // of a sample (every lane's maximum over its first U chunks: each is an
-// element of the row), then any warp's k-th largest candidate so far (shared
-// through s_thr).  One vote per step on the packed maxima decides whether
+// element of the row), then any warp's k-th largest candidate so far (the
+// maximum of both in s_thr).  One vote per step on the packed maxima decides whether
 // any element can pass (the common case: none); otherwise a ballot per chunk
 // skips the chunks without one, and the lanes that have some append them, by
 // bit mask, to the warp's buffer with shared-memory atomics.  A buffer that
@@ -162,20 +162,30 @@ __global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkPar
   const int c0 = (int)((long long)nchunks * warp / kWarps), c1 = (int)((long long)nchunks * (warp + 1) / kWarps);
   const int trigger = 2 * k > 64 ? 2 * k : 64;  // <= 128 = kBuf - 32 * 8
   const unsigned valid_bits = vec ? (1u << E) - 1u : 1u;  // the scalar path fills elements 1.. with -inf
-  unsigned long long bound = 0ull;
 
   // chunk c of this lane: valid iff c < c1 and its first element is in the row
-  auto load = [&](CT& ch, int c) {
-    const int base = c * span + lane * per;
-    ch.fill();
-    if (c < c1 && base < V) {
-      if (vec) ch.load(x + base);
-      else ch.set_single(to_f32(x[base]));
+  auto load_checked = [&](CT (&ch)[U], int c) {
+#pragma unroll
+    for (int q = 0; q < U; ++q) {
+      const int base = (c + q) * span + lane * per;
+      ch[q].fill();
+      if (c + q < c1 && base < V) {
+        if (vec) ch[q].load(x + base);
+        else ch[q].set_single(to_f32(x[base]));
+      }
     }
   };
-  auto process = [&](const CT (&ch)[U], int c) {
-    const unsigned long long shared_thr = *(volatile unsigned long long*)&s_thr;
-    const unsigned long long t = bound > shared_thr ? bound : shared_thr;
+  // U chunks that lie inside the row and the warp's range (the main loop)
+  auto load_full = [&](CT (&ch)[U], int c) {
+    const T* ptr = x + c * span + lane * per;
+#pragma unroll
+    for (int q = 0; q < U; ++q) {
+      if (vec) ch[q].load(ptr + q * span);
+      else ch[q].set_single(to_f32(ptr[q * span]));
+    }
+  };
+  auto process = [&](const CT (&ch)[U], int c, bool full) {
+    const unsigned long long t = *(volatile unsigned long long*)&s_thr;
     const float tv = t ? key_value(t) : -INFINITY;
     Part m = ch[0].part();
 #pragma unroll
@@ -185,8 +195,9 @@ __global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkPar
 #pragma unroll
     for (int q = 0; q < U; ++q) {
       const int base = (c + q) * span + lane * per;
-      const unsigned bits = (c + q < c1 && base < V) ? ch[q].mask(tv) & valid_bits : 0u;
-      if (!__ballot_sync(FULL, bits != 0u)) continue;
+      const bool has = CT::finish(ch[q].part()) >= tv && (full || (c + q < c1 && base < V));
+      if (!__ballot_sync(FULL, has)) continue;
+      const unsigned bits = has ? ch[q].mask(tv) & valid_bits : 0u;
       for (unsigned r = bits; r; r &= r - 1) {
         const int e = __ffs(r) - 1;
         const unsigned long long key = make_key(ch[q].value(e), (uint32_t)(base + e));
@@ -197,18 +208,14 @@ __global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkPar
       if (n > trigger) {  // keep the top k so far (kBuf leaves room for one more chunk)
         n = warp_compact(buf, tmp, n, k, lane);
         if (lane == 0) s_n[warp] = n;
-        if (n >= k) {
-          bound = buf[k - 1];
-          if (lane == 0) atomicMax(&s_thr, bound);
-        }
+        if (n >= k && lane == 0) atomicMax(&s_thr, buf[k - 1]);
         __syncwarp();
       }
     }
   };
 
   CT ch[U];
-#pragma unroll
-  for (int q = 0; q < U; ++q) load(ch[q], c0 + q);
+  load_checked(ch, c0);
   {
     // Sampling: each lane's maximum over its first U chunks, sorted within
     // the warp (bitonic, by shuffles); warp 0 merges the 16 sorted lists up
@@ -248,11 +255,17 @@ __global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkPar
     }
     __syncthreads();
   }
-  process(ch, c0);
-  for (int c = c0 + U; c < c1; c += U) {
-#pragma unroll
-    for (int q = 0; q < U; ++q) load(ch[q], c + q);
-    process(ch, c);
+  process(ch, c0, false);
+  // chunks [0, nfull) lie wholly inside the row
+  const int cfull = c1 < V / span ? c1 : V / span;
+  int c = c0 + U;
+  for (; c + U <= cfull; c += U) {
+    load_full(ch, c);
+    process(ch, c, true);
+  }
+  for (; c < c1; c += U) {
+    load_checked(ch, c);
+    process(ch, c, false);
   }
   int n = warp_compact(buf, tmp, *(volatile int*)&s_n[warp], k, lane);
   if (lane == 0) s_n[warp] = n;
