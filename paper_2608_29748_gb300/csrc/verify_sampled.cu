@@ -140,14 +140,14 @@ __global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkPar
   __shared__ int s_n[kWarps];
   __shared__ unsigned long long s_thr;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long row = blockIdx.x;
-  const long long nt = (long long)p.B * (p.K + 1);
+  const int row = blockIdx.x;  // B (2K+1) rows: a grid dimension, below 2^31
+  const int nt = p.B * (p.K + 1);
   const T* x;
   if (row < nt) {
-    const long long b = row / (p.K + 1), i = row % (p.K + 1);
+    const int b = row / (p.K + 1), i = row - b * (p.K + 1);
     x = reinterpret_cast<const T*>(p.tlogits) + b * p.t_batch + i * p.t_row;
   } else {
-    const long long r = row - nt, b = r / p.K, i = r % p.K;
+    const int r = row - nt, b = r / p.K, i = r - b * p.K;
     x = reinterpret_cast<const T*>(p.dlogits) + b * p.d_batch + i * p.d_row;
   }
   const int V = p.V, k = p.k;
@@ -273,7 +273,7 @@ __global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkPar
   // Merge the warps' sorted lists: lane w of warp 0 holds the head of list w;
   // the largest head is the next key of the row.
   if (warp == 0) {
-    unsigned long long* out = p.keys + row * kMaxTopK;
+    unsigned long long* out = p.keys + (long long)row * kMaxTopK;
     int pos = 0;
     const int len = lane < kWarps ? s_n[lane] : 0;
     for (int r = 0; r < k; ++r) {
