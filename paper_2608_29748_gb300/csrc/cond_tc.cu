@@ -226,6 +226,73 @@ __device__ void gate_bias_rows(const CondParams& p, int d, int lane, uint32_t* n
   }
 }
 
+// Correction epilogue of one tile row (Eq. 7): r = m + beta * c for the 256
+// accumulator columns n0.., m = the first d columns of the packed row g.
+__device__ __forceinline__ void epilogue_correction(const CondParams& p, uint32_t taddr, int g, bool valid, int n0,
+                                                    int d) {
+  const __nv_bfloat16* mrow = p.apack + (long long)g * 2 * d;
+  const long long orow = valid ? (p.compact_out ? g : __ldcg(p.rowmap + g)) : 0;
+  for (int cc = 0; cc < 8; ++cc) {
+    float c[32];
+    tmem_ld_32cols(taddr + (uint32_t)(cc * 32), c);
+    if (valid) {
+      const int n = n0 + cc * 32;
+      const uint4* mv = reinterpret_cast<const uint4*>(mrow + n);
+      uint4* ov = reinterpret_cast<uint4*>(p.r_out + orow * d + n);
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        const uint4 mw = __ldcg(mv + v);
+        const uint32_t mwords[4] = {mw.x, mw.y, mw.z, mw.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          const float lo = bf16_lo(mwords[w]) + p.beta * c[v * 8 + 2 * w];
+          const float hi = bf16_hi(mwords[w]) + p.beta * c[v * 8 + 2 * w + 1];
+          o[w] = pack_bf16x2(lo, hi);
+        }
+        ov[v] = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+    }
+  }
+}
+
+// Gated-fusion epilogue of one tile row (Eq. 8): e~ = e + v * sigmoid(g) for
+// the 128 features n0.., v in accumulator columns 0..127, the r half of the
+// gate in 128..255 (plus W_g[:, :d] e from ge for a broadcast e).
+__device__ __forceinline__ void epilogue_gate(const CondParams& p, uint32_t taddr, int g, bool valid, int n0, int d) {
+  const long long orow = valid ? __ldcg(p.rowmap + g) : 0;
+  const __nv_bfloat16* erow = p.e + (p.e_dense ? (long long)g * d : 0);
+  for (int cc = 0; cc < 4; ++cc) {
+    float v[32], gt[32];
+    tmem_ld_32cols(taddr + (uint32_t)(cc * 32), v);
+    tmem_ld_32cols(taddr + 128u + (uint32_t)(cc * 32), gt);
+    if (valid) {
+      const int n = n0 + cc * 32;
+      const uint4* ev = reinterpret_cast<const uint4*>(erow + n);
+      uint4* ov = reinterpret_cast<uint4*>(p.e_out + orow * d + n);
+#pragma unroll
+      for (int x = 0; x < 4; ++x) {
+        const uint4 ew = __ldcg(ev + x);
+        const uint32_t ewords[4] = {ew.x, ew.y, ew.z, ew.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          const int c0 = x * 8 + 2 * w;
+          float g0 = gt[c0], g1 = gt[c0 + 1];
+          if (!p.e_dense) {
+            g0 += __ldcg(p.ge + n + c0);
+            g1 += __ldcg(p.ge + n + c0 + 1);
+          }
+          const float s0 = 1.f / (1.f + expf(-g0));
+          const float s1 = 1.f / (1.f + expf(-g1));
+          o[w] = pack_bf16x2(bf16_lo(ewords[w]) + v[c0] * s0, bf16_hi(ewords[w]) + v[c0 + 1] * s1);
+        }
+        ov[x] = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+    }
+  }
+}
+
 // Tile t < T0: correction tile (row block t / nt0, 256 output columns t % nt0);
 // T0 <= t < T0 + T1: gate tile (row block (t-T0) / nt1, 128 features).  Tiles
 // are handed out in this order by a global counter, so every gate tile's row
@@ -559,31 +626,7 @@ __global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
       const bool valid = FUSED ? q < tile_rows : g < R;
       const uint32_t taddr = tmem + acc * ACC_COLS + lane_base;
       if (corr) {
-        // r = m + beta * c   (Eq. 7), m = first d columns of the packed row
-        const __nv_bfloat16* mrow = p.apack + (long long)g * 2 * d;
-        const long long orow = valid ? (p.compact_out ? g : __ldcg(p.rowmap + g)) : 0;
-        for (int cc = 0; cc < 8; ++cc) {
-          float c[32];
-          tmem_ld_32cols(taddr + (uint32_t)(cc * 32), c);
-          if (valid) {
-            const int n = n0 + cc * 32;
-            const uint4* mv = reinterpret_cast<const uint4*>(mrow + n);
-            uint4* ov = reinterpret_cast<uint4*>(p.r_out + orow * d + n);
-#pragma unroll
-            for (int v = 0; v < 4; ++v) {
-              const uint4 mw = __ldcg(mv + v);
-              const uint32_t mwords[4] = {mw.x, mw.y, mw.z, mw.w};
-              uint32_t o[4];
-#pragma unroll
-              for (int w = 0; w < 4; ++w) {
-                const float lo = bf16_lo(mwords[w]) + p.beta * c[v * 8 + 2 * w];
-                const float hi = bf16_hi(mwords[w]) + p.beta * c[v * 8 + 2 * w + 1];
-                o[w] = pack_bf16x2(lo, hi);
-              }
-              ov[v] = make_uint4(o[0], o[1], o[2], o[3]);
-            }
-          }
-        }
+        epilogue_correction(p, taddr, g, valid, n0, d);
         if (p.do_gate) {
           // Publish this warp's 32 rows of the (row block, column block) of r
           // to the gate tiles: one count per epilogue warp, no wait.
@@ -593,38 +636,7 @@ __global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
           if (lane == 0) atomicAdd(block_done + m0 / BM, 1u);
         }
       } else {
-        // e~ = e + v * sigmoid(g)   (Eq. 8)
-        const long long orow = valid ? __ldcg(p.rowmap + g) : 0;
-        const __nv_bfloat16* erow = p.e + (p.e_dense ? (long long)g * d : 0);
-        for (int cc = 0; cc < 4; ++cc) {
-          float v[32], gt[32];
-          tmem_ld_32cols(taddr + (uint32_t)(cc * 32), v);
-          tmem_ld_32cols(taddr + 128u + (uint32_t)(cc * 32), gt);
-          if (valid) {
-            const int n = n0 + cc * 32;
-            const uint4* ev = reinterpret_cast<const uint4*>(erow + n);
-            uint4* ov = reinterpret_cast<uint4*>(p.e_out + orow * d + n);
-#pragma unroll
-            for (int x = 0; x < 4; ++x) {
-              const uint4 ew = __ldcg(ev + x);
-              const uint32_t ewords[4] = {ew.x, ew.y, ew.z, ew.w};
-              uint32_t o[4];
-#pragma unroll
-              for (int w = 0; w < 4; ++w) {
-                const int c0 = x * 8 + 2 * w;
-                float g0 = gt[c0], g1 = gt[c0 + 1];
-                if (!p.e_dense) {
-                  g0 += __ldcg(p.ge + n + c0);
-                  g1 += __ldcg(p.ge + n + c0 + 1);
-                }
-                const float s0 = 1.f / (1.f + expf(-g0));
-                const float s1 = 1.f / (1.f + expf(-g1));
-                o[w] = pack_bf16x2(bf16_lo(ewords[w]) + v[c0] * s0, bf16_hi(ewords[w]) + v[c0 + 1] * s1);
-              }
-              ov[x] = make_uint4(o[0], o[1], o[2], o[3]);
-            }
-          }
-        }
+        epilogue_gate(p, taddr, g, valid, n0, d);
       }
       tc_fence_before();
       __syncwarp();
@@ -637,6 +649,384 @@ __global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
   if (warp == 2) {
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// CTA-pair projections: tcgen05.mma.cta_group::2, M = 256 over two SMs
+// ---------------------------------------------------------------------------
+// The same tiles as cond_kernel<false> with twice the rows: a cluster of two
+// CTAs takes a 256-row pair tile, each CTA staging its own 128 rows of A and
+// half of the N = 256 weight tile (correction: W_c rows n0.. and n0+128..;
+// gate: the W_v rows in the leader, the matching W_g[:, d:2d] rows in the
+// follower), so a stage is 32 KB per SM instead of 48 KB and six stages fit.
+// The leader's MMA thread issues M256 N256 K16 MMAs that read both CTAs'
+// shared memory and accumulate into both CTAs' tensor memory (each CTA's
+// TMEM lanes are its own 128 rows); its commits arrive on both CTAs'
+// barriers (multicast).  Stage-full barriers live in the leader and count the
+// bytes of both CTAs' copies.  The leader takes tiles from the global queue
+// and hands each to the follower through the follower's shared memory.  A
+// broadcast e only (per-position e takes cond_kernel).  Every wait is bounded.
+constexpr int PSTAGES = 6;
+constexpr int P_THREADS = 256;
+constexpr int P_A_BYTES = BM * BK * 2;   // 16 KB: this CTA's 128 rows
+constexpr int P_B_BYTES = 128 * BK * 2;  // 16 KB: this CTA's half of the weight tile
+constexpr int P_STAGE_BYTES = P_A_BYTES + P_B_BYTES;
+constexpr int P_SMEM_BYTES = PSTAGES * P_STAGE_BYTES + 1024;  // + slack for 1024-B alignment
+constexpr uint32_t IDESC_M256_N256 = idesc_bf16_f32(256, 256);
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// The shared::cluster address of `addr` (this CTA's shared memory) in CTA `rank`.
+__device__ __forceinline__ uint32_t map_rank(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+__device__ __forceinline__ void st_remote_u32(uint32_t cluster_addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cluster_addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_acq_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// mbar_wait_bounded for a barrier that the peer CTA arrives on.
+__device__ __forceinline__ bool mbar_wait_cluster_bounded(uint32_t bar, uint32_t parity, volatile int* abort) {
+  unsigned long long t0 = 0ull;
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait_acq_cluster(bar, parity)) return true;
+    if ((it & 255u) == 0u) {
+      if (*abort) return false;
+      const unsigned long long now = global_ns();
+      if (t0 == 0ull)
+        t0 = now;
+      else if (now - t0 > kWaitLimitNs)
+        return false;
+    }
+  }
+}
+__device__ __forceinline__ bool warp_wait_cluster(uint32_t bar, uint32_t parity, volatile int* abort) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait_cluster_bounded(bar, parity, abort) ? 1 : 0;
+  ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+  __syncwarp();
+  return ok != 0;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t slot_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(slot_smem), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_mma_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive once on the barrier at `bar` in both CTAs of the pair when the MMAs
+// issued so far complete.
+__device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "h"((uint16_t)0x3)
+      : "memory");
+}
+// A 2D tile load into this CTA's shared memory that completes on a barrier
+// of either CTA of the pair (`bar` a shared::cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(map), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+__global__ void __launch_bounds__(P_THREADS, 1)
+    cond_pair_kernel(const __grid_constant__ CUtensorMap tmApack, const __grid_constant__ CUtensorMap tmWc,
+                     const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmWv,
+                     const __grid_constant__ CUtensorMap tmWg, const CondParams p) {
+  extern __shared__ uint8_t dsmem[];
+  __shared__ __align__(8) uint64_t bar_full[PSTAGES];           // leader: both CTAs' bytes of a stage
+  __shared__ __align__(8) uint64_t bar_empty[PSTAGES];          // stage free (leader's commit, both CTAs)
+  __shared__ __align__(8) uint64_t bar_tfull[2];                // accumulator ready (both CTAs)
+  __shared__ __align__(8) uint64_t bar_tempty[2];               // leader: eight epilogue warps done
+  __shared__ __align__(8) uint64_t bar_tile_full[TILE_SLOTS];   // tile index published (both CTAs)
+  __shared__ __align__(8) uint64_t bar_tile_empty[TILE_SLOTS];  // leader: ten readers done
+  __shared__ int s_tile[TILE_SLOTS];
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t rank = cluster_rank();
+  const bool leader = rank == 0;
+  const int d = p.d;
+  const int nt0 = d / 256, nt1 = d / 128;
+  const int R = *(volatile const int32_t*)p.R;
+  const int pairs_m = (R + 2 * BM - 1) / (2 * BM);
+  const int T0 = p.do_correct ? pairs_m * nt0 : 0;
+  const int T = T0 + (p.do_gate ? pairs_m * nt1 : 0);
+  if (T == 0) return;  // both CTAs read the same R
+  uint32_t* tile_queue = p.sync + kSyncTileQueue;
+  uint32_t* gemv_next = p.sync + kSyncGemvNext;
+  uint32_t* gemv_done = p.sync + kSyncGemvDone;
+  uint32_t* block_done = p.block_done;
+  const bool need_ge = p.do_gate;  // broadcast e
+
+  if (tid == 0) {
+    s_abort = 0;
+    for (int s = 0; s < PSTAGES; ++s) {
+      mbar_init(smem_u32(&bar_full[s]), 1);  // the leader's expect_tx
+      mbar_init(smem_u32(&bar_empty[s]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(smem_u32(&bar_tfull[a]), 1);
+      mbar_init(smem_u32(&bar_tempty[a]), 8);  // four epilogue warps in each CTA
+    }
+    for (int a = 0; a < TILE_SLOTS; ++a) {
+      mbar_init(smem_u32(&bar_tile_full[a]), 1);
+      mbar_init(smem_u32(&bar_tile_empty[a]), 10);  // MMA + 4 epilogue warps; producer + 4 epilogue warps
+    }
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    if (p.do_correct) {
+      tma_prefetch_desc(&tmApack);
+      tma_prefetch_desc(&tmWc);
+    }
+    if (p.do_gate) {
+      tma_prefetch_desc(&tmR);
+      tma_prefetch_desc(&tmWv);
+      tma_prefetch_desc(&tmWg);
+    }
+  }
+  if (warp == 2) {
+    tmem_alloc_pair(smem_u32(&s_tmem), TMEM_COLS);  // one warp of each CTA of the pair
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // both CTAs' barriers initialised before any remote arrive
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+  const uint32_t base = (smem_u32(dsmem) + 1023u) & ~1023u;
+  const int kb_half = d / BK;
+  // the leader's barriers as seen from either CTA
+  auto leader_addr = [&](const void* local) { return map_rank(smem_u32(local), 0); };
+
+  if (warp == 0) {
+    // ---------------- tile hand-off + TMA producer (both CTAs) ----------------
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (uint32_t lt = 0;; ++lt) {
+        const uint32_t slot = lt % TILE_SLOTS, sph = (lt / TILE_SLOTS) & 1u;
+        int t;
+        if (leader) {
+          t = (int)atomicAdd(tile_queue, 1u);
+          if (t >= T) t = -1;
+          if (!mbar_wait_cluster_bounded(smem_u32(&bar_tile_empty[slot]), sph ^ 1u, &s_abort)) {
+            ok = false;
+            break;
+          }
+          s_tile[slot] = t;
+          st_remote_u32(map_rank(smem_u32(&s_tile[slot]), 1), (uint32_t)t);
+          mbar_arrive(smem_u32(&bar_tile_full[slot]));
+          mbar_arrive_remote(map_rank(smem_u32(&bar_tile_full[slot]), 1));  // release orders the store
+        } else {
+          if (!mbar_wait_cluster_bounded(smem_u32(&bar_tile_full[slot]), sph, &s_abort)) {
+            ok = false;
+            break;
+          }
+          t = s_tile[slot];
+          mbar_arrive_remote(leader_addr(&bar_tile_empty[slot]));
+        }
+        if (t < 0) break;
+        const bool corr = t < T0;
+        const int tt = corr ? t : t - T0;
+        const int m0 = (corr ? tt / nt0 : tt / nt1) * 2 * BM + (int)rank * BM;  // this CTA's rows
+        const int n0 = corr ? (tt % nt0) * 256 : (tt % nt1) * 128;
+        const int nkb = corr ? 2 * kb_half : kb_half;
+        if (!corr && p.do_correct) {
+          // the r rows of this CTA's block are written by the correction epilogues
+          if (!wait_counter(block_done + m0 / BM, (uint32_t)(4 * nt0), &s_abort)) {
+            ok = false;
+            break;
+          }
+          fence_proxy_async_global();
+        }
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const uint32_t s = it % PSTAGES, ph = (it / PSTAGES) & 1u;
+          if (!mbar_wait_bounded(smem_u32(&bar_empty[s]), ph ^ 1u, &s_abort)) {
+            ok = false;
+            break;
+          }
+          const uint32_t a_dst = base + s * P_STAGE_BYTES, b_dst = a_dst + P_A_BYTES;
+          const uint32_t full = leader_addr(&bar_full[s]);
+          if (leader) mbar_arrive_expect_tx(smem_u32(&bar_full[s]), 2 * P_STAGE_BYTES);  // both CTAs' bytes
+          if (corr) {
+            tma_load_2d_pair(a_dst, &tmApack, kb * BK, m0, full);                   // [m; u] rows
+            tma_load_2d_pair(b_dst, &tmWc, kb * BK, n0 + (int)rank * 128, full);    // W_c rows
+          } else {
+            tma_load_2d_pair(a_dst, &tmR, kb * BK, m0, full);  // r rows
+            if (leader)
+              tma_load_2d_pair(b_dst, &tmWv, kb * BK, n0, full);  // W_v rows: accumulator columns 0..127
+            else
+              tma_load_2d_pair(b_dst, &tmWg, d + kb * BK, n0, full);  // W_g[:, d:2d] rows: columns 128..255
+          }
+        }
+        if (!ok) break;
+      }
+      if (!ok) {
+        raise_abort(&s_abort, p.status);
+        if (leader) {
+          volatile int never = 0;  // wait for the copies in flight into the pair's stages
+          const uint32_t first = it > PSTAGES ? it - PSTAGES : 0;
+          for (uint32_t k = first; k < it; ++k)
+            mbar_wait_bounded(smem_u32(&bar_full[k % PSTAGES]), (k / PSTAGES) & 1u, &never);
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---------------- MMA issuer (leader) ----------------
+    if (leader && lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (uint32_t lt = 0;; ++lt) {
+        const uint32_t slot = lt % TILE_SLOTS, sph = (lt / TILE_SLOTS) & 1u;
+        if (!mbar_wait_bounded(smem_u32(&bar_tile_full[slot]), sph, &s_abort)) {
+          ok = false;
+          break;
+        }
+        const int t = s_tile[slot];
+        mbar_arrive(smem_u32(&bar_tile_empty[slot]));
+        if (t < 0) break;
+        const int nkb = t < T0 ? 2 * kb_half : kb_half;
+        const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
+        if (!mbar_wait_cluster_bounded(smem_u32(&bar_tempty[acc]), aph ^ 1u, &s_abort)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem + acc * ACC_COLS;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const uint32_t s = it % PSTAGES, ph = (it / PSTAGES) & 1u;
+          if (!mbar_wait_bounded(smem_u32(&bar_full[s]), ph, &s_abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_base = base + s * P_STAGE_BYTES, b_base = a_base + P_A_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint64_t adesc = sw128_kmajor_desc(a_base + (uint32_t)k * 32u);
+            const uint64_t bdesc = sw128_kmajor_desc(b_base + (uint32_t)k * 32u);
+            tc_mma_pair(d_tmem, adesc, bdesc, IDESC_M256_N256, (kb > 0 || k > 0) ? 1u : 0u);
+          }
+          tc_commit_pair(smem_u32(&bar_empty[s]));
+        }
+        tc_commit_pair(smem_u32(&bar_tfull[acc]));  // accumulator ready (also after a failure)
+        if (!ok) break;
+      }
+      if (!ok) raise_abort(&s_abort, p.status);
+    }
+    __syncwarp();
+  } else if (warp == 2 || warp == 3) {
+    // ---------------- W_g[:, :d] e for the broadcast e (idle warps) ----------------
+    if (need_ge) gate_bias_rows(p, d, lane, gemv_next, gemv_done);
+  } else {
+    // ---------------- epilogue (warps 4-7 of both CTAs) ----------------
+    const int q = (warp - 4) * 32 + lane;  // tile row = TMEM lane
+    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    bool have_ge = !need_ge;
+    for (uint32_t lt = 0;; ++lt) {
+      const uint32_t slot = lt % TILE_SLOTS, sph = (lt / TILE_SLOTS) & 1u;
+      bool ok = warp_wait_cluster(smem_u32(&bar_tile_full[slot]), sph, &s_abort);
+      if (!ok) {
+        if (lane == 0) raise_abort(&s_abort, p.status);
+        break;
+      }
+      const int t = s_tile[slot];
+      __syncwarp();
+      if (lane == 0) {
+        if (leader) mbar_arrive(smem_u32(&bar_tile_empty[slot]));
+        else mbar_arrive_remote(leader_addr(&bar_tile_empty[slot]));
+      }
+      if (t < 0) break;
+      const bool corr = t < T0;
+      const int tt = corr ? t : t - T0;
+      const int m0 = (corr ? tt / nt0 : tt / nt1) * 2 * BM + (int)rank * BM;
+      const int n0 = corr ? (tt % nt0) * 256 : (tt % nt1) * 128;
+      const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
+      ok = warp_wait(smem_u32(&bar_tfull[acc]), aph, &s_abort);
+      tc_fence_after();
+      if (!ok) {
+        if (lane == 0) raise_abort(&s_abort, p.status);
+        break;
+      }
+      if (s_abort) break;
+      if (!corr && !have_ge) {
+        int got = 1;
+        if (lane == 0) got = wait_counter(gemv_done, (uint32_t)d, &s_abort) ? 1 : 0;
+        got = __shfl_sync(0xFFFFFFFFu, got, 0);
+        if (!got) {
+          if (lane == 0) raise_abort(&s_abort, p.status);
+          break;
+        }
+        have_ge = true;
+      }
+      const int g = m0 + q;
+      const bool valid = g < R;
+      const uint32_t taddr = tmem + acc * ACC_COLS + lane_base;
+      if (corr) {
+        epilogue_correction(p, taddr, g, valid, n0, d);
+        if (p.do_gate) {
+          __threadfence();
+          fence_proxy_async_global();
+          __syncwarp();
+          if (lane == 0) atomicAdd(block_done + m0 / BM, 1u);
+        }
+      } else {
+        epilogue_gate(p, taddr, g, valid, n0, d);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (leader) mbar_arrive(smem_u32(&bar_tempty[acc]));
+        else mbar_arrive_remote(leader_addr(&bar_tempty[acc]));
+      }
+    }
+  }
+  // ---------------- teardown ----------------
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // the peer is done with this CTA's shared and tensor memory
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, TMEM_COLS);
   }
 }
 
@@ -681,10 +1071,99 @@ cudaError_t launch_pack(const PackArgs& a, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
+static cudaError_t launch_cond_pair(const TcCondArgs& a, int clusters, cudaStream_t stream) {
+  const long long rmax = (long long)a.B * (a.K - 1);
+  const uint64_t d = (uint64_t)a.d;
+  CUtensorMap mApack, mWc, mR, mWv, mWg;
+  // Maps of operands a call does not use point at a used buffer (never read).
+  const void* apack = a.do_correct ? a.apack : a.rpack;
+  const void* wc = a.do_correct ? a.Wc : a.Wv;
+  const void* rp = a.do_gate ? a.rpack : a.apack;
+  const void* wv = a.do_gate ? a.Wv : a.Wc;
+  const void* wg = a.do_gate ? a.Wg : a.Wc;
+  if (encode_tensor_map_2d(&mApack, apack, a.do_correct ? 2 * d : d, (uint64_t)rmax, (a.do_correct ? 4 : 2) * d, BK, BM) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWc, wc, a.do_correct ? 2 * d : d, d, (a.do_correct ? 4 : 2) * d, BK, 128) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mR, rp, d, (uint64_t)rmax, 2 * (a.r_row_stride ? (uint64_t)a.r_row_stride : d), BK, BM) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWv, wv, a.do_gate ? d : 2 * d, d, (a.do_gate ? 2 : 4) * d, BK, 128) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWg, wg, 2 * d, d, 4 * d, BK, 128) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  CondParams p{};
+  p.d = a.d;
+  p.do_correct = a.do_correct;
+  p.do_gate = a.do_gate;
+  p.R = a.R;
+  p.rowmap = a.rowmap;
+  p.apack = reinterpret_cast<const __nv_bfloat16*>(a.apack);
+  p.beta = a.beta;
+  p.r_out = reinterpret_cast<__nv_bfloat16*>(a.r_out);
+  p.compact_out = a.compact_out;
+  p.e = reinterpret_cast<const __nv_bfloat16*>(a.e);
+  p.e_dense = 0;
+  p.Wg = reinterpret_cast<const __nv_bfloat16*>(a.Wg);
+  p.ge = a.ge;
+  p.e_out = reinterpret_cast<__nv_bfloat16*>(a.e_out);
+  p.sync = a.sync;
+  p.block_done = a.sync + kSyncBlocks;
+  p.block_ready = a.sync + kSyncBlocks + blocks_max(a.B, a.K);
+  p.status = a.status;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * (unsigned)clusters, 1, 1);
+  cfg.blockDim = dim3(P_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = P_SMEM_BYTES;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, cond_pair_kernel, mApack, mWc, mR, mWv, mWg, p);
+}
+
+// The CTA-pair kernel: broadcast e (or no gate), and a device that can keep
+// at least one pair of its CTAs resident.  Returns the pair count (0: use
+// cond_kernel).
+static int pair_clusters(const TcCondArgs& a, long long tiles_max_pairs, cudaError_t* err) {
+  *err = cudaSuccess;
+  if (a.do_gate && a.e_dense) return 0;
+  static int max_clusters[64] = {0};  // per device; -1: none fits
+  int dev = 0;
+  if ((*err = cudaGetDevice(&dev)) != cudaSuccess) return 0;
+  if (max_clusters[dev & 63] == 0) {
+    if ((*err = cudaFuncSetAttribute(cond_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES)) !=
+        cudaSuccess)
+      return 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2, 1, 1);
+    cfg.blockDim = dim3(P_THREADS, 1, 1);
+    cfg.dynamicSmemBytes = P_SMEM_BYTES;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if ((*err = cudaOccupancyMaxActiveClusters(&n, cond_pair_kernel, &cfg)) != cudaSuccess) return 0;
+    max_clusters[dev & 63] = n > 0 ? n : -1;
+  }
+  const int n = max_clusters[dev & 63];
+  if (n <= 0) return 0;
+  return (int)(tiles_max_pairs < n ? tiles_max_pairs : n);
+}
+
 cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream) {
   const long long rmax = (long long)a.B * (a.K - 1);
   if (rmax <= 0 || (!a.do_correct && !a.do_gate)) return cudaSuccess;
-  cudaError_t err = ensure_smem_attr<false>();
+  const long long tiles_max_pairs =
+      (rmax + 2 * BM - 1) / (2 * BM) * ((a.do_correct ? a.d / 256 : 0) + (a.do_gate ? a.d / 128 : 0));
+  cudaError_t err;
+  const int clusters = pair_clusters(a, tiles_max_pairs, &err);
+  if (err != cudaSuccess) return err;
+  if (clusters > 0) return launch_cond_pair(a, clusters, stream);
+  err = ensure_smem_attr<false>();
   if (err != cudaSuccess) return err;
   const uint64_t d = (uint64_t)a.d;
   CUtensorMap mApack, mWc, mR, mE, mWv, mWg;
