@@ -51,6 +51,14 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Logistic function from the fast exponential and division intrinsics: their
+// relative error (a few fp32 ulp) is far below the bf16 rounding of the
+// outputs it feeds.  The argument is clamped to [-80, 80], where the fp32
+// logistic is already 0 or 1 to within its rounding.
+__device__ __forceinline__ float fast_sigmoid(float x) {
+  return __fdividef(1.f, 1.f + __expf(-fminf(fmaxf(x, -80.f), 80.f)));
+}
+
 // ---------------------------------------------------------------------------
 // Argmax keys.  A 64-bit key orders (value, index) pairs by value, then by
 // LOWER index: the high word maps the float to an unsigned integer with the

@@ -258,7 +258,8 @@ __device__ __forceinline__ void epilogue_correction(const CondParams& p, uint32_
 
 // Gated-fusion epilogue of one tile row (Eq. 8): e~ = e + v * sigmoid(g) for
 // the 128 features n0.., v in accumulator columns 0..127, the r half of the
-// gate in 128..255 (plus W_g[:, :d] e from ge for a broadcast e).
+// gate in 128..255 (plus W_g[:, :d] e from ge for a broadcast e, the same
+// 32 values for every lane: one 16-byte broadcast load per four features).
 __device__ __forceinline__ void epilogue_gate(const CondParams& p, uint32_t taddr, int g, bool valid, int n0, int d) {
   const long long orow = valid ? __ldcg(p.rowmap + g) : 0;
   const __nv_bfloat16* erow = p.e + (p.e_dense ? (long long)g * d : 0);
@@ -268,6 +269,17 @@ __device__ __forceinline__ void epilogue_gate(const CondParams& p, uint32_t tadd
     tmem_ld_32cols(taddr + 128u + (uint32_t)(cc * 32), gt);
     if (valid) {
       const int n = n0 + cc * 32;
+      if (!p.e_dense) {
+        const float4* gb = reinterpret_cast<const float4*>(p.ge + n);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float4 b = __ldcg(gb + j);
+          gt[4 * j] += b.x;
+          gt[4 * j + 1] += b.y;
+          gt[4 * j + 2] += b.z;
+          gt[4 * j + 3] += b.w;
+        }
+      }
       const uint4* ev = reinterpret_cast<const uint4*>(erow + n);
       uint4* ov = reinterpret_cast<uint4*>(p.e_out + orow * d + n);
 #pragma unroll
@@ -278,13 +290,7 @@ __device__ __forceinline__ void epilogue_gate(const CondParams& p, uint32_t tadd
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
           const int c0 = x * 8 + 2 * w;
-          float g0 = gt[c0], g1 = gt[c0 + 1];
-          if (!p.e_dense) {
-            g0 += __ldcg(p.ge + n + c0);
-            g1 += __ldcg(p.ge + n + c0 + 1);
-          }
-          const float s0 = 1.f / (1.f + expf(-g0));
-          const float s1 = 1.f / (1.f + expf(-g1));
+          const float s0 = fast_sigmoid(gt[c0]), s1 = fast_sigmoid(gt[c0 + 1]);
           o[w] = pack_bf16x2(bf16_lo(ewords[w]) + v[c0] * s0, bf16_hi(ewords[w]) + v[c0 + 1] * s1);
         }
         ov[x] = make_uint4(o[0], o[1], o[2], o[3]);
@@ -532,16 +538,15 @@ __global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
           tc_fence_after();
           const uint32_t a_base = base + s * STAGE_BYTES, b_base = a_base + A_BYTES;
           const bool e_part = !corr && kb >= kb_half;
+          // K16 steps advance the start address by 32 bytes: + 2 in the descriptor's address field
+          const uint64_t adesc0 = sw128_kmajor_desc(a_base);
+          const uint64_t bdesc0 = sw128_kmajor_desc(e_part ? b_base + B_BYTES / 2 : b_base);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
-            const uint64_t adesc = sw128_kmajor_desc(a_base + (uint32_t)k * 32u);
-            if (!e_part) {
-              const uint64_t bdesc = sw128_kmajor_desc(b_base + (uint32_t)k * 32u);
-              tc_mma_bf16(d_tmem, adesc, bdesc, IDESC_N256, (kb > 0 || k > 0) ? 1u : 0u);
-            } else {
-              const uint64_t bdesc = sw128_kmajor_desc(b_base + B_BYTES / 2 + (uint32_t)k * 32u);
-              tc_mma_bf16(d_tmem + 128u, adesc, bdesc, IDESC_N128, 1u);
-            }
+            if (!e_part)
+              tc_mma_bf16(d_tmem, adesc0 + 2u * k, bdesc0 + 2u * k, IDESC_N256, (kb > 0 || k > 0) ? 1u : 0u);
+            else
+              tc_mma_bf16(d_tmem + 128u, adesc0 + 2u * k, bdesc0 + 2u * k, IDESC_N128, 1u);
           }
           tc_commit(smem_u32(&bar_empty[s]));
         }
@@ -940,12 +945,11 @@ __global__ void __launch_bounds__(P_THREADS, 1)
           }
           tc_fence_after();
           const uint32_t a_base = base + s * P_STAGE_BYTES, b_base = a_base + P_A_BYTES;
+          // K16 steps advance the start address by 32 bytes: + 2 in the descriptor's address field
+          const uint64_t adesc0 = sw128_kmajor_desc(a_base), bdesc0 = sw128_kmajor_desc(b_base);
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k) {
-            const uint64_t adesc = sw128_kmajor_desc(a_base + (uint32_t)k * 32u);
-            const uint64_t bdesc = sw128_kmajor_desc(b_base + (uint32_t)k * 32u);
-            tc_mma_pair(d_tmem, adesc, bdesc, IDESC_M256_N256, (kb > 0 || k > 0) ? 1u : 0u);
-          }
+          for (int k = 0; k < BK / 16; ++k)
+            tc_mma_pair(d_tmem, adesc0 + 2u * k, bdesc0 + 2u * k, IDESC_M256_N256, (kb > 0 || k > 0) ? 1u : 0u);
           tc_commit_pair(smem_u32(&bar_empty[s]));
         }
         tc_commit_pair(smem_u32(&bar_tfull[acc]));  // accumulator ready (also after a failure)

@@ -100,13 +100,6 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 
 __device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
-// Logistic function from the fast exponential and division intrinsics: their
-// relative error (a few fp32 ulp) is far below the bf16 rounding of the
-// output.  The argument is clamped to [-80, 80], where the fp32 logistic is
-// already 0 or 1 to within its rounding.
-__device__ __forceinline__ float fast_sigmoid(float x) {
-  return __fdividef(1.f, 1.f + __expf(-fminf(fmaxf(x, -80.f), 80.f)));
-}
 
 // grid (row blocks, 2H): blockIdx.y < H reduces over the m half against P,
 // the rest over the u half against B_c[:, 64:].
