@@ -63,11 +63,11 @@ VERIFY_TRAFFIC_SHAPE = (16, 151936, 4096, "bf16")
 # DRAM traffic of the single-kernel round per sequence (same shapes, same
 # profiling workload and method); None until measured for the current kernel.
 ROUND_TRAFFIC_PER_SEQUENCE = None
-# DRAM traffic (read + write) of one cond_kernel launch, by workload, measured
-# with ncu on that workload.  It does not scale with the batch (weights and L2
-# reuse dominate), so it is only reported where it was measured.  Must be
-# re-measured whenever cond_kernel changes.
-COND_TRAFFIC = {"qwen3-8b-B256-K16": 655573504 + 41077248}
+# DRAM traffic (read + write) of one conditioning launch (cond_pair_kernel),
+# by workload, measured with ncu on that workload.  It does not scale with the
+# batch (weights and L2 reuse dominate), so it is only reported where it was
+# measured.  Must be re-measured whenever the conditioning kernel changes.
+COND_TRAFFIC = {"qwen3-8b-B256-K16": 593758208 + 43461120}
 
 
 # ---------------------------------------------------------------------------
@@ -476,7 +476,8 @@ def run_gpu(args) -> dict | None:
             }
         elif cflops:
             c_roof = {
-                "kernel": "cond_kernel: correction + gated-fusion projections (+ gate-bias GEMV), one persistent launch",
+                "kernel": "cond_pair_kernel: correction + gated-fusion projections (+ gate-bias GEMV), one persistent "
+                          "launch on CTA pairs (tcgen05.mma.cta_group::2)",
                 "bound": "tensor",
                 "achieved": round(c_tflops, 2),
                 "peak": peaks["bf16_tflops"],
@@ -486,7 +487,7 @@ def run_gpu(args) -> dict | None:
                 "frac_of_sustained": round(c_tflops / peaks["bf16_tflops_sustained"], 4),
                 "algorithmic_flops": cflops,
                 "avg_launch_us": round(c_avg_s * 1e6, 2),
-                "traffic": (COND_TRAFFIC.get(cfg.name) if args.variant == "corrected" else None),
+                "traffic": (COND_TRAFFIC.get(cfg.name) if args.variant == "corrected" and not args.sampled else None),
                 "traffic_source": "ncu dram read+write of one launch on this workload",
             }
         # `roofline` is the kernel that takes the larger share of the round
