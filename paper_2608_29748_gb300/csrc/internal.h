@@ -46,7 +46,7 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   L.status = off;
   off = align_up(off + 64 * 4, 256);
   L.sync = off;
-  L.sync_bytes = align_up((size_t)(32 + 2 * ((rmax + 127) / 128)) * 4, 256);
+  L.sync_bytes = align_up((size_t)(32 + 2 * ((rmax + 255) / 256 * 2)) * 4, 256);  // 2 x blocks_max
   off += L.sync_bytes;
   L.keys = off;
   off = align_up(off + (size_t)(B * (K + 1)) * 8, 256);
@@ -222,9 +222,11 @@ constexpr int kSyncSeqDone = 4;
 constexpr int kSyncChunkNext = 5;
 constexpr int kSyncBlocks = 32;
 
+// 128-row blocks of the largest packed-row count, rounded up to whole pairs
+// (the CTA-pair kernel counts per 128-row block over 256-row pair tiles).
 inline long long blocks_max(long long B, long long K) {
   const long long rmax = B * (K > 1 ? K - 1 : 0);
-  return (rmax + 127) / 128;
+  return (rmax + 255) / 256 * 2;
 }
 
 struct TcCondArgs {
