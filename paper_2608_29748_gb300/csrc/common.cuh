@@ -94,6 +94,17 @@ __device__ __forceinline__ unsigned long long warp_max_key(unsigned long long k)
 }
 
 // ---------------------------------------------------------------------------
+// Programmatic dependent launch: a kernel launched with the programmatic
+// stream-serialisation attribute may start once every CTA of the previous
+// kernel in the stream has called pdl_launch_dependents (or exited); it must
+// call pdl_wait before it reads anything the previous kernel writes, and
+// pdl_wait returns once that kernel has completed and its writes are visible.
+// Both are no-ops for a kernel launched without the attribute.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// ---------------------------------------------------------------------------
 // Shared-memory address helpers
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

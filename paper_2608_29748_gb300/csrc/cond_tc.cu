@@ -789,11 +789,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
   const bool leader = rank == 0;
   const int d = p.d;
   const int nt0 = d / 256, nt1 = d / 128;
-  const int R = *(volatile const int32_t*)p.R;
-  const int pairs_m = (R + 2 * BM - 1) / (2 * BM);
-  const int T0 = p.do_correct ? pairs_m * nt0 : 0;
-  const int T = T0 + (p.do_gate ? pairs_m * nt1 : 0);
-  if (T == 0) return;  // both CTAs read the same R
+  pdl_launch_dependents();
   uint32_t* tile_queue = p.sync + kSyncTileQueue;
   uint32_t* gemv_next = p.sync + kSyncGemvNext;
   uint32_t* gemv_done = p.sync + kSyncGemvDone;
@@ -838,6 +834,19 @@ __global__ void __launch_bounds__(P_THREADS, 1)
   const uint32_t tmem = s_tmem;
   const uint32_t base = (smem_u32(dsmem) + 1023u) & ~1023u;
   const int kb_half = d / BK;
+  // The set-up above may overlap the end of the previous kernel (programmatic
+  // dependent launch).  R, the packed rows and the row map are its outputs:
+  // every role that reads them waits here first.  The gate-bias GEMV (warps
+  // 2-3) reads only the inputs and starts at once.  With R = 0 the queue's
+  // first claim already ends every role.
+  int R = 0, T0 = 0, T = 0;
+  if (warp != 2 && warp != 3) {
+    pdl_wait();
+    R = *(volatile const int32_t*)p.R;
+    const int pairs_m = (R + 2 * BM - 1) / (2 * BM);
+    T0 = p.do_correct ? pairs_m * nt0 : 0;
+    T = T0 + (p.do_gate ? pairs_m * nt1 : 0);
+  }
   // the leader's barriers as seen from either CTA
   auto leader_addr = [&](const void* local) { return map_rank(smem_u32(local), 0); };
 
@@ -1110,19 +1119,9 @@ static cudaError_t launch_cond_pair(const TcCondArgs& a, int clusters, cudaStrea
   p.block_done = a.sync + kSyncBlocks;
   p.block_ready = a.sync + kSyncBlocks + blocks_max(a.B, a.K);
   p.status = a.status;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(2 * (unsigned)clusters, 1, 1);
-  cfg.blockDim = dim3(P_THREADS, 1, 1);
-  cfg.dynamicSmemBytes = P_SMEM_BYTES;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, cond_pair_kernel, mApack, mWc, mR, mWv, mWg, p);
+  // clusters of two CTAs; set-up may overlap the previous kernel's end
+  return launch_dependent(cond_pair_kernel, dim3(2 * (unsigned)clusters), dim3(P_THREADS), P_SMEM_BYTES, stream, 2,
+                          mApack, mWc, mR, mWv, mWg, p);
 }
 
 // The CTA-pair kernel: broadcast e (or no gate), and a device that can keep

@@ -114,6 +114,8 @@ __global__ void __launch_bounds__(256, 1)
   __shared__ volatile int s_abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_launch_dependents();
+  pdl_wait();  // the packed rows and R come from verification
   const int R = *(volatile const int32_t*)p.R;
   const int m0 = blockIdx.x * BM;
   if (m0 >= R) return;
@@ -308,13 +310,17 @@ __device__ __forceinline__ void lr_gemv_rows(const LrParams& p, int d, int lane)
   }
 }
 
-// grid >= ceil(R_max / 8) and >= two CTAs per SM: rows first, then the GEMV.
+// grid >= ceil(R_max / 8) and >= two CTAs per SM.  The GEMV reads only the
+// inputs, so it runs first, while the projection may still be running
+// (programmatic dependent launch); the rows wait for the projection's partials.
 __global__ void __launch_bounds__(256) lr_finish_kernel(const LrParams p) {
-  const int R = *(volatile const int32_t*)p.R;
+  pdl_launch_dependents();
   const long long g = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int d = p.d, lane = threadIdx.x & 31;
-  if ((long long)blockIdx.x * 8 < R) finish_rows(p, g, R, d, lane);  // uniform over the CTA
   lr_gemv_rows(p, d, lane);
+  pdl_wait();
+  const int R = *(volatile const int32_t*)p.R;
+  if ((long long)blockIdx.x * 8 < R) finish_rows(p, g, R, d, lane);  // uniform over the CTA
 }
 
 // Persistent: CTA c takes tiles c, c + G, ... of the (row block, 64-feature
@@ -333,6 +339,8 @@ __global__ void __launch_bounds__(kFuseThreads, 2)
   __shared__ volatile int s_abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_launch_dependents();
+  pdl_wait();  // rho and W_g[:, :d] e come from the finishing kernel
   const int R = *(volatile const int32_t*)p.R;
   const int d = p.d;
   const int nb = d / kFuseFeat;
@@ -617,11 +625,14 @@ cudaError_t launch_lowrank(const LowRankArgs& a, bool tc, cudaStream_t stream) {
   p.ge = a.ge;
   p.gemv_next = a.gemv_next;
   p.status = a.status;
-  lr_project_kernel<<<dim3(mt, 2 * H), 256, SMEM_PROJECT, stream>>>(mA, mP, mBc, p);
-  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  // Each of the three kernels may start while the previous one finishes
+  // (programmatic dependent launch), and waits for its outputs in the kernel.
+  if ((err = launch_dependent(lr_project_kernel, dim3(mt, 2 * H), dim3(256), SMEM_PROJECT, stream, 1, mA, mP, mBc,
+                              p)) != cudaSuccess)
+    return err;
   const long long fgrid = (rmax + 7) / 8 > 2LL * info.sm_count ? (rmax + 7) / 8 : 2LL * info.sm_count;
-  lr_finish_kernel<<<(unsigned)fgrid, 256, 0, stream>>>(p);
-  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  if ((err = launch_dependent(lr_finish_kernel, dim3((unsigned)fgrid), dim3(256), 0, stream, 1, p)) != cudaSuccess)
+    return err;
   LrFuseParams f{};
   f.d = a.d;
   f.R = a.R;
@@ -633,8 +644,7 @@ cudaError_t launch_lowrank(const LowRankArgs& a, bool tc, cudaStream_t stream) {
   const long long tiles_max = (long long)mt * (a.d / kFuseFeat);
   const long long slots = 2LL * info.sm_count;  // two CTAs per SM
   const unsigned grid = (unsigned)(tiles_max < slots ? tiles_max : slots);
-  lr_fuse_kernel<<<grid, kFuseThreads, SMEM_FUSE, stream>>>(mRho, mWv, mWg, f);
-  return cudaGetLastError();
+  return launch_dependent(lr_fuse_kernel, dim3(grid), dim3(kFuseThreads), SMEM_FUSE, stream, 1, mRho, mWv, mWg, f);
 }
 
 }  // namespace retrace

@@ -258,6 +258,7 @@ __global__ void __launch_bounds__(kThreads) verify_kernel(const VerifyParams p) 
   __shared__ int s_t[kMaxK + 1];
   __shared__ int s_A[2];  // accepted length, packed-row offset
   __shared__ int s_last;
+  pdl_launch_dependents();  // the next kernel may take SMs as this grid's CTAs finish
 
   const long long T_ = p.total_slots;
   const long long G = gridDim.x;

@@ -139,6 +139,7 @@ __global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkPar
   __shared__ float s_sample[kThreads];
   __shared__ int s_n[kWarps];
   __shared__ unsigned long long s_thr;
+  pdl_launch_dependents();  // the finalize kernel may take SMs as these CTAs finish
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = blockIdx.x;  // B (2K+1) rows: a grid dimension, below 2^31
   const int nt = p.B * (p.K + 1);
@@ -423,6 +424,8 @@ __device__ int draw(const RowDist& r, const float wt[2], float u, int lane) {
 // every thread writes the outputs and, for a round, copies and packs rows.
 __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizeParams p) {
   __shared__ int s_A, s_y, s_off;
+  pdl_launch_dependents();
+  pdl_wait();  // the sorted lists come from the top-k kernel
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int b = blockIdx.x;
   const int K = p.K, K1 = K + 1;
@@ -594,8 +597,7 @@ cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cud
   fp.epack = a.epack;
   fp.rowmap = a.rowmap;
   fp.R_count = a.R_count;
-  sampled_finalize_kernel<<<(unsigned)a.B, 256, 0, stream>>>(fp);
-  return cudaGetLastError();
+  return launch_dependent(sampled_finalize_kernel, dim3((unsigned)a.B), dim3(256), 0, stream, 1, fp);
 }
 
 }  // namespace retrace
