@@ -94,6 +94,29 @@ __device__ __forceinline__ unsigned long long warp_max_key(unsigned long long k)
 }
 
 // ---------------------------------------------------------------------------
+// Block-wide copy of n 16-byte vectors: element i = load(i) goes to store(i, .).
+// Each thread keeps kInFlight independent loads in flight before it stores,
+// so a copy of a few hundred KB per block is not a chain of memory latencies.
+// ---------------------------------------------------------------------------
+template <int kInFlight = 8, typename Load, typename Store>
+__device__ __forceinline__ void copy_vectors(long long n, Load load, Store store) {
+  const long long stride = blockDim.x;
+  for (long long i0 = threadIdx.x; i0 < n; i0 += kInFlight * stride) {
+    uint4 v[kInFlight];
+#pragma unroll
+    for (int q = 0; q < kInFlight; ++q) {
+      const long long i = i0 + q * stride;
+      if (i < n) v[q] = load(i);
+    }
+#pragma unroll
+    for (int q = 0; q < kInFlight; ++q) {
+      const long long i = i0 + q * stride;
+      if (i < n) store(i, v[q]);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Programmatic dependent launch: a kernel launched with the programmatic
 // stream-serialisation attribute may start once every CTA of the previous
 // kernel in the stream has called pdl_launch_dependents (or exited); it must

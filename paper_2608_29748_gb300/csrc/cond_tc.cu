@@ -11,22 +11,35 @@
 //    GEMMs stream their A operand with tiled TMA boxes (per-row gathers were
 //    measured to starve the tensor pipe).
 //
-// 2. tc_gemm_kernel, persistent (one CTA per SM, static tile schedule):
-//    MODE 0, correction (Eq. 6-7):  r = m + beta * W_c [m; u]
-//        A = Apack [R, 2d]; B = W_c [d, 2d] (K-major); 128 x 256 tiles of c;
+// 2. one persistent launch runs both projections from a dynamic tile queue
+//    (every correction tile, then every gate tile; a gate tile of a row block
+//    waits until the correction epilogues of that block have written r):
+//    correction (Eq. 6-7):  r = m + beta * W_c [m; u]
+//        A = Apack [R, 2d]; B = W_c [d, 2d] (K-major); N = 256 tiles of c;
 //        the epilogue adds m (the first d columns of Apack) and writes r bf16.
-//    MODE 1, gated fusion (Eq. 8):  e~ = e + (W_v r) .* sigmoid(W_g [e; r])
+//    gated fusion (Eq. 8):  e~ = e + (W_v r) .* sigmoid(W_g [e; r])
 //        A = r rows; the B tile stacks 128 rows of W_v over the matching 128
 //        rows of W_g[:, d:2d], so one N = 256 MMA yields v (accumulator
 //        columns 0..127) and the r half of the gate (128..255) for the same
 //        output features.  The e half of the gate is a broadcast vector
-//        precomputed once (added in the epilogue) or, for per-position e,
-//        extra K blocks (Epack x W_g[:, :d]) accumulated into the gate columns.
+//        computed once by idle warps (W_g[:, :d] e, added in the epilogue)
+//        or, for per-position e, extra K blocks (Epack x W_g[:, :d])
+//        accumulated into the gate columns.
+//    Two kernels implement it:
+//    cond_pair_kernel   (broadcast e) clusters of two CTAs, 256-row tiles,
+//                       tcgen05.mma.cta_group::2 M256 N256 K16; each CTA
+//                       stages its own 128 rows and half of the weight tile
+//                       (described at the kernel);
+//    cond_kernel<false> (per-position e) one CTA per SM, 128-row tiles,
+//                       tcgen05.mma.cta_group::1 M128 N256 K16;
+//    cond_kernel<true>  the overlapped round: the same plus verification
+//                       streamed through shared memory (verify_stream.cuh).
 //
-// Warp roles of the GEMM (256 threads):
-//   warp 0     TMA producer (one elected lane): A box + weight box(es) per stage;
-//   warp 1     MMA issuer (one lane): 4 x tcgen05.mma M128 N256 K16 per stage;
+// Warp roles of cond_kernel<false> (256 threads; the pair kernel's are alike):
+//   warp 0     tile scheduler + TMA producer (one elected lane);
+//   warp 1     MMA issuer (one lane): 4 x tcgen05.mma per 64-deep stage;
 //   warp 2     TMEM allocation: 2 accumulators x 256 fp32 columns = 512 columns;
+//   warps 2-3  the broadcast-e GEMV W_g[:, :d] e, rows claimed from a counter;
 //   warps 4-7  epilogue: tcgen05.ld of their 32 TMEM lanes (= tile rows).
 // The two accumulators alternate between tiles, so a tile's epilogue overlaps
 // the next tile's main loop.  Every mbarrier wait is bounded; on expiry the CTA

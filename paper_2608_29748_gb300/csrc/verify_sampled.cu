@@ -14,9 +14,11 @@
 //                            k-th largest (a sample's k-th largest, then the
 //                            best warp's k-th largest candidate) go to per-warp
 //                            buffers; the CTA merges the warps' lists by rank;
-//   sampled_finalize_kernel  one warp per sequence: the filtered
-//                            probabilities from the sorted lists, the accept
-//                            tests in order, and the draw.
+//   sampled_finalize_kernel  one CTA per sequence: the filtered
+//                            probabilities of the draft tokens from the sorted
+//                            lists (eight positions at a time, one per warp),
+//                            the accept tests in order, the draw, and for a
+//                            round the copies and packing of e~ and [m; u].
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -420,33 +422,60 @@ __device__ int draw(const RowDist& r, const float wt[2], float u, int lane) {
   return h == 0 ? t0 : t1;
 }
 
-// One CTA per sequence: warp 0 takes the accept decisions and the draw; then
-// every thread writes the outputs and, for a round, copies and packs rows.
+// One CTA per sequence.  The accept tests need only p_i(x_i) and q_i(x_i):
+// the warps compute them for eight positions at a time, one position each,
+// and thread 0 takes the decisions in order, so the chain of dependent
+// distributions is one per chunk instead of one per position.  Warp 0 then
+// draws the appended token; every thread writes the outputs and, for a round,
+// copies and packs rows.
 __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizeParams p) {
+  constexpr int kFinWarps = 8;
   __shared__ int s_A, s_y, s_off;
+  __shared__ float s_px[kFinWarps], s_qx[kFinWarps];
   pdl_launch_dependents();
   pdl_wait();  // the sorted lists come from the top-k kernel
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int b = blockIdx.x;
   const int K = p.K, K1 = K + 1;
   const int32_t* dr = p.draft + (long long)b * K;
-  if (warp == 0) {
-    const long long tbase = (long long)b * K1, dbase = (long long)p.B * K1 + (long long)b * K;
-    const float* u = p.uniforms + (long long)b * K1;
-    int A = K;
-    for (int i = 0; i < K; ++i) {
+  const long long tbase = (long long)b * K1, dbase = (long long)p.B * K1 + (long long)b * K;
+  const float* u = p.uniforms + (long long)b * K1;
+  int A = K;
+  for (int c0 = 0; c0 < K; c0 += kFinWarps) {
+    const int i = c0 + warp;
+    if (i < K) {
       const int x = dr[i];
-      bool ok = false;
+      float px = -1.f, qx = 0.f;  // px < 0: a token outside [0, V) is rejected
       if (x >= 0 && x < p.V) {
         const RowDist pt = row_dist(p, tbase + i, lane);
         const RowDist qd = row_dist(p, dbase + i, lane);
-        ok = u[i] * dist_prob(qd, x) < dist_prob(pt, x);
+        px = dist_prob(pt, x);
+        qx = dist_prob(qd, x);
       }
-      if (!ok) {
-        A = i;
-        break;
+      if (lane == 0) {
+        s_px[warp] = px;
+        s_qx[warp] = qx;
       }
     }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int a = -1;
+      for (int j = 0; j < kFinWarps && c0 + j < K; ++j) {
+        if (!(s_px[j] >= 0.f && u[c0 + j] * s_qx[j] < s_px[j])) {
+          a = c0 + j;
+          break;
+        }
+      }
+      s_A = a;
+    }
+    __syncthreads();
+    const int a = s_A;
+    if (a >= 0) {
+      A = a;
+      break;
+    }
+  }
+  if (warp == 0) {
     const RowDist pt = row_dist(p, tbase + A, lane);
     int y;
     if (A < K) {
@@ -473,14 +502,13 @@ __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizePar
       y = draw(pt, pt.w, u[K], lane);
     }
     if (lane == 0) {
-      s_A = A;
       s_y = y;
       const int nb = K - 1 - A > 0 ? K - 1 - A : 0;
       s_off = (p.R_count && nb > 0) ? atomicAdd(p.R_count, nb) : 0;
     }
   }
   __syncthreads();
-  const int A = s_A, y = s_y;
+  const int y = s_y;
   for (int i = threadIdx.x; i < K1; i += blockDim.x) {
     const long long o = (long long)b * K1 + i;
     p.committed[o] = i < A ? dr[i] : (i == A ? y : -1);
@@ -503,10 +531,8 @@ __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizePar
     const long long pos_vec = p.e_pos_stride * p.elem / 16;
     const uint4* src = reinterpret_cast<const uint4*>(e_b);
     uint4* dst = reinterpret_cast<uint4*>(p.e_out) + (base_row + nb) * vpr;
-    for (long long i = threadIdx.x; i < rows * vpr; i += blockDim.x) {
-      const long long j = nb + i / vpr, c = i % vpr;
-      dst[i] = __ldg(src + j * pos_vec + c);
-    }
+    copy_vectors(rows * vpr, [&](long long i) { return __ldg(src + (nb + i / vpr) * pos_vec + i % vpr); },
+                 [&](long long i, const uint4& v) { dst[i] = v; });
   } else if (p.elem == 2) {
     const uint16_t* src = reinterpret_cast<const uint16_t*>(e_b);
     uint16_t* dst = reinterpret_cast<uint16_t*>(p.e_out) + (base_row + nb) * p.d;
@@ -533,17 +559,17 @@ __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizePar
   const uint4* hD = reinterpret_cast<const uint4*>(p.hD);
   const uint4* hT = reinterpret_cast<const uint4*>(p.hT);
   uint4* ap = reinterpret_cast<uint4*>(p.apack);
-  for (long long i = threadIdx.x; i < (long long)nb * 2 * vpr; i += blockDim.x) {
-    const long long j = i / (2 * vpr), c = i % (2 * vpr);
-    ap[(off + j) * 2 * vpr + c] = c < vpr ? __ldg(hD + (base_row + A + 1 + j) * vpr + c)
-                                          : __ldg(hT + (base_row + A + j) * vpr + c - vpr);
-  }
+  copy_vectors(
+      (long long)nb * 2 * vpr,
+      [&](long long i) {
+        const long long j = i / (2 * vpr), c = i % (2 * vpr);
+        return c < vpr ? __ldg(hD + (base_row + A + 1 + j) * vpr + c) : __ldg(hT + (base_row + A + j) * vpr + c - vpr);
+      },
+      [&](long long i, const uint4& v) { ap[(long long)off * 2 * vpr + i] = v; });
   if (p.e_dense) {
     uint4* ep = reinterpret_cast<uint4*>(p.epack);
-    for (long long i = threadIdx.x; i < (long long)nb * vpr; i += blockDim.x) {
-      const long long j = i / vpr, c = i % vpr;
-      ep[(off + j) * vpr + c] = __ldg(e_v + j * pos_vec + c);
-    }
+    copy_vectors((long long)nb * vpr, [&](long long i) { return __ldg(e_v + (i / vpr) * pos_vec + i % vpr); },
+                 [&](long long i, const uint4& v) { ep[(long long)off * vpr + i] = v; });
   }
 }
 
