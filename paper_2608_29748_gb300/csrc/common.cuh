@@ -135,6 +135,38 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
 }
 
 // ---------------------------------------------------------------------------
+// Block-wide copy of n 16-byte vectors through shared memory: thread t copies
+// vectors t, t + blockDim.x, ... .  kStage of them at a time go from global
+// memory into the thread's own slots of `staging` (kStage * blockDim.x
+// vectors) with cp.async, which holds no registers while in flight, then from
+// the slots to their destination.  No block barrier: each thread reads back
+// only the slots it filled.  src(i) and dst(i) give 16-byte aligned addresses.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void cp_async16(uint32_t smem_dst, const void* gsrc) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_dst), "l"(gsrc) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+template <int kStage, typename Src, typename Dst>
+__device__ __forceinline__ void copy_vectors_staged(long long n, uint4* staging, Src src, Dst dst) {
+  const long long stride = blockDim.x;
+  for (long long i0 = threadIdx.x; i0 < n; i0 += kStage * stride) {
+#pragma unroll
+    for (int q = 0; q < kStage; ++q) {
+      const long long i = i0 + q * stride;
+      if (i < n) cp_async16(smem_u32(staging + q * stride + threadIdx.x), src(i));
+    }
+    cp_async_wait_all();
+#pragma unroll
+    for (int q = 0; q < kStage; ++q) {
+      const long long i = i0 + q * stride;
+      if (i < n) *dst(i) = staging[q * stride + threadIdx.x];
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
 // mbarrier
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {

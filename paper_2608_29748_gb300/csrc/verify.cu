@@ -149,11 +149,17 @@ __device__ __forceinline__ unsigned long long block_max_key(unsigned long long k
   return s_red[0];
 }
 
+// Row copies of the finalising CTA go through shared memory with cp.async,
+// four 16-byte vectors per thread in flight (32 KB per CTA; more would make
+// this kernel spill at its two-CTAs-per-SM register budget).
+constexpr int kCopyStage = 4;
+constexpr int kCopyStageBytes = kCopyStage * kThreads * 16;
+
 // Copy of rows [j0, K) of sequence b into e_out: rows j < j_m from the
 // aligned drafter states m_j = hD[b, A+1+j] (the overwrite ablation), the
 // others from the drafter inputs e.
 template <typename T>
-__device__ void copy_rows(const VerifyParams& p, int b, int A, int j0, int j_m) {
+__device__ void copy_rows(const VerifyParams& p, int b, int A, int j0, int j_m, uint4* staging) {
   const int K = p.K, d = p.d;
   const long long rows = K - j0;
   if (rows <= 0) return;
@@ -165,11 +171,15 @@ __device__ void copy_rows(const VerifyParams& p, int b, int A, int j0, int j_m) 
                    (j_m <= j0 || (uintptr_t)p.hD % 16 == 0);
   if (vec) {
     const int vpr = d * (int)sizeof(T) / 16;
-    for (long long i = threadIdx.x; i < rows * vpr; i += kThreads) {
-      const long long j = j0 + i / vpr, q = i % vpr;
-      const T* row = (j < j_m) ? m_b + j * d : src_b + j * p.e_pos_stride;
-      reinterpret_cast<uint4*>(dst)[i] = reinterpret_cast<const uint4*>(row)[q];
-    }
+    copy_vectors_staged<kCopyStage>(
+        rows * vpr,
+        staging,
+        [&](long long i) {
+          const long long j = j0 + i / vpr, q = i % vpr;
+          const T* row = (j < j_m) ? m_b + j * d : src_b + j * p.e_pos_stride;
+          return reinterpret_cast<const uint4*>(row) + q;
+        },
+        [&](long long i) { return reinterpret_cast<uint4*>(dst) + i; });
   } else {
     for (long long i = threadIdx.x; i < rows * d; i += kThreads) {
       const long long j = j0 + i / d, q = i % d;
@@ -183,7 +193,7 @@ __device__ void copy_rows(const VerifyParams& p, int b, int A, int j0, int j_m) 
 // (Eq. 4-5) and, for per-position e, e[b, j]; rows land at a block of n_b rows
 // claimed with one atomic (row order across sequences does not matter: every
 // packed row carries its position in rowmap).
-__device__ void pack_sequence_rows(const VerifyParams& p, int b, int A, int nb, int* s_off) {
+__device__ void pack_sequence_rows(const VerifyParams& p, int b, int A, int nb, int* s_off, uint4* staging) {
   const int K = p.K, d = p.d;
   if (threadIdx.x == 0) *s_off = atomicAdd(p.R_count, nb);
   __syncthreads();
@@ -194,23 +204,23 @@ __device__ void pack_sequence_rows(const VerifyParams& p, int b, int A, int nb, 
   const uint4* hD = reinterpret_cast<const uint4*>(p.hD);
   const uint4* hT = reinterpret_cast<const uint4*>(p.hT);
   uint4* out = reinterpret_cast<uint4*>(p.apack);
-  for (int i = threadIdx.x; i < nb * 2 * vpr; i += kThreads) {
-    const int j = i / (2 * vpr), c = i - j * 2 * vpr;
-    const uint4 v = (c < vpr) ? __ldg(hD + (base + A + 1 + j) * vpr + c) : __ldg(hT + (base + A + j) * vpr + c - vpr);
-    out[(long long)(off + j) * 2 * vpr + c] = v;
-  }
+  copy_vectors_staged<kCopyStage>(
+      (long long)nb * 2 * vpr, staging,
+      [&](long long i) {
+        const long long j = i / (2 * vpr), c = i - j * 2 * vpr;
+        return (c < vpr) ? hD + (base + A + 1 + j) * vpr + c : hT + (base + A + j) * vpr + c - vpr;
+      },
+      [&](long long i) { return out + (long long)off * 2 * vpr + i; });
   if (p.e_dense) {
     const uint4* e = reinterpret_cast<const uint4*>(p.e);
     uint4* eo = reinterpret_cast<uint4*>(p.epack);
-    for (int i = threadIdx.x; i < nb * vpr; i += kThreads) {
-      const int j = i / vpr, c = i - j * vpr;
-      eo[(long long)(off + j) * vpr + c] = __ldg(e + (base + j) * vpr + c);
-    }
+    copy_vectors_staged<kCopyStage>((long long)nb * vpr, staging, [&](long long i) { return e + base * vpr + i; },
+                                    [&](long long i) { return eo + (long long)off * vpr + i; });
   }
 }
 
 template <typename T>
-__device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s_A) {
+__device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s_A, uint4* staging) {
   const int K = p.K, K1 = K + 1;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int i = threadIdx.x; i < K1; i += kThreads)
@@ -245,19 +255,20 @@ __device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s
     p.tickets[b] = 0u;
   }
   if (p.e_out) {
-    if (p.cond_copy == kCondCopyKeep) copy_rows<T>(p, b, A, nb, 0);
-    else if (p.cond_copy == kCondCopyE) copy_rows<T>(p, b, A, 0, 0);
-    else copy_rows<T>(p, b, A, 0, nb);
+    if (p.cond_copy == kCondCopyKeep) copy_rows<T>(p, b, A, nb, 0, staging);
+    else if (p.cond_copy == kCondCopyE) copy_rows<T>(p, b, A, 0, 0, staging);
+    else copy_rows<T>(p, b, A, 0, nb, staging);
   }
-  if (p.R_count && nb > 0) pack_sequence_rows(p, b, A, nb, s_A + 1);
+  if (p.R_count && nb > 0) pack_sequence_rows(p, b, A, nb, s_A + 1, staging);
 }
 
 template <typename T, bool VEC>
-__global__ void __launch_bounds__(kThreads) verify_kernel(const VerifyParams p) {
+__global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams p) {
   __shared__ unsigned long long s_red[kThreads / 32];
   __shared__ int s_t[kMaxK + 1];
   __shared__ int s_A[2];  // accepted length, packed-row offset
   __shared__ int s_last;
+  extern __shared__ uint4 s_stage[];  // kCopyStage * kThreads vectors: row copies of the finaliser
   pdl_launch_dependents();  // the next kernel may take SMs as this grid's CTAs finish
 
   const long long T_ = p.total_slots;
@@ -299,7 +310,7 @@ __global__ void __launch_bounds__(kThreads) verify_kernel(const VerifyParams p) 
       __syncthreads();
       if (s_last) {
         __threadfence();
-        finalize_sequence<T>(p, b, s_t, s_A);
+        finalize_sequence<T>(p, b, s_t, s_A, s_stage);
       }
       __syncthreads();
     }
@@ -314,7 +325,9 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
   static int occ_cache[64] = {0};
   int& occ = occ_cache[info.device & 63];
   if (occ == 0) {
-    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, verify_kernel<T, VEC>, kThreads, 0);
+    err = cudaFuncSetAttribute(verify_kernel<T, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize, kCopyStageBytes);
+    if (err != cudaSuccess) return err;
+    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, verify_kernel<T, VEC>, kThreads, kCopyStageBytes);
     if (err != cudaSuccess) return err;
     if (occ < 1) occ = 1;
   }
@@ -357,7 +370,7 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
   if (by_bytes < grid) grid = by_bytes;
   if (grid > p.total_slots) grid = p.total_slots;
   if (grid < 1) grid = 1;
-  verify_kernel<T, VEC><<<(unsigned)grid, kThreads, 0, stream>>>(p);
+  verify_kernel<T, VEC><<<(unsigned)grid, kThreads, kCopyStageBytes, stream>>>(p);
   return cudaGetLastError();
 }
 
