@@ -58,7 +58,7 @@ L2_FLUSH_BYTES = 256 << 20
 # + 3.10 MB written (the packed rows it writes stay in L2 during the launch).
 # Traffic grows in proportion to the sequences (the logits dominate).  Must be
 # re-measured whenever verify_kernel changes.
-VERIFY_TRAFFIC_PER_SEQUENCE = (685663232 + 3102720) / 128
+VERIFY_TRAFFIC_PER_SEQUENCE = (685742592 + 2950912) / 128
 VERIFY_TRAFFIC_SHAPE = (16, 151936, 4096, "bf16")
 # DRAM traffic of the single-kernel round per sequence (same shapes, same
 # profiling workload and method); None until measured for the current kernel.
@@ -67,7 +67,7 @@ ROUND_TRAFFIC_PER_SEQUENCE = None
 # by workload, measured with ncu on that workload.  It does not scale with the
 # batch (weights and L2 reuse dominate), so it is only reported where it was
 # measured.  Must be re-measured whenever the conditioning kernel changes.
-COND_TRAFFIC = {"qwen3-8b-B256-K16": 593758208 + 43461120}
+COND_TRAFFIC = {"qwen3-8b-B256-K16": 616099328 + 42992640}
 
 
 # ---------------------------------------------------------------------------
