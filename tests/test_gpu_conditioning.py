@@ -152,3 +152,40 @@ def test_half_gate_identity_value_is_exact(rt, d, dtype):
     if dtype == torch.bfloat16:
         want = oracle.round_to_bf16(want)
     assert np.array_equal(got, want)
+
+
+def accept_for_rows(B, K, R):
+    """Accepted lengths whose carried rows n_b = max(0, K-1-A_b) sum to R."""
+    a = torch.full((B,), K, dtype=torch.int32)
+    left = R
+    for b in range(B):
+        n = min(K - 1, left)
+        a[b] = K - 1 - n if n > 0 else K
+        left -= n
+    assert left == 0
+    return a.cuda()
+
+
+@pytest.mark.parametrize("R", [1, 127, 128, 129, 255, 256, 257, 384, 513])
+def test_pair_tile_boundaries(rt, R):
+    """Row counts around the 128-row halves and 256-row pairs of the
+    tensor-core kernel (one CTA's half empty, odd block counts)."""
+    B, K, d, dtype = 40, 16, 256, torch.bfloat16
+    x = make_inputs(B, K, d, dtype, seed=R, accept=accept_for_rows(B, K, R))
+    A = host_int(x["accept"])
+    n_host = oracle.carried_rows(A, K)
+    assert n_host.sum() == R
+    ws = rt.Workspace(B, K, 8, d, dtype)
+    r = torch.full((B, K, d), 9.0, dtype=dtype, device="cuda")
+    n = torch.empty((B,), dtype=torch.int32, device="cuda")
+    rt.retrace_align_refine(x["hD"], x["hT"], x["accept"], x["Wc"], 0.5, r, n, ws)
+    out = torch.full((B, K, d), 7.0, dtype=dtype, device="cuda")
+    rt.retrace_gate_fuse(x["e_vec"], r, n, x["Wv"], x["Wg"], out, ws)
+    torch.cuda.synchronize()
+    assert ws.check() == 0
+    m, u = oracle.align(host_f64(x["hD"]), host_f64(x["hT"]), A)
+    r_ref = oracle.correct(m, u, host_f64(x["Wc"]), 0.5, round_r_bf16=False)
+    assert_close(r, r_ref, f"r, R={R}")
+    e_full = np.broadcast_to(host_f64(x["e_vec"]), (B, K, d))
+    want = oracle.gate_fuse(e_full, host_f64(r), n_host, host_f64(x["Wv"]), host_f64(x["Wg"]))
+    assert_close(out, want, f"e~, R={R}")
