@@ -31,7 +31,8 @@ namespace {
 
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
-constexpr int kBuf = 384;  // candidate keys per warp: the compaction trigger (<= 128) + one chunk
+constexpr int kTrigger = kMaxTopK;       // a warp's buffer is cut to its top k once it holds more keys
+constexpr int kBuf = kTrigger + 32 * 8;  // candidate keys per warp: the trigger + one bf16 chunk of the warp
 
 struct TopkParams {
   const void* tlogits;
@@ -163,7 +164,9 @@ __global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkPar
   const int span = 32 * per;
   const int nchunks = (V + span - 1) / span;
   const int c0 = (int)((long long)nchunks * warp / kWarps), c1 = (int)((long long)nchunks * (warp + 1) / kWarps);
-  const int trigger = 2 * k > 64 ? 2 * k : 64;  // <= 128 = kBuf - 32 * 8
+  // k <= kMaxTopK = kTrigger: a compaction leaves at most kTrigger keys, so
+  // the buffer has room for the next chunk
+  const int trigger = kTrigger;
   const unsigned valid_bits = vec ? (1u << E) - 1u : 1u;  // the scalar path fills elements 1.. with -inf
 
   // chunk c of this lane: valid iff c < c1 and its first element is in the row
