@@ -618,6 +618,88 @@ def run_reference(args) -> dict | None:
     }
 
 
+def run_sweep(args) -> None:
+    """Every workload (configs 1-5): verification alone and the whole round,
+    the median of max(steps, 50) CUDA-event timings after warm-up, cold (a
+    256 MB L2 flush before every call) and warm (back to back, so whatever
+    fits stays in L2), plus CUDA-graph replay of the round for B <= 8.  Also
+    the bytes verification needs at least, sum_b (A_b + 1) V s (the rows up to
+    the first mismatch), against the B (K+1) V s a parallel kernel reads.  One
+    JSON line per workload; an extra report, not the benchmark line."""
+    from paper_2608_29748_gb300 import binding as rt
+
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    peaks = load_peaks()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    iters = max(args.steps, 50)
+
+    def timed(fn, cold: bool) -> float:
+        for _ in range(max(args.warmup, 3)):
+            fn()
+        torch.cuda.synchronize(dev)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(iters)]
+        for i in range(iters):
+            if cold:
+                flush.fill_(i & 0xFF)
+            ev[i][0].record()
+            fn()
+            ev[i][1].record()
+        torch.cuda.synchronize(dev)
+        return statistics.median(a.elapsed_time(b) for a, b in ev) * 1e3  # µs
+
+    for cid in sorted(CONFIGS):
+        cfg = CONFIGS[cid]
+        x = make_round_inputs(cfg, device=dev)
+        ws = rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype, device=dev)
+        out = rt.RoundBuffers(cfg.B, cfg.K, cfg.d, cfg.torch_dtype, device=dev)
+
+        def verify():
+            rt.retrace_verify(x["logits"], x["draft"], out.accept_len, out.committed, out.bonus, ws)
+
+        def round_():
+            rt.run_round(x, ws, out=out)
+
+        v = {"cold": timed(verify, True), "warm": timed(verify, False)}
+        r = {"cold": timed(round_, True), "warm": timed(round_, False)}
+        graph = None
+        if cfg.B <= 8:
+            s = torch.cuda.Stream(dev)
+            s.wait_stream(torch.cuda.current_stream(dev))
+            with torch.cuda.stream(s):
+                rt.run_round(x, ws, out=out, stream=s)
+            torch.cuda.current_stream(dev).wait_stream(s)
+            torch.cuda.synchronize(dev)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s):
+                rt.run_round(x, ws, out=out, stream=s)
+            graph = {"cold": timed(g.replay, True), "warm": timed(g.replay, False)}
+        round_()
+        torch.cuda.synchronize(dev)
+        A = out.accept_len.cpu().numpy().astype(np.int64)
+        n = out.n.cpu().numpy().astype(np.int64)
+        s_b = cfg.elem_bytes
+        logits = cfg.logits_bytes()
+        needed = int(np.sum(np.minimum(A, cfg.K) + 1)) * cfg.V * s_b
+        line = {
+            "config": cid, "workload": cfg.name, "B": cfg.B, "K": cfg.K, "V": cfg.V, "d": cfg.d,
+            "dtype": cfg.dtype, "conditioned_rows_R": int(n.sum()), "iters": iters, "statistic": "median",
+            "verify_us": {k: round(t, 2) for k, t in v.items()},
+            "logits_gbs": {k: round(logits / t / 1e3, 1) for k, t in v.items()},
+            "logits_frac_of_hbm": {k: round(logits / t / 1e3 / peaks["hbm_gbs"], 4) for k, t in v.items()},
+            "round_us": {k: round(t, 2) for k, t in r.items()},
+            "rounds_per_s": {k: round(1e6 / t, 1) for k, t in r.items()},
+            "graph_round_us": None if graph is None else {k: round(t, 2) for k, t in graph.items()},
+            "logits_bytes": logits,
+            "needed_bytes_rows_to_first_mismatch": needed,
+            "needed_us_at_hbm_peak": round(needed / (peaks["hbm_gbs"] * 1e3), 2),
+            "hbm_peak_gbs": peaks["hbm_gbs"], "peak_source": peaks["source"],
+        }
+        print(json.dumps(line), flush=True)
+        del x, ws, out
+        torch.cuda.empty_cache()
+
+
 def workload(name: str) -> RoundConfig:
     return PROFILE_CONFIG if name == "profile" else CONFIGS[int(name)]
 
@@ -642,6 +724,9 @@ def parse_args(argv=None):
                     help="time the low-rank conditioning path (retrace_round_lowrank)")
     ap.add_argument("--variant", choices=sorted(VARIANT_FLAGS), default="corrected",
                     help="conditioning variant of the component ablation (default: the method)")
+    ap.add_argument("--sweep", action="store_true",
+                    help="report every workload (1-5): verification and round, cold and warm medians, "
+                         "graph replay for B <= 8; one JSON line each (not the benchmark line)")
     return ap.parse_args(argv)
 
 
@@ -649,6 +734,9 @@ def main(argv=None) -> None:
     args = parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    if args.sweep:
+        run_sweep(args)
+        return
     line = run_reference(args) if args.impl == "reference" else run_gpu(args)
     if line is not None:
         print(json.dumps(line), flush=True)
