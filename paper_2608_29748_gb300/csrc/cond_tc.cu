@@ -209,7 +209,8 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 constexpr int TILE_SLOTS = 2;
 
 // One warp: rows i of ge = W_g[:, :d] e (broadcast e), claimed from a global
-// counter until all d rows are taken; each finished row is counted.
+// counter until all d rows are taken; each finished row is counted.  Eight
+// 16-byte loads per lane are in flight (d a multiple of 8).
 __device__ void gate_bias_rows(const CondParams& p, int d, int lane, uint32_t* next, uint32_t* done) {
   const int vpr = d / 8;
   const uint4* ev = reinterpret_cast<const uint4*>(p.e);
@@ -220,13 +221,25 @@ __device__ void gate_bias_rows(const CondParams& p, int d, int lane, uint32_t* n
     if (i >= d) break;
     const uint4* wr = reinterpret_cast<const uint4*>(p.Wg + (long long)i * 2 * d);
     float acc = 0.f;
-    for (int v = lane; v < vpr; v += 32) {
-      const uint4 w = __ldcs(wr + v), x = __ldg(ev + v);
-      const uint32_t ww[4] = {w.x, w.y, w.z, w.w}, xx[4] = {x.x, x.y, x.z, x.w};
+    for (int v0 = 0; v0 < vpr; v0 += 8 * 32) {
+      uint4 w[8];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        acc = fmaf(bf16_lo(ww[q]), bf16_lo(xx[q]), acc);
-        acc = fmaf(bf16_hi(ww[q]), bf16_hi(xx[q]), acc);
+      for (int u = 0; u < 8; ++u) {
+        const int v = v0 + u * 32 + lane;
+        w[u] = v < vpr ? __ldcs(wr + v) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int v = v0 + u * 32 + lane;
+        if (v < vpr) {
+          const uint4 x = __ldg(ev + v);
+          const uint32_t ww[4] = {w[u].x, w[u].y, w[u].z, w[u].w}, xx[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            acc = fmaf(bf16_lo(ww[q]), bf16_lo(xx[q]), acc);
+            acc = fmaf(bf16_hi(ww[q]), bf16_hi(xx[q]), acc);
+          }
+        }
       }
     }
 #pragma unroll
@@ -660,6 +673,8 @@ __global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&bar_tempty[acc]));
     }
+    // out of tiles: help finish W_g[:, :d] e (the rows left on the counter)
+    if (!FUSED && need_ge && !s_abort) gate_bias_rows(p, d, lane, gemv_next, gemv_done);
   }
   // ---------------- teardown ----------------
   tc_fence_before();
@@ -1045,6 +1060,8 @@ __global__ void __launch_bounds__(P_THREADS, 1)
         else mbar_arrive_remote(leader_addr(&bar_tempty[acc]));
       }
     }
+    // out of tiles: help finish W_g[:, :d] e (the rows left on the counter)
+    if (need_ge && !s_abort) gate_bias_rows(p, d, lane, gemv_next, gemv_done);
   }
   // ---------------- teardown ----------------
   tc_fence_before();
@@ -1167,6 +1184,8 @@ static int pair_clusters(const TcCondArgs& a, long long tiles_max_pairs, cudaErr
   }
   const int n = max_clusters[dev & 63];
   if (n <= 0) return 0;
+  // every pair when the gate-bias GEMV is needed: pairs without tiles compute it
+  if (a.do_gate) return n;
   return (int)(tiles_max_pairs < n ? tiles_max_pairs : n);
 }
 
@@ -1220,7 +1239,9 @@ cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream) {
   err = device_info(&info);
   if (err != cudaSuccess) return err;
   const long long tiles_max = (rmax + BM - 1) / BM * ((a.do_correct ? a.d / 256 : 0) + (a.do_gate ? a.d / 128 : 0));
-  const unsigned grid = (unsigned)(tiles_max < info.sm_count ? tiles_max : info.sm_count);
+  // every SM when the broadcast-e GEMV is needed: CTAs without tiles compute it
+  const bool need_ge = a.do_gate && !a.e_dense;
+  const unsigned grid = (unsigned)(need_ge || tiles_max >= info.sm_count ? info.sm_count : tiles_max);
   VerifyStreamParams vp{};
   cond_kernel<false><<<grid, THREADS, SMEM_BYTES, stream>>>(mApack, mWc, mR, mE, mWv, mWg, p, vp);
   return cudaGetLastError();
