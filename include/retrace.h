@@ -309,6 +309,23 @@ retrace_status retrace_round_lowrank(const void* logits, int64_t logits_row_stri
                                      size_t ws_bytes, const cudaEvent_t* phase_events,
                                      cudaStream_t stream);
 
+/* Self-test of the bounded device waits.  The pipelined tensor-core kernels
+ * wait on mbarrier phases and on counters that other CTAs raise, and none of
+ * those waits may spin forever: each gives up after about one second, sets
+ * bit 0 of the workspace status word (reported by retrace_workspace_check),
+ * and its kernel returns normally, so the CUDA context stays usable.  This
+ * call runs the same wait code in one thread on a condition the caller
+ * controls:
+ *   kind 0  waits until the device word *flag >= target (the counter wait);
+ *   kind 1  waits for an mbarrier phase that completes only if target == 0
+ *           (the phase wait; flag is not read and may be NULL).
+ * A condition that is already met returns at once; one that never becomes
+ * true takes the full bound and sets the flag.  Only the status word of `ws`
+ * (at least 256 bytes, 256-byte aligned) is written; call
+ * retrace_workspace_init before reusing the workspace after a set flag. */
+retrace_status retrace_wait_selftest(int kind, const uint32_t* flag, uint32_t target, void* ws, size_t ws_bytes,
+                                     cudaStream_t stream);
+
 /* Size in bytes of the fixed device scratch used by retrace_verify_noalloc. */
 #define RETRACE_NOALLOC_SCRATCH_BYTES 65536
 

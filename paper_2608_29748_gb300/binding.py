@@ -57,11 +57,12 @@ def _load() -> ctypes.CDLL:
     lib.retrace_round_lowrank.argtypes = [P, I64, I64, P, P, P, P, P, P, P, P, P, F, I, I, I, I, I,
                                           P, P, P, P, P, P, P, SZ, P, P]
     lib.retrace_verify_sampled.argtypes = [P, I64, I64, P, I64, I64, I, I, I, I, P, P, F, I, F, P, P, P, P, SZ, P]
+    lib.retrace_wait_selftest.argtypes = [I, P, ctypes.c_uint32, P, SZ, P]
     lib.retrace_round_sampled.argtypes = [P, I64, I64, P, I64, I64, P, P, F, I, F, P, P, P, I64, I64, P, P, P, F,
                                           I, I, I, I, I, P, P, P, P, P, P, SZ, P, P]
     for name in ("retrace_workspace_init", "retrace_workspace_check", "retrace_verify",
                  "retrace_align_refine", "retrace_gate_fuse", "retrace_round", "retrace_round_lowrank",
-                 "retrace_verify_sampled", "retrace_round_sampled"):
+                 "retrace_verify_sampled", "retrace_round_sampled", "retrace_wait_selftest"):
         getattr(lib, name).restype = I
     return lib
 
@@ -272,6 +273,13 @@ def retrace_round_lowrank(logits, draft, hD, hT, e, P, Bc, Ac, Wv, Wg, beta, acc
                                      ws.ptr, ws.nbytes,
                                      ctypes.cast(ev, ctypes.c_void_p) if ev is not None else None,
                                      _stream(stream)))
+
+
+def retrace_wait_selftest(kind, flag, target, ws, stream=None):
+    """Runs the kernels' bounded wait on a caller-controlled condition (see include/retrace.h)."""
+    if flag is not None and flag.dtype != torch.int32:
+        raise TypeError("flag must be an int32 device tensor")
+    _check(lib.retrace_wait_selftest(int(kind), _ptr(flag), int(target), ws.ptr, ws.nbytes, _stream(stream)))
 
 
 class RoundBuffers:

@@ -516,6 +516,17 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   return RETRACE_OK;
 }
 
+retrace_status retrace_wait_selftest(int kind, const uint32_t* flag, uint32_t target, void* ws, size_t ws_bytes,
+                                    cudaStream_t stream) {
+  g_err[0] = '\0';
+  if (kind != 0 && kind != 1) return fail(RETRACE_ERR_INVALID_ARG, "kind must be 0 (counter) or 1 (mbarrier)");
+  if (kind == 0 && !flag) return fail(RETRACE_ERR_INVALID_ARG, "NULL flag");
+  retrace_status st = check_ws(ws, ws_bytes, 256);
+  if (st != RETRACE_OK) return st;
+  RT_CUDA(launch_wait_selftest(kind, flag, target, status_word(ws), stream), "wait self-test launch");
+  return RETRACE_OK;
+}
+
 retrace_status retrace_verify_sampled(const void* target_logits, int64_t target_row_stride,
                                       int64_t target_batch_stride, const void* draft_logits,
                                       int64_t draft_row_stride, int64_t draft_batch_stride,

@@ -1073,6 +1073,28 @@ __global__ void __launch_bounds__(P_THREADS, 1)
   }
 }
 
+// One thread runs the pipelined kernels' bounded waits on a condition the
+// caller controls (retrace_wait_selftest): kind 0 waits until *flag >= target
+// (the counter wait), kind 1 for an mbarrier phase that completes only if
+// target == 0 (the phase wait).  An expired wait sets the status flag, as in
+// the kernels, and the kernel returns.
+__global__ void wait_selftest_kernel(int kind, const uint32_t* flag, uint32_t target, uint32_t* status) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ volatile int s_abort;
+  if (threadIdx.x != 0) return;
+  s_abort = 0;
+  bool ok;
+  if (kind == 0) {
+    ok = wait_counter(flag, target, &s_abort);
+  } else {
+    mbar_init(smem_u32(&bar), 1);
+    fence_mbar_init();
+    if (target == 0) mbar_arrive(smem_u32(&bar));  // phase 0 completes: the wait returns at once
+    ok = mbar_wait_bounded(smem_u32(&bar), 0, &s_abort);
+  }
+  if (!ok) atomicOr(status, kFlagWaitTimeout);
+}
+
 template <bool FUSED>
 cudaError_t ensure_smem_attr() {
   static int done[64] = {0};
@@ -1089,6 +1111,12 @@ cudaError_t ensure_smem_attr() {
 }
 
 }  // namespace
+
+cudaError_t launch_wait_selftest(int kind, const uint32_t* flag, uint32_t target, uint32_t* status,
+                                 cudaStream_t stream) {
+  wait_selftest_kernel<<<1, 32, 0, stream>>>(kind, flag, target, status);
+  return cudaGetLastError();
+}
 
 bool tc_supported(retrace_dtype dtype, int d) {
   return dtype == RETRACE_BF16 && d >= 256 && d % 256 == 0;

@@ -283,6 +283,9 @@ struct TcCondArgs {
   uint32_t* status;
 };
 cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream);
+// The bounded waits of the pipelined kernels on a caller-controlled condition.
+cudaError_t launch_wait_selftest(int kind, const uint32_t* flag, uint32_t target, uint32_t* status,
+                                 cudaStream_t stream);
 
 // Low-rank conditioning (rank-64 latents, rank-32 correction; broadcast e).
 struct LowRankArgs {

@@ -182,6 +182,14 @@ def test_sampled_round_argument_errors(lib):
     assert call(B=0) == OK
 
 
+def test_wait_selftest_argument_errors(lib):
+    P, U32 = ctypes.c_void_p, ctypes.c_uint32
+    assert lib.retrace_wait_selftest(2, P(16), U32(1), P(256), ctypes.c_size_t(1 << 20), None) == INVALID
+    assert lib.retrace_wait_selftest(0, None, U32(1), P(256), ctypes.c_size_t(1 << 20), None) == INVALID
+    assert lib.retrace_wait_selftest(1, None, U32(1), P(256), ctypes.c_size_t(64), None) == WORKSPACE
+    assert lib.retrace_wait_selftest(1, None, U32(1), P(100), ctypes.c_size_t(1 << 20), None) == WORKSPACE
+
+
 def test_lowrank_round_argument_errors(lib):
     P, I64 = ctypes.c_void_p, ctypes.c_int64
 
