@@ -134,6 +134,29 @@ retrace_status retrace_verify(const void* logits, retrace_dtype dtype, int B, in
                               int32_t* bonus, int32_t* target_argmax, void* ws,
                               size_t ws_bytes, cudaStream_t stream);
 
+/* Schedules of greedy verification (every entry point that verifies greedily).
+ * They differ in the rows they read, never in the results.
+ *   RETRACE_VERIFY_FULL     one pass over every row of every sequence.
+ *   RETRACE_VERIFY_WINDOWS  passes over windows of 4 rows (more for long
+ *                           blocks, at most 16 passes): pass k reads rows
+ *                           [4k, 4k+4) of the sequences whose draft tokens
+ *                           matched every earlier row, so rows past the first
+ *                           mismatch's window are never read.  Applies when
+ *                           target_argmax is NULL (every row is an output
+ *                           otherwise) and K+1 > 4; other calls take the full
+ *                           pass.
+ *   RETRACE_VERIFY_AUTO     (default) WINDOWS where it applies and one row of
+ *                           the whole batch is at least 32 MiB (B * V *
+ *                           element size), FULL otherwise (each extra pass
+ *                           costs a few microseconds, which small batches
+ *                           do not win back).
+ * Process-wide.  Returns the previous mode, or -1 (nothing changes) for an
+ * unknown one. */
+#define RETRACE_VERIFY_AUTO 0
+#define RETRACE_VERIFY_FULL 1
+#define RETRACE_VERIFY_WINDOWS 2
+int retrace_set_verify_schedule(int mode);
+
 /* Rejected-trajectory alignment and target-aware correction (Eq. 3-7,
  * Algorithm 1 carry/reset steps).
  *   hD, hT      [B, K, d] of `dtype`, contiguous.

@@ -58,11 +58,13 @@ def _load() -> ctypes.CDLL:
                                           P, P, P, P, P, P, P, SZ, P, P]
     lib.retrace_verify_sampled.argtypes = [P, I64, I64, P, I64, I64, I, I, I, I, P, P, F, I, F, P, P, P, P, SZ, P]
     lib.retrace_wait_selftest.argtypes = [I, P, ctypes.c_uint32, P, SZ, P]
+    lib.retrace_set_verify_schedule.argtypes = [I]
     lib.retrace_round_sampled.argtypes = [P, I64, I64, P, I64, I64, P, P, F, I, F, P, P, P, I64, I64, P, P, P, F,
                                           I, I, I, I, I, P, P, P, P, P, P, SZ, P, P]
     for name in ("retrace_workspace_init", "retrace_workspace_check", "retrace_verify",
                  "retrace_align_refine", "retrace_gate_fuse", "retrace_round", "retrace_round_lowrank",
-                 "retrace_verify_sampled", "retrace_round_sampled", "retrace_wait_selftest"):
+                 "retrace_verify_sampled", "retrace_round_sampled", "retrace_wait_selftest",
+                 "retrace_set_verify_schedule"):
         getattr(lib, name).restype = I
     return lib
 
@@ -309,6 +311,18 @@ def run_round(x: dict, ws: Workspace, out: RoundBuffers | None = None, target_ar
 
 def version() -> str:
     return lib.retrace_version().decode()
+
+
+VERIFY_AUTO, VERIFY_FULL, VERIFY_WINDOWS = 0, 1, 2
+
+
+def retrace_set_verify_schedule(mode: int) -> int:
+    """Selects the greedy verification schedule (VERIFY_AUTO / VERIFY_FULL /
+    VERIFY_WINDOWS); returns the previous one."""
+    prev = lib.retrace_set_verify_schedule(int(mode))
+    if prev < 0:
+        raise RetraceError(1, f"unknown verification schedule {mode}")
+    return prev
 
 
 def run_round_lowrank(x: dict, w: dict, ws: Workspace, out: RoundBuffers | None = None, target_argmax=None,

@@ -134,6 +134,14 @@ retrace_status e_mode(int64_t ebs, int64_t eps, int K, int d, int* dense) {
 
 uint32_t* status_word(void* ws) { return reinterpret_cast<uint32_t*>(ws); }
 
+// Workspace pointers of the greedy verification kernels.
+void verify_workspace(VerifyArgs* a, char* w, const WsLayout& L) {
+  a->keys = reinterpret_cast<unsigned long long*>(w + L.keys);
+  a->tickets = reinterpret_cast<uint32_t*>(w + L.tickets);
+  a->live = reinterpret_cast<int32_t*>(w + L.live);
+  a->pass_counts = reinterpret_cast<uint32_t*>(w + L.counts);
+}
+
 
 retrace_status check_sampling(int B, int K, int V, const void* draft_logits, int64_t draft_row_stride,
                               int64_t draft_batch_stride, const float* uniforms, float temperature, int top_k,
@@ -226,6 +234,8 @@ const char* retrace_last_error(void) { return g_err; }
 
 const char* retrace_version(void) { return "retrace 0.1.0 sm_103a"; }
 
+int retrace_set_verify_schedule(int mode) { return set_verify_schedule(mode); }
+
 size_t retrace_workspace_bytes(int B, int K, int V, int d, retrace_dtype dtype) {
   if (B < 0 || K < 0 || V < 1 || d < 0 || !dtype_ok(dtype)) return 0;
   return ws_layout(B, K, d, elem_size(dtype)).total;
@@ -271,8 +281,7 @@ retrace_status retrace_verify(const void* logits, retrace_dtype dtype, int B, in
   a.committed = committed;
   a.bonus = bonus;
   a.target_argmax = target_argmax;
-  a.keys = reinterpret_cast<unsigned long long*>((char*)ws + L.keys);
-  a.tickets = reinterpret_cast<uint32_t*>((char*)ws + L.tickets);
+  verify_workspace(&a, reinterpret_cast<char*>(ws), L);
   RT_CUDA(launch_verify(a, dtype, stream), "verify kernel launch");
   return RETRACE_OK;
 }
@@ -479,8 +488,7 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   va.bonus = bonus;
   va.target_argmax = target_argmax;
   va.n_out = n_out;
-  va.keys = reinterpret_cast<unsigned long long*>(w + L.keys);
-  va.tickets = reinterpret_cast<uint32_t*>(w + L.tickets);
+  verify_workspace(&va, w, L);
   va.e = e;
   va.e_batch_stride = e_batch_stride;
   va.e_pos_stride = e_pos_stride;
@@ -685,8 +693,7 @@ retrace_status retrace_round_lowrank(const void* logits, int64_t logits_row_stri
   va.bonus = bonus;
   va.target_argmax = target_argmax;
   va.n_out = n_out;
-  va.keys = reinterpret_cast<unsigned long long*>(w + Lw.keys);
-  va.tickets = reinterpret_cast<uint32_t*>(w + Lw.tickets);
+  verify_workspace(&va, w, Lw);
   va.e = e;
   va.e_batch_stride = 0;
   va.e_pos_stride = 0;

@@ -20,6 +20,9 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 //                               gate-bias progress, per-128-row-block progress)
 //   keys     uint64 [B*(K+1)]   per-row argmax keys, zero between calls
 //   tickets  uint32 [B]         per-sequence CTA arrival counters, zero between calls
+//   live     int32  [2*B]       windowed verification: live sequence lists of two passes
+//   counts   uint32 [1+passes]  windowed verification: [0] CTAs out of the last pass,
+//                               [k] sequences live into pass k; zero between calls
 //   ge       fp32   [d]         W_g[:, :d] e for a broadcast e
 //   r        elem   [R_max, d]  compacted corrected signal, R_max = B*(K-1)
 //   apack    elem   [R_max, 2d] packed [m; u] rows (tensor-core path)
@@ -33,8 +36,10 @@ constexpr int kLowRankCorrection = 32;  // rank of the target-aware correction
 constexpr int kLowRankSplits = 8;       // split-K parts per half of the [m; u] reduction
 //   skeys    uint64 [B*(2K+1), 64]  sampled verification: top-k keys per target and drafter row
 constexpr int kMaxTopK = 64;            // largest top_k of sampled verification
+constexpr int kWindowRows = 4;          // rows per pass of windowed verification
+constexpr int kMaxWindowPasses = 16;    // most passes of windowed verification
 struct WsLayout {
-  size_t status, sync, sync_bytes, keys, tickets, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, skeys, total;
+  size_t status, sync, sync_bytes, keys, tickets, live, counts, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, skeys, total;
 };
 
 inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
@@ -52,6 +57,10 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   off = align_up(off + (size_t)(B * (K + 1)) * 8, 256);
   L.tickets = off;
   off = align_up(off + (size_t)B * 4, 256);
+  L.live = off;
+  off = align_up(off + (size_t)B * 2 * 4, 256);
+  L.counts = off;
+  off = align_up(off + (size_t)(kMaxWindowPasses + 1) * 4, 256);
   L.ge = off;
   off = align_up(off + dd * 4, 256);
   L.r = off;
@@ -137,6 +146,10 @@ struct VerifyArgs {
   void* epack;     // [R_max, d]: e rows (dense e only)
   int32_t* rowmap; // [R_max]: packed row -> b*K + j
   int32_t* R_count;
+  // Windowed schedule (NULL live: one pass over every row only): two live
+  // lists of B sequences and the passes' counters, from the workspace.
+  int32_t* live;
+  uint32_t* pass_counts;
   // Rows j < n_b of e_out in the copy above (no packing then): kCondCopyKeep
   // leaves them to the conditioning kernels, kCondCopyE writes e (no
   // conditioning), kCondCopyM writes m_j = hD[b, A_b+1+j] (overwrite).
@@ -146,6 +159,7 @@ constexpr int kCondCopyKeep = 0;
 constexpr int kCondCopyE = 1;
 constexpr int kCondCopyM = 2;
 cudaError_t launch_verify(const VerifyArgs& a, retrace_dtype dtype, cudaStream_t stream);
+int set_verify_schedule(int mode);  // RETRACE_VERIFY_*; previous mode, or -1
 
 // Stochastic verification (speculative sampling on top-k / top-p filtered
 // distributions at temperature T).

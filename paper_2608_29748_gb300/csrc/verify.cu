@@ -11,6 +11,17 @@
 // finds the first mismatch with a warp ballot and writes the accepted length,
 // committed tokens and bonus, resets the keys and ticket to zero for the next
 // call and, inside a fused round, copies the unconditioned drafter inputs.
+//
+//
+// The outputs depend only on rows 0..A_b of each sequence.  The windowed
+// schedule runs the same kernel as a chain of passes over row windows
+// [i0, i1): the finaliser of a sequence whose draft tokens matched every row
+// of the window appends it to the next pass's live list instead of
+// finalising it, and the next pass (launched programmatically dependent)
+// streams only the listed sequences' rows.  Rows past the window holding the
+// first mismatch are never read.  Same keys, same finaliser, same results.
+#include <atomic>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -46,6 +57,16 @@ struct VerifyParams {
   int32_t* rowmap;
   int32_t* R_count;
   int cond_copy;
+  // Row window of this pass (windowed schedule; [0, K+1) in one pass).
+  int i0, i1;
+  const int32_t* live_in;    // sequences of this pass (NULL: 0..B-1)
+  const uint32_t* count_in;  // their number, written by the previous pass (NULL: B)
+  int32_t* live_out;         // sequences that matched every row of the window (NULL: last pass)
+  uint32_t* count_out;
+  uint32_t* pass_counts;     // last pass: counters of every pass, zeroed by its last CTA out
+  int n_counts;
+  uint32_t* exits;           // last pass: CTAs out (zero between calls)
+  int defer_copies;          // the finaliser leaves the copies to verify_copy_kernel
 };
 
 // 16-byte vector helpers: the maximum of the vector's elements and element q.
@@ -219,18 +240,59 @@ __device__ void pack_sequence_rows(const VerifyParams& p, int b, int A, int nb, 
   }
 }
 
+// Copies of sequence b once A is known: the unconditioned rows of e_out and
+// the packing of the conditioned ones (in a fused round).
+template <typename T>
+__device__ void copy_sequence(const VerifyParams& p, int b, int A, int* s_off, uint4* staging) {
+  const int nb = (p.K - 1 - A) > 0 ? (p.K - 1 - A) : 0;
+  if (p.e_out) {
+    if (p.cond_copy == kCondCopyKeep) copy_rows<T>(p, b, A, nb, 0, staging);
+    else if (p.cond_copy == kCondCopyE) copy_rows<T>(p, b, A, 0, 0, staging);
+    else copy_rows<T>(p, b, A, 0, nb, staging);
+  }
+  if (p.R_count && nb > 0) pack_sequence_rows(p, b, A, nb, s_off, staging);
+}
+
+// Outputs of sequence b once its accepted length A and the argmaxes s_t[0..A]
+// are known: committed tokens, accepted length, bonus, n_b and (unless a
+// later kernel does them) the copies.  The argmax keys of rows 0..rows-1 are
+// reset for the next call.
+template <typename T>
+__device__ void finish_sequence(const VerifyParams& p, int b, int A, int rows, const int* s_t, int* s_off,
+                                uint4* staging) {
+  const int K = p.K, K1 = K + 1;
+  for (int i = threadIdx.x; i < K1; i += kThreads) {
+    const long long o = (long long)b * K1 + i;
+    p.committed[o] = (i <= A) ? s_t[i] : -1;
+    if (p.target_argmax) p.target_argmax[o] = s_t[i];
+    if (i < rows) p.keys[o] = 0ull;
+  }
+  const int nb = (K - 1 - A) > 0 ? (K - 1 - A) : 0;
+  if (threadIdx.x == 0) {
+    p.accept_len[b] = A;
+    p.bonus[b] = s_t[A];
+    if (p.n_out) p.n_out[b] = nb;
+  }
+  if (!p.defer_copies) copy_sequence<T>(p, b, A, s_off, staging);
+}
+
+// Every row of sequence b in the window [i0, i1) has its key (rows before
+// i0 matched their draft tokens in earlier passes): the first mismatch in the
+// window by ballot, then the outputs; a sequence without one, when rows
+// remain, goes on to the next pass instead.
 template <typename T>
 __device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s_A, uint4* staging) {
   const int K = p.K, K1 = K + 1;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int i = threadIdx.x; i < K1; i += kThreads)
+  for (int i = threadIdx.x; i < p.i1; i += kThreads)
     s_t[i] = (int)key_index(__ldcg(&p.keys[(long long)b * K1 + i]));
   __syncthreads();
   if (warp == 0) {
-    int A = K;
-    for (int base = 0; base < K; base += 32) {
+    int A = p.i1 == K1 ? K : -1;  // -1: every row of the window matched, more rows to read
+    const int hi = min(p.i1, K);
+    for (int base = p.i0; base < hi; base += 32) {
       const int i = base + lane;
-      const bool mismatch = (i < K) && (s_t[i] != p.draft[(long long)b * K + i]);
+      const bool mismatch = (i < hi) && (s_t[i] != p.draft[(long long)b * K + i]);
       const unsigned bal = __ballot_sync(0xFFFFFFFFu, mismatch);
       if (bal) {
         A = base + __ffs(bal) - 1;
@@ -241,25 +303,11 @@ __device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s
   }
   __syncthreads();
   const int A = *s_A;
-  for (int i = threadIdx.x; i < K1; i += kThreads) {
-    const long long o = (long long)b * K1 + i;
-    p.committed[o] = (i <= A) ? s_t[i] : -1;
-    if (p.target_argmax) p.target_argmax[o] = s_t[i];
-    p.keys[o] = 0ull;
-  }
-  const int nb = (K - 1 - A) > 0 ? (K - 1 - A) : 0;
   if (threadIdx.x == 0) {
-    p.accept_len[b] = A;
-    p.bonus[b] = s_t[A];
-    if (p.n_out) p.n_out[b] = nb;
     p.tickets[b] = 0u;
+    if (A < 0) p.live_out[atomicAdd(p.count_out, 1u)] = b;
   }
-  if (p.e_out) {
-    if (p.cond_copy == kCondCopyKeep) copy_rows<T>(p, b, A, nb, 0, staging);
-    else if (p.cond_copy == kCondCopyE) copy_rows<T>(p, b, A, 0, 0, staging);
-    else copy_rows<T>(p, b, A, 0, nb, staging);
-  }
-  if (p.R_count && nb > 0) pack_sequence_rows(p, b, A, nb, s_A + 1, staging);
+  if (A >= 0) finish_sequence<T>(p, b, A, p.i1, s_t, s_A + 1, staging);
 }
 
 template <typename T, bool VEC>
@@ -271,34 +319,42 @@ __global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams 
   extern __shared__ uint4 s_stage[];  // kCopyStage * kThreads vectors: row copies of the finaliser
   pdl_launch_dependents();  // the next kernel may take SMs as this grid's CTAs finish
 
-  const long long T_ = p.total_slots;
-  const long long G = gridDim.x;
-  const long long c = blockIdx.x;
-  const long long s_begin = c * T_ / G, s_end = (c + 1) * T_ / G;
+  long long n_live = p.B;
+  if (p.count_in) {  // a later pass: the previous pass wrote the live list
+    pdl_wait();
+    n_live = (long long)__ldcg(p.count_in);
+  }
   const long long VV = p.slots_per_row;
-  const int K1 = p.K + 1;
-  const long long per_seq = (long long)K1 * VV;
+  const int K1 = p.K + 1, W = p.i1 - p.i0;
+  const long long per_seq = (long long)W * VV;
+  const long long T_ = n_live * per_seq;
+  // Active CTAs: at least ~32 KB of logits each, no more than there are slots.
+  const long long by_bytes = (T_ * (VEC ? 16 : (long long)sizeof(T)) + 32767) / 32768;
+  const long long G = min((long long)gridDim.x, min(by_bytes, T_));
+  const long long c = blockIdx.x;
 
-  long long s = s_begin;
+  long long s = c < G ? c * T_ / G : 0;
+  const long long s_end = c < G ? (c + 1) * T_ / G : 0;
   while (s < s_end) {
-    const long long row = s / VV;
-    const int b = (int)(row / K1);
-    const int i = (int)(row - (long long)b * K1);
-    const long long seg_end = min(s_end, (row + 1) * VV);
-    const int v0 = (int)(s - row * VV), v1 = (int)(seg_end - row * VV);
+    const long long vrow = s / VV;  // row of the pass: sequence vrow / W, window row vrow % W
+    const long long l = vrow / W;
+    const int b = p.live_in ? __ldg(p.live_in + l) : (int)l;
+    const int i = p.i0 + (int)(vrow - l * W);
+    const long long seg_end = min(s_end, (vrow + 1) * VV);
+    const int v0 = (int)(s - vrow * VV), v1 = (int)(seg_end - vrow * VV);
     const T* rowp = reinterpret_cast<const T*>(p.logits) + (long long)b * p.batch_stride +
                     (long long)i * p.row_stride;
 
     unsigned long long key = segment_key<T, VEC>(rowp, v0, v1, p.V);
     key = block_max_key(key, s_red);
-    if (threadIdx.x == 0) atomicMax(&p.keys[row], key);
+    if (threadIdx.x == 0) atomicMax(&p.keys[(long long)b * K1 + i], key);
     s = seg_end;
 
     if (s == s_end || s % per_seq == 0) {
       // This CTA has folded in all of its rows of sequence b.  The CTAs that
       // own slots of b are those from the owner of its first slot to the
-      // owner of its last (every CTA range is non-empty: G <= total slots).
-      const long long first = (long long)b * per_seq, last = first + per_seq - 1;
+      // owner of its last (every active CTA range is non-empty: G <= T_).
+      const long long first = l * per_seq, last = first + per_seq - 1;
       const long long c_first = ((first + 1) * G - 1) / T_;
       const long long c_last = ((last + 1) * G - 1) / T_;
       const uint32_t count = (uint32_t)(c_last - c_first + 1);
@@ -315,6 +371,51 @@ __global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams 
       __syncthreads();
     }
   }
+  // The last pass's last CTA out zeroes the passes' live counters.
+  if (p.exits && threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(p.exits, 1u) == gridDim.x - 1u) {
+      for (int k = 0; k < p.n_counts; ++k) p.pass_counts[k] = 0u;
+      *p.exits = 0u;
+    }
+  }
+}
+
+// The copies of a windowed verification, after its last pass: one sequence
+// per CTA at a time (accept_len holds every A_b by then).
+template <typename T>
+__global__ void __launch_bounds__(kThreads, 2) verify_copy_kernel(const VerifyParams p) {
+  __shared__ int s_off;
+  extern __shared__ uint4 s_stage[];
+  pdl_launch_dependents();
+  pdl_wait();
+  for (int b = blockIdx.x; b < p.B; b += gridDim.x) {
+    const int A = __ldcg(p.accept_len + b);
+    copy_sequence<T>(p, b, A, &s_off, s_stage);
+    __syncthreads();
+  }
+}
+
+std::atomic<int> g_schedule{RETRACE_VERIFY_AUTO};
+constexpr long long kWindowMinBatchRowBytes = 32ll << 20;  // B * V * element size
+
+// Row windows of the windowed schedule: the first kWindowRows rows, then
+// windows half as long again as the one before (fewer, longer passes as the
+// live sequences thin out), the last one stretched to row K when what would
+// remain is shorter than half a window.  Writes the window starts (n + 1
+// entries, the last = K1) and returns the number of passes n (1: one window
+// holds every row).
+inline int window_bounds(int K1, int* start) {
+  int n = 0, i = 0, w = kWindowRows;
+  start[0] = 0;
+  while (i < K1 && n < kMaxWindowPasses) {
+    int e = i + w;
+    if (e >= K1 || 2 * (K1 - e) < w || n == kMaxWindowPasses - 1) e = K1;
+    start[++n] = e;
+    i = e;
+    w += w / 2;
+  }
+  return n;
 }
 
 template <typename T, bool VEC>
@@ -362,19 +463,85 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
   p.rowmap = a.rowmap;
   p.R_count = a.R_count;
   p.cond_copy = a.cond_copy;
-  // Enough CTAs to fill every SM at full occupancy, but at least ~32 KB of
-  // logits per CTA so that small batches do not pay for idle CTAs.
-  const long long bytes = (long long)a.B * (a.K + 1) * a.V * (long long)sizeof(T);
-  long long grid = (long long)info.sm_count * occ;
-  const long long by_bytes = (bytes + 32767) / 32768;
-  if (by_bytes < grid) grid = by_bytes;
-  if (grid > p.total_slots) grid = p.total_slots;
-  if (grid < 1) grid = 1;
-  verify_kernel<T, VEC><<<(unsigned)grid, kThreads, kCopyStageBytes, stream>>>(p);
-  return cudaGetLastError();
+  p.i0 = 0;
+  p.i1 = a.K + 1;
+  p.live_in = nullptr;
+  p.count_in = nullptr;
+  p.live_out = nullptr;
+  p.count_out = nullptr;
+  p.pass_counts = nullptr;
+  p.n_counts = 0;
+  p.exits = nullptr;
+  p.defer_copies = 0;
+  const int K1 = a.K + 1;
+  int start[kMaxWindowPasses + 1];
+  const int n_pass = window_bounds(K1, start);
+  const int mode = g_schedule.load(std::memory_order_relaxed);
+  const long long wave = (long long)a.B * a.V * (long long)sizeof(T);
+  const bool windowed = a.live && !a.target_argmax && n_pass > 1 &&
+                        (mode == RETRACE_VERIFY_WINDOWS || (mode == RETRACE_VERIFY_AUTO && wave >= kWindowMinBatchRowBytes));
+  const long long grid_full = (long long)info.sm_count * occ;
+  if (!windowed) {
+    // Enough CTAs to fill every SM at full occupancy, but at least ~32 KB of
+    // logits per CTA so that small batches do not pay for idle CTAs (the
+    // kernel trims its active CTAs the same way).
+    const long long bytes = (long long)a.B * K1 * a.V * (long long)sizeof(T);
+    long long grid = grid_full;
+    const long long by_bytes = (bytes + 32767) / 32768;
+    if (by_bytes < grid) grid = by_bytes;
+    if (grid > p.total_slots) grid = p.total_slots;
+    if (grid < 1) grid = 1;
+    verify_kernel<T, VEC><<<(unsigned)grid, kThreads, kCopyStageBytes, stream>>>(p);
+    return cudaGetLastError();
+  }
+  // Windowed: pass k reads rows [start[k], start[k+1]) of the sequences that
+  // matched every earlier row; each pass after the first waits for its
+  // predecessor inside the kernel (programmatic dependent launch) and sizes
+  // its work from the live count that pass wrote.  The copies of a fused
+  // round follow in one more kernel, balanced over sequences.
+  const bool copies = a.e_out || a.R_count;
+  p.defer_copies = copies ? 1 : 0;
+  for (int k = 0; k < n_pass; ++k) {
+    const bool last = k == n_pass - 1;
+    p.i0 = start[k];
+    p.i1 = start[k + 1];
+    p.live_in = k == 0 ? nullptr : a.live + (size_t)((k - 1) & 1) * a.B;
+    p.count_in = k == 0 ? nullptr : a.pass_counts + k;
+    p.live_out = last ? nullptr : a.live + (size_t)(k & 1) * a.B;
+    p.count_out = last ? nullptr : a.pass_counts + k + 1;
+    p.pass_counts = last ? a.pass_counts + 1 : nullptr;
+    p.n_counts = last ? n_pass - 1 : 0;
+    p.exits = last ? a.pass_counts : nullptr;
+    if (k == 0) {
+      verify_kernel<T, VEC><<<(unsigned)grid_full, kThreads, kCopyStageBytes, stream>>>(p);
+      err = cudaGetLastError();
+    } else {
+      err = launch_dependent(verify_kernel<T, VEC>, dim3((unsigned)grid_full), dim3(kThreads), kCopyStageBytes,
+                             stream, 1u, p);
+    }
+    if (err != cudaSuccess) return err;
+  }
+  if (copies) {
+    static int copy_attr[64] = {0};
+    if (!copy_attr[info.device & 63]) {
+      err = cudaFuncSetAttribute(verify_copy_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, kCopyStageBytes);
+      if (err != cudaSuccess) return err;
+      copy_attr[info.device & 63] = 1;
+    }
+    const long long grid = a.B < grid_full ? a.B : grid_full;
+    err = launch_dependent(verify_copy_kernel<T>, dim3((unsigned)grid), dim3(kThreads), kCopyStageBytes, stream, 1u,
+                           p);
+    if (err != cudaSuccess) return err;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace
+
+int set_verify_schedule(int mode) {
+  if (mode != RETRACE_VERIFY_AUTO && mode != RETRACE_VERIFY_FULL && mode != RETRACE_VERIFY_WINDOWS) return -1;
+  return g_schedule.exchange(mode);
+}
 
 cudaError_t launch_verify(const VerifyArgs& a, retrace_dtype dtype, cudaStream_t stream) {
   const size_t es = dtype == RETRACE_BF16 ? 2 : 4;
