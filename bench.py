@@ -50,15 +50,16 @@ from paper_2608_29748_gb300.workloads import CONFIGS, PROFILE_CONFIG, RoundConfi
 METRIC = "verify+ReTrace rounds/sec at 1 GB300; logits HBM GB/s and % of roofline"
 UNIT = "rounds/s"
 KERNELS_PER_ROUND_FUSED = 1  # cond_kernel<FUSED>: the whole round
-KERNELS_PER_ROUND = 2  # verify_kernel (+ row packing), cond_kernel (both projections + gate-bias GEMV)
+KERNELS_PER_ROUND = 2  # one-pass verify_kernel (+ row packing), cond_kernel (both projections + gate-bias GEMV)
 L2_FLUSH_BYTES = 256 << 20
-# DRAM traffic of one verify_kernel launch per sequence of the serving shapes
-# (K=16, V=151936, d=4096, bf16), measured with ncu (dram__bytes_read.sum +
-# dram__bytes_write.sum) on the 128-sequence profiling workload: 685.66 MB read
-# + 3.10 MB written (the packed rows it writes stay in L2 during the launch).
-# Traffic grows in proportion to the sequences (the logits dominate).  Must be
-# re-measured whenever verify_kernel changes.
-VERIFY_TRAFFIC_PER_SEQUENCE = (685742592 + 2950912) / 128
+# DRAM traffic of the verification kernels of one round per sequence of the
+# serving shapes (K=16, V=151936, d=4096, bf16; windowed schedule), measured
+# with ncu (dram__bytes_read.sum + dram__bytes_write.sum, summed over the
+# passes and the copy kernel) on the 128-sequence profiling workload, whose
+# accepted lengths follow the serving workload's distribution; scaled by
+# B/128 (profiles/verify_windowed_launch_list-B128.md): 285.56 MB at B = 128.
+VERIFY_TRAFFIC_PER_SEQUENCE = 285564928 / 128
+VERIFY_TRAFFIC_PASSES = 3  # the schedule the traffic was measured on (passes of verify_kernel)
 VERIFY_TRAFFIC_SHAPE = (16, 151936, 4096, "bf16")
 # DRAM traffic of the single-kernel round per sequence (same shapes, same
 # profiling workload and method); None until measured for the current kernel.
@@ -250,11 +251,28 @@ VARIANT_FLAGS = {"corrected": 0, "raw": 0x2, "overwrite": 0x4, "none": 0x8}  # i
 ROUND_OVERLAP_FLAG = 0x1
 
 
-def verify_bytes(cfg: RoundConfig, n: np.ndarray, packs_rows: bool, variant: str = "corrected") -> int:
-    """Algorithmic bytes of one verification launch of a round."""
+def needed_logits_bytes(cfg: RoundConfig, accept: np.ndarray) -> int:
+    """Logits the verification outputs depend on: rows 0..A_b of each
+    sequence (the argmaxes of later rows change nothing)."""
+    return int(np.sum(accept.astype(np.int64) + 1)) * cfg.V * cfg.elem_bytes
+
+
+def read_logits_bytes(cfg: RoundConfig, accept: np.ndarray, windows: list[int]) -> int:
+    """Logits a greedy verification schedule streams: window k's rows for the
+    sequences whose draft tokens matched every row before it."""
+    rows = 0
+    for k in range(len(windows) - 1):
+        rows += int(np.sum(accept >= windows[k])) * (windows[k + 1] - windows[k])
+    return rows * cfg.V * cfg.elem_bytes
+
+
+def verify_bytes(cfg: RoundConfig, n: np.ndarray, packs_rows: bool, variant: str = "corrected",
+                 accept: np.ndarray | None = None) -> int:
+    """Algorithmic bytes of the verification phase of a round: the logits rows
+    the outputs depend on, tokens, and the row copies / packing."""
     es = cfg.elem_bytes
     B, K, V, d = cfg.B, cfg.K, cfg.V, cfg.d
-    logits = B * (K + 1) * V * es
+    logits = needed_logits_bytes(cfg, accept) if accept is not None else B * (K + 1) * V * es
     tokens_in = B * K * 4
     tokens_out = B * (K + 1) * 4 + 3 * B * 4  # committed; accept_len, bonus, n
     R = int(np.sum(n))
@@ -278,7 +296,7 @@ def conditioning_flops(cfg: RoundConfig, R: int, dense_e: bool, variant: str = "
 
 LOWRANK_L, LOWRANK_C = 64, 32
 KERNELS_PER_ROUND_SAMPLED = 3  # sampled top-k, sampled finalize (copies + packing), cond_kernel
-KERNELS_PER_ROUND_LOWRANK = 4  # verify_kernel, latent projection, finish (+ GEMV), latent fusion (tensor cores)
+KERNELS_PER_ROUND_LOWRANK = 4  # one-pass verify_kernel, latent projection, finish (+ GEMV), latent fusion
 
 
 def lowrank_flops(cfg: RoundConfig, R: int) -> int:
@@ -392,7 +410,13 @@ def run_gpu(args) -> dict | None:
     value = aggregate_value(steps, world, round_s_max)
 
     n = out.n.cpu().numpy().astype(np.int64)
+    accept = out.accept_len.cpu().numpy().astype(np.int64)
     R = int(n.sum())
+    # greedy verification: one pass, or passes over row windows plus one copy kernel
+    windows = ([0, cfg.K + 1] if (fused or args.sampled)
+               else rt.retrace_verify_plan(cfg.B, cfg.K, cfg.V, cfg.torch_dtype))
+    n_pass = len(windows) - 1
+    verify_launches = n_pass + (1 if n_pass > 1 else 0)
     step_avg_s = statistics.mean(step_ms) / 1e3
     cflops = (lowrank_flops(cfg, R) if args.lowrank
               else conditioning_flops(cfg, R, dense_e=False, variant=args.variant))
@@ -428,16 +452,20 @@ def run_gpu(args) -> dict | None:
         logits_gbs = cfg.logits_bytes() / step_avg_s / 1e9
     else:
         packs_rows = cfg.dtype == "bf16" and cfg.d % 256 == 0  # tensor-core path: verify packs the rows
-        vbytes = verify_bytes(cfg, n, packs_rows and args.variant in ("corrected", "raw"), args.variant)
+        vbytes = verify_bytes(cfg, n, packs_rows and args.variant in ("corrected", "raw"), args.variant, accept)
+        rbytes = vbytes - needed_logits_bytes(cfg, accept) + read_logits_bytes(cfg, accept, windows)
         v_avg_s = statistics.mean(verify_ms) / 1e3
-        v_gbs = vbytes / v_avg_s / 1e9
         c_avg_s = statistics.mean(cond_ms) / 1e3
         c_tflops = cflops / c_avg_s / 1e12
-        if args.sampled:  # the drafter's logits and the uniforms are read too
-            vbytes += cfg.B * cfg.K * cfg.V * cfg.elem_bytes + cfg.B * (cfg.K + 1) * 4
-            v_gbs = vbytes / v_avg_s / 1e9
+        if args.sampled:  # drafter rows 0..min(A_b, K-1) and the uniforms are needed too; every row is read
+            d_needed = int(np.sum(np.minimum(accept + 1, cfg.K))) * cfg.V * cfg.elem_bytes
+            vbytes += d_needed + cfg.B * (cfg.K + 1) * 4
+            rbytes += cfg.B * cfg.K * cfg.V * cfg.elem_bytes + cfg.B * (cfg.K + 1) * 4
+        v_gbs = vbytes / v_avg_s / 1e9
         v_roof = {
-            "kernel": "verify_kernel (argmax/compare/commit + copy of unconditioned rows + row packing)",
+            "kernel": (f"verify_kernel x{n_pass} passes over row windows {windows} + verify_copy_kernel (copy of "
+                       "unconditioned rows + row packing)" if n_pass > 1 else
+                       "verify_kernel (argmax/compare/commit + copy of unconditioned rows + row packing)"),
             "bound": "hbm",
             "achieved": round(v_gbs, 1),
             "peak": peaks["hbm_gbs"],
@@ -445,14 +473,21 @@ def run_gpu(args) -> dict | None:
             "frac": round(v_gbs / peaks["hbm_gbs"], 4),
             "peak_source": peaks["source"] + " HBM copy bandwidth",
             "algorithmic_bytes": vbytes,
+            "algorithmic_bytes_note": "logits rows 0..A_b of each sequence (what the outputs depend on), tokens, "
+                                      "row copies and packing",
+            "bytes_streamed": rbytes,
+            "streamed_frac": round(rbytes / v_avg_s / 1e9 / peaks["hbm_gbs"], 4),
+            "launches": verify_launches if not args.sampled else 2,
             "avg_launch_us": round(v_avg_s * 1e6, 2),
             "traffic": (round(VERIFY_TRAFFIC_PER_SEQUENCE * cfg.B)
                         if VERIFY_TRAFFIC_PER_SEQUENCE and (cfg.K, cfg.V, cfg.d, cfg.dtype) == VERIFY_TRAFFIC_SHAPE
-                        and args.variant == "corrected" else None),
-            "traffic_source": "ncu dram read+write on B=128 profiling workload, scaled by B/128",
+                        and args.variant == "corrected" and n_pass == VERIFY_TRAFFIC_PASSES else None),
+            "traffic_source": "ncu dram read+write of the verification kernels on the B=128 profiling workload, "
+                              "scaled by B/128",
         }
         if args.variant in ("overwrite", "none"):
-            v_roof["kernel"] = "verify_kernel (argmax/compare/commit + every row of e~ copied)"
+            v_roof["kernel"] = v_roof["kernel"].replace("copy of unconditioned rows + row packing",
+                                                        "every row of e~ copied")
         if args.sampled:
             v_roof["kernel"] = ("sampled_topk_kernel + sampled_finalize_kernel (top-k of every target and drafter "
                                 "row, accept tests, draw, copy of unconditioned rows + row packing)")
@@ -522,19 +557,22 @@ def run_gpu(args) -> dict | None:
             "variant": ("low-rank (rank-64 latents, rank-32 correction)" if args.lowrank
                         else f"temperature {x['temperature']}, top_k {x['top_k']}, top_p {x['top_p']} "
                              "(speculative sampling)" if args.sampled else args.variant),
+            "verify_windows": windows,
             "round_kernel": ("overlapped (one persistent launch)" if fused
-                             else "verify, latent projection, finish + GEMV, latent fusion" if args.lowrank
+                             else f"verify ({verify_launches} launches), latent projection, finish + GEMV, "
+                                  "latent fusion" if args.lowrank
                              else "three launches (sampled top-k, sampled finalize, projections)" if args.sampled
-                             else "two launches (verify, projections)"),
+                             else f"verify ({verify_launches} launches), projections" if cflops
+                             else f"verify ({verify_launches} launches)"),
         },
         "roofline": roofline,
         **line_extra,
         "logits_gbs": round(logits_gbs, 1),
         "e2e": e2e,
         "gpu_launches": (KERNELS_PER_ROUND_FUSED if fused
-                         else KERNELS_PER_ROUND_LOWRANK if args.lowrank
+                         else KERNELS_PER_ROUND_LOWRANK - 1 + verify_launches if args.lowrank
                          else KERNELS_PER_ROUND_SAMPLED if args.sampled
-                         else KERNELS_PER_ROUND if cflops else 1) * steps,
+                         else KERNELS_PER_ROUND - 1 + verify_launches if cflops else verify_launches) * steps,
         "wall_s_timed_region": round(t_wall, 4),
         "device_status_flags": status_flags,
         "impl": "ours",
@@ -624,8 +662,9 @@ def run_sweep(args) -> None:
     256 MB L2 flush before every call) and warm (back to back, so whatever
     fits stays in L2), plus CUDA-graph replay of the round for B <= 8.  Also
     the bytes verification needs at least, sum_b (A_b + 1) V s (the rows up to
-    the first mismatch), against the B (K+1) V s a parallel kernel reads.  One
-    JSON line per workload; an extra report, not the benchmark line."""
+    the first mismatch), against the bytes its schedule streams (every row in
+    one pass, or the row windows of the still-matching sequences).  One JSON
+    line per workload; an extra report, not the benchmark line."""
     from paper_2608_29748_gb300 import binding as rt
 
     torch.cuda.set_device(0)
@@ -678,19 +717,21 @@ def run_sweep(args) -> None:
         torch.cuda.synchronize(dev)
         A = out.accept_len.cpu().numpy().astype(np.int64)
         n = out.n.cpu().numpy().astype(np.int64)
-        s_b = cfg.elem_bytes
-        logits = cfg.logits_bytes()
-        needed = int(np.sum(np.minimum(A, cfg.K) + 1)) * cfg.V * s_b
+        windows = rt.retrace_verify_plan(cfg.B, cfg.K, cfg.V, cfg.torch_dtype)
+        logits = read_logits_bytes(cfg, A, windows)  # what the schedule streams
+        needed = needed_logits_bytes(cfg, A)
         line = {
             "config": cid, "workload": cfg.name, "B": cfg.B, "K": cfg.K, "V": cfg.V, "d": cfg.d,
             "dtype": cfg.dtype, "conditioned_rows_R": int(n.sum()), "iters": iters, "statistic": "median",
+            "verify_windows": windows,
             "verify_us": {k: round(t, 2) for k, t in v.items()},
             "logits_gbs": {k: round(logits / t / 1e3, 1) for k, t in v.items()},
             "logits_frac_of_hbm": {k: round(logits / t / 1e3 / peaks["hbm_gbs"], 4) for k, t in v.items()},
+            "needed_gbs": {k: round(needed / t / 1e3, 1) for k, t in v.items()},
             "round_us": {k: round(t, 2) for k, t in r.items()},
             "rounds_per_s": {k: round(1e6 / t, 1) for k, t in r.items()},
             "graph_round_us": None if graph is None else {k: round(t, 2) for k, t in graph.items()},
-            "logits_bytes": logits,
+            "logits_bytes_streamed": logits,
             "needed_bytes_rows_to_first_mismatch": needed,
             "needed_us_at_hbm_peak": round(needed / (peaks["hbm_gbs"] * 1e3), 2),
             "hbm_peak_gbs": peaks["hbm_gbs"], "peak_source": peaks["source"],

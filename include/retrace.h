@@ -137,16 +137,19 @@ retrace_status retrace_verify(const void* logits, retrace_dtype dtype, int B, in
 /* Schedules of greedy verification (every entry point that verifies greedily).
  * They differ in the rows they read, never in the results.
  *   RETRACE_VERIFY_FULL     one pass over every row of every sequence.
- *   RETRACE_VERIFY_WINDOWS  passes over windows of 4 rows (more for long
- *                           blocks, at most 16 passes): pass k reads rows
- *                           [4k, 4k+4) of the sequences whose draft tokens
- *                           matched every earlier row, so rows past the first
- *                           mismatch's window are never read.  Applies when
- *                           target_argmax is NULL (every row is an output
- *                           otherwise) and K+1 > 4; other calls take the full
- *                           pass.
+ *   RETRACE_VERIFY_WINDOWS  passes over row windows: rows [0, 4), then
+ *                           windows half as long again as the one before
+ *                           (4, 6, 9, ... rows; at most 16 passes; a short
+ *                           remainder joins the last window).  Pass k reads
+ *                           its window only for the sequences whose draft
+ *                           tokens matched every earlier row, so rows past
+ *                           the window of the first mismatch are never
+ *                           read.  Applies when target_argmax is NULL (every
+ *                           row is an output otherwise) and K+1 > 5; other
+ *                           calls take the full pass.  retrace_verify_plan
+ *                           gives the windows.
  *   RETRACE_VERIFY_AUTO     (default) WINDOWS where it applies and one row of
- *                           the whole batch is at least 32 MiB (B * V *
+ *                           the whole batch is at least 16 MiB (B * V *
  *                           element size), FULL otherwise (each extra pass
  *                           costs a few microseconds, which small batches
  *                           do not win back).
@@ -156,6 +159,16 @@ retrace_status retrace_verify(const void* logits, retrace_dtype dtype, int B, in
 #define RETRACE_VERIFY_FULL 1
 #define RETRACE_VERIFY_WINDOWS 2
 int retrace_set_verify_schedule(int mode);
+
+/* The greedy verification schedule a call with this shape takes under the
+ * current mode, given a workspace: returns the number of passes n (1 = the
+ * one-pass schedule; -1 for an invalid shape or dtype) and, when
+ * window_starts is not NULL, writes the n + 1 window boundaries (at most 17
+ * entries: pass k reads rows [window_starts[k], window_starts[k+1]) of the
+ * sequences that matched every row before it).  A windowed round launches n
+ * verification kernels plus one for the row copies; the one-pass round, one.
+ * Host arithmetic only. */
+int retrace_verify_plan(int B, int K, int V, retrace_dtype dtype, int target_argmax, int* window_starts);
 
 /* Rejected-trajectory alignment and target-aware correction (Eq. 3-7,
  * Algorithm 1 carry/reset steps).

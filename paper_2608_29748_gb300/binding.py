@@ -59,12 +59,13 @@ def _load() -> ctypes.CDLL:
     lib.retrace_verify_sampled.argtypes = [P, I64, I64, P, I64, I64, I, I, I, I, P, P, F, I, F, P, P, P, P, SZ, P]
     lib.retrace_wait_selftest.argtypes = [I, P, ctypes.c_uint32, P, SZ, P]
     lib.retrace_set_verify_schedule.argtypes = [I]
+    lib.retrace_verify_plan.argtypes = [I, I, I, I, I, ctypes.POINTER(ctypes.c_int)]
     lib.retrace_round_sampled.argtypes = [P, I64, I64, P, I64, I64, P, P, F, I, F, P, P, P, I64, I64, P, P, P, F,
                                           I, I, I, I, I, P, P, P, P, P, P, SZ, P, P]
     for name in ("retrace_workspace_init", "retrace_workspace_check", "retrace_verify",
                  "retrace_align_refine", "retrace_gate_fuse", "retrace_round", "retrace_round_lowrank",
                  "retrace_verify_sampled", "retrace_round_sampled", "retrace_wait_selftest",
-                 "retrace_set_verify_schedule"):
+                 "retrace_set_verify_schedule", "retrace_verify_plan"):
         getattr(lib, name).restype = I
     return lib
 
@@ -314,6 +315,17 @@ def version() -> str:
 
 
 VERIFY_AUTO, VERIFY_FULL, VERIFY_WINDOWS = 0, 1, 2
+
+
+def retrace_verify_plan(B: int, K: int, V: int, dtype: torch.dtype, target_argmax: bool = False) -> list[int]:
+    """Window boundaries greedy verification takes for this shape under the
+    current schedule ([0, K+1] for the one-pass schedule)."""
+    starts = (ctypes.c_int * 17)()
+    code = RETRACE_BF16 if dtype == torch.bfloat16 else RETRACE_F32 if dtype == torch.float32 else -1
+    n = lib.retrace_verify_plan(B, K, V, code, int(bool(target_argmax)), starts)
+    if n < 1:
+        raise RetraceError(1, "invalid shape or dtype for retrace_verify_plan")
+    return list(starts[: n + 1])
 
 
 def retrace_set_verify_schedule(mode: int) -> int:

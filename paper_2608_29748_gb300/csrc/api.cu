@@ -140,6 +140,7 @@ void verify_workspace(VerifyArgs* a, char* w, const WsLayout& L) {
   a->tickets = reinterpret_cast<uint32_t*>(w + L.tickets);
   a->live = reinterpret_cast<int32_t*>(w + L.live);
   a->pass_counts = reinterpret_cast<uint32_t*>(w + L.counts);
+  a->pack_off = reinterpret_cast<int32_t*>(w + L.poff);
 }
 
 
@@ -235,6 +236,15 @@ const char* retrace_last_error(void) { return g_err; }
 const char* retrace_version(void) { return "retrace 0.1.0 sm_103a"; }
 
 int retrace_set_verify_schedule(int mode) { return set_verify_schedule(mode); }
+
+int retrace_verify_plan(int B, int K, int V, retrace_dtype dtype, int target_argmax, int* window_starts) {
+  if (B < 0 || K < 0 || V < 1 || K > kMaxK || (dtype != RETRACE_BF16 && dtype != RETRACE_F32)) return -1;
+  int start[kMaxWindowPasses + 1];
+  const int n = verify_windows(B, K, V, (int)elem_size(dtype), true, target_argmax != 0, start);
+  if (window_starts)
+    for (int k = 0; k <= n; ++k) window_starts[k] = start[k];
+  return n;
+}
 
 size_t retrace_workspace_bytes(int B, int K, int V, int d, retrace_dtype dtype) {
   if (B < 0 || K < 0 || V < 1 || d < 0 || !dtype_ok(dtype)) return 0;

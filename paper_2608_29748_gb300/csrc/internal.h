@@ -21,6 +21,7 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 //   keys     uint64 [B*(K+1)]   per-row argmax keys, zero between calls
 //   tickets  uint32 [B]         per-sequence CTA arrival counters, zero between calls
 //   live     int32  [2*B]       windowed verification: live sequence lists of two passes
+//   poff     int32  [B]         windowed verification: first packed row of each sequence
 //   counts   uint32 [1+passes]  windowed verification: [0] CTAs out of the last pass,
 //                               [k] sequences live into pass k; zero between calls
 //   ge       fp32   [d]         W_g[:, :d] e for a broadcast e
@@ -39,7 +40,7 @@ constexpr int kMaxTopK = 64;            // largest top_k of sampled verification
 constexpr int kWindowRows = 4;          // rows per pass of windowed verification
 constexpr int kMaxWindowPasses = 16;    // most passes of windowed verification
 struct WsLayout {
-  size_t status, sync, sync_bytes, keys, tickets, live, counts, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, skeys, total;
+  size_t status, sync, sync_bytes, keys, tickets, live, poff, counts, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, skeys, total;
 };
 
 inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
@@ -59,6 +60,8 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   off = align_up(off + (size_t)B * 4, 256);
   L.live = off;
   off = align_up(off + (size_t)B * 2 * 4, 256);
+  L.poff = off;
+  off = align_up(off + (size_t)B * 4, 256);
   L.counts = off;
   off = align_up(off + (size_t)(kMaxWindowPasses + 1) * 4, 256);
   L.ge = off;
@@ -150,6 +153,7 @@ struct VerifyArgs {
   // lists of B sequences and the passes' counters, from the workspace.
   int32_t* live;
   uint32_t* pass_counts;
+  int32_t* pack_off;
   // Rows j < n_b of e_out in the copy above (no packing then): kCondCopyKeep
   // leaves them to the conditioning kernels, kCondCopyE writes e (no
   // conditioning), kCondCopyM writes m_j = hD[b, A_b+1+j] (overwrite).
@@ -160,6 +164,10 @@ constexpr int kCondCopyE = 1;
 constexpr int kCondCopyM = 2;
 cudaError_t launch_verify(const VerifyArgs& a, retrace_dtype dtype, cudaStream_t stream);
 int set_verify_schedule(int mode);  // RETRACE_VERIFY_*; previous mode, or -1
+// Row windows greedy verification takes for this call: writes the window
+// starts (n + 1 entries, at most kMaxWindowPasses + 1) and returns the number
+// of passes n (1: the one-pass schedule).
+int verify_windows(int B, int K, int V, int elem_bytes, bool have_workspace, bool argmax_out, int* start);
 
 // Stochastic verification (speculative sampling on top-k / top-p filtered
 // distributions at temperature T).

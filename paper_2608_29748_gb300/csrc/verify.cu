@@ -67,6 +67,7 @@ struct VerifyParams {
   int n_counts;
   uint32_t* exits;           // last pass: CTAs out (zero between calls)
   int defer_copies;          // the finaliser leaves the copies to verify_copy_kernel
+  int32_t* pack_off;         // [B] first packed row of each sequence (deferred copies)
 };
 
 // 16-byte vector helpers: the maximum of the vector's elements and element q.
@@ -272,6 +273,7 @@ __device__ void finish_sequence(const VerifyParams& p, int b, int A, int rows, c
     p.accept_len[b] = A;
     p.bonus[b] = s_t[A];
     if (p.n_out) p.n_out[b] = nb;
+    if (p.defer_copies && p.R_count) p.pack_off[b] = nb > 0 ? atomicAdd(p.R_count, nb) : 0;
   }
   if (!p.defer_copies) copy_sequence<T>(p, b, A, s_off, staging);
 }
@@ -381,23 +383,88 @@ __global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams 
   }
 }
 
-// The copies of a windowed verification, after its last pass: one sequence
-// per CTA at a time (accept_len holds every A_b by then).
-template <typename T>
+// The copies of a windowed verification, after its last pass (accept_len
+// and the packed-row offsets hold every sequence's values by then).  Work
+// items are row segments: (sequence b, position j, segment), the segments in
+// order the row of e_out (when this position's e_out row is written here: e,
+// or m_j in the overwrite variant), then, for conditioned positions of a
+// packing round, the halves m_j and u_j of the packed row and the packed e
+// row.  Each warp takes items in turn and copies one with its 32 lanes, each
+// lane kCopyBatch 16-byte vectors in flight at a time (elements when CV is
+// false); inactive items cost one decode.
+constexpr int kCopyBatch = 8;
+template <typename T, bool CV>
 __global__ void __launch_bounds__(kThreads, 2) verify_copy_kernel(const VerifyParams p) {
-  __shared__ int s_off;
-  extern __shared__ uint4 s_stage[];
   pdl_launch_dependents();
   pdl_wait();
-  for (int b = blockIdx.x; b < p.B; b += gridDim.x) {
-    const int A = __ldcg(p.accept_len + b);
-    copy_sequence<T>(p, b, A, &s_off, s_stage);
-    __syncthreads();
+  const int K = p.K, d = p.d;
+  constexpr int E = CV ? 16 / (int)sizeof(T) : 1;  // elements per copy slot
+  const int vpr = d / E;
+  const bool pack = p.R_count != nullptr;
+  const int nseg = (p.e_out ? 1 : 0) + (pack ? (p.e_dense ? 3 : 2) : 0);
+  const long long items = (long long)p.B * K * nseg;
+  const int lane = threadIdx.x & 31;
+  const long long warps = (long long)gridDim.x * (kThreads / 32);
+  const T* e = reinterpret_cast<const T*>(p.e);
+  const T* hD = reinterpret_cast<const T*>(p.hD);
+  const T* hT = reinterpret_cast<const T*>(p.hT);
+  T* e_out = reinterpret_cast<T*>(p.e_out);
+  T* apack = reinterpret_cast<T*>(p.apack);
+  T* epack = reinterpret_cast<T*>(p.epack);
+  for (long long it = (long long)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5); it < items; it += warps) {
+    const long long u = it / nseg;
+    const int seg = (int)(it - u * nseg);
+    const int b = (int)(u / K), j = (int)(u - (long long)b * K);
+    const int A = __ldg(p.accept_len + b);
+    const int nb = (K - 1 - A) > 0 ? (K - 1 - A) : 0;
+    const long long pos = (long long)b * K + j;
+    const int kind = p.e_out ? seg : seg + 1;  // 0 e_out row, 1 m half, 2 u half, 3 packed e
+    const T* src;
+    T* dst;
+    if (kind == 0) {
+      if (p.cond_copy == kCondCopyKeep && j < nb) continue;  // the conditioning kernels write it
+      src = (p.cond_copy == kCondCopyM && j < nb) ? hD + (pos + A + 1) * d
+                                                  : e + (long long)b * p.e_batch_stride + (long long)j * p.e_pos_stride;
+      dst = e_out + pos * d;
+    } else {
+      if (j >= nb) continue;
+      const long long row = (long long)__ldg(p.pack_off + b) + j;
+      if (kind == 1) {
+        src = hD + (pos + A + 1) * d;
+        dst = apack + row * 2 * d;
+        if (lane == 0) p.rowmap[row] = (int32_t)pos;
+      } else if (kind == 2) {
+        src = hT + (pos + A) * d;
+        dst = apack + row * 2 * d + d;
+      } else {
+        src = e + pos * d;
+        dst = epack + row * d;
+      }
+    }
+    if constexpr (CV) {
+      const uint4* s4 = reinterpret_cast<const uint4*>(src);
+      uint4* d4 = reinterpret_cast<uint4*>(dst);
+      for (int v0 = 0; v0 < vpr; v0 += 32 * kCopyBatch) {
+        uint4 x[kCopyBatch];
+#pragma unroll
+        for (int k = 0; k < kCopyBatch; ++k) {
+          const int v = v0 + k * 32 + lane;
+          if (v < vpr) x[k] = __ldcs(s4 + v);
+        }
+#pragma unroll
+        for (int k = 0; k < kCopyBatch; ++k) {
+          const int v = v0 + k * 32 + lane;
+          if (v < vpr) d4[v] = x[k];
+        }
+      }
+    } else {
+      for (int v = lane; v < d; v += 32) dst[v] = src[v];
+    }
   }
 }
 
 std::atomic<int> g_schedule{RETRACE_VERIFY_AUTO};
-constexpr long long kWindowMinBatchRowBytes = 32ll << 20;  // B * V * element size
+constexpr long long kWindowMinBatchRowBytes = 16ll << 20;  // B * V * element size
 
 // Row windows of the windowed schedule: the first kWindowRows rows, then
 // windows half as long again as the one before (fewer, longer passes as the
@@ -417,6 +484,23 @@ inline int window_bounds(int K1, int* start) {
   }
   return n;
 }
+
+}  // namespace
+
+int verify_windows(int B, int K, int V, int elem_bytes, bool have_workspace, bool argmax_out, int* start) {
+  const int K1 = K + 1;
+  const int n = window_bounds(K1, start);
+  const int mode = g_schedule.load(std::memory_order_relaxed);
+  const long long wave = (long long)B * V * elem_bytes;
+  const bool windowed = have_workspace && !argmax_out && B > 0 && n > 1 &&
+                        (mode == RETRACE_VERIFY_WINDOWS || (mode == RETRACE_VERIFY_AUTO && wave >= kWindowMinBatchRowBytes));
+  if (windowed) return n;
+  start[0] = 0;
+  start[1] = K1;
+  return 1;
+}
+
+namespace {
 
 template <typename T, bool VEC>
 cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
@@ -473,13 +557,11 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
   p.n_counts = 0;
   p.exits = nullptr;
   p.defer_copies = 0;
+  p.pack_off = a.pack_off;
   const int K1 = a.K + 1;
   int start[kMaxWindowPasses + 1];
-  const int n_pass = window_bounds(K1, start);
-  const int mode = g_schedule.load(std::memory_order_relaxed);
-  const long long wave = (long long)a.B * a.V * (long long)sizeof(T);
-  const bool windowed = a.live && !a.target_argmax && n_pass > 1 &&
-                        (mode == RETRACE_VERIFY_WINDOWS || (mode == RETRACE_VERIFY_AUTO && wave >= kWindowMinBatchRowBytes));
+  const int n_pass = verify_windows(a.B, a.K, a.V, (int)sizeof(T), a.live != nullptr, a.target_argmax != nullptr, start);
+  const bool windowed = n_pass > 1;
   const long long grid_full = (long long)info.sm_count * occ;
   if (!windowed) {
     // Enough CTAs to fill every SM at full occupancy, but at least ~32 KB of
@@ -522,15 +604,13 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
     if (err != cudaSuccess) return err;
   }
   if (copies) {
-    static int copy_attr[64] = {0};
-    if (!copy_attr[info.device & 63]) {
-      err = cudaFuncSetAttribute(verify_copy_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, kCopyStageBytes);
-      if (err != cudaSuccess) return err;
-      copy_attr[info.device & 63] = 1;
-    }
-    const long long grid = a.B < grid_full ? a.B : grid_full;
-    err = launch_dependent(verify_copy_kernel<T>, dim3((unsigned)grid), dim3(kThreads), kCopyStageBytes, stream, 1u,
-                           p);
+    const size_t es = sizeof(T);
+    auto al = [](const void* q) { return (uintptr_t)q % 16 == 0; };
+    const bool cv = (a.d * es) % 16 == 0 && al(a.e) && al(a.e_out) && (a.e_pos_stride * (long long)es) % 16 == 0 &&
+                    (a.e_batch_stride * (long long)es) % 16 == 0 && (a.cond_copy != kCondCopyM || al(a.hD)) &&
+                    (!a.R_count || (al(a.hD) && al(a.hT) && al(a.apack) && (!a.e_dense || al(a.epack))));
+    auto kern = cv ? verify_copy_kernel<T, true> : verify_copy_kernel<T, false>;
+    err = launch_dependent(kern, dim3((unsigned)grid_full), dim3(kThreads), 0, stream, 1u, p);
     if (err != cudaSuccess) return err;
   }
   return cudaSuccess;

@@ -203,3 +203,41 @@ def test_lowrank_round_argument_errors(lib):
     assert call(K=0) == INVALID
     assert call(d=0) == INVALID
     assert call(B=0) == OK
+
+
+def _plan(lib, B, K, V, dtype=BF16, argmax=0):
+    starts = (ctypes.c_int * 17)()
+    lib.retrace_verify_plan.argtypes = [ctypes.c_int] * 5 + [ctypes.POINTER(ctypes.c_int)]
+    n = lib.retrace_verify_plan(B, K, V, dtype, argmax, starts)
+    return n, list(starts[: n + 1]) if n > 0 else []
+
+
+def test_verify_schedule_plan(lib):
+    """Windows of the windowed schedule: 4 rows, then half as long again each
+    pass, a short remainder joining the last window; the automatic choice by
+    batch size; target_argmax and short blocks keep one pass."""
+    AUTO, FULL, WINDOWS = 0, 1, 2
+    prev = lib.retrace_set_verify_schedule(AUTO)
+    try:
+        assert _plan(lib, 256, 16, 151936) == (3, [0, 4, 10, 17])      # 74 MiB per row of the batch
+        assert _plan(lib, 64, 16, 151936) == (3, [0, 4, 10, 17])       # 18.5 MiB
+        assert _plan(lib, 8, 16, 151936) == (1, [0, 17])               # 2.3 MiB: one pass
+        assert _plan(lib, 256, 16, 151936, argmax=1) == (1, [0, 17])   # every row is an output
+        assert lib.retrace_set_verify_schedule(WINDOWS) == AUTO
+        assert _plan(lib, 8, 16, 151936) == (3, [0, 4, 10, 17])
+        assert _plan(lib, 1, 4, 100) == (1, [0, 5])                    # K+1 = 5: one window
+        assert _plan(lib, 1, 5, 100) == (2, [0, 4, 6])
+        assert _plan(lib, 1, 6, 100) == (2, [0, 4, 7])
+        assert _plan(lib, 1, 9, 100) == (2, [0, 4, 10])
+        assert _plan(lib, 1, 11, 100) == (2, [0, 4, 12])               # 2 rows left < 6 / 2: joined
+        assert _plan(lib, 1, 12, 100) == (3, [0, 4, 10, 13])
+        n, s = _plan(lib, 2, 1024, 100)
+        assert 2 <= n <= 16 and s[0] == 0 and s[-1] == 1025 and all(a < b for a, b in zip(s, s[1:]))
+        assert _plan(lib, 0, 16, 100) == (1, [0, 17])
+        assert _plan(lib, 1, 16, 0)[0] == -1 and _plan(lib, 1, 1025, 10)[0] == -1
+        assert _plan(lib, 1, 16, 10, dtype=7)[0] == -1
+        assert lib.retrace_set_verify_schedule(FULL) == WINDOWS
+        assert _plan(lib, 256, 16, 151936) == (1, [0, 17])
+        assert lib.retrace_set_verify_schedule(9) == -1
+    finally:
+        lib.retrace_set_verify_schedule(prev)

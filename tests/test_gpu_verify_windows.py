@@ -228,3 +228,28 @@ def test_round_outputs_identical_under_both_schedules(rt, cfg_id, flags):
         for name in ("accept_len", "committed", "bonus", "n", "e_out"):
             assert torch.equal(getattr(o, name), getattr(outs[0], name)), name
     assert ws.check() == 0
+
+
+@pytest.mark.parametrize("flags", ["default", "overwrite"])
+def test_round_unaligned_e_out_both_schedules(rt, flags):
+    """e_out one element off a 16-byte boundary: the copies after the windowed
+    passes take their element-wise path; the bits equal the one-pass round's."""
+    f = {"default": 0, "overwrite": rt.COND_OVERWRITE}[flags]
+    x = make_round_inputs(CONFIGS[4], device="cuda")
+    cfg = x["cfg"]
+    ws = rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype)
+    outs = []
+    prev = rt.retrace_set_verify_schedule(rt.VERIFY_FULL)
+    try:
+        for mode in (rt.VERIFY_FULL, rt.VERIFY_WINDOWS):
+            rt.retrace_set_verify_schedule(mode)
+            out = rt.RoundBuffers(cfg.B, cfg.K, cfg.d, cfg.torch_dtype)
+            big = torch.empty(cfg.B * cfg.K * cfg.d + 1, dtype=cfg.torch_dtype, device="cuda")
+            out.e_out = big[1:].view(cfg.B, cfg.K, cfg.d)
+            outs.append(rt.run_round(x, ws, out=out, flags=f))
+            torch.cuda.synchronize()
+    finally:
+        rt.retrace_set_verify_schedule(prev)
+    for name in ("accept_len", "committed", "bonus", "n", "e_out"):
+        assert torch.equal(getattr(outs[1], name), getattr(outs[0], name)), name
+    assert ws.check() == 0
