@@ -295,7 +295,6 @@ def conditioning_flops(cfg: RoundConfig, R: int, dense_e: bool, variant: str = "
 
 
 LOWRANK_L, LOWRANK_C = 64, 32
-KERNELS_PER_ROUND_SAMPLED = 3  # sampled top-k, sampled finalize (copies + packing), cond_kernel
 KERNELS_PER_ROUND_LOWRANK = 4  # one-pass verify_kernel, latent projection, finish (+ GEMV), latent fusion
 
 
@@ -412,11 +411,11 @@ def run_gpu(args) -> dict | None:
     n = out.n.cpu().numpy().astype(np.int64)
     accept = out.accept_len.cpu().numpy().astype(np.int64)
     R = int(n.sum())
-    # greedy verification: one pass, or passes over row windows plus one copy kernel
-    windows = ([0, cfg.K + 1] if (fused or args.sampled)
-               else rt.retrace_verify_plan(cfg.B, cfg.K, cfg.V, cfg.torch_dtype))
+    # verification: one pass, or passes over row windows plus one copy kernel
+    # (a pass is one kernel greedy, top-k + finalize at temperature 1)
+    windows = [0, cfg.K + 1] if fused else rt.retrace_verify_plan(cfg.B, cfg.K, cfg.V, cfg.torch_dtype)
     n_pass = len(windows) - 1
-    verify_launches = n_pass + (1 if n_pass > 1 else 0)
+    verify_launches = n_pass * (2 if args.sampled else 1) + (1 if n_pass > 1 else 0)
     step_avg_s = statistics.mean(step_ms) / 1e3
     cflops = (lowrank_flops(cfg, R) if args.lowrank
               else conditioning_flops(cfg, R, dense_e=False, variant=args.variant))
@@ -457,10 +456,12 @@ def run_gpu(args) -> dict | None:
         v_avg_s = statistics.mean(verify_ms) / 1e3
         c_avg_s = statistics.mean(cond_ms) / 1e3
         c_tflops = cflops / c_avg_s / 1e12
-        if args.sampled:  # drafter rows 0..min(A_b, K-1) and the uniforms are needed too; every row is read
+        if args.sampled:  # drafter rows 0..min(A_b, K-1) and the uniforms are needed too
             d_needed = int(np.sum(np.minimum(accept + 1, cfg.K))) * cfg.V * cfg.elem_bytes
+            d_rows = sum(int(np.sum(accept >= windows[k])) * max(0, min(windows[k + 1], cfg.K) - windows[k])
+                         for k in range(n_pass))
             vbytes += d_needed + cfg.B * (cfg.K + 1) * 4
-            rbytes += cfg.B * cfg.K * cfg.V * cfg.elem_bytes + cfg.B * (cfg.K + 1) * 4
+            rbytes += d_rows * cfg.V * cfg.elem_bytes + cfg.B * (cfg.K + 1) * 4
         v_gbs = vbytes / v_avg_s / 1e9
         v_roof = {
             "kernel": (f"verify_kernel x{n_pass} passes over row windows {windows} + verify_copy_kernel (copy of "
@@ -477,7 +478,7 @@ def run_gpu(args) -> dict | None:
                                       "row copies and packing",
             "bytes_streamed": rbytes,
             "streamed_frac": round(rbytes / v_avg_s / 1e9 / peaks["hbm_gbs"], 4),
-            "launches": verify_launches if not args.sampled else 2,
+            "launches": verify_launches,
             "avg_launch_us": round(v_avg_s * 1e6, 2),
             "traffic": (round(VERIFY_TRAFFIC_PER_SEQUENCE * cfg.B)
                         if VERIFY_TRAFFIC_PER_SEQUENCE and (cfg.K, cfg.V, cfg.d, cfg.dtype) == VERIFY_TRAFFIC_SHAPE
@@ -489,8 +490,10 @@ def run_gpu(args) -> dict | None:
             v_roof["kernel"] = v_roof["kernel"].replace("copy of unconditioned rows + row packing",
                                                         "every row of e~ copied")
         if args.sampled:
-            v_roof["kernel"] = ("sampled_topk_kernel + sampled_finalize_kernel (top-k of every target and drafter "
-                                "row, accept tests, draw, copy of unconditioned rows + row packing)")
+            v_roof["kernel"] = (f"sampled_topk_kernel + sampled_finalize_kernel x{n_pass} passes over row windows "
+                                f"{windows} (top-k of the window's target and drafter rows, accept tests, draw)"
+                                + (" + verify_copy_kernel (copy of unconditioned rows + row packing)"
+                                   if n_pass > 1 else " (+ copy of unconditioned rows + row packing)"))
             v_roof["traffic"] = None
         c_roof = None
         if args.lowrank:
@@ -561,7 +564,8 @@ def run_gpu(args) -> dict | None:
             "round_kernel": ("overlapped (one persistent launch)" if fused
                              else f"verify ({verify_launches} launches), latent projection, finish + GEMV, "
                                   "latent fusion" if args.lowrank
-                             else "three launches (sampled top-k, sampled finalize, projections)" if args.sampled
+                             else f"verify ({verify_launches} launches: sampled top-k + finalize per pass), "
+                                  "projections" if args.sampled
                              else f"verify ({verify_launches} launches), projections" if cflops
                              else f"verify ({verify_launches} launches)"),
         },
@@ -571,7 +575,7 @@ def run_gpu(args) -> dict | None:
         "e2e": e2e,
         "gpu_launches": (KERNELS_PER_ROUND_FUSED if fused
                          else KERNELS_PER_ROUND_LOWRANK - 1 + verify_launches if args.lowrank
-                         else KERNELS_PER_ROUND_SAMPLED if args.sampled
+                         else verify_launches + 1 if args.sampled
                          else KERNELS_PER_ROUND - 1 + verify_launches if cflops else verify_launches) * steps,
         "wall_s_timed_region": round(t_wall, 4),
         "device_status_flags": status_flags,

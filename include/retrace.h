@@ -134,20 +134,21 @@ retrace_status retrace_verify(const void* logits, retrace_dtype dtype, int B, in
                               int32_t* bonus, int32_t* target_argmax, void* ws,
                               size_t ws_bytes, cudaStream_t stream);
 
-/* Schedules of greedy verification (every entry point that verifies greedily).
- * They differ in the rows they read, never in the results.
+/* Schedules of verification (every entry point that verifies, greedy or at
+ * temperature T).  They differ in the rows they read, never in the results.
  *   RETRACE_VERIFY_FULL     one pass over every row of every sequence.
  *   RETRACE_VERIFY_WINDOWS  passes over row windows: rows [0, 4), then
  *                           windows half as long again as the one before
  *                           (4, 6, 9, ... rows; at most 16 passes; a short
  *                           remainder joins the last window).  Pass k reads
  *                           its window only for the sequences whose draft
- *                           tokens matched every earlier row, so rows past
- *                           the window of the first mismatch are never
- *                           read.  Applies when target_argmax is NULL (every
- *                           row is an output otherwise) and K+1 > 5; other
- *                           calls take the full pass.  retrace_verify_plan
- *                           gives the windows.
+ *                           tokens matched (greedy) or were accepted (at
+ *                           temperature T) in every earlier row, so rows past
+ *                           the window of the first mismatch are never read.
+ *                           Applies when target_argmax is NULL (every row is
+ *                           an output otherwise) and K+1 > 5; other calls take
+ *                           the full pass.  retrace_verify_plan gives the
+ *                           windows.
  *   RETRACE_VERIFY_AUTO     (default) WINDOWS where it applies and one row of
  *                           the whole batch is at least 16 MiB (B * V *
  *                           element size), FULL otherwise (each extra pass
@@ -165,9 +166,10 @@ int retrace_set_verify_schedule(int mode);
  * one-pass schedule; -1 for an invalid shape or dtype) and, when
  * window_starts is not NULL, writes the n + 1 window boundaries (at most 17
  * entries: pass k reads rows [window_starts[k], window_starts[k+1]) of the
- * sequences that matched every row before it).  A windowed round launches n
- * verification kernels plus one for the row copies; the one-pass round, one.
- * Host arithmetic only. */
+ * sequences that matched every row before it).  A windowed greedy round
+ * launches n verification kernels plus one for the row copies (one kernel in
+ * one pass); at temperature T, 2n kernels (top-k scan and accept tests per
+ * pass) plus the copies (two in one pass).  Host arithmetic only. */
 int retrace_verify_plan(int B, int K, int V, retrace_dtype dtype, int target_argmax, int* window_starts);
 
 /* Rejected-trajectory alignment and target-aware correction (Eq. 3-7,

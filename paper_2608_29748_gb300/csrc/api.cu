@@ -134,6 +134,13 @@ retrace_status e_mode(int64_t ebs, int64_t eps, int K, int d, int* dense) {
 
 uint32_t* status_word(void* ws) { return reinterpret_cast<uint32_t*>(ws); }
 
+// Workspace pointers of the windowed schedule of sampled verification.
+void sampled_workspace(SampledArgs* a, char* w, const WsLayout& L) {
+  a->live = reinterpret_cast<int32_t*>(w + L.live);
+  a->pass_counts = reinterpret_cast<uint32_t*>(w + L.counts);
+  a->pack_off = reinterpret_cast<int32_t*>(w + L.poff);
+}
+
 // Workspace pointers of the greedy verification kernels.
 void verify_workspace(VerifyArgs* a, char* w, const WsLayout& L) {
   a->keys = reinterpret_cast<unsigned long long*>(w + L.keys);
@@ -581,6 +588,7 @@ retrace_status retrace_verify_sampled(const void* target_logits, int64_t target_
   a.committed = committed;
   a.bonus = bonus;
   a.keys = reinterpret_cast<unsigned long long*>(reinterpret_cast<char*>(ws) + Lw.skeys);
+  sampled_workspace(&a, reinterpret_cast<char*>(ws), Lw);
   RT_CUDA(launch_verify_sampled(a, dtype, stream), "sampled verification launch");
   return RETRACE_OK;
 }
@@ -636,6 +644,7 @@ retrace_status retrace_round_sampled(const void* target_logits, int64_t target_r
   a.committed = committed;
   a.bonus = bonus;
   a.keys = reinterpret_cast<unsigned long long*>(w + L.skeys);
+  sampled_workspace(&a, w, L);
   a.n_out = n_out;
   a.e = e;
   a.e_batch_stride = e_batch_stride;

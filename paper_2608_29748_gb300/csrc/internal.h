@@ -163,6 +163,10 @@ constexpr int kCondCopyKeep = 0;
 constexpr int kCondCopyE = 1;
 constexpr int kCondCopyM = 2;
 cudaError_t launch_verify(const VerifyArgs& a, retrace_dtype dtype, cudaStream_t stream);
+// The copies of a windowed verification after its last pass (accept_len and
+// pack_off complete): unconditioned rows of e_out and the packed rows, from
+// the copy fields of `a` (B, K, d, accept_len, e..., cond_copy, pack_off).
+cudaError_t launch_verify_copies(const VerifyArgs& a, retrace_dtype dtype, cudaStream_t stream);
 int set_verify_schedule(int mode);  // RETRACE_VERIFY_*; previous mode, or -1
 // Row windows greedy verification takes for this call: writes the window
 // starts (n + 1 entries, at most kMaxWindowPasses + 1) and returns the number
@@ -200,6 +204,11 @@ struct SampledArgs {
   void* epack;
   int32_t* rowmap;
   int32_t* R_count;
+  // Windowed schedule (NULL live: one pass): live lists, pass counters and
+  // packed-row offsets from the workspace, as for greedy verification.
+  int32_t* live;
+  uint32_t* pass_counts;
+  int32_t* pack_off;
 };
 cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cudaStream_t stream);
 

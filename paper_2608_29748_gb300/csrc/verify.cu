@@ -502,6 +502,20 @@ int verify_windows(int B, int K, int V, int elem_bytes, bool have_workspace, boo
 
 namespace {
 
+// verify_copy_kernel after the last pass (programmatically dependent): the
+// 16-byte path when every copied tensor allows it.
+template <typename T>
+cudaError_t launch_copies(const VerifyArgs& a, const VerifyParams& p, long long grid, cudaStream_t stream) {
+  const size_t es = sizeof(T);
+  auto al = [](const void* q) { return (uintptr_t)q % 16 == 0; };
+  const bool cv = (a.d * es) % 16 == 0 && (!a.e_out || (al(a.e) && al(a.e_out))) &&
+                  (a.e_pos_stride * (long long)es) % 16 == 0 && (a.e_batch_stride * (long long)es) % 16 == 0 &&
+                  (a.cond_copy != kCondCopyM || al(a.hD)) &&
+                  (!a.R_count || (al(a.hD) && al(a.hT) && al(a.apack) && (!a.e_dense || al(a.epack))));
+  auto kern = cv ? verify_copy_kernel<T, true> : verify_copy_kernel<T, false>;
+  return launch_dependent(kern, dim3((unsigned)grid), dim3(kThreads), 0, stream, 1u, p);
+}
+
 template <typename T, bool VEC>
 cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
   DeviceInfo info;
@@ -603,20 +617,39 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
     }
     if (err != cudaSuccess) return err;
   }
-  if (copies) {
-    const size_t es = sizeof(T);
-    auto al = [](const void* q) { return (uintptr_t)q % 16 == 0; };
-    const bool cv = (a.d * es) % 16 == 0 && al(a.e) && al(a.e_out) && (a.e_pos_stride * (long long)es) % 16 == 0 &&
-                    (a.e_batch_stride * (long long)es) % 16 == 0 && (a.cond_copy != kCondCopyM || al(a.hD)) &&
-                    (!a.R_count || (al(a.hD) && al(a.hT) && al(a.apack) && (!a.e_dense || al(a.epack))));
-    auto kern = cv ? verify_copy_kernel<T, true> : verify_copy_kernel<T, false>;
-    err = launch_dependent(kern, dim3((unsigned)grid_full), dim3(kThreads), 0, stream, 1u, p);
-    if (err != cudaSuccess) return err;
-  }
+  if (copies) return launch_copies<T>(a, p, grid_full, stream);
   return cudaSuccess;
 }
 
 }  // namespace
+
+cudaError_t launch_verify_copies(const VerifyArgs& a, retrace_dtype dtype, cudaStream_t stream) {
+  DeviceInfo info;
+  cudaError_t err = device_info(&info);
+  if (err != cudaSuccess) return err;
+  VerifyParams p{};
+  p.B = a.B;
+  p.K = a.K;
+  p.V = a.V;
+  p.accept_len = a.accept_len;
+  p.e = a.e;
+  p.e_batch_stride = a.e_batch_stride;
+  p.e_pos_stride = a.e_pos_stride;
+  p.e_out = a.e_out;
+  p.d = a.d;
+  p.hD = a.hD;
+  p.hT = a.hT;
+  p.e_dense = a.e_dense;
+  p.apack = a.apack;
+  p.epack = a.epack;
+  p.rowmap = a.rowmap;
+  p.R_count = a.R_count;
+  p.cond_copy = a.cond_copy;
+  p.pack_off = a.pack_off;
+  const long long grid = (long long)info.sm_count * 2;
+  return dtype == RETRACE_BF16 ? launch_copies<__nv_bfloat16>(a, p, grid, stream)
+                               : launch_copies<float>(a, p, grid, stream);
+}
 
 int set_verify_schedule(int mode) {
   if (mode != RETRACE_VERIFY_AUTO && mode != RETRACE_VERIFY_FULL && mode != RETRACE_VERIFY_WINDOWS) return -1;

@@ -41,6 +41,12 @@ struct TopkParams {
   long long d_row, d_batch;
   int B, K, V, k;
   unsigned long long* keys;  // [B (2K+1), kMaxTopK]: target rows b*(K+1)+i, then drafter rows
+  // Row window of this pass ([0, K+1) in one pass): target rows [i0, i1) and
+  // drafter rows [i0, min(i1, K)) of the listed sequences (NULL: 0..B-1;
+  // count_in NULL: B of them, else written by the previous pass).
+  int i0, i1;
+  const int32_t* live_in;
+  const uint32_t* count_in;
 };
 
 // The largest key whose value is below v: every element of value >= v beats it.
@@ -144,15 +150,29 @@ __global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkPar
   __shared__ unsigned long long s_thr;
   pdl_launch_dependents();  // the finalize kernel may take SMs as these CTAs finish
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int row = blockIdx.x;  // B (2K+1) rows: a grid dimension, below 2^31
-  const int nt = p.B * (p.K + 1);
+  // This CTA's row of the pass: the window's target rows of each listed
+  // sequence, then its drafter rows; `row` is the row's slot in p.keys.
+  int n_live = p.B;
+  if (p.count_in) {  // a later pass: the previous finalize wrote the live list
+    pdl_wait();
+    n_live = (int)__ldcg(p.count_in);
+  }
+  const int wt = p.i1 - p.i0, wd = min(p.i1, p.K) - p.i0;
+  const int r0 = blockIdx.x;  // B (2K+1) rows at most: a grid dimension, below 2^31
+  int row;
   const T* x;
-  if (row < nt) {
-    const int b = row / (p.K + 1), i = row - b * (p.K + 1);
+  if (r0 < n_live * wt) {
+    const int l = r0 / wt, i = p.i0 + (r0 - l * wt);
+    const int b = p.live_in ? __ldg(p.live_in + l) : l;
+    row = b * (p.K + 1) + i;
     x = reinterpret_cast<const T*>(p.tlogits) + b * p.t_batch + i * p.t_row;
-  } else {
-    const int r = row - nt, b = r / p.K, i = r - b * p.K;
+  } else if (r0 < n_live * (wt + wd)) {
+    const int r = r0 - n_live * wt, l = r / wd, i = p.i0 + (r - l * wd);
+    const int b = p.live_in ? __ldg(p.live_in + l) : l;
+    row = p.B * (p.K + 1) + b * p.K + i;
     x = reinterpret_cast<const T*>(p.dlogits) + b * p.d_batch + i * p.d_row;
+  } else {
+    return;  // past the live rows of this pass
   }
   const int V = p.V, k = p.k;
   unsigned long long* buf = s_buf[warp];
@@ -314,6 +334,21 @@ struct FinalizeParams {
   void* epack;
   int32_t* rowmap;
   int32_t* R_count;
+  // Windowed schedule: accept tests over rows [i0, min(i1, K)) of the listed
+  // sequences (live_in NULL: 0..B-1, count_in NULL: B); a sequence that
+  // accepts them all, with rows left, goes to live_out.  The last pass's last
+  // CTA out zeroes the passes' counters.  With defer_copies the finaliser
+  // only claims the packed rows (pack_off) and a later kernel copies.
+  int i0, i1;
+  const int32_t* live_in;
+  const uint32_t* count_in;
+  int32_t* live_out;
+  uint32_t* count_out;
+  uint32_t* pass_counts;
+  int n_counts;
+  uint32_t* exits;
+  int defer_copies;
+  int32_t* pack_off;
 };
 
 // The filtered distribution of one row, lane j holding entries j and 32 + j
@@ -431,22 +466,21 @@ __device__ int draw(const RowDist& r, const float wt[2], float u, int lane) {
 // distributions is one per chunk instead of one per position.  Warp 0 then
 // draws the appended token; every thread writes the outputs and, for a round,
 // copies and packs rows.
-__global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizeParams p) {
+__device__ void sampled_finalize_sequence(const FinalizeParams& p, int b) {
   constexpr int kFinWarps = 8;
   __shared__ int s_A, s_y, s_off;
   __shared__ float s_px[kFinWarps], s_qx[kFinWarps];
-  pdl_launch_dependents();
-  pdl_wait();  // the sorted lists come from the top-k kernel
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int b = blockIdx.x;
   const int K = p.K, K1 = K + 1;
   const int32_t* dr = p.draft + (long long)b * K;
   const long long tbase = (long long)b * K1, dbase = (long long)p.B * K1 + (long long)b * K;
   const float* u = p.uniforms + (long long)b * K1;
-  int A = K;
-  for (int c0 = 0; c0 < K; c0 += kFinWarps) {
+  // rows before i0 were accepted in earlier passes
+  int A = p.i1 == K1 ? K : -1;  // -1: every row of the window accepted, rows left
+  const int hi = min(p.i1, K);
+  for (int c0 = p.i0; c0 < hi; c0 += kFinWarps) {
     const int i = c0 + warp;
-    if (i < K) {
+    if (i < hi) {
       const int x = dr[i];
       float px = -1.f, qx = 0.f;  // px < 0: a token outside [0, V) is rejected
       if (x >= 0 && x < p.V) {
@@ -463,7 +497,7 @@ __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizePar
     __syncthreads();
     if (threadIdx.x == 0) {
       int a = -1;
-      for (int j = 0; j < kFinWarps && c0 + j < K; ++j) {
+      for (int j = 0; j < kFinWarps && c0 + j < hi; ++j) {
         if (!(s_px[j] >= 0.f && u[c0 + j] * s_qx[j] < s_px[j])) {
           a = c0 + j;
           break;
@@ -477,6 +511,10 @@ __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizePar
       A = a;
       break;
     }
+  }
+  if (A < 0) {  // every draft of the window accepted: on to the next pass
+    if (threadIdx.x == 0) p.live_out[atomicAdd(p.count_out, 1u)] = b;
+    return;
   }
   if (warp == 0) {
     const RowDist pt = row_dist(p, tbase + A, lane);
@@ -508,6 +546,7 @@ __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizePar
       s_y = y;
       const int nb = K - 1 - A > 0 ? K - 1 - A : 0;
       s_off = (p.R_count && nb > 0) ? atomicAdd(p.R_count, nb) : 0;
+      if (p.defer_copies && p.R_count) p.pack_off[b] = s_off;
     }
   }
   __syncthreads();
@@ -522,7 +561,7 @@ __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizePar
     p.bonus[b] = y;
     if (p.n_out) p.n_out[b] = nb;
   }
-  if (!p.e_out) return;
+  if (!p.e_out || p.defer_copies) return;
   // rows j >= n_b keep the drafter input, bit for bit
   const long long base_row = (long long)b * K;
   const char* e_b = static_cast<const char*>(p.e) + b * p.e_batch_stride * p.elem;
@@ -576,6 +615,22 @@ __global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizePar
   }
 }
 
+__global__ void __launch_bounds__(256) sampled_finalize_kernel(const FinalizeParams p) {
+  pdl_launch_dependents();
+  pdl_wait();  // the sorted lists come from the top-k kernel
+  const int n_live = p.count_in ? (int)__ldcg(p.count_in) : p.B;
+  if ((int)blockIdx.x < n_live) {
+    sampled_finalize_sequence(p, p.live_in ? __ldg(p.live_in + blockIdx.x) : (int)blockIdx.x);
+  }
+  if (p.exits && threadIdx.x == 0) {  // the last pass's last CTA out resets the live counters
+    __threadfence();
+    if (atomicAdd(p.exits, 1u) == gridDim.x - 1u) {
+      for (int k = 0; k < p.n_counts; ++k) p.pass_counts[k] = 0u;
+      *p.exits = 0u;
+    }
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cudaStream_t stream) {
@@ -592,13 +647,6 @@ cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cud
   tp.V = a.V;
   tp.k = a.top_k;
   tp.keys = a.keys;
-  const long long rows = (long long)a.B * (2 * a.K + 1);
-  if (dtype == RETRACE_BF16)
-    sampled_topk_kernel<__nv_bfloat16><<<(unsigned)rows, kThreads, 0, stream>>>(tp);
-  else
-    sampled_topk_kernel<float><<<(unsigned)rows, kThreads, 0, stream>>>(tp);
-  cudaError_t err = cudaGetLastError();
-  if (err != cudaSuccess) return err;
   FinalizeParams fp{};
   fp.keys = a.keys;
   fp.B = a.B;
@@ -626,7 +674,64 @@ cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cud
   fp.epack = a.epack;
   fp.rowmap = a.rowmap;
   fp.R_count = a.R_count;
-  return launch_dependent(sampled_finalize_kernel, dim3((unsigned)a.B), dim3(256), 0, stream, 1, fp);
+  fp.pack_off = a.pack_off;
+  // The outputs depend only on the target rows 0..A_b and the drafter rows
+  // 0..min(A_b, K-1): the same row windows as greedy verification.  Pass k
+  // scans the window's rows of the sequences that accepted every earlier
+  // draft (top-k kernel), then runs their accept tests (finalize kernel).
+  int start[kMaxWindowPasses + 1];
+  const int K1 = a.K + 1;
+  const int n_pass = verify_windows(a.B, a.K, a.V, (int)fp.elem, a.live != nullptr, false, start);
+  const bool defer = n_pass > 1 && a.e_out;
+  fp.defer_copies = defer ? 1 : 0;
+  for (int k = 0; k < n_pass; ++k) {
+    const bool last = k == n_pass - 1;
+    tp.i0 = fp.i0 = start[k];
+    tp.i1 = fp.i1 = start[k + 1];
+    tp.live_in = fp.live_in = k == 0 ? nullptr : a.live + (size_t)((k - 1) & 1) * a.B;
+    tp.count_in = fp.count_in = k == 0 ? nullptr : a.pass_counts + k;
+    fp.live_out = last ? nullptr : a.live + (size_t)(k & 1) * a.B;
+    fp.count_out = last ? nullptr : a.pass_counts + k + 1;
+    fp.pass_counts = last && n_pass > 1 ? a.pass_counts + 1 : nullptr;
+    fp.n_counts = last ? n_pass - 1 : 0;
+    fp.exits = last && n_pass > 1 ? a.pass_counts : nullptr;
+    const int wt = tp.i1 - tp.i0, wd = (tp.i1 < a.K ? tp.i1 : a.K) - tp.i0;
+    const dim3 grid((unsigned)((long long)a.B * (wt + wd)));
+    cudaError_t err;
+    auto topk = dtype == RETRACE_BF16 ? sampled_topk_kernel<__nv_bfloat16> : sampled_topk_kernel<float>;
+    if (k == 0) {
+      topk<<<grid, kThreads, 0, stream>>>(tp);
+      err = cudaGetLastError();
+    } else {
+      err = launch_dependent(topk, grid, dim3(kThreads), 0, stream, 1, tp);
+    }
+    if (err != cudaSuccess) return err;
+    err = launch_dependent(sampled_finalize_kernel, dim3((unsigned)a.B), dim3(256), 0, stream, 1, fp);
+    if (err != cudaSuccess) return err;
+  }
+  (void)K1;
+  if (!defer) return cudaSuccess;
+  // the row copies and packing, balanced over the grid
+  VerifyArgs c{};
+  c.B = a.B;
+  c.K = a.K;
+  c.V = a.V;
+  c.accept_len = a.accept_len;
+  c.e = a.e;
+  c.e_batch_stride = a.e_batch_stride;
+  c.e_pos_stride = a.e_pos_stride;
+  c.e_out = a.e_out;
+  c.d = a.d;
+  c.hD = a.hD;
+  c.hT = a.hT;
+  c.e_dense = a.e_dense;
+  c.apack = a.apack;
+  c.epack = a.epack;
+  c.rowmap = a.rowmap;
+  c.R_count = a.R_count;
+  c.pack_off = a.pack_off;
+  c.cond_copy = kCondCopyKeep;
+  return launch_verify_copies(c, dtype, stream);
 }
 
 }  // namespace retrace

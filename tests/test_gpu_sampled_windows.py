@@ -1,0 +1,122 @@
+"""Windowed schedule of stochastic verification vs the one-pass schedule and the oracle.
+
+The outputs of speculative sampling depend only on the target rows 0..A_b and
+the drafter rows 0..min(A_b, K-1): the accept tests stop at the first
+rejection, whose row also gives the residual draw.  The windowed schedule
+scans the row windows of the sequences that accepted every earlier draft, and
+its outputs must equal the one-pass schedule's bit for bit (both decide from
+the same per-row top-k lists) and the oracle's.  Acceptance is planted here
+so that every window boundary is crossed: drafter rows equal to the target's
+(q = p, so a draft in the kept set is always accepted) and, at row a_b, a
+draft outside the target's top k (p = 0: always rejected).
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from parity import host_int
+from test_gpu_sampled import check_against_oracle
+from paper_2608_29748_gb300.workloads import CONFIGS, make_round_inputs, make_sampled_inputs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def rt():
+    from paper_2608_29748_gb300 import binding
+
+    return binding
+
+
+@pytest.fixture
+def windows(rt):
+    prev = rt.retrace_set_verify_schedule(rt.VERIFY_WINDOWS)
+    yield
+    rt.retrace_set_verify_schedule(prev)
+
+
+def sampled(rt, x, s, ws, T, k, p):
+    B, K1, _ = x["logits"].shape
+    outs = [torch.full((B,), -7, dtype=torch.int32, device="cuda"),
+            torch.full((B, K1), -7, dtype=torch.int32, device="cuda"),
+            torch.full((B,), -7, dtype=torch.int32, device="cuda")]
+    rt.retrace_verify_sampled(x["logits"], s["draft_logits"], s["draft"], s["uniforms"], T, k, p, *outs, ws)
+    torch.cuda.synchronize()
+    return outs
+
+
+def planted(cfg, accept):
+    """Target logits of cfg; drafter rows = target rows; drafts = the target's
+    argmax in rows i < a_b and its smallest logit's index in row a_b."""
+    x = make_round_inputs(cfg, device="cuda")
+    tl = x["logits"]
+    B, K1, V = tl.shape
+    K = K1 - 1
+    s = make_sampled_inputs(cfg, tl, device="cuda")
+    s["draft_logits"] = tl[:, :K].contiguous()
+    top = torch.argmax(tl[:, :K].float(), dim=-1)
+    low = torch.argmin(tl[:, :K].float(), dim=-1)
+    i = torch.arange(K, device="cuda")[None, :]
+    a = accept.to("cuda")[:, None]
+    s["draft"] = torch.where(i < a, top, low).to(torch.int32)
+    return x, s
+
+
+@pytest.mark.parametrize("cfg_id", [1, 3, 4])
+@pytest.mark.parametrize("T,k,p", [(1.0, 20, 0.95), (0.7, 64, 0.8), (1.3, 5, 1.0)])
+def test_windowed_equals_one_pass(rt, cfg_id, T, k, p):
+    cfg = CONFIGS[cfg_id]
+    x = make_round_inputs(cfg, device="cuda")
+    s = make_sampled_inputs(cfg, x["logits"], device="cuda")
+    ws = rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype)
+    prev = rt.retrace_set_verify_schedule(rt.VERIFY_FULL)
+    try:
+        full = sampled(rt, x, s, ws, T, k, p)
+        rt.retrace_set_verify_schedule(rt.VERIFY_WINDOWS)
+        for _ in range(2):  # and again on the same workspace
+            win = sampled(rt, x, s, ws, T, k, p)
+            for a, b in zip(win, full):
+                assert torch.equal(a, b)
+    finally:
+        rt.retrace_set_verify_schedule(prev)
+    assert ws.check() == 0
+
+
+@pytest.mark.parametrize("cfg_id", [3, 4])
+def test_windowed_planted_acceptance_every_boundary(rt, windows, cfg_id):
+    cfg = CONFIGS[cfg_id]
+    accept = torch.arange(cfg.B) % (cfg.K + 1)  # every accepted length 0..K
+    x, s = planted(cfg, accept)
+    acc = check_against_oracle(rt, x, s)
+    np.testing.assert_array_equal(acc, accept.numpy())
+
+
+def test_windowed_all_accepted(rt, windows):
+    cfg = CONFIGS[4]
+    x, s = planted(cfg, torch.full((cfg.B,), cfg.K))
+    acc = check_against_oracle(rt, x, s)
+    assert (acc == cfg.K).all()
+
+
+@pytest.mark.parametrize("cfg_id", [1, 3, 4])
+def test_windowed_round_equals_one_pass(rt, cfg_id):
+    """The round: outputs, n and e~ (copies and packing after the last pass,
+    then the projections) equal the one-pass round's bit for bit."""
+    cfg = CONFIGS[cfg_id]
+    x = make_round_inputs(cfg, device="cuda")
+    s = make_sampled_inputs(cfg, x["logits"], device="cuda")
+    ws = rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype)
+    outs = []
+    prev = rt.retrace_set_verify_schedule(rt.VERIFY_FULL)
+    try:
+        for mode in (rt.VERIFY_FULL, rt.VERIFY_WINDOWS):
+            rt.retrace_set_verify_schedule(mode)
+            outs.append(rt.run_round_sampled(x, s, ws))
+            torch.cuda.synchronize()
+    finally:
+        rt.retrace_set_verify_schedule(prev)
+    for name in ("accept_len", "committed", "bonus", "n", "e_out"):
+        assert torch.equal(getattr(outs[1], name), getattr(outs[0], name)), name
+    assert host_int(outs[1].n).sum() > 0
+    assert ws.check() == 0
