@@ -137,43 +137,27 @@ __device__ int warp_compact(unsigned long long* buf, unsigned long long* tmp, in
 // bit mask, to the warp's buffer with shared-memory atomics.  A buffer that
 // passes a trigger is cut to its top k.  The row's top k are merged from the
 // warps' sorted lists.
+struct TopkSmem {
+  unsigned long long buf[kWarps][kBuf];
+  unsigned long long tmp[kWarps][kMaxTopK];
+  float sample[kThreads];
+  int n[kWarps];
+  unsigned long long thr;
+};
+
+// The top-k list of one row x into p.keys slot `row` (the whole CTA).
 template <typename T>
-__global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkParams p) {
+__device__ __forceinline__ void topk_row(const TopkParams& p, const T* x, int row, TopkSmem& sm) {
   using CT = Chunk<T>;
   using Part = typename CT::Part;
   constexpr int E = CT::E;
   constexpr int U = 4;
-  __shared__ unsigned long long s_buf[kWarps][kBuf];
-  __shared__ unsigned long long s_tmp[kWarps][kMaxTopK];
-  __shared__ float s_sample[kThreads];
-  __shared__ int s_n[kWarps];
-  __shared__ unsigned long long s_thr;
-  pdl_launch_dependents();  // the finalize kernel may take SMs as these CTAs finish
+  auto& s_buf = sm.buf;
+  auto& s_tmp = sm.tmp;
+  auto& s_sample = sm.sample;
+  auto& s_n = sm.n;
+  auto& s_thr = sm.thr;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // This CTA's row of the pass: the window's target rows of each listed
-  // sequence, then its drafter rows; `row` is the row's slot in p.keys.
-  int n_live = p.B;
-  if (p.count_in) {  // a later pass: the previous finalize wrote the live list
-    pdl_wait();
-    n_live = (int)__ldcg(p.count_in);
-  }
-  const int wt = p.i1 - p.i0, wd = min(p.i1, p.K) - p.i0;
-  const int r0 = blockIdx.x;  // B (2K+1) rows at most: a grid dimension, below 2^31
-  int row;
-  const T* x;
-  if (r0 < n_live * wt) {
-    const int l = r0 / wt, i = p.i0 + (r0 - l * wt);
-    const int b = p.live_in ? __ldg(p.live_in + l) : l;
-    row = b * (p.K + 1) + i;
-    x = reinterpret_cast<const T*>(p.tlogits) + b * p.t_batch + i * p.t_row;
-  } else if (r0 < n_live * (wt + wd)) {
-    const int r = r0 - n_live * wt, l = r / wd, i = p.i0 + (r - l * wd);
-    const int b = p.live_in ? __ldg(p.live_in + l) : l;
-    row = p.B * (p.K + 1) + b * p.K + i;
-    x = reinterpret_cast<const T*>(p.dlogits) + b * p.d_batch + i * p.d_row;
-  } else {
-    return;  // past the live rows of this pass
-  }
   const int V = p.V, k = p.k;
   unsigned long long* buf = s_buf[warp];
   unsigned long long* tmp = s_tmp[warp];
@@ -307,6 +291,50 @@ __global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkPar
       const unsigned long long best = warp_max_key(head);
       if (lane == 0) out[r] = best;  // 0 once every list is exhausted (V < k)
       if (head == best && best != 0ull) ++pos;
+    }
+  }
+}
+
+// One row per CTA (the first pass: every row of the window), or a grid of
+// resident CTAs looping over the rows of a later pass (its live count is
+// known only on the device; a grid of the whole batch's rows would spend
+// whole waves of CTAs that only find they have nothing to do).  The rows of
+// a pass: the window's target rows of each listed sequence, then its drafter
+// rows; `row` is the row's slot in p.keys.
+template <typename T, bool LOOP>
+__global__ void __launch_bounds__(kThreads, 3) sampled_topk_kernel(const TopkParams p) {
+  __shared__ TopkSmem sm;
+  pdl_launch_dependents();  // the finalize kernel may take SMs as these CTAs finish
+  int n_live = p.B;
+  if (p.count_in) {  // a later pass: the previous finalize wrote the live list
+    pdl_wait();
+    n_live = (int)__ldcg(p.count_in);
+  }
+  const int wt = p.i1 - p.i0, wd = min(p.i1, p.K) - p.i0;
+  const int rows = n_live * (wt + wd);  // B (2K+1) at most, below 2^31
+  auto row_of = [&](int r0, const T*& x) -> int {
+    if (r0 < n_live * wt) {
+      const int l = r0 / wt, i = p.i0 + (r0 - l * wt);
+      const int b = p.live_in ? __ldg(p.live_in + l) : l;
+      x = reinterpret_cast<const T*>(p.tlogits) + b * p.t_batch + i * p.t_row;
+      return b * (p.K + 1) + i;
+    }
+    const int r = r0 - n_live * wt, l = r / wd, i = p.i0 + (r - l * wd);
+    const int b = p.live_in ? __ldg(p.live_in + l) : l;
+    x = reinterpret_cast<const T*>(p.dlogits) + b * p.d_batch + i * p.d_row;
+    return p.B * (p.K + 1) + b * p.K + i;
+  };
+  if constexpr (!LOOP) {
+    if ((int)blockIdx.x >= rows) return;
+    const T* x;
+    const int row = row_of(blockIdx.x, x);
+    topk_row<T>(p, x, row, sm);
+  } else {
+    for (int r0 = blockIdx.x; r0 < rows; r0 += gridDim.x) {
+      const T* x;
+      const int row = row_of(r0, x);
+      topk_row<T>(p, x, row, sm);
+      __syncthreads();  // the row's shared buffers are read to the end before the next row
     }
   }
 }
@@ -683,6 +711,13 @@ cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cud
   const int K1 = a.K + 1;
   const int n_pass = verify_windows(a.B, a.K, a.V, (int)fp.elem, a.live != nullptr, false, start);
   const bool defer = n_pass > 1 && a.e_out;
+  long long topk_resident = 0;
+  if (n_pass > 1) {
+    DeviceInfo info;
+    cudaError_t e0 = device_info(&info);
+    if (e0 != cudaSuccess) return e0;
+    topk_resident = (long long)info.sm_count * 3;  // __launch_bounds__(kThreads, 3)
+  }
   fp.defer_copies = defer ? 1 : 0;
   for (int k = 0; k < n_pass; ++k) {
     const bool last = k == n_pass - 1;
@@ -696,9 +731,15 @@ cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cud
     fp.n_counts = last ? n_pass - 1 : 0;
     fp.exits = last && n_pass > 1 ? a.pass_counts : nullptr;
     const int wt = tp.i1 - tp.i0, wd = (tp.i1 < a.K ? tp.i1 : a.K) - tp.i0;
-    const dim3 grid((unsigned)((long long)a.B * (wt + wd)));
+    // the first pass: one CTA per row; later passes: resident CTAs looping
+    const long long rows_max = (long long)a.B * (wt + wd);
+    const long long grid_n = k == 0 ? rows_max : (rows_max < topk_resident ? rows_max : topk_resident);
+    const dim3 grid((unsigned)(grid_n > 0 ? grid_n : 1));
     cudaError_t err;
-    auto topk = dtype == RETRACE_BF16 ? sampled_topk_kernel<__nv_bfloat16> : sampled_topk_kernel<float>;
+    auto topk = k == 0 ? (dtype == RETRACE_BF16 ? sampled_topk_kernel<__nv_bfloat16, false>
+                                                 : sampled_topk_kernel<float, false>)
+                       : (dtype == RETRACE_BF16 ? sampled_topk_kernel<__nv_bfloat16, true>
+                                                 : sampled_topk_kernel<float, true>);
     if (k == 0) {
       topk<<<grid, kThreads, 0, stream>>>(tp);
       err = cudaGetLastError();
