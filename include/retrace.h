@@ -54,8 +54,16 @@
  *               retrace_workspace_check.
  *   Workspace   `ws` must be zeroed once by retrace_workspace_init before its
  *               first use.  Every successful call leaves the workspace ready for
- *               the next call.  Calls sharing one workspace must be ordered on
- *               one stream (or otherwise serialised); after an error status,
+ *               the next call, also of another shape (a workspace sized for the
+ *               largest shape serves every smaller one): a call whose (B, K)
+ *               differs from the previous call's on the same workspace first
+ *               re-zeroes the workspace's small counter regions (one
+ *               cudaMemsetAsync; the library keeps each workspace's last shape
+ *               on the host, in call order).  A CUDA graph replays what was
+ *               captured, so between replays and calls of other shapes on the
+ *               same workspace call retrace_workspace_init (or give each shape
+ *               its own workspace).  Calls sharing one workspace must be ordered
+ *               on one stream (or otherwise serialised); after an error status,
  *               call retrace_workspace_init again.
  *   Errors      arguments are checked on the host before anything is enqueued;
  *               a bad argument returns a status and enqueues nothing.  A CUDA

@@ -3,6 +3,9 @@
 #include <stdarg.h>
 #include <stdio.h>
 
+#include <mutex>
+#include <unordered_map>
+
 #include "internal.h"
 
 namespace retrace {
@@ -90,6 +93,47 @@ retrace_status check_ws(const void* ws, size_t ws_bytes, size_t need) {
   if (ws_bytes < need)
     return fail(RETRACE_ERR_WORKSPACE, "workspace too small: %zu bytes given, %zu needed", ws_bytes, need);
   return RETRACE_OK;
+}
+
+// The regions that must be zero between calls (sync counters, argmax keys,
+// tickets, pass counters) lie before L.ge, at offsets that depend on B and K
+// (the live lists and packed-row offsets between them hold data).  A call of
+// another (B, K) than the previous call on the same workspace would find some
+// of them over the previous layout's data, so it first re-zeroes
+// [256, max(old, new) L.ge) -- the status word at 0 is kept.  The previous
+// shape of each workspace is kept here, on the host, in enqueue order (calls
+// on one workspace are ordered on one stream); retrace_workspace_init
+// forgets it.
+struct WsMemo {
+  long long B, K;
+  size_t zero_end;
+};
+static std::mutex g_ws_mu;
+static std::unordered_map<uintptr_t, WsMemo> g_ws_memo;
+
+retrace_status prepare_ws(void* ws, size_t ws_bytes, const WsLayout& L, long long B, long long K,
+                          cudaStream_t stream) {
+  size_t clear_end = 0;
+  {
+    std::lock_guard<std::mutex> lock(g_ws_mu);
+    auto it = g_ws_memo.find((uintptr_t)ws);
+    if (it == g_ws_memo.end()) {
+      g_ws_memo[(uintptr_t)ws] = WsMemo{B, K, L.ge};
+    } else if (it->second.B != B || it->second.K != K) {
+      clear_end = it->second.zero_end > L.ge ? it->second.zero_end : L.ge;
+      it->second = WsMemo{B, K, L.ge};
+    }
+  }
+  if (clear_end > ws_bytes) clear_end = ws_bytes;
+  if (clear_end > 256)
+    RT_CUDA(cudaMemsetAsync(static_cast<char*>(ws) + 256, 0, clear_end - 256, stream),
+            "cudaMemsetAsync(workspace, shape change)");
+  return RETRACE_OK;
+}
+
+void forget_ws(const void* ws) {
+  std::lock_guard<std::mutex> lock(g_ws_mu);
+  g_ws_memo.erase((uintptr_t)ws);
 }
 
 retrace_status check_verify_args(const void* logits, retrace_dtype dtype, int B, int K, int V,
@@ -262,6 +306,7 @@ retrace_status retrace_workspace_init(void* ws, size_t ws_bytes, cudaStream_t st
   g_err[0] = '\0';
   if (!ws || ws_bytes == 0) return fail(RETRACE_ERR_INVALID_ARG, "NULL or empty workspace");
   RT_CUDA(cudaMemsetAsync(ws, 0, ws_bytes, stream), "cudaMemsetAsync(workspace)");
+  forget_ws(ws);
   return RETRACE_OK;
 }
 
@@ -286,6 +331,7 @@ retrace_status retrace_verify(const void* logits, retrace_dtype dtype, int B, in
   if (st != RETRACE_OK || B == 0) return st;
   const WsLayout L = ws_layout(B, K, 0, elem_size(dtype));
   if ((st = check_ws(ws, ws_bytes, L.ge)) != RETRACE_OK) return st;
+  if ((st = prepare_ws(ws, ws_bytes, L, B, K, stream)) != RETRACE_OK) return st;
   VerifyArgs a{};
   a.logits = logits;
   a.B = B;
@@ -314,6 +360,7 @@ retrace_status retrace_align_refine(const void* hD, const void* hT, retrace_dtyp
     return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
   const WsLayout L = ws_layout(B, K, d, elem_size(dtype));
   if ((st = check_ws(ws, ws_bytes, L.total)) != RETRACE_OK) return st;
+  if ((st = prepare_ws(ws, ws_bytes, L, B, K, stream)) != RETRACE_OK) return st;
   const RowSource rows{accept_len, 1};
   RT_CUDA(launch_fill_rows(B, K, d, rows, n_out, r_out, nullptr, 0, nullptr, dtype, stream),
           "fill kernel launch");
@@ -360,6 +407,7 @@ retrace_status retrace_gate_fuse(const void* e, int64_t e_batch_stride, int64_t 
   if ((st = e_mode(e_batch_stride, e_pos_stride, K, d, &dense)) != RETRACE_OK) return st;
   const WsLayout L = ws_layout(B, K, d, elem_size(dtype));
   if ((st = check_ws(ws, ws_bytes, L.total)) != RETRACE_OK) return st;
+  if ((st = prepare_ws(ws, ws_bytes, L, B, K, stream)) != RETRACE_OK) return st;
   char* w = reinterpret_cast<char*>(ws);
   float* ge = reinterpret_cast<float*>(w + L.ge);
   const RowSource rows{n, 0};
@@ -430,6 +478,7 @@ retrace_status retrace_round(const void* logits, int64_t logits_row_stride,
   if ((st = e_mode(e_batch_stride, e_pos_stride, K, d, &dense)) != RETRACE_OK) return st;
   const WsLayout L = ws_layout(B, K, d, elem_size(dtype));
   if ((st = check_ws(ws, ws_bytes, L.total)) != RETRACE_OK) return st;
+  if ((st = prepare_ws(ws, ws_bytes, L, B, K, stream)) != RETRACE_OK) return st;
   char* w = reinterpret_cast<char*>(ws);
   float* ge = reinterpret_cast<float*>(w + L.ge);
   void* r_ws = w + L.r;
@@ -569,6 +618,7 @@ retrace_status retrace_verify_sampled(const void* target_logits, int64_t target_
   if (B == 0) return RETRACE_OK;
   const WsLayout Lw = ws_layout(B, K, 1, elem_size(dtype));
   if ((st = check_ws(ws, ws_bytes, Lw.total)) != RETRACE_OK) return st;
+  if ((st = prepare_ws(ws, ws_bytes, Lw, B, K, stream)) != RETRACE_OK) return st;
   SampledArgs a{};
   a.tlogits = target_logits;
   a.t_row = target_row_stride;
@@ -617,6 +667,7 @@ retrace_status retrace_round_sampled(const void* target_logits, int64_t target_r
   if ((st = e_mode(e_batch_stride, e_pos_stride, K, d, &dense)) != RETRACE_OK) return st;
   const WsLayout L = ws_layout(B, K, d, elem_size(dtype));
   if ((st = check_ws(ws, ws_bytes, L.total)) != RETRACE_OK) return st;
+  if ((st = prepare_ws(ws, ws_bytes, L, B, K, stream)) != RETRACE_OK) return st;
   char* w = reinterpret_cast<char*>(ws);
   const bool tc = tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(Wc) && aligned16(Wv) &&
                   aligned16(Wg) && aligned16(e) && aligned16(e_out);
@@ -689,6 +740,7 @@ retrace_status retrace_round_lowrank(const void* logits, int64_t logits_row_stri
     return fail(RETRACE_ERR_INVALID_ARG, "NULL tensor pointer");
   const WsLayout Lw = ws_layout(B, K, d, elem_size(dtype));
   if ((st = check_ws(ws, ws_bytes, Lw.total)) != RETRACE_OK) return st;
+  if ((st = prepare_ws(ws, ws_bytes, Lw, B, K, stream)) != RETRACE_OK) return st;
   char* w = reinterpret_cast<char*>(ws);
   const bool tc = lowrank_tc_supported(dtype, d) && aligned16(hD) && aligned16(hT) && aligned16(e) &&
                   aligned16(P) && aligned16(Bc) && aligned16(Ac) && aligned16(Wv) && aligned16(Wg) &&
