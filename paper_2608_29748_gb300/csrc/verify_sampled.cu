@@ -19,6 +19,11 @@
 //                            lists (eight positions at a time, one per warp),
 //                            the accept tests in order, the draw, and for a
 //                            round the copies and packing of e~ and [m; u].
+// The outputs depend only on the target rows 0..A_b and the drafter rows
+// 0..min(A_b, K-1).  In the windowed schedule the pair of kernels runs once
+// per row window, over the sequences that accepted every earlier draft (live
+// lists in the workspace); the copies and packing then follow in the greedy
+// path's copy kernel.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -708,7 +713,6 @@ cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cud
   // scans the window's rows of the sequences that accepted every earlier
   // draft (top-k kernel), then runs their accept tests (finalize kernel).
   int start[kMaxWindowPasses + 1];
-  const int K1 = a.K + 1;
   const int n_pass = verify_windows(a.B, a.K, a.V, (int)fp.elem, a.live != nullptr, false, start);
   const bool defer = n_pass > 1 && a.e_out;
   long long topk_resident = 0;
@@ -750,7 +754,6 @@ cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cud
     err = launch_dependent(sampled_finalize_kernel, dim3((unsigned)a.B), dim3(256), 0, stream, 1, fp);
     if (err != cudaSuccess) return err;
   }
-  (void)K1;
   if (!defer) return cudaSuccess;
   // the row copies and packing, balanced over the grid
   VerifyArgs c{};
