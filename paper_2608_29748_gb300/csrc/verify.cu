@@ -12,7 +12,6 @@
 // committed tokens and bonus, resets the keys and ticket to zero for the next
 // call and, inside a fused round, copies the unconditioned drafter inputs.
 //
-//
 // The outputs depend only on rows 0..A_b of each sequence.  The windowed
 // schedule runs the same kernel as a chain of passes over row windows
 // [i0, i1): the finaliser of a sequence whose draft tokens matched every row
@@ -20,6 +19,8 @@
 // finalising it, and the next pass (launched programmatically dependent)
 // streams only the listed sequences' rows.  Rows past the window holding the
 // first mismatch are never read.  Same keys, same finaliser, same results.
+// The finalisers of a windowed round only claim their packed rows; the row
+// copies follow in verify_copy_kernel, spread over the whole grid.
 #include <atomic>
 
 #include "common.cuh"
