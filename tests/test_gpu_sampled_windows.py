@@ -120,3 +120,27 @@ def test_windowed_round_equals_one_pass(rt, cfg_id):
         assert torch.equal(getattr(outs[1], name), getattr(outs[0], name)), name
     assert host_int(outs[1].n).sum() > 0
     assert ws.check() == 0
+
+
+@pytest.mark.parametrize("K", [5, 6, 9, 11])
+def test_windowed_short_blocks(rt, K):
+    """Windows [0,4),[4,6) at K = 5 (the last window has one target row, K,
+    and one drafter row, 4), [0,4),[4,7) at K = 6, [0,4),[4,10) at K = 9 and
+    [0,4),[4,12) at K = 11: equal to the one-pass schedule, accepted lengths
+    from 0 to K planted."""
+    cfg = CONFIGS[2].__class__(f"sampled-K{K}", K + 1, K, 3001, 8, "bf16", 1.0, "uniform", seed_offset=40 + K)
+    accept = torch.arange(cfg.B) % (K + 1)
+    x, s = planted(cfg, accept)
+    ws = rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype)
+    prev = rt.retrace_set_verify_schedule(rt.VERIFY_FULL)
+    try:
+        full = sampled(rt, x, s, ws, 1.0, 20, 0.95)
+        rt.retrace_set_verify_schedule(rt.VERIFY_WINDOWS)
+        assert len(rt.retrace_verify_plan(cfg.B, K, cfg.V, cfg.torch_dtype)) == 3
+        win = sampled(rt, x, s, ws, 1.0, 20, 0.95)
+    finally:
+        rt.retrace_set_verify_schedule(prev)
+    for a, b in zip(win, full):
+        assert torch.equal(a, b)
+    np.testing.assert_array_equal(host_int(win[0]), accept.numpy())
+    assert ws.check() == 0
