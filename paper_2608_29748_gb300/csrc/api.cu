@@ -264,6 +264,7 @@ retrace_status enqueue_conditioning(const ConditioningArgs& c, retrace_dtype dty
     a.rowmap = reinterpret_cast<int32_t*>(w + L.rowmap);
     a.sync = sync;
     a.status = status_word(ws);
+    a.part = swap_part_bytes(B, K, d) ? reinterpret_cast<float*>(reinterpret_cast<char*>(ws) + L.swp) : nullptr;
     RT_CUDA(launch_cond_tc(a, stream), "conditioning kernel launch");
     if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
   } else {
@@ -387,6 +388,7 @@ retrace_status retrace_align_refine(const void* hD, const void* hT, retrace_dtyp
     a.rowmap = rowmap;
     a.sync = sync;
     a.status = status_word(ws);
+    a.part = swap_part_bytes(B, K, d) ? reinterpret_cast<float*>(reinterpret_cast<char*>(ws) + L.swp) : nullptr;
     RT_CUDA(launch_cond_tc(a, stream), "correction kernel launch");
   } else {
     CorrectArgs a{hD, hT, Wc, beta, B, K, d, rows, r_out, 0};
@@ -439,6 +441,7 @@ retrace_status retrace_gate_fuse(const void* e, int64_t e_batch_stride, int64_t 
     a.rowmap = rowmap;
     a.sync = sync;
     a.status = status_word(ws);
+    a.part = swap_part_bytes(B, K, d) ? reinterpret_cast<float*>(reinterpret_cast<char*>(ws) + L.swp) : nullptr;
     RT_CUDA(launch_cond_tc(a, stream), "gate kernel launch");
   } else {
     if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");

@@ -1095,6 +1095,284 @@ __global__ void wait_selftest_kernel(int kind, const uint32_t* flag, uint32_t ta
   if (!ok) atomicOr(status, kFlagWaitTimeout);
 }
 
+// ---------------------------------------------------------------------------
+// Small R (B (K-1) <= kSwapMaxRows conditioned rows): the weights on the M side
+// ---------------------------------------------------------------------------
+// With few rows the 256-row pair tiles are mostly padding and only d/256
+// correction tiles exist, so a handful of SMs stream the weights.  Here the
+// GEMMs run transposed: c^T = W_c [m; u]^T and [v; g_r]^T = [W_v; W_g,r] r^T,
+// the weights as the A operand in 128-row tiles (M = 128, no padding), the
+// rows as B in tiles of up to 256 (N = R rounded up to 16, read on the
+// device), and the K range split so that one resident wave of CTAs streams
+// the weights.  Each CTA writes its fp32 partial [split][row][feature]; a
+// reduction kernel sums the splits in a fixed order (results repeat bit for
+// bit) and applies the epilogue.
+constexpr int SW_STAGES = 4;
+constexpr int SW_THREADS = 256;
+
+// How a GEMM of R rows is cut, the same in the GEMM and its reduction: N
+// tiles of up to 256 rows, work = weight tiles x N tiles, each split `grid /
+// work` ways along K (no empty split).
+struct SwapPlan {
+  int nrows, ntiles, work, splits, kb_split;
+};
+__device__ __forceinline__ SwapPlan swap_plan(int R, int mtiles, int nkb, int grid) {
+  SwapPlan s;
+  s.nrows = (R + 15) / 16 * 16;
+  s.ntiles = (s.nrows + 255) / 256;
+  s.work = mtiles * s.ntiles;
+  int splits = s.work > 0 ? grid / s.work : 1;
+  if (splits < 1) splits = 1;
+  if (splits > nkb) splits = nkb;
+  s.kb_split = (nkb + splits - 1) / splits;
+  s.splits = (nkb + s.kb_split - 1) / s.kb_split;
+  return s;
+}
+
+struct SwapParams {
+  const int32_t* R;
+  int nkb;        // k-blocks of the reduction
+  int mtiles;     // 128-row weight tiles in all
+  int mt_a;       // tiles taken from map A (the others from map A2)
+  int a2_x0;      // column offset of map A2's operand (d: the r half of W_g)
+  int box_n;      // rows of a B box (min(256, the largest R rounded to 16))
+  uint32_t tmem_cols;
+  uint32_t stage_stride;  // bytes per pipeline stage (A tile + B box, 1024-aligned)
+  float* part;            // [splits][nrows][mtiles * 128]
+  uint32_t* status;
+};
+
+__global__ void __launch_bounds__(SW_THREADS, 1)
+    swap_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
+                     const __grid_constant__ CUtensorMap tmB, const SwapParams p) {
+  extern __shared__ uint8_t dsmem[];
+  __shared__ __align__(8) uint64_t bar_full[SW_STAGES];
+  __shared__ __align__(8) uint64_t bar_empty[SW_STAGES];
+  __shared__ __align__(8) uint64_t bar_acc;
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_launch_dependents();
+  if (threadIdx.x == 0) {
+    s_abort = 0;
+    for (int s = 0; s < SW_STAGES; ++s) {
+      mbar_init(smem_u32(&bar_full[s]), 1);
+      mbar_init(smem_u32(&bar_empty[s]), 1);
+    }
+    mbar_init(smem_u32(&bar_acc), 1);
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmA2);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 2) {
+    tmem_alloc(smem_u32(&s_tmem), p.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+  const uint32_t base = (smem_u32(dsmem) + 1023u) & ~1023u;
+  pdl_wait();  // R and the activation rows come from the previous kernels
+  const int R = *(volatile const int32_t*)p.R;
+  const SwapPlan pl = swap_plan(R, p.mtiles, p.nkb, (int)gridDim.x);
+  const int c = blockIdx.x;
+  const bool active = c < pl.work * pl.splits;
+  const int sp = c % pl.splits, w = c / pl.splits;
+  const int mt = w / (pl.ntiles > 0 ? pl.ntiles : 1), nt = w - mt * (pl.ntiles > 0 ? pl.ntiles : 1);
+  const int kb0 = sp * pl.kb_split, kb1 = min(p.nkb, kb0 + pl.kb_split);
+  const int tn = active ? min(256, pl.nrows - nt * 256) : 0;  // rows of this N tile (MMA N)
+
+  if (!active) {
+    // nothing to do: fall through to the teardown
+  } else if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      const bool second = mt >= p.mt_a;
+      const CUtensorMap* ma = second ? &tmA2 : &tmA;
+      const int ay = (second ? mt - p.mt_a : mt) * 128, ax0 = second ? p.a2_x0 : 0;
+      const uint32_t tx = (uint32_t)(BM * BK * 2) + (uint32_t)p.box_n * BK * 2;
+      int kb = kb0;
+      for (; kb < kb1; ++kb) {
+        const int i = kb - kb0;
+        const uint32_t s = (uint32_t)(i % SW_STAGES), ph = (uint32_t)((i / SW_STAGES) & 1);
+        if (!mbar_wait_bounded(smem_u32(&bar_empty[s]), ph ^ 1u, &s_abort)) break;
+        const uint32_t a_dst = base + s * p.stage_stride, b_dst = a_dst + (uint32_t)(BM * BK * 2);
+        mbar_arrive_expect_tx(smem_u32(&bar_full[s]), tx);
+        tma_load_2d(a_dst, ma, ax0 + kb * BK, ay, smem_u32(&bar_full[s]));
+        tma_load_2d(b_dst, &tmB, kb * BK, nt * 256, smem_u32(&bar_full[s]));
+      }
+      if (kb < kb1) {  // a wait expired: flag it, let the copies in flight land
+        raise_abort(&s_abort, p.status);
+        volatile int never = 0;
+        const int first = kb - kb0 > SW_STAGES ? kb - kb0 - SW_STAGES : 0;
+        for (int i = first; i < kb - kb0; ++i)
+          mbar_wait_bounded(smem_u32(&bar_full[i % SW_STAGES]), (uint32_t)((i / SW_STAGES) & 1), &never);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(128, tn);
+      bool ok = true;
+      for (int kb = kb0; kb < kb1; ++kb) {
+        const int i = kb - kb0;
+        const uint32_t s = (uint32_t)(i % SW_STAGES), ph = (uint32_t)((i / SW_STAGES) & 1);
+        if (!mbar_wait_bounded(smem_u32(&bar_full[s]), ph, &s_abort)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a_base = base + s * p.stage_stride, b_base = a_base + (uint32_t)(BM * BK * 2);
+        const uint64_t adesc0 = sw128_kmajor_desc(a_base), bdesc0 = sw128_kmajor_desc(b_base);
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k)
+          tc_mma_bf16(tmem, adesc0 + 2u * k, bdesc0 + 2u * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+        tc_commit(smem_u32(&bar_empty[s]));
+      }
+      tc_commit(smem_u32(&bar_acc));  // accumulator ready (also after a failure)
+      if (!ok) raise_abort(&s_abort, p.status);
+    }
+    __syncwarp();
+  } else if (warp >= 4) {
+    // ---------------- epilogue: the partial of this (weight tile, N tile, split) ----------------
+    const int q = (warp - 4) * 32 + lane;  // weight row of the tile = TMEM lane
+    const bool ok = warp_wait(smem_u32(&bar_acc), 0u, &s_abort);
+    tc_fence_after();
+    if (ok && !s_abort) {
+      const uint32_t taddr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+      const long long mtot = (long long)p.mtiles * 128;
+      float* out = p.part + ((long long)sp * pl.nrows + nt * 256) * mtot + mt * 128 + q;
+      for (int c0 = 0; c0 < tn; c0 += 32) {
+        float v[32];
+        tmem_ld_32cols(taddr + (uint32_t)c0, v);
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (c0 + j < tn) out[(long long)(c0 + j) * mtot] = v[j];  // 32 lanes: 128 contiguous bytes
+      }
+    } else if (!ok && lane == 0) {
+      raise_abort(&s_abort, p.status);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, p.tmem_cols);
+  }
+}
+
+struct SwapReduceParams {
+  int d;
+  const int32_t* R;
+  // the GEMM's cut (swap_plan): weight tiles, k-blocks, grid
+  int mtiles, nkb, grid;
+  const float* part;  // [splits][nrows][mtiles * 128]
+  // correction: r = m + beta * c
+  const __nv_bfloat16* apack;  // m = the first d columns of each packed row
+  float beta;
+  __nv_bfloat16* r_out;
+  int compact_out;
+  // gate: e~ = e + v * sigmoid(g_r + ge)
+  const __nv_bfloat16* e;
+  const float* ge;
+  __nv_bfloat16* e_out;
+  const int32_t* rowmap;
+  // W_g[:, :d] e for a broadcast e, before the wait (it reads inputs only)
+  int do_gemv;
+  CondParams gemv;
+  uint32_t* gemv_next;
+  uint32_t* gemv_done;
+};
+
+// r rows of the packed correction (Eq. 7): eight features per thread; the
+// splits summed in order.  Before it waits for the correction GEMM, every
+// warp takes rows of the gate-bias GEMV W_g[:, :d] e, which thereby overlaps
+// the GEMM.
+__global__ void __launch_bounds__(256) swap_reduce_correction_kernel(const SwapReduceParams p) {
+  pdl_launch_dependents();
+  if (p.do_gemv) gate_bias_rows(p.gemv, p.d, threadIdx.x & 31, p.gemv_next, p.gemv_done);
+  pdl_wait();
+  const int R = *(volatile const int32_t*)p.R;
+  const SwapPlan pl = swap_plan(R, p.mtiles, p.nkb, p.grid);
+  const int d = p.d, vpr = d / 8;
+  const long long n_units = (long long)R * vpr;
+  for (long long u = blockIdx.x * (long long)blockDim.x + threadIdx.x; u < n_units;
+       u += (long long)gridDim.x * blockDim.x) {
+    const int g = (int)(u / vpr), n = (int)(u - (long long)g * vpr) * 8;
+    float c[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) c[j] = 0.f;
+    for (int s = 0; s < pl.splits; ++s) {
+      const float4* src = reinterpret_cast<const float4*>(p.part + ((long long)s * pl.nrows + g) * d + n);
+      const float4 x0 = __ldcg(src), x1 = __ldcg(src + 1);
+      c[0] += x0.x; c[1] += x0.y; c[2] += x0.z; c[3] += x0.w;
+      c[4] += x1.x; c[5] += x1.y; c[6] += x1.z; c[7] += x1.w;
+    }
+    const uint4 mw = __ldcg(reinterpret_cast<const uint4*>(p.apack + (long long)g * 2 * d + n));
+    const uint32_t mwords[4] = {mw.x, mw.y, mw.z, mw.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int w = 0; w < 4; ++w)
+      o[w] = pack_bf16x2(bf16_lo(mwords[w]) + p.beta * c[2 * w], bf16_hi(mwords[w]) + p.beta * c[2 * w + 1]);
+    const long long orow = p.compact_out ? g : __ldcg(p.rowmap + g);
+    *reinterpret_cast<uint4*>(p.r_out + orow * d + n) = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// W_g[:, :d] e alone (a gate-only call: no correction kernel to overlap it
+// with), by the same per-row code, so the bits match the correction path's.
+__global__ void __launch_bounds__(256) swap_gemv_kernel(const SwapReduceParams p) {
+  pdl_launch_dependents();
+  gate_bias_rows(p.gemv, p.d, threadIdx.x & 31, p.gemv_next, p.gemv_done);
+}
+
+// e~ rows of the gated fusion (Eq. 8), broadcast e: v in features 0..d-1 of
+// the partials, the r half of the gate in d..2d-1.
+__global__ void __launch_bounds__(256) swap_reduce_gate_kernel(const SwapReduceParams p) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int R = *(volatile const int32_t*)p.R;
+  const SwapPlan pl = swap_plan(R, p.mtiles, p.nkb, p.grid);
+  const int d = p.d, vpr = d / 8;
+  const long long n_units = (long long)R * vpr;
+  for (long long u = blockIdx.x * (long long)blockDim.x + threadIdx.x; u < n_units;
+       u += (long long)gridDim.x * blockDim.x) {
+    const int g = (int)(u / vpr), n = (int)(u - (long long)g * vpr) * 8;
+    float v[8], gt[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] = gt[j] = 0.f;
+    for (int s = 0; s < pl.splits; ++s) {
+      const float* row = p.part + ((long long)s * pl.nrows + g) * 2 * d;
+      const float4* vs = reinterpret_cast<const float4*>(row + n);
+      const float4* gs = reinterpret_cast<const float4*>(row + d + n);
+      const float4 v0 = __ldcg(vs), v1 = __ldcg(vs + 1), g0 = __ldcg(gs), g1 = __ldcg(gs + 1);
+      v[0] += v0.x; v[1] += v0.y; v[2] += v0.z; v[3] += v0.w;
+      v[4] += v1.x; v[5] += v1.y; v[6] += v1.z; v[7] += v1.w;
+      gt[0] += g0.x; gt[1] += g0.y; gt[2] += g0.z; gt[3] += g0.w;
+      gt[4] += g1.x; gt[5] += g1.y; gt[6] += g1.z; gt[7] += g1.w;
+    }
+    const float4 b0 = __ldcg(reinterpret_cast<const float4*>(p.ge + n));
+    const float4 b1 = __ldcg(reinterpret_cast<const float4*>(p.ge + n) + 1);
+    gt[0] += b0.x; gt[1] += b0.y; gt[2] += b0.z; gt[3] += b0.w;
+    gt[4] += b1.x; gt[5] += b1.y; gt[6] += b1.z; gt[7] += b1.w;
+    const uint4 ew = __ldg(reinterpret_cast<const uint4*>(p.e + n));
+    const uint32_t ewords[4] = {ew.x, ew.y, ew.z, ew.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const float s0 = fast_sigmoid(gt[2 * w]), s1 = fast_sigmoid(gt[2 * w + 1]);
+      o[w] = pack_bf16x2(bf16_lo(ewords[w]) + v[2 * w] * s0, bf16_hi(ewords[w]) + v[2 * w + 1] * s1);
+    }
+    const long long orow = __ldcg(p.rowmap + g);
+    *reinterpret_cast<uint4*>(p.e_out + orow * d + n) = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
 template <bool FUSED>
 cudaError_t ensure_smem_attr() {
   static int done[64] = {0};
@@ -1217,9 +1495,133 @@ static int pair_clusters(const TcCondArgs& a, long long tiles_max_pairs, cudaErr
   return (int)(tiles_max_pairs < n ? tiles_max_pairs : n);
 }
 
+// The small-R path (B (K-1) <= kSwapMaxRows, broadcast e or no gate): each
+// GEMM as split-K tiles of 128 weight rows against the R rows, then its
+// reduction kernel; four launches, each waiting on the one before inside the
+// kernel, which cut the work from the R they read.
+static cudaError_t launch_cond_swap(const TcCondArgs& a, cudaStream_t stream) {
+  const long long rmax = (long long)a.B * (a.K - 1);
+  const int d = a.d;
+  const int rows_max = (int)((rmax + 15) / 16 * 16);
+  const int box_n = rows_max < 256 ? rows_max : 256;
+  const int ntiles_max = (rows_max + 255) / 256;
+  DeviceInfo info;
+  cudaError_t err = device_info(&info);
+  if (err != cudaSuccess) return err;
+  static int attr_done[64] = {0};
+  const int max_smem = SW_STAGES * (BM * BK * 2 + 256 * BK * 2) + 1024;
+  if (!attr_done[info.device & 63]) {
+    err = cudaFuncSetAttribute(swap_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem);
+    if (err != cudaSuccess) return err;
+    attr_done[info.device & 63] = 1;
+  }
+  const uint32_t stage_stride = (uint32_t)((BM * BK * 2 + box_n * BK * 2 + 1023) / 1024 * 1024);
+  const int smem = SW_STAGES * (int)stage_stride + 1024;
+  uint32_t tmem_cols = 32;
+  while ((int)tmem_cols < box_n) tmem_cols <<= 1;
+  // One resident wave when it can carry every work tile: a split's CTA
+  // streams its whole K range, so a second wave would double the time.
+  static int occ_cache[64][256 / 16 + 1] = {};
+  int& occ = occ_cache[info.device & 63][box_n / 16];
+  if (occ == 0) {
+    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, swap_gemm_kernel, SW_THREADS, (size_t)smem);
+    if (err != cudaSuccess) return err;
+    if (occ < 1) occ = 1;
+  }
+  int resident = info.sm_count * occ;
+  if (resident > kSwapMaxCtas) resident = kSwapMaxCtas;
+  const uint64_t du = (uint64_t)d;
+  auto params = [&](SwapParams& sp, int mtiles, int nkb) {
+    sp.R = a.R;
+    sp.nkb = nkb;
+    sp.mtiles = mtiles;
+    sp.box_n = box_n;
+    sp.tmem_cols = tmem_cols;
+    sp.stage_stride = stage_stride;
+    sp.part = a.part;
+    sp.status = a.status;
+    const int work_max = mtiles * ntiles_max;
+    return work_max > resident ? work_max : resident;  // the grid
+  };
+  SwapReduceParams rp{};
+  rp.d = d;
+  rp.R = a.R;
+  rp.part = a.part;
+  rp.rowmap = a.rowmap;
+  const int red_grid = info.sm_count * 4;
+  const bool gemv = a.do_gate && !a.e_dense;
+  if (a.do_correct) {
+    CUtensorMap mA, mB;
+    if (encode_tensor_map_2d(&mA, a.Wc, 2 * du, du, 4 * du, BK, 128) != CUDA_SUCCESS ||
+        encode_tensor_map_2d(&mB, a.apack, 2 * du, (uint64_t)rmax, 4 * du, BK, (uint32_t)box_n) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+    SwapParams sp{};
+    const int grid = params(sp, d / 128, 2 * d / BK);
+    sp.mt_a = d / 128;
+    sp.a2_x0 = 0;
+    err = launch_dependent(swap_gemm_kernel, dim3((unsigned)grid), dim3(SW_THREADS), (size_t)smem, stream, 1u, mA,
+                           mA, mB, sp);
+    if (err != cudaSuccess) return err;
+    rp.mtiles = sp.mtiles;
+    rp.nkb = sp.nkb;
+    rp.grid = grid;
+    rp.do_gemv = gemv ? 1 : 0;  // overlapping the correction GEMM
+    rp.gemv.d = d;
+    rp.gemv.e = reinterpret_cast<const __nv_bfloat16*>(a.e);
+    rp.gemv.Wg = reinterpret_cast<const __nv_bfloat16*>(a.Wg);
+    rp.gemv.ge = a.ge;
+    rp.gemv_next = a.sync + kSyncGemvNext;
+    rp.gemv_done = a.sync + kSyncGemvDone;
+    rp.apack = reinterpret_cast<const __nv_bfloat16*>(a.apack);
+    rp.beta = a.beta;
+    rp.r_out = reinterpret_cast<__nv_bfloat16*>(a.r_out);
+    rp.compact_out = a.compact_out;
+    err = launch_dependent(swap_reduce_correction_kernel, dim3((unsigned)red_grid), dim3(256), 0, stream, 1u, rp);
+    if (err != cudaSuccess) return err;
+  }
+  if (a.do_gate) {
+    const uint64_t rstride = 2 * (a.r_row_stride ? (uint64_t)a.r_row_stride : du);
+    CUtensorMap mA, mA2, mB;
+    if (encode_tensor_map_2d(&mA, a.Wv, du, du, 2 * du, BK, 128) != CUDA_SUCCESS ||
+        encode_tensor_map_2d(&mA2, a.Wg, 2 * du, du, 4 * du, BK, 128) != CUDA_SUCCESS ||
+        encode_tensor_map_2d(&mB, a.rpack, du, (uint64_t)rmax, rstride, BK, (uint32_t)box_n) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+    if (gemv && !a.do_correct) {  // no correction kernel to overlap the GEMV with
+      SwapReduceParams gp{};
+      gp.d = d;
+      gp.gemv.d = d;
+      gp.gemv.e = reinterpret_cast<const __nv_bfloat16*>(a.e);
+      gp.gemv.Wg = reinterpret_cast<const __nv_bfloat16*>(a.Wg);
+      gp.gemv.ge = a.ge;
+      gp.gemv_next = a.sync + kSyncGemvNext;
+      gp.gemv_done = a.sync + kSyncGemvDone;
+      err = launch_dependent(swap_gemv_kernel, dim3((unsigned)red_grid), dim3(256), 0, stream, 1u, gp);
+      if (err != cudaSuccess) return err;
+    }
+    SwapParams sp{};
+    const int grid = params(sp, 2 * d / 128, d / BK);
+    sp.mt_a = d / 128;  // W_v rows first, then the r half of W_g
+    sp.a2_x0 = d;
+    err = launch_dependent(swap_gemm_kernel, dim3((unsigned)grid), dim3(SW_THREADS), (size_t)smem, stream, 1u, mA,
+                           mA2, mB, sp);
+    if (err != cudaSuccess) return err;
+    rp.mtiles = sp.mtiles;
+    rp.nkb = sp.nkb;
+    rp.grid = grid;
+    rp.do_gemv = 0;
+    rp.e = reinterpret_cast<const __nv_bfloat16*>(a.e);
+    rp.ge = a.ge;
+    rp.e_out = reinterpret_cast<__nv_bfloat16*>(a.e_out);
+    err = launch_dependent(swap_reduce_gate_kernel, dim3((unsigned)red_grid), dim3(256), 0, stream, 1u, rp);
+    if (err != cudaSuccess) return err;
+  }
+  return cudaSuccess;
+}
+
 cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream) {
   const long long rmax = (long long)a.B * (a.K - 1);
   if (rmax <= 0 || (!a.do_correct && !a.do_gate)) return cudaSuccess;
+  if (a.part && !(a.do_gate && a.e_dense)) return launch_cond_swap(a, stream);
   const long long tiles_max_pairs =
       (rmax + 2 * BM - 1) / (2 * BM) * ((a.do_correct ? a.d / 256 : 0) + (a.do_gate ? a.d / 128 : 0));
   cudaError_t err;

@@ -36,11 +36,28 @@ constexpr int kLowRankLatent = 64;      // rank of the rejected-suffix latents
 constexpr int kLowRankCorrection = 32;  // rank of the target-aware correction
 constexpr int kLowRankSplits = 8;       // split-K parts per half of the [m; u] reduction
 //   skeys    uint64 [B*(2K+1), 64]  sampled verification: top-k keys per target and drafter row
+//   swp      fp32   (small R only)  split partials of the small-R conditioning GEMMs
 constexpr int kMaxTopK = 64;            // largest top_k of sampled verification
 constexpr int kWindowRows = 4;          // rows per pass of windowed verification
 constexpr int kMaxWindowPasses = 16;    // most passes of windowed verification
+// Small-R conditioning (at most kSwapMaxRows packed rows): the GEMMs as
+// split-K tiles of 128 weight rows against N tiles of up to 256 rows, one
+// grid of at most max(kSwapMaxCtas, work tiles) CTAs, each writing an fp32
+// partial of at most 128 x min(256, rows) values.  Taken while the gate
+// GEMM's work tiles (2d/128 x N tiles) fit in kSwapMaxCtas.
+constexpr int kSwapMaxRows = 1024;
+constexpr int kSwapMaxCtas = 256;
+inline size_t swap_part_bytes(long long B, long long K, long long d) {
+  const long long rmax = B * (K > 1 ? K - 1 : 0);
+  if (rmax <= 0 || rmax > kSwapMaxRows || d <= 0) return 0;
+  const long long rows = (rmax + 15) / 16 * 16;
+  const long long ntiles = (rows + 255) / 256;
+  if ((2 * d / 128) * ntiles > kSwapMaxCtas) return 0;
+  const long long box = rows < 256 ? rows : 256;
+  return (size_t)(kSwapMaxCtas * 128 * box * 4);
+}
 struct WsLayout {
-  size_t status, sync, sync_bytes, keys, tickets, live, poff, counts, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, skeys, total;
+  size_t status, sync, sync_bytes, keys, tickets, live, poff, counts, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, skeys, swp, total;
 };
 
 inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
@@ -82,6 +99,8 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   off = align_up(off + rmax * kLowRankLatent * elem, 256);
   L.skeys = off;
   off = align_up(off + (size_t)(B * (2 * K + 1)) * kMaxTopK * 8, 256);
+  L.swp = off;
+  off = align_up(off + swap_part_bytes(B, K, d), 256);
   L.total = off;
   return L;
 }
@@ -312,6 +331,8 @@ struct TcCondArgs {
   const int32_t* rowmap;
   uint32_t* sync;
   uint32_t* status;
+  // small-R path (B (K-1) <= kSwapMaxRows): fp32 split partials, swap_part_bytes (NULL: not taken)
+  float* part;
 };
 cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream);
 // The bounded waits of the pipelined kernels on a caller-controlled condition.

@@ -169,8 +169,9 @@ def accept_for_rows(B, K, R):
 @pytest.mark.parametrize("R", [1, 127, 128, 129, 255, 256, 257, 384, 513])
 def test_pair_tile_boundaries(rt, R):
     """Row counts around the 128-row halves and 256-row pairs of the
-    tensor-core kernel (one CTA's half empty, odd block counts)."""
-    B, K, d, dtype = 40, 16, 256, torch.bfloat16
+    CTA-pair kernel (one CTA's half empty, odd block counts).  B (K-1) = 1200
+    possible rows keeps the call off the small-R path."""
+    B, K, d, dtype = 80, 16, 256, torch.bfloat16
     x = make_inputs(B, K, d, dtype, seed=R, accept=accept_for_rows(B, K, R))
     A = host_int(x["accept"])
     n_host = oracle.carried_rows(A, K)
@@ -189,3 +190,38 @@ def test_pair_tile_boundaries(rt, R):
     e_full = np.broadcast_to(host_f64(x["e_vec"]), (B, K, d))
     want = oracle.gate_fuse(e_full, host_f64(r), n_host, host_f64(x["Wv"]), host_f64(x["Wg"]))
     assert_close(out, want, f"e~, R={R}")
+
+
+@pytest.mark.parametrize("B,K,d", [(1, 2, 256), (3, 6, 512), (16, 16, 256), (16, 17, 256), (8, 16, 2560),
+                                   (17, 16, 256), (40, 16, 256), (64, 17, 256)])
+def test_small_r_path(rt, B, K, d):
+    """At most 1024 conditioned rows (B (K-1) <= 1024): the GEMMs run with the
+    weights as the 128-row side against N tiles of up to 256 rows, split over
+    K, the partials summed in a fixed order.  Every draft rejected at once
+    (A_b = 0), so all B (K-1) rows are carried: 1, 15, 240, 256, 255, 600 and
+    1024 rows (one to four N tiles, the last one partial) and d up to 2560;
+    both entry points against the oracle, repeatable bit for bit."""
+    dtype = torch.bfloat16
+    x = make_inputs(B, K, d, dtype, seed=B * 100 + K, accept=torch.zeros(B, dtype=torch.int32).cuda())
+    A = host_int(x["accept"])
+    n_host = oracle.carried_rows(A, K)
+    assert n_host.sum() == B * (K - 1)
+    ws = rt.Workspace(B, K, 8, d, dtype)
+    outs = []
+    for _ in range(2):
+        r = torch.full((B, K, d), 9.0, dtype=dtype, device="cuda")
+        n = torch.empty((B,), dtype=torch.int32, device="cuda")
+        rt.retrace_align_refine(x["hD"], x["hT"], x["accept"], x["Wc"], 0.75, r, n, ws)
+        out = torch.full((B, K, d), 7.0, dtype=dtype, device="cuda")
+        rt.retrace_gate_fuse(x["e_vec"], r, n, x["Wv"], x["Wg"], out, ws)
+        torch.cuda.synchronize()
+        outs.append((r, out))
+    assert ws.check() == 0
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+    r, out = outs[0]
+    m, u = oracle.align(host_f64(x["hD"]), host_f64(x["hT"]), A)
+    r_ref = oracle.correct(m, u, host_f64(x["Wc"]), 0.75, round_r_bf16=False)
+    assert_close(r, r_ref, f"r, B={B} K={K}")
+    e_full = np.broadcast_to(host_f64(x["e_vec"]), (B, K, d))
+    want = oracle.gate_fuse(e_full, host_f64(r), n_host, host_f64(x["Wv"]), host_f64(x["Wg"]))
+    assert_close(out, want, f"e~, B={B} K={K}")

@@ -24,6 +24,14 @@ def rt():
     return binding
 
 
+def small_r_path(B, K, d):
+    """Whether the conditioning of a bf16 round with a broadcast e takes the
+    small-R GEMMs: at most 1024 possible rows, and the gate GEMM's work tiles
+    (2d/128 weight tiles x N tiles of 256 rows) at most 256."""
+    rows = (B * (K - 1) + 15) // 16 * 16
+    return 0 < rows <= 1024 and (2 * d // 128) * ((rows + 255) // 256) <= 256
+
+
 def run(rt, x, ws=None, **kw):
     cfg = x["cfg"]
     if ws is None:
@@ -143,7 +151,9 @@ def test_overlapped_round_equals_separate_entry_points(rt, cfg_id):
     projections overlapped in one persistent kernel) against retrace_verify +
     retrace_align_refine + retrace_gate_fuse on the same inputs: identical
     bits, since every output element is computed by the same arithmetic in
-    the same order."""
+    the same order -- except where the separate entry points take the
+    small-R path (split-K sums, another fp32 summation order), where both
+    must match the oracle instead."""
     x = make_round_inputs(CONFIGS[cfg_id], device="cuda")
     cfg = x["cfg"]
     fused, targ, ws = run(rt, x, flags=rt.ROUND_OVERLAP)
@@ -163,12 +173,19 @@ def test_overlapped_round_equals_separate_entry_points(rt, cfg_id):
     assert torch.equal(com, fused.committed)
     assert torch.equal(bon, fused.bonus)
     assert torch.equal(n, fused.n)
-    assert torch.equal(e_out, fused.e_out)
+    if small_r_path(B, K, d):
+        want = oracle_round(x)
+        assert_close(fused.e_out, want["e_tilde"], "overlapped round")
+        assert_close(e_out, want["e_tilde"], "separate entry points, small-R path")
+    else:
+        assert torch.equal(e_out, fused.e_out)
 
 
 def test_overlapped_round_matches_the_oracle_and_the_default_path(rt):
     """The overlapped kernel on the serving shape's sibling (B = 64): oracle
-    parity, and the same bits as the default two-launch round."""
+    parity, and the default round's outputs (the same bits where both take
+    the same GEMMs; at B = 64 the default round takes the small-R path, so
+    both are held to the oracle)."""
     x = make_round_inputs(CONFIGS[4], device="cuda")
     over, targ, ws = run(rt, x, flags=rt.ROUND_OVERLAP)
     assert ws.check() == 0
@@ -176,8 +193,12 @@ def test_overlapped_round_matches_the_oracle_and_the_default_path(rt):
     assert_verify_exact(want, over.accept_len, over.committed, over.bonus, targ)
     assert_close(over.e_out, want["e_tilde"], "overlapped round")
     plain, _, _ = run(rt, x, ws=ws)
-    assert torch.equal(plain.e_out, over.e_out)
     assert torch.equal(plain.n, over.n)
+    cfg = x["cfg"]
+    if small_r_path(cfg.B, cfg.K, cfg.d):
+        assert_close(plain.e_out, want["e_tilde"], "default round, small-R path")
+    else:
+        assert torch.equal(plain.e_out, over.e_out)
 
 
 def test_overlap_flag_rejects_what_the_kernel_does_not_cover(rt):
