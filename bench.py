@@ -642,13 +642,20 @@ def run_e2e(cfg, x, dev, steps, world, round_fn, names) -> dict:
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps}
 
 
+CPU_BASELINE_SECONDS = 10.0  # the oracle's sample is repeated until it has run this long
+
+
 def cpu_baseline(cfg: RoundConfig, args) -> dict:
     host = prepare_oracle_sample(cfg, args.cpu_sample, seed=1234, lowrank=args.lowrank, sampled=args.sampled)
-    secs = time_oracle(host, args.variant)
+    times = []
+    while sum(times) < CPU_BASELINE_SECONDS and len(times) < 200:
+        times.append(time_oracle(host, args.variant))
+    secs = sum(times) / len(times)
     rounds = host["B"] / cfg.B
     return {"value": round(rounds / secs, 6), "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
-            "sample": f"{host['B']} of {cfg.B} sequences of {cfg.name}, full-size weights; one round of the "
-                      f"sample took {secs:.2f} s, scaled by {host['B']}/{cfg.B} to rounds/s"}
+            "sample": f"{host['B']} of {cfg.B} sequences of {cfg.name}, full-size weights, run {len(times)} times "
+                      f"({sum(times):.1f} s of CPU work); one round of the sample took {secs:.2f} s on average, "
+                      f"scaled by {host['B']}/{cfg.B} to rounds/s"}
 
 
 # ---------------------------------------------------------------------------
