@@ -241,3 +241,17 @@ def test_verify_schedule_plan(lib):
         assert lib.retrace_set_verify_schedule(9) == -1
     finally:
         lib.retrace_set_verify_schedule(prev)
+
+
+def test_workspace_holds_small_r_partials(lib):
+    """At most 1024 conditioned rows (and the gate GEMM's work tiles within 256
+    CTAs) the workspace also holds the split partials of the small-R GEMMs:
+    256 CTAs x 128 weight rows x min(256, rows rounded to 16) fp32."""
+    ws = lib.retrace_workspace_bytes
+    for B, K, d in ((1, 16, 2560), (8, 16, 4096), (64, 16, 2560), (64, 17, 4096)):
+        rows = (B * (K - 1) + 15) // 16 * 16
+        part = 256 * 128 * min(256, rows) * 4
+        assert ws(B, K, 1000, d, BF16) >= part
+    small = ws(64, 17, 1000, 4096, BF16)   # 1024 rows: partials of 32 MiB
+    large = ws(65, 17, 1000, 4096, BF16)   # 1040 rows: the CTA-pair path, no partials
+    assert small - large > 30 << 20

@@ -265,3 +265,28 @@ def test_raw_variant_equals_zero_beta_on_the_default_path(rt):
     raw, _, ws = run(rt, x, flags=rt.COND_RAW)
     zero, _, _ = run(rt, {**x, "beta": 0.0}, ws=ws)
     assert torch.equal(raw.e_out, zero.e_out)
+
+
+@pytest.mark.parametrize("R", [0, 1])
+def test_small_r_round_with_almost_nothing_to_condition(rt, R):
+    """Config 3's shapes (small-R GEMMs) with every draft accepted (R = 0: no
+    row is conditioned, the GEMMs' CTAs all idle) or all but one row (R = 1):
+    e~ keeps e bit for bit wherever no signal is carried, and the one
+    conditioned row matches the oracle."""
+    cfg = CONFIGS[3]
+    x = make_round_inputs(cfg, device="cuda")
+    top = torch.argmax(x["logits"][:, : cfg.K].float(), dim=-1).to(torch.int32)
+    x["draft"] = top.clone()
+    if R == 1:  # sequence 0 rejects its draft at position K-2: n_0 = 1
+        x["draft"][0, cfg.K - 2] = (top[0, cfg.K - 2] + 1) % cfg.V
+    out, targ, ws = run(rt, x)
+    assert ws.check() == 0
+    want = oracle_round(x)
+    assert_verify_exact(want, out.accept_len, out.committed, out.bonus, targ)
+    assert int(out.n.sum()) == R
+    assert_close(out.e_out, want["e_tilde"], f"R={R}")
+    got = host_f64(out.e_out)
+    e = host_f64(x["e"])
+    for b in range(cfg.B):
+        nb = int(want["n"][b])
+        assert np.array_equal(got[b, nb:], np.broadcast_to(e, got[b, nb:].shape))
