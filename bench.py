@@ -436,6 +436,15 @@ def run_gpu(args) -> dict | None:
     windows = [0, cfg.K + 1] if fused else rt.retrace_verify_plan(cfg.B, cfg.K, cfg.V, cfg.torch_dtype)
     n_pass = len(windows) - 1
     verify_launches = n_pass * (2 if args.sampled else 1) + (1 if n_pass > 1 else 0)
+    # conditioning launches of the greedy and temperature-1 rounds, by path
+    rows = (cfg.B * (cfg.K - 1) + 15) // 16 * 16
+    small_r = 0 < rows <= 1024 and (2 * cfg.d // 128) * ((rows + 255) // 256) <= 256
+    if cfg.dtype != "bf16" or cfg.d % 256:
+        cond_launches = 3  # correction, gate bias, gate (FFMA)
+    elif small_r:
+        cond_launches = 4 if args.variant == "corrected" else 3  # GEMM + reduction each; raw: GEMV, GEMM, reduction
+    else:
+        cond_launches = 1  # cond_pair_kernel
     step_avg_s = statistics.mean(step_ms) / 1e3
     cflops = (lowrank_flops(cfg, R) if args.lowrank
               else conditioning_flops(cfg, R, dense_e=False, variant=args.variant))
@@ -534,8 +543,8 @@ def run_gpu(args) -> dict | None:
             }
         elif cflops:
             c_roof = {
-                "kernel": "cond_pair_kernel: correction + gated-fusion projections (+ gate-bias GEMV), one persistent "
-                          "launch on CTA pairs (tcgen05.mma.cta_group::2)",
+                "kernel": ("cond_pair_kernel: correction + gated-fusion projections (+ gate-bias GEMV), one persistent "
+                           "launch on CTA pairs (tcgen05.mma.cta_group::2)"),
                 "bound": "tensor",
                 "achieved": round(c_tflops, 2),
                 "peak": peaks["bf16_tflops"],
@@ -548,6 +557,30 @@ def run_gpu(args) -> dict | None:
                 "traffic": (COND_TRAFFIC.get(cfg.name) if args.variant == "corrected" and not args.sampled else None),
                 "traffic_source": "ncu dram read+write of one launch on this workload",
             }
+            if cfg.dtype != "bf16" or cfg.d % 256:
+                # fp32 (no TF32) or shapes the tensor-core kernels do not take: plain FFMA
+                props = torch.cuda.get_device_properties(dev)
+                max_mhz = (clocks.summary() or {}).get("sm_max_mhz") or 2070.0
+                ffma_peak = props.multi_processor_count * 128 * 2 * max_mhz * 1e6 / 1e12
+                c_roof.update({
+                    "kernel": "FFMA path: simt_correct_kernel, gate_bias_kernel, simt_gate_kernel",
+                    "bound": "alu", "peak": round(ffma_peak, 1), "frac": round(c_tflops / ffma_peak, 4),
+                    "peak_source": "derived: SMs x 128 FP32 lanes x 2 flop per FMA x maximum SM clock",
+                    "frac_of_sustained": None, "traffic": None})
+            elif small_r:
+                # weights streamed once dominate: HBM-bound at these row counts
+                es, d = cfg.elem_bytes, cfg.d
+                cbytes = 5 * d * d * es + R * (2 * d + d + d) * es + R * d * 2
+                c_roof.update({
+                    "kernel": ("small-R GEMMs: swap_gemm_kernel (tcgen05, weights as the 128-row side, split-K) for "
+                               "each projection, each followed by its reduction kernel"),
+                    "bound": "hbm", "achieved": round(cbytes / c_avg_s / 1e9, 1), "peak": peaks["hbm_gbs"],
+                    "unit": "GB/s", "frac": round(cbytes / c_avg_s / 1e9 / peaks["hbm_gbs"], 4),
+                    "peak_source": peaks["source"] + " HBM copy bandwidth",
+                    "algorithmic_bytes": cbytes,
+                    "algorithmic_bytes_note": "W_c, W_v, W_g once; packed [m; u] rows read, r written and read, "
+                                              "e~ rows written",
+                    "achieved_tflops": round(c_tflops, 3), "frac_of_sustained": None, "traffic": None})
         # `roofline` is the kernel that takes the larger share of the round
         roofline = c_roof if (c_roof and c_avg_s > v_avg_s) else v_roof
         line_extra = {"roofline_verify": v_roof, "roofline_conditioning": c_roof}
@@ -596,8 +629,8 @@ def run_gpu(args) -> dict | None:
         "e2e": e2e,
         "gpu_launches": (KERNELS_PER_ROUND_FUSED if fused
                          else KERNELS_PER_ROUND_LOWRANK - 1 + verify_launches if args.lowrank
-                         else verify_launches + 1 if args.sampled
-                         else KERNELS_PER_ROUND - 1 + verify_launches if cflops else verify_launches) * steps,
+                         else verify_launches + cond_launches if (args.sampled or cflops)
+                         else verify_launches) * steps,
         "wall_s_timed_region": round(t_wall, 4),
         "device_status_flags": status_flags,
         "impl": "ours",
