@@ -217,6 +217,155 @@ __global__ void __launch_bounds__(kNT) simt_gate_kernel(const SimtGateParams p) 
   }
 }
 
+// ---------------------------------------------------------------------------
+// Few rows (B (K-1) <= kRowsMax): one warp per output feature
+// ---------------------------------------------------------------------------
+// With a handful of rows the 32 x 64 tiles above leave all but d/64 SMs idle
+// and walk the reduction in 32-deep steps, one load latency each.  Here each
+// warp owns one output feature n and all rows: its lanes stride the
+// reduction index (coalesced loads of the weight row, the operand rows read
+// through L1), each lane keeps kRowGroup row sums, and a butterfly of
+// shuffles adds the lanes in a fixed order (results repeat bit for bit).
+// The rows are taken kRowGroup at a time; the weight row is re-read per group.
+constexpr int kRowsMax = 32;  // one plan tile
+constexpr int kRowGroup = 8;
+constexpr int kRowsWarps = kNT / 32;
+
+__device__ __forceinline__ float warp_sum(float s) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, off);
+  return s;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kNT) simt_rows_correct_kernel(const SimtCorrectParams p) {
+  __shared__ int s_b[kRowsMax], s_j[kRowsMax], s_nb[kRowsMax], s_scan[kNT / 32 + 1];
+  __shared__ long long s_m[kRowsMax], s_u[kRowsMax];
+  const int R = plan_tile<kNT, kRowsMax>(p.rows, p.B, p.K, 0, s_b, s_j, s_nb, s_scan);
+  const int K = p.K, d = p.d, tid = threadIdx.x, lane = tid & 31;
+  if (tid < kRowsMax) {
+    const int b = s_b[tid];
+    const int A = K - 1 - s_nb[tid];
+    s_m[tid] = b >= 0 ? ((long long)b * K + A + 1 + s_j[tid]) * d : 0;  // m_j = hD[b, A+1+j]
+    s_u[tid] = b >= 0 ? ((long long)b * K + A + s_j[tid]) * d : 0;      // u_j = hT[b, A+j]
+  }
+  __syncthreads();
+  const int n = blockIdx.x * kRowsWarps + (tid >> 5);
+  if (n >= d) return;
+  const T* hD = reinterpret_cast<const T*>(p.hD);
+  const T* hT = reinterpret_cast<const T*>(p.hT);
+  const T* w = reinterpret_cast<const T*>(p.Wc) + (long long)n * 2 * d;
+  T* out = reinterpret_cast<T*>(p.out);
+  const int nrows = R < kRowsMax ? R : kRowsMax;
+  for (int g0 = 0; g0 < nrows; g0 += kRowGroup) {
+    const int gn = nrows - g0 < kRowGroup ? nrows - g0 : kRowGroup;
+    float acc[kRowGroup];
+#pragma unroll
+    for (int q = 0; q < kRowGroup; ++q) acc[q] = 0.f;
+    if (!p.raw) {
+      // c = W_c [m; u]: the m half (k < d), then the u half
+      for (int half = 0; half < 2; ++half) {
+        const T* wh = w + half * d;
+#pragma unroll 4
+        for (int k = lane; k < d; k += 32) {
+          const float wk = to_f32(wh[k]);
+#pragma unroll
+          for (int q = 0; q < kRowGroup; ++q) {
+            if (q < gn) {
+              const T* src = half == 0 ? hD + s_m[g0 + q] : hT + s_u[g0 + q];
+              acc[q] = fmaf(wk, to_f32(src[k]), acc[q]);
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < kRowGroup; ++q) acc[q] = warp_sum(acc[q]);
+    }
+    if (lane < gn) {
+      float a = acc[0];
+#pragma unroll
+      for (int q = 1; q < kRowGroup; ++q)
+        if (lane == q) a = acc[q];
+      const int row = g0 + lane;
+      const long long orow = p.compact_out ? row : ((long long)s_b[row] * K + s_j[row]);
+      const T m = hD[s_m[row] + n];
+      out[orow * d + n] = p.raw ? m : from_f32<T>(to_f32(m) + p.beta * a);
+    }
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kNT) simt_rows_gate_kernel(const SimtGateParams p) {
+  __shared__ int s_b[kRowsMax], s_j[kRowsMax], s_nb[kRowsMax], s_scan[kNT / 32 + 1];
+  __shared__ long long s_r[kRowsMax], s_e[kRowsMax];
+  const int R = plan_tile<kNT, kRowsMax>(p.rows, p.B, p.K, 0, s_b, s_j, s_nb, s_scan);
+  const int K = p.K, d = p.d, tid = threadIdx.x, lane = tid & 31;
+  if (tid < kRowsMax) {
+    const int b = s_b[tid];
+    const long long pos = b >= 0 ? (long long)b * K + s_j[tid] : 0;
+    s_r[tid] = (p.r_compact ? tid : pos) * d;
+    s_e[tid] = p.e_dense ? pos * d : 0;
+  }
+  __syncthreads();
+  const int n = blockIdx.x * kRowsWarps + (tid >> 5);
+  if (n >= d) return;
+  const T* r = reinterpret_cast<const T*>(p.r);
+  const T* e = reinterpret_cast<const T*>(p.e);
+  const T* wv = reinterpret_cast<const T*>(p.Wv) + (long long)n * d;
+  const T* wg = reinterpret_cast<const T*>(p.Wg) + (long long)n * 2 * d;
+  T* out = reinterpret_cast<T*>(p.out);
+  const int nrows = R < kRowsMax ? R : kRowsMax;
+  for (int g0 = 0; g0 < nrows; g0 += kRowGroup) {
+    const int gn = nrows - g0 < kRowGroup ? nrows - g0 : kRowGroup;
+    float av[kRowGroup], ag[kRowGroup];
+#pragma unroll
+    for (int q = 0; q < kRowGroup; ++q) av[q] = ag[q] = 0.f;
+    // v = W_v r and the r half of the gate, W_g[:, d:2d] r
+#pragma unroll 2
+    for (int k = lane; k < d; k += 32) {
+      const float wvk = to_f32(wv[k]), wgk = to_f32(wg[d + k]);
+#pragma unroll
+      for (int q = 0; q < kRowGroup; ++q) {
+        if (q < gn) {
+          const float x = to_f32(r[s_r[g0 + q] + k]);
+          av[q] = fmaf(wvk, x, av[q]);
+          ag[q] = fmaf(wgk, x, ag[q]);
+        }
+      }
+    }
+    // per-position e: the e half of the gate, W_g[:, 0:d] e
+    if (p.e_dense) {
+#pragma unroll 4
+      for (int k = lane; k < d; k += 32) {
+        const float wk = to_f32(wg[k]);
+#pragma unroll
+        for (int q = 0; q < kRowGroup; ++q)
+          if (q < gn) ag[q] = fmaf(wk, to_f32(e[s_e[g0 + q] + k]), ag[q]);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < kRowGroup; ++q) {
+      av[q] = warp_sum(av[q]);
+      ag[q] = warp_sum(ag[q]);
+    }
+    if (lane < gn) {
+      float v = av[0], gs = ag[0];
+#pragma unroll
+      for (int q = 1; q < kRowGroup; ++q)
+        if (lane == q) {
+          v = av[q];
+          gs = ag[q];
+        }
+      const int row = g0 + lane;
+      const long long orow = (long long)s_b[row] * K + s_j[row];
+      const float g = gs + (p.e_dense ? 0.f : p.ge[n]);
+      const float ev = to_f32(e[s_e[row] + n]);
+      const float gate = 1.f / (1.f + expf(-g));
+      out[orow * d + n] = from_f32<T>(ev + v * gate);
+    }
+  }
+}
+
 // ge[i] = sum_k W_g[i, k] e[k] over the e half (k < d), one warp per output.
 template <typename T>
 __global__ void __launch_bounds__(256) gate_bias_kernel(const T* __restrict__ Wg,
@@ -255,6 +404,10 @@ cudaError_t correct_typed(const CorrectArgs& a, cudaStream_t stream) {
   SimtCorrectParams p{a.hD, a.hT, a.Wc, a.beta, a.B, a.K, a.d, a.rows, a.r_out, a.compact_out, a.raw};
   const long long rmax = (long long)a.B * (a.K - 1);
   if (rmax <= 0) return cudaSuccess;
+  if (rmax <= kRowsMax) {
+    simt_rows_correct_kernel<T><<<(unsigned)((a.d + kRowsWarps - 1) / kRowsWarps), kNT, 0, stream>>>(p);
+    return cudaGetLastError();
+  }
   dim3 grid((unsigned)((rmax + TM - 1) / TM), (unsigned)((a.d + TN - 1) / TN));
   simt_correct_kernel<T><<<grid, kNT, 0, stream>>>(p);
   return cudaGetLastError();
@@ -265,6 +418,10 @@ cudaError_t gate_typed(const GateArgs& a, cudaStream_t stream) {
   SimtGateParams p{a.e, a.e_dense, a.r, a.r_compact, a.Wv, a.Wg, a.ge, a.B, a.K, a.d, a.rows, a.e_out};
   const long long rmax = (long long)a.B * (a.K - 1);
   if (rmax <= 0) return cudaSuccess;
+  if (rmax <= kRowsMax) {
+    simt_rows_gate_kernel<T><<<(unsigned)((a.d + kRowsWarps - 1) / kRowsWarps), kNT, 0, stream>>>(p);
+    return cudaGetLastError();
+  }
   dim3 grid((unsigned)((rmax + TM - 1) / TM), (unsigned)((a.d + TN - 1) / TN));
   simt_gate_kernel<T><<<grid, kNT, 0, stream>>>(p);
   return cudaGetLastError();

@@ -53,6 +53,8 @@ SHAPES = [
     (3, 5, 100, torch.bfloat16),
     (2, 8, 256, torch.float32),
     (6, 16, 96, torch.float32),
+    (4, 9, 160, torch.float32),  # B (K-1) = 32: the last shape of the warp-per-feature kernel
+    (3, 12, 160, torch.bfloat16),  # B (K-1) = 33: the first of the 32 x 64 tiles
 ]
 
 
