@@ -436,6 +436,13 @@ def run_gpu(args) -> dict | None:
     windows = [0, cfg.K + 1] if fused else rt.retrace_verify_plan(cfg.B, cfg.K, cfg.V, cfg.torch_dtype)
     n_pass = len(windows) - 1
     verify_launches = n_pass * (2 if args.sampled else 1) + (1 if n_pass > 1 else 0)
+    # one greedy pass that packs rows for the tensor-core projections hands its
+    # copies to the copy kernel when there are fewer sequences than SMs
+    packs = cfg.dtype == "bf16" and (cfg.d % 64 == 0 if args.lowrank
+                                     else cfg.d % 256 == 0 and args.variant in ("corrected", "raw"))
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    if n_pass == 1 and not (fused or args.sampled) and packs and cfg.B < sms:
+        verify_launches += 1
     # conditioning launches of the greedy and temperature-1 rounds, by path
     rows = (cfg.B * (cfg.K - 1) + 15) // 16 * 16
     small_r = 0 < rows <= 1024 and (2 * cfg.d // 128) * ((rows + 255) // 256) <= 256
@@ -495,6 +502,8 @@ def run_gpu(args) -> dict | None:
         v_roof = {
             "kernel": (f"verify_kernel x{n_pass} passes over row windows {windows} + verify_copy_kernel (copy of "
                        "unconditioned rows + row packing)" if n_pass > 1 else
+                       "verify_kernel (argmax/compare/commit) + verify_copy_kernel (copy of unconditioned rows + "
+                       "row packing)" if verify_launches == 2 and not args.sampled else
                        "verify_kernel (argmax/compare/commit + copy of unconditioned rows + row packing)"),
             "bound": "hbm",
             "achieved": round(v_gbs, 1),
@@ -563,7 +572,9 @@ def run_gpu(args) -> dict | None:
                 max_mhz = (clocks.summary() or {}).get("sm_max_mhz") or 2070.0
                 ffma_peak = props.multi_processor_count * 128 * 2 * max_mhz * 1e6 / 1e12
                 c_roof.update({
-                    "kernel": "FFMA path: simt_correct_kernel, gate_bias_kernel, simt_gate_kernel",
+                    "kernel": ("FFMA path: simt_rows_correct_kernel, gate_bias_kernel, simt_rows_gate_kernel (a warp per "
+                               "feature)" if cfg.B * (cfg.K - 1) <= 32 else
+                               "FFMA path: simt_correct_kernel, gate_bias_kernel, simt_gate_kernel"),
                     "bound": "alu", "peak": round(ffma_peak, 1), "frac": round(c_tflops / ffma_peak, 4),
                     "peak_source": "derived: SMs x 128 FP32 lanes x 2 flop per FMA x maximum SM clock",
                     "frac_of_sustained": None, "traffic": None})

@@ -19,8 +19,9 @@
 // finalising it, and the next pass (launched programmatically dependent)
 // streams only the listed sequences' rows.  Rows past the window holding the
 // first mismatch are never read.  Same keys, same finaliser, same results.
-// The finalisers of a windowed round only claim their packed rows; the row
-// copies follow in verify_copy_kernel, spread over the whole grid.
+// The finalisers of a windowed round, and of a one-pass round that packs rows
+// for fewer sequences than there are SMs, only claim their packed rows; the
+// row copies follow in verify_copy_kernel, spread over the whole grid.
 #include <atomic>
 
 #include "common.cuh"
@@ -588,8 +589,16 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
     if (by_bytes < grid) grid = by_bytes;
     if (grid > p.total_slots) grid = p.total_slots;
     if (grid < 1) grid = 1;
+    // Row packing for the tensor-core projections with fewer sequences than
+    // SMs: each finaliser would copy its sequence's rows on one SM after the
+    // stream has ended, so the copies go to the balanced copy kernel instead.
+    const bool defer = a.R_count && a.B < info.sm_count;
+    p.defer_copies = defer ? 1 : 0;
     verify_kernel<T, VEC><<<(unsigned)grid, kThreads, kCopyStageBytes, stream>>>(p);
-    return cudaGetLastError();
+    err = cudaGetLastError();
+    if (err != cudaSuccess || !defer) return err;
+    const long long copy_grid = ((long long)a.B * a.K * 4 + 15) / 16;  // a warp per row segment
+    return launch_copies<T>(a, p, copy_grid < grid_full ? copy_grid : grid_full, stream);
   }
   // Windowed: pass k reads rows [start[k], start[k+1]) of the sequences that
   // matched every earlier row; each pass after the first waits for its
