@@ -253,3 +253,36 @@ def test_round_unaligned_e_out_both_schedules(rt, flags):
     for name in ("accept_len", "committed", "bonus", "n", "e_out"):
         assert torch.equal(getattr(outs[1], name), getattr(outs[0], name)), name
     assert ws.check() == 0
+
+
+# More sequences than the GB300's 152 SMs at a size the automatic schedule
+# verifies in one pass: there the finalisers pack their own rows.
+MANY_SEQUENCES = CONFIGS[2].__class__("bf16 B160 K8 d256 (one pass, copies in the finalisers)",
+                                      160, 8, 4099, 256, "bf16", 1.0, "uniform", seed_offset=21)
+
+
+@pytest.mark.parametrize("flags", ["default", "overwrite"])
+def test_round_copies_in_finalisers_equal_copy_kernel(rt, flags):
+    """One pass with at least as many sequences as SMs copies and packs rows
+    inside the finalisers; the windowed schedule leaves them to the copy
+    kernel.  Both give the same bits."""
+    f = {"default": 0, "overwrite": rt.COND_OVERWRITE}[flags]
+    x = make_round_inputs(MANY_SEQUENCES, device="cuda")
+    cfg = x["cfg"]
+    assert cfg.B >= torch.cuda.get_device_properties(0).multi_processor_count
+    ws = rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype)
+    outs = []
+    prev = rt.retrace_set_verify_schedule(rt.VERIFY_FULL)
+    try:
+        for mode in (rt.VERIFY_FULL, rt.VERIFY_WINDOWS, rt.VERIFY_FULL):
+            rt.retrace_set_verify_schedule(mode)
+            outs.append(rt.run_round(x, ws, flags=f))
+            torch.cuda.synchronize()
+    finally:
+        rt.retrace_set_verify_schedule(prev)
+    want = oracle.verify(host_f64(x["logits"]), host_int(x["draft"]))
+    np.testing.assert_array_equal(host_int(outs[0].accept_len), want["accept_len"])
+    for o in outs[1:]:
+        for name in ("accept_len", "committed", "bonus", "n", "e_out"):
+            assert torch.equal(getattr(o, name), getattr(outs[0], name)), name
+    assert ws.check() == 0
