@@ -439,9 +439,9 @@ def run_gpu(args) -> dict | None:
     # one greedy pass that packs rows for the tensor-core projections hands its
     # copies to the copy kernel when there are fewer sequences than SMs
     packs = cfg.dtype == "bf16" and (cfg.d % 64 == 0 if args.lowrank
-                                     else cfg.d % 256 == 0 and args.variant in ("corrected", "raw"))
+                                     else cfg.d % 256 == 0 and (args.sampled or args.variant in ("corrected", "raw")))
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    if n_pass == 1 and not (fused or args.sampled) and packs and cfg.B < sms:
+    if n_pass == 1 and not fused and packs and cfg.B < sms:
         verify_launches += 1
     # conditioning launches of the greedy and temperature-1 rounds, by path
     rows = (cfg.B * (cfg.K - 1) + 15) // 16 * 16
@@ -499,12 +499,16 @@ def run_gpu(args) -> dict | None:
             vbytes += d_needed + cfg.B * (cfg.K + 1) * 4
             rbytes += d_rows * cfg.V * cfg.elem_bytes + cfg.B * (cfg.K + 1) * 4
         v_gbs = vbytes / v_avg_s / 1e9
+        copies = " + verify_copy_kernel (copy of unconditioned rows + row packing)"
+        passes = "sampled_topk_kernel + sampled_finalize_kernel" if args.sampled else "verify_kernel"
+        if n_pass > 1:
+            v_kernel = f"{passes} x{n_pass} passes over row windows {windows}{copies}"
+        elif verify_launches > (2 if args.sampled else 1):
+            v_kernel = f"{passes} (one pass){copies}"
+        else:
+            v_kernel = f"{passes} (one pass; the finalisers copy unconditioned rows and pack rows)"
         v_roof = {
-            "kernel": (f"verify_kernel x{n_pass} passes over row windows {windows} + verify_copy_kernel (copy of "
-                       "unconditioned rows + row packing)" if n_pass > 1 else
-                       "verify_kernel (argmax/compare/commit) + verify_copy_kernel (copy of unconditioned rows + "
-                       "row packing)" if verify_launches == 2 and not args.sampled else
-                       "verify_kernel (argmax/compare/commit + copy of unconditioned rows + row packing)"),
+            "kernel": v_kernel,
             "bound": "hbm",
             "achieved": round(v_gbs, 1),
             "peak": peaks["hbm_gbs"],

@@ -714,14 +714,14 @@ cudaError_t launch_verify_sampled(const SampledArgs& a, retrace_dtype dtype, cud
   // draft (top-k kernel), then runs their accept tests (finalize kernel).
   int start[kMaxWindowPasses + 1];
   const int n_pass = verify_windows(a.B, a.K, a.V, (int)fp.elem, a.live != nullptr, false, start);
-  const bool defer = n_pass > 1 && a.e_out;
-  long long topk_resident = 0;
-  if (n_pass > 1) {
-    DeviceInfo info;
-    cudaError_t e0 = device_info(&info);
-    if (e0 != cudaSuccess) return e0;
-    topk_resident = (long long)info.sm_count * 3;  // __launch_bounds__(kThreads, 3)
-  }
+  DeviceInfo info;
+  cudaError_t e0 = device_info(&info);
+  if (e0 != cudaSuccess) return e0;
+  // Copies after the last pass, balanced over the grid: always with windows;
+  // in one pass when it packs rows for fewer sequences than SMs (otherwise
+  // each finalising CTA copies its own sequence's rows).
+  const bool defer = a.e_out && (n_pass > 1 || (a.R_count && a.B < info.sm_count));
+  const long long topk_resident = (long long)info.sm_count * 3;  // __launch_bounds__(kThreads, 3)
   fp.defer_copies = defer ? 1 : 0;
   for (int k = 0; k < n_pass; ++k) {
     const bool last = k == n_pass - 1;

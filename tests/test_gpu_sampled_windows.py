@@ -144,3 +144,28 @@ def test_windowed_short_blocks(rt, K):
         assert torch.equal(a, b)
     np.testing.assert_array_equal(host_int(win[0]), accept.numpy())
     assert ws.check() == 0
+
+
+def test_one_pass_round_many_sequences_equals_windowed(rt):
+    """More sequences than the GB300's 152 SMs: the one-pass round's finalisers
+    copy and pack their own rows, the windowed round leaves them to the copy
+    kernel.  Both give the same bits."""
+    cfg = CONFIGS[2].__class__("sampled bf16 B160 K8 d256", 160, 8, 4096, 256, "bf16", 1.0, "uniform",
+                               seed_offset=23)
+    assert cfg.B >= torch.cuda.get_device_properties(0).multi_processor_count
+    x = make_round_inputs(cfg, device="cuda")
+    s = make_sampled_inputs(cfg, x["logits"], device="cuda")
+    ws = rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype)
+    outs = []
+    prev = rt.retrace_set_verify_schedule(rt.VERIFY_FULL)
+    try:
+        for mode in (rt.VERIFY_FULL, rt.VERIFY_WINDOWS, rt.VERIFY_FULL):
+            rt.retrace_set_verify_schedule(mode)
+            outs.append(rt.run_round_sampled(x, s, ws))
+            torch.cuda.synchronize()
+    finally:
+        rt.retrace_set_verify_schedule(prev)
+    for o in outs[1:]:
+        for name in ("accept_len", "committed", "bonus", "n", "e_out"):
+            assert torch.equal(getattr(o, name), getattr(outs[0], name)), name
+    assert ws.check() == 0
