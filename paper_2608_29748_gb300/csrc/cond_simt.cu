@@ -226,9 +226,12 @@ __global__ void __launch_bounds__(kNT) simt_gate_kernel(const SimtGateParams p) 
 // reduction index (coalesced loads of the weight row, the operand rows read
 // through L1), each lane keeps kRowGroup row sums, and a butterfly of
 // shuffles adds the lanes in a fixed order (results repeat bit for bit).
-// The rows are taken kRowGroup at a time; the weight row is re-read per group.
+// The rows are taken kRowGroup at a time (the weight row is re-read per
+// group), and each lane issues the loads of kBatch reduction steps for the
+// weight and every row of the group before it multiplies.
 constexpr int kRowsMax = 32;  // one plan tile
 constexpr int kRowGroup = 8;
+constexpr int kBatch = 4;  // reduction steps per lane with their loads issued together
 constexpr int kRowsWarps = kNT / 32;
 
 __device__ __forceinline__ float warp_sum(float s) {
@@ -266,16 +269,25 @@ __global__ void __launch_bounds__(kNT) simt_rows_correct_kernel(const SimtCorrec
       // c = W_c [m; u]: the m half (k < d), then the u half
       for (int half = 0; half < 2; ++half) {
         const T* wh = w + half * d;
-#pragma unroll 4
-        for (int k = lane; k < d; k += 32) {
-          const float wk = to_f32(wh[k]);
+        const T* src[kRowGroup];
 #pragma unroll
-          for (int q = 0; q < kRowGroup; ++q) {
-            if (q < gn) {
-              const T* src = half == 0 ? hD + s_m[g0 + q] : hT + s_u[g0 + q];
-              acc[q] = fmaf(wk, to_f32(src[k]), acc[q]);
-            }
+        for (int q = 0; q < kRowGroup; ++q) {  // rows past the group repeat its first (discarded)
+          const int row = g0 + (q < gn ? q : 0);
+          src[q] = half == 0 ? hD + s_m[row] : hT + s_u[row];
+        }
+        for (int k0 = lane; k0 < d; k0 += 32 * kBatch) {
+          float wk[kBatch], x[kRowGroup][kBatch];
+#pragma unroll
+          for (int u = 0; u < kBatch; ++u) {
+            const int k = k0 + 32 * u;
+            wk[u] = k < d ? to_f32(wh[k]) : 0.f;
+#pragma unroll
+            for (int q = 0; q < kRowGroup; ++q) x[q][u] = k < d ? to_f32(src[q][k]) : 0.f;
           }
+#pragma unroll
+          for (int q = 0; q < kRowGroup; ++q)
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u) acc[q] = fmaf(wk[u], x[q][u], acc[q]);
         }
       }
 #pragma unroll
@@ -321,26 +333,47 @@ __global__ void __launch_bounds__(kNT) simt_rows_gate_kernel(const SimtGateParam
 #pragma unroll
     for (int q = 0; q < kRowGroup; ++q) av[q] = ag[q] = 0.f;
     // v = W_v r and the r half of the gate, W_g[:, d:2d] r
-#pragma unroll 2
-    for (int k = lane; k < d; k += 32) {
-      const float wvk = to_f32(wv[k]), wgk = to_f32(wg[d + k]);
+    const T* rs[kRowGroup];
+    const T* es[kRowGroup];
 #pragma unroll
-      for (int q = 0; q < kRowGroup; ++q) {
-        if (q < gn) {
-          const float x = to_f32(r[s_r[g0 + q] + k]);
-          av[q] = fmaf(wvk, x, av[q]);
-          ag[q] = fmaf(wgk, x, ag[q]);
-        }
+    for (int q = 0; q < kRowGroup; ++q) {  // rows past the group repeat its first (discarded)
+      const int row = g0 + (q < gn ? q : 0);
+      rs[q] = r + s_r[row];
+      es[q] = e + s_e[row];
+    }
+    for (int k0 = lane; k0 < d; k0 += 32 * kBatch) {
+      float wvk[kBatch], wgk[kBatch], x[kRowGroup][kBatch];
+#pragma unroll
+      for (int u = 0; u < kBatch; ++u) {
+        const int k = k0 + 32 * u;
+        wvk[u] = k < d ? to_f32(wv[k]) : 0.f;
+        wgk[u] = k < d ? to_f32(wg[d + k]) : 0.f;
+#pragma unroll
+        for (int q = 0; q < kRowGroup; ++q) x[q][u] = k < d ? to_f32(rs[q][k]) : 0.f;
       }
+#pragma unroll
+      for (int q = 0; q < kRowGroup; ++q)
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+          av[q] = fmaf(wvk[u], x[q][u], av[q]);
+          ag[q] = fmaf(wgk[u], x[q][u], ag[q]);
+        }
     }
     // per-position e: the e half of the gate, W_g[:, 0:d] e
     if (p.e_dense) {
-#pragma unroll 4
-      for (int k = lane; k < d; k += 32) {
-        const float wk = to_f32(wg[k]);
+      for (int k0 = lane; k0 < d; k0 += 32 * kBatch) {
+        float wk[kBatch], x[kRowGroup][kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+          const int k = k0 + 32 * u;
+          wk[u] = k < d ? to_f32(wg[k]) : 0.f;
+#pragma unroll
+          for (int q = 0; q < kRowGroup; ++q) x[q][u] = k < d ? to_f32(es[q][k]) : 0.f;
+        }
 #pragma unroll
         for (int q = 0; q < kRowGroup; ++q)
-          if (q < gn) ag[q] = fmaf(wk, to_f32(e[s_e[g0 + q] + k]), ag[q]);
+#pragma unroll
+          for (int u = 0; u < kBatch; ++u) ag[q] = fmaf(wk[u], x[q][u], ag[q]);
       }
     }
 #pragma unroll

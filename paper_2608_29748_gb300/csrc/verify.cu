@@ -32,6 +32,9 @@ namespace {
 
 constexpr int kThreads = 512;
 constexpr int kUnroll = 4;
+// Least logits bytes per active CTA: small problems spread one row or so per
+// CTA instead of streaming several rows one after another on a few CTAs.
+constexpr long long kMinCtaBytes = 4096;
 
 struct VerifyParams {
   const void* logits;
@@ -332,8 +335,8 @@ __global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams 
   const int K1 = p.K + 1, W = p.i1 - p.i0;
   const long long per_seq = (long long)W * VV;
   const long long T_ = n_live * per_seq;
-  // Active CTAs: at least ~32 KB of logits each, no more than there are slots.
-  const long long by_bytes = (T_ * (VEC ? 16 : (long long)sizeof(T)) + 32767) / 32768;
+  // Active CTAs: at least kMinCtaBytes of logits each, no more than there are slots.
+  const long long by_bytes = (T_ * (VEC ? 16 : (long long)sizeof(T)) + kMinCtaBytes - 1) / kMinCtaBytes;
   const long long G = min((long long)gridDim.x, min(by_bytes, T_));
   const long long c = blockIdx.x;
 
@@ -580,12 +583,12 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
   const bool windowed = n_pass > 1;
   const long long grid_full = (long long)info.sm_count * occ;
   if (!windowed) {
-    // Enough CTAs to fill every SM at full occupancy, but at least ~32 KB of
+    // Enough CTAs to fill every SM at full occupancy, but at least kMinCtaBytes of
     // logits per CTA so that small batches do not pay for idle CTAs (the
     // kernel trims its active CTAs the same way).
     const long long bytes = (long long)a.B * K1 * a.V * (long long)sizeof(T);
     long long grid = grid_full;
-    const long long by_bytes = (bytes + 32767) / 32768;
+    const long long by_bytes = (bytes + kMinCtaBytes - 1) / kMinCtaBytes;
     if (by_bytes < grid) grid = by_bytes;
     if (grid > p.total_slots) grid = p.total_slots;
     if (grid < 1) grid = 1;
