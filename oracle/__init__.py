@@ -15,7 +15,6 @@ from .retrace_oracle import (  # noqa: F401
     condition,
     conditioned_rows,
     correct,
-    f64_to_bf16_bits,
     filtered_distribution,
     gate_fuse,
     LOWRANK_CORRECTION,

@@ -75,14 +75,14 @@ def round_to_bf16(x: np.ndarray) -> np.ndarray:
     return out
 
 
-def f64_to_bf16_bits(x: np.ndarray) -> np.ndarray:
-    """Bit patterns (uint16) of float64 values that are exact bfloat16 values."""
-    f32 = np.asarray(x, dtype=np.float64).astype(np.float32)
-    return (f32.view(np.uint32) >> np.uint32(16)).astype(np.uint16)
-
-
 def bf16_ulp(x: np.ndarray) -> np.ndarray:
-    """Spacing of bfloat16 values at |x| (one unit in the last place)."""
+    """Spacing of bfloat16 values at |x| (one unit in the last place).
+
+    For |x| in [2^(e-1), 2^e) the next larger bf16 value is 2^(e-8) away (8
+    significant bits); below the normal range the spacing stays at the
+    subnormal quantum 2^-133, which is also the spacing at 0.  Used for the
+    bf16 output tolerance where |reference| >= 4.
+    """
     x = np.abs(np.asarray(x, dtype=np.float64))
     _, e = np.frexp(np.where(x == 0.0, np.ldexp(1.0, -126), x))
     return np.ldexp(1.0, np.maximum(e - 8, -133))

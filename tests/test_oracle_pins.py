@@ -69,6 +69,25 @@ def test_round_to_bf16_matches_torch_float32_conversion():
     assert np.array_equal(ours, ref)
 
 
+def test_bf16_ulp_is_the_spacing_torch_gives():
+    """bf16_ulp(x) sets the bf16 output tolerance where |reference| >= 4.  It
+    must be the distance from x's bf16 interval floor to the next bf16 value:
+    taken here from torch's decoding of consecutive bit patterns, over every
+    positive finite pattern (zero, subnormals, every binade up to the largest
+    finite value), for those values negated, and for points strictly inside
+    each interval."""
+    bits = np.arange(0, 0x7F7F, dtype=np.int32)  # 0x7F7F is the largest finite bf16
+    lo = torch.from_numpy(bits.astype(np.int16)).view(torch.bfloat16).double().numpy()
+    hi = torch.from_numpy((bits + 1).astype(np.int16)).view(torch.bfloat16).double().numpy()
+    spacing = hi - lo
+    assert np.array_equal(oracle.bf16_ulp(lo), spacing)
+    assert np.array_equal(oracle.bf16_ulp(-lo), spacing)
+    inside = lo + 0.5 * spacing  # exact in float64: both ends are bf16 values
+    assert np.array_equal(oracle.bf16_ulp(inside), spacing)
+    # the tolerance band the GPU tests use: 2^-5 in [4, 8), 2^-4 in [8, 16)
+    assert oracle.bf16_ulp(np.array([4.0, 7.99, 8.0, 15.9]))[[0, 1, 2, 3]].tolist() == [2**-5, 2**-5, 2**-4, 2**-4]
+
+
 # ---------------------------------------------------------------------------
 # Verification
 # ---------------------------------------------------------------------------
@@ -561,7 +580,14 @@ def _pins():
         test_sampled_verification_brute_force,
         test_sampled_verification_with_top_k_one_is_greedy,
         test_sampled_verification_accepts_everything_when_draft_equals_target,
+        test_bf16_ulp_is_the_spacing_torch_gives,
     ]
+
+
+def _mut_ulp_below(x):
+    a = np.abs(np.asarray(x, dtype=np.float64))
+    mant, _ = np.frexp(a)
+    return orc.__dict__["_orig_bf16_ulp"](x) * np.where(mant == 0.5, 0.5, 1.0)
 
 
 def _mut_argmax_last(logits):
@@ -644,6 +670,8 @@ def _mut_filtered(kind):
 
 
 MUTATIONS = {
+    "bf16 ulp exponent off by one": ("bf16_ulp", lambda x: 2.0 * orc.__dict__["_orig_bf16_ulp"](x)),
+    "bf16 ulp measured below x (half at powers of two)": ("bf16_ulp", _mut_ulp_below),
     "temperature ignored": ("filtered_distribution", _mut_filtered("no_temperature")),
     "top-p drops the crossing token": ("filtered_distribution", _mut_filtered("top_p_drops_crossing")),
     "top-p ignored": ("filtered_distribution", _mut_filtered("no_top_p")),
@@ -691,6 +719,7 @@ def test_planted_mistakes_are_caught(name, monkeypatch):
     monkeypatch.setitem(orc.__dict__, "_orig_condition", orc.condition)
     monkeypatch.setitem(orc.__dict__, "_orig_lowrank", orc.lowrank_condition)
     monkeypatch.setitem(orc.__dict__, "_orig_filtered", orc.filtered_distribution)
+    monkeypatch.setitem(orc.__dict__, "_orig_bf16_ulp", orc.bf16_ulp)
     monkeypatch.setattr(orc, attr, fn)
     monkeypatch.setattr(oracle, attr, fn, raising=False)
     caught = 0
