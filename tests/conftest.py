@@ -31,3 +31,16 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+def pytest_terminal_summary(terminalreporter):
+    # bf16 comparisons: how many elements needed the 1-ulp allowance above the
+    # 2e-2 bound (|reference| >= 4), next to the largest error of each check
+    parity = sys.modules.get("parity")
+    rows = getattr(parity, "RELAXED", None)
+    if not rows:
+        return
+    terminalreporter.section("bf16 elements above 2e-2 (allowed: 1 bf16 ulp where |ref| >= 4)")
+    for what, count, total, worst in rows:
+        terminalreporter.write_line(f"{what or '(unnamed)'}: {count} of {total} elements above 2e-2; "
+                                    f"largest error {worst:.4g}")

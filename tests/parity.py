@@ -53,6 +53,13 @@ def bf16_tolerance(ref_rounded: np.ndarray) -> np.ndarray:
     return np.where(np.abs(ref_rounded) >= 4.0, np.maximum(BF16_ABS_TOL, oracle.bf16_ulp(ref_rounded)), BF16_ABS_TOL)
 
 
+# Elements that pass only through the 1-ulp allowance for |ref| >= 4, i.e.
+# whose error exceeds the plain 2e-2 bound: (check, count, compared, worst
+# error) for every bf16 comparison, printed in the test session's summary so
+# that the relaxation is visible beside the stated bound.
+RELAXED = []
+
+
 def assert_close(gpu: torch.Tensor, ref64: np.ndarray, what: str = "") -> float:
     """Checks gpu (bf16 or fp32) against the float64 oracle; returns max |gpu - ref64|."""
     got = host_f64(gpu)
@@ -61,6 +68,8 @@ def assert_close(gpu: torch.Tensor, ref64: np.ndarray, what: str = "") -> float:
         ref_r = oracle.round_to_bf16(ref64)
         err = np.abs(got - ref_r)
         tol = bf16_tolerance(ref_r)
+        over = err > BF16_ABS_TOL
+        RELAXED.append((what, int(over.sum()), int(err.size), float(err.max(initial=0.0))))
         bad = err > tol
         assert not bad.any(), f"{what}: {bad.sum()} elements out of tolerance; worst err {err.max():.4g}"
     else:

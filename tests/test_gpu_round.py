@@ -1,9 +1,11 @@
 """GPU parity of the fused round (retrace_round) on the five workloads vs the oracle.
 
 Configs 1-4 are checked in full.  Config 5 (B = 256, 1.3 GB of logits) is
-checked in the launch configuration the benchmark times: verification outputs
-in full, the unconditioned rows in full (bit-exact copies of e), and a seeded
-sample of conditioned rows computed one by one by the oracle.
+checked twice: in full in the launch configuration the benchmark times
+(target_argmax not requested, so the default schedule verifies in row
+windows, copies and packs rows in the copy kernel and runs both projections
+in cond_pair_kernel), and with target_argmax requested (one verification
+pass) on a seeded sample of conditioned rows.
 """
 
 import numpy as np
@@ -58,8 +60,38 @@ def test_round_workloads_full(rt, cfg_id):
         assert np.array_equal(got[b, want["n"][b]:], np.broadcast_to(e, got[b, want["n"][b]:].shape))
 
 
+def test_round_serving_batch_benched_path(rt):
+    """Config 5 at full size (B=256, K=16, V=151936, d=4096) through exactly
+    the call bench.py times: retrace_round with target_argmax NULL under the
+    default schedule.  That composition is the row-window verification passes,
+    verify_copy_kernel (unconditioned rows of e~, packing of [m; u]) and
+    cond_pair_kernel (both projections; R = 2876 rows, so the last 256-row
+    pair block is partial).  Every output is compared with the oracle: the
+    verification outputs and n bit-exact, every row of e~ within the bf16
+    tolerance, and the unconditioned rows bit-exact copies of e."""
+    cfg = CONFIGS[5]
+    windows = rt.retrace_verify_plan(cfg.B, cfg.K, cfg.V, cfg.torch_dtype)
+    assert len(windows) > 2, "the default schedule verifies this workload in row windows"
+    x = make_round_inputs(cfg, device="cuda")
+    ws = rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype)
+    out = rt.run_round(x, ws)  # no target_argmax: the benchmark's call
+    torch.cuda.synchronize()
+    assert ws.check() == 0
+    want = oracle_round(x)
+    assert_verify_exact(want, out.accept_len, out.committed, out.bonus)
+    np.testing.assert_array_equal(host_int(out.n), want["n"])
+    R = int(want["n"].sum())
+    assert R % 256 != 0 and R > 256, R  # several pair blocks and a partial last one
+    assert_close(out.e_out, want["e_tilde"], "config 5 benched round, every row")
+    pos = torch.arange(cfg.K, device="cuda")[None, :]
+    mask = pos >= out.n.long()[:, None]
+    assert torch.equal(out.e_out[mask], x["e"].expand(int(mask.sum()), cfg.d))
+
+
 def test_round_serving_batch_sampled(rt):
-    """Config 5 at full size: B=256, K=16, V=151936, d=4096."""
+    """Config 5 at full size with target_argmax requested (which makes the
+    verification a single pass over every row): verification outputs in full,
+    the unconditioned rows in full, a seeded sample of conditioned rows."""
     cfg = CONFIGS[5]
     x = make_round_inputs(cfg, device="cuda")
     out, targ, ws = run(rt, x)
