@@ -56,23 +56,38 @@ UNIT = "rounds/s"
 KERNELS_PER_ROUND_FUSED = 1  # cond_kernel<FUSED>: the whole round
 KERNELS_PER_ROUND = 2  # one-pass verify_kernel (+ row packing), cond_kernel (both projections + gate-bias GEMV)
 L2_FLUSH_BYTES = 256 << 20
-# DRAM traffic of the verification kernels of one round per sequence of the
-# serving shapes (K=16, V=151936, d=4096, bf16; windowed schedule), measured
-# with ncu (dram__bytes_read.sum + dram__bytes_write.sum, summed over the
-# passes and the copy kernel) on the 128-sequence profiling workload, whose
-# accepted lengths follow the serving workload's distribution; scaled by
-# B/128 (profiles/verify_windowed_launch_list-B128.md): 285.56 MB at B = 128.
-VERIFY_TRAFFIC_PER_SEQUENCE = 285564928 / 128
-VERIFY_TRAFFIC_PASSES = 3  # the schedule the traffic was measured on (passes of verify_kernel)
-VERIFY_TRAFFIC_SHAPE = (16, 151936, 4096, "bf16")
-# DRAM traffic of the single-kernel round per sequence (same shapes, same
-# profiling workload and method); None until measured for the current kernel.
-ROUND_TRAFFIC_PER_SEQUENCE = None
-# DRAM traffic (read + write) of one conditioning launch (cond_pair_kernel),
-# by workload, measured with ncu on that workload.  It does not scale with the
-# batch (weights and L2 reuse dominate), so it is only reported where it was
-# measured.  Must be re-measured whenever the conditioning kernel changes.
-COND_TRAFFIC = {"qwen3-8b-B256-K16": 616099328 + 42992640}
+# DRAM traffic per round (ncu dram__bytes_read.sum + dram__bytes_write.sum,
+# summed over the kernels of the phase) of the phase a roofline object names,
+# measured once with ncu on that workload.  Each figure holds only for the
+# kernel sources it was measured on: `sources` is kernel_sources_hash() at the
+# time, and the line reports null traffic once the sources differ.
+TRAFFIC = {
+    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311331584 + 3026944 + 184293120 + 65792 + 55385600 + 1024
+                                      + 47148032 + 3488512, "sources": "32ff2909d7391a9f"},
+    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 611928576 + 39502080, "sources": "32ff2909d7391a9f"},
+}
+
+
+def kernel_sources_hash() -> str:
+    """Hash of every CUDA source of the library (kernels and their headers)."""
+    import hashlib
+
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_29748_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode() + b"\0" + f.read())
+    return h.hexdigest()[:16]
+
+
+def measured_traffic(phase: str, workload_name: str, variant: str) -> int | None:
+    """ncu DRAM bytes per round of `phase` on this workload, if measured on
+    the current kernel sources (the default, corrected variant only)."""
+    t = TRAFFIC.get((phase, workload_name))
+    if variant != "corrected" or t is None or t["sources"] != kernel_sources_hash():
+        return None
+    return t["bytes"]
 
 
 # ---------------------------------------------------------------------------
@@ -475,16 +490,13 @@ def run_gpu(args) -> dict | None:
             "algorithmic_flops": cflops,
             "floor_us": {"hbm": round(t_hbm * 1e6, 1), "tensor": round(t_tc * 1e6, 1)},
             "avg_launch_us": round(step_avg_s * 1e6, 2),
-            "traffic": (round(ROUND_TRAFFIC_PER_SEQUENCE * cfg.B)
-                        if ROUND_TRAFFIC_PER_SEQUENCE and (cfg.K, cfg.V, cfg.d, cfg.dtype) == VERIFY_TRAFFIC_SHAPE
-                        else None),
-            "traffic_source": "ncu dram read+write on B=128 profiling workload, scaled by B/128",
+            "traffic": measured_traffic("overlapped", cfg.name, args.variant),
+            "traffic_source": "ncu dram read+write of the round's kernel on this workload",
         }
         line_extra = {"hbm_view": {"achieved_gbs": round(hbytes / step_avg_s / 1e9, 1),
                                    "frac": round(t_hbm / step_avg_s, 4)},
                       "tensor_view": {"achieved_tflops": round(cflops / step_avg_s / 1e12, 2),
                                       "frac": round(t_tc / step_avg_s, 4)}}
-        logits_gbs = cfg.logits_bytes() / step_avg_s / 1e9
     else:
         packs_rows = cfg.dtype == "bf16" and cfg.d % 256 == 0  # tensor-core path: verify packs the rows
         vbytes = verify_bytes(cfg, n, packs_rows and args.variant in ("corrected", "raw"), args.variant, accept)
@@ -522,11 +534,9 @@ def run_gpu(args) -> dict | None:
             "streamed_frac": round(rbytes / v_avg_s / 1e9 / peaks["hbm_gbs"], 4),
             "launches": verify_launches,
             "avg_launch_us": round(v_avg_s * 1e6, 2),
-            "traffic": (round(VERIFY_TRAFFIC_PER_SEQUENCE * cfg.B)
-                        if VERIFY_TRAFFIC_PER_SEQUENCE and (cfg.K, cfg.V, cfg.d, cfg.dtype) == VERIFY_TRAFFIC_SHAPE
-                        and args.variant == "corrected" and n_pass == VERIFY_TRAFFIC_PASSES else None),
-            "traffic_source": "ncu dram read+write of the verification kernels on the B=128 profiling workload, "
-                              "scaled by B/128",
+            "traffic": None if args.sampled else measured_traffic("verify", cfg.name, args.variant),
+            "traffic_source": "ncu dram read+write of the verification kernels (passes + copy kernel) of one round "
+                              "on this workload",
         }
         if args.variant in ("overwrite", "none"):
             v_roof["kernel"] = v_roof["kernel"].replace("copy of unconditioned rows + row packing",
@@ -567,7 +577,7 @@ def run_gpu(args) -> dict | None:
                 "frac_of_sustained": round(c_tflops / peaks["bf16_tflops_sustained"], 4),
                 "algorithmic_flops": cflops,
                 "avg_launch_us": round(c_avg_s * 1e6, 2),
-                "traffic": (COND_TRAFFIC.get(cfg.name) if args.variant == "corrected" and not args.sampled else None),
+                "traffic": None if args.sampled else measured_traffic("conditioning", cfg.name, args.variant),
                 "traffic_source": "ncu dram read+write of one launch on this workload",
             }
             if cfg.dtype != "bf16" or cfg.d % 256:
@@ -599,7 +609,6 @@ def run_gpu(args) -> dict | None:
         # `roofline` is the kernel that takes the larger share of the round
         roofline = c_roof if (c_roof and c_avg_s > v_avg_s) else v_roof
         line_extra = {"roofline_verify": v_roof, "roofline_conditioning": c_roof}
-        logits_gbs = cfg.logits_bytes() / v_avg_s / 1e9
 
     # ---- end to end through the public API with host buffers ----
     names = ["logits", "draft", "hD", "hT"] + (["draft_logits", "uniforms"] if args.sampled else [])
@@ -640,7 +649,6 @@ def run_gpu(args) -> dict | None:
         },
         "roofline": roofline,
         **line_extra,
-        "logits_gbs": round(logits_gbs, 1),
         "e2e": e2e,
         "gpu_launches": (KERNELS_PER_ROUND_FUSED if fused
                          else KERNELS_PER_ROUND_LOWRANK - 1 + verify_launches if args.lowrank
@@ -805,7 +813,7 @@ def run_sweep(args) -> None:
             "dtype": cfg.dtype, "conditioned_rows_R": int(n.sum()), "iters": iters, "statistic": "median",
             "verify_windows": windows,
             "verify_us": {k: round(t, 2) for k, t in v.items()},
-            "logits_gbs": {k: round(logits / t / 1e3, 1) for k, t in v.items()},
+            "streamed_gbs": {k: round(logits / t / 1e3, 1) for k, t in v.items()},
             "logits_frac_of_hbm": {k: round(logits / t / 1e3 / peaks["hbm_gbs"], 4) for k, t in v.items()},
             "needed_gbs": {k: round(needed / t / 1e3, 1) for k, t in v.items()},
             "round_us": {k: round(t, 2) for k, t in r.items()},
