@@ -393,7 +393,17 @@ retrace_status retrace_wait_selftest(int kind, const uint32_t* flag, uint32_t ta
  *              RETRACE_ERR_UNSUPPORTED and enqueues nothing.
  *   Set-up     the first call on each device looks up the array's device
  *              address (cudaGetSymbolAddress) with that device current; make
- *              that first call before any stream capture on the device.
+ *              that first call before any stream capture on the device.  The
+ *              address is kept per device together with the identity of the
+ *              context it belongs to: after a device reset (cudaDeviceReset)
+ *              the next call looks it up again, so that call too should come
+ *              before any capture.
+ *   Schedule   always one pass over every row (RETRACE_VERIFY_FULL): the
+ *              row-window schedule keeps live lists in the workspace, which
+ *              this entry point does not have.  At large batches it is
+ *              therefore slower than retrace_verify with a workspace and
+ *              target_argmax NULL, which reads only the windows up to each
+ *              sequence's first mismatch.
  *   Sharing    every call on a device uses the same array and clears the part
  *              it needs (cudaMemsetAsync on `stream`) before its kernel runs.
  *              Calls whose work may overlap on the GPU (different streams with

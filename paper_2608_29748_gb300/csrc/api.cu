@@ -11,14 +11,15 @@
 namespace retrace {
 
 cudaError_t device_info(DeviceInfo* out) {
-  static int sm_cache[64] = {0};
+  static std::atomic<int> sm_cache[64];  // 0: not yet read (threads may race to fill it)
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
-  int& sm = sm_cache[dev & 63];
+  int sm = sm_cache[dev & 63].load(std::memory_order_relaxed);
   if (sm == 0) {
     err = cudaDeviceGetAttribute(&sm, cudaDevAttrMultiProcessorCount, dev);
     if (err != cudaSuccess) return err;
+    sm_cache[dev & 63].store(sm, std::memory_order_relaxed);
   }
   out->device = dev;
   out->sm_count = sm;
@@ -31,16 +32,19 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 static EncodeTiledFn encode_fn() {
-  static EncodeTiledFn fn = nullptr;
-  if (!fn) {
+  static std::atomic<EncodeTiledFn> fn{nullptr};
+  EncodeTiledFn f = fn.load(std::memory_order_acquire);
+  if (!f) {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
                                          &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(p);
+        q == cudaDriverEntryPointSuccess) {
+      f = reinterpret_cast<EncodeTiledFn>(p);
+      fn.store(f, std::memory_order_release);
+    }
   }
-  return fn;
+  return f;
 }
 
 // bf16 2D tensor [rows, inner], 128-byte swizzle, box {box_inner, box_rows}.

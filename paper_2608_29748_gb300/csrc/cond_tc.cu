@@ -1375,15 +1375,15 @@ __global__ void __launch_bounds__(256) swap_reduce_gate_kernel(const SwapReduceP
 
 template <bool FUSED>
 cudaError_t ensure_smem_attr() {
-  static int done[64] = {0};
+  static std::atomic<int> done[64];
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
-  if (!done[dev & 63]) {
+  if (!done[dev & 63].load(std::memory_order_acquire)) {
     err = cudaFuncSetAttribute(cond_kernel<FUSED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                FUSED ? SMEM_BYTES_FUSED : SMEM_BYTES);
     if (err != cudaSuccess) return err;
-    done[dev & 63] = 1;
+    done[dev & 63].store(1, std::memory_order_release);
   }
   return cudaSuccess;
 }
@@ -1466,10 +1466,10 @@ static cudaError_t launch_cond_pair(const TcCondArgs& a, int clusters, cudaStrea
 static int pair_clusters(const TcCondArgs& a, long long tiles_max_pairs, cudaError_t* err) {
   *err = cudaSuccess;
   if (a.do_gate && a.e_dense) return 0;
-  static int max_clusters[64] = {0};  // per device; -1: none fits
+  static std::atomic<int> max_clusters[64];  // per device; 0: not yet known; -1: none fits
   int dev = 0;
   if ((*err = cudaGetDevice(&dev)) != cudaSuccess) return 0;
-  if (max_clusters[dev & 63] == 0) {
+  if (max_clusters[dev & 63].load(std::memory_order_acquire) == 0) {
     if ((*err = cudaFuncSetAttribute(cond_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES)) !=
         cudaSuccess)
       return 0;
@@ -1486,9 +1486,9 @@ static int pair_clusters(const TcCondArgs& a, long long tiles_max_pairs, cudaErr
     cfg.numAttrs = 1;
     int n = 0;
     if ((*err = cudaOccupancyMaxActiveClusters(&n, cond_pair_kernel, &cfg)) != cudaSuccess) return 0;
-    max_clusters[dev & 63] = n > 0 ? n : -1;
+    max_clusters[dev & 63].store(n > 0 ? n : -1, std::memory_order_release);
   }
-  const int n = max_clusters[dev & 63];
+  const int n = max_clusters[dev & 63].load(std::memory_order_acquire);
   if (n <= 0) return 0;
   // every pair when the gate-bias GEMV is needed: pairs without tiles compute it
   if (a.do_gate) return n;
@@ -1508,12 +1508,12 @@ static cudaError_t launch_cond_swap(const TcCondArgs& a, cudaStream_t stream) {
   DeviceInfo info;
   cudaError_t err = device_info(&info);
   if (err != cudaSuccess) return err;
-  static int attr_done[64] = {0};
+  static std::atomic<int> attr_done[64];
   const int max_smem = SW_STAGES * (BM * BK * 2 + 256 * BK * 2) + 1024;
-  if (!attr_done[info.device & 63]) {
+  if (!attr_done[info.device & 63].load(std::memory_order_acquire)) {
     err = cudaFuncSetAttribute(swap_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem);
     if (err != cudaSuccess) return err;
-    attr_done[info.device & 63] = 1;
+    attr_done[info.device & 63].store(1, std::memory_order_release);
   }
   const uint32_t stage_stride = (uint32_t)((BM * BK * 2 + box_n * BK * 2 + 1023) / 1024 * 1024);
   const int smem = SW_STAGES * (int)stage_stride + 1024;
@@ -1521,12 +1521,13 @@ static cudaError_t launch_cond_swap(const TcCondArgs& a, cudaStream_t stream) {
   while ((int)tmem_cols < box_n) tmem_cols <<= 1;
   // One resident wave when it can carry every work tile: a split's CTA
   // streams its whole K range, so a second wave would double the time.
-  static int occ_cache[64][256 / 16 + 1] = {};
-  int& occ = occ_cache[info.device & 63][box_n / 16];
+  static std::atomic<int> occ_cache[64][256 / 16 + 1];
+  int occ = occ_cache[info.device & 63][box_n / 16].load(std::memory_order_relaxed);
   if (occ == 0) {
     err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, swap_gemm_kernel, SW_THREADS, (size_t)smem);
     if (err != cudaSuccess) return err;
     if (occ < 1) occ = 1;
+    occ_cache[info.device & 63][box_n / 16].store(occ, std::memory_order_relaxed);
   }
   int resident = info.sm_count * occ;
   if (resident > kSwapMaxCtas) resident = kSwapMaxCtas;

@@ -590,15 +590,15 @@ cudaError_t launch_lowrank(const LowRankArgs& a, bool tc, cudaStream_t stream) {
   }
   DeviceInfo info{0, 148};
   if ((err = device_info(&info)) != cudaSuccess) return err;
-  static bool attr_done[64] = {false};
-  if (!attr_done[info.device & 63]) {
+  static std::atomic<int> attr_done[64];
+  if (!attr_done[info.device & 63].load(std::memory_order_acquire)) {
     if ((err = cudaFuncSetAttribute(lr_project_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_PROJECT)) !=
         cudaSuccess)
       return err;
     if ((err = cudaFuncSetAttribute(lr_fuse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_FUSE)) !=
         cudaSuccess)
       return err;
-    attr_done[info.device & 63] = true;
+    attr_done[info.device & 63].store(1, std::memory_order_release);
   }
   const uint64_t d = (uint64_t)a.d;
   CUtensorMap mA, mP, mBc, mRho, mWv, mWg;

@@ -526,14 +526,17 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
   DeviceInfo info;
   cudaError_t err = device_info(&info);
   if (err != cudaSuccess) return err;
-  static int occ_cache[64] = {0};
-  int& occ = occ_cache[info.device & 63];
+  // Per device, filled by the first call (concurrent first calls may both
+  // fill it; both set the same attribute and store the same value).
+  static std::atomic<int> occ_cache[64];
+  int occ = occ_cache[info.device & 63].load(std::memory_order_acquire);
   if (occ == 0) {
     err = cudaFuncSetAttribute(verify_kernel<T, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize, kCopyStageBytes);
     if (err != cudaSuccess) return err;
     err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, verify_kernel<T, VEC>, kThreads, kCopyStageBytes);
     if (err != cudaSuccess) return err;
     if (occ < 1) occ = 1;
+    occ_cache[info.device & 63].store(occ, std::memory_order_release);
   }
   VerifyParams p;
   p.logits = a.logits;

@@ -31,7 +31,46 @@ constexpr int kMaxDevices = 64;
 static __device__ __align__(256) unsigned char g_scratch[kNoAllocScratchBytes];
 
 std::mutex g_setup_mutex;
-void* g_scratch_addr[kMaxDevices] = {nullptr};
+
+// Device address of g_scratch per device, with the identity of the context it
+// was looked up in.  A device reset destroys the primary context and the
+// module with it; a new context loads the module again, possibly elsewhere,
+// so an address is only reused while the same context is current.
+struct ScratchEntry {
+  void* addr;
+  unsigned long long ctx_id;
+};
+ScratchEntry g_scratch_entry[kMaxDevices] = {};
+
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+
+// Unique identifier of the context current on this thread, through the
+// driver entry points the runtime exposes; 0 when there is none or the
+// driver cannot tell (the address is then looked up on every call).
+unsigned long long current_context_id() {
+  static CtxGetCurrentFn get_current = nullptr;  // resolved under g_setup_mutex
+  static CtxGetIdFn get_id = nullptr;
+  static bool resolved = false;
+  if (!resolved) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(p);
+    resolved = true;
+  }
+  if (!get_current || !get_id) return 0;
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return 0;
+  if (get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
 
 // Errors are reported through retrace_last_error(), like every other entry point.
 retrace_status fail(retrace_status s, const char* msg) {
@@ -39,16 +78,21 @@ retrace_status fail(retrace_status s, const char* msg) {
   return s;
 }
 
-// Device address of g_scratch on the current device, looked up once per device.
+// Device address of g_scratch on the current device: looked up with
+// cudaGetSymbolAddress the first time, and again whenever the current context
+// differs from the one the cached address came from.
 cudaError_t scratch_address(int dev, void** out) {
   std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (!g_scratch_addr[dev]) {
+  ScratchEntry& e = g_scratch_entry[dev];
+  const unsigned long long id = current_context_id();
+  if (!e.addr || id == 0 || e.ctx_id != id) {
     void* p = nullptr;
-    const cudaError_t err = cudaGetSymbolAddress(&p, g_scratch);
+    const cudaError_t err = cudaGetSymbolAddress(&p, g_scratch);  // makes the primary context current if needed
     if (err != cudaSuccess) return err;
-    g_scratch_addr[dev] = p;
+    e.addr = p;
+    e.ctx_id = current_context_id();
   }
-  *out = g_scratch_addr[dev];
+  *out = e.addr;
   return cudaSuccess;
 }
 

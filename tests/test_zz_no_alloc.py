@@ -80,6 +80,31 @@ def test_noalloc_matches_workspace_verify_on_consecutive_calls(rt):
             assert torch.equal(a, b), name
 
 
+def test_noalloc_without_argmax_output_matches_the_windowed_schedule(rt):
+    """With target_argmax NULL at the serving shape (B = 256, K = 16,
+    V = 151936, bf16), retrace_verify with a workspace verifies in row
+    windows while retrace_verify_noalloc, which has no live lists, reads every
+    row in one pass.  The integer outputs must still agree bit for bit, on two
+    calls in a row."""
+    B, K, V = 256, 16, 151936  # 256 * 17 keys + 256 counters: 35,840 bytes of scratch
+    assert len(rt.retrace_verify_plan(B, K, V, torch.bfloat16)) > 2  # the workspace path is windowed
+    logits, draft = case(B, K, V, torch.bfloat16, seed=5)
+    code = rt.RETRACE_BF16
+    stream = torch.cuda.current_stream().cuda_stream
+    ws = rt.Workspace(B, K, V, 8, logits.dtype)
+    for _ in range(2):
+        got = outputs(B, K)[:3]
+        st = rt.lib.retrace_verify_noalloc(logits.data_ptr(), code, B, K, V, logits.stride(1), logits.stride(0),
+                                           draft.data_ptr(), got[0].data_ptr(), got[1].data_ptr(),
+                                           got[2].data_ptr(), None, stream)
+        assert st == 0, rt.lib.retrace_last_error().decode()
+        want = outputs(B, K)[:3]
+        rt.retrace_verify(logits, draft, want[0], want[1], want[2], ws)  # no target_argmax: windowed
+        torch.cuda.synchronize()
+        for name, a, b in zip(("accept_len", "committed", "bonus"), got, want):
+            assert torch.equal(a, b), name
+
+
 def test_noalloc_rejects_batches_beyond_the_fixed_scratch(rt):
     B, K, V = 512, 16, 64  # 512 * 17 keys of 8 bytes = 69632 bytes > 65536
     logits, draft = case(B, K, V, torch.bfloat16, seed=4)
