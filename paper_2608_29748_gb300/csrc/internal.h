@@ -24,8 +24,9 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 //   tickets  uint32 [B]         per-sequence CTA arrival counters, zero between calls
 //   live     int32  [2*B]       windowed verification: live sequence lists of two passes
 //   poff     int32  [B]         windowed verification: first packed row of each sequence
-//   counts   uint32 [1+passes]  windowed verification: [0] CTAs out of the last pass,
-//                               [k] sequences live into pass k; zero between calls
+//   counts   uint32 [2(1+passes)] windowed verification: [0] CTAs out of the finish
+//                               kernel, [k] sequences live into pass k, [17 + k] packed
+//                               rows claimed before pass k's window; zero between calls
 //   ge       fp32   [d]         W_g[:, :d] e for a broadcast e
 //   r        elem   [R_max, d]  compacted corrected signal, R_max = B*(K-1)
 //   apack    elem   [R_max, 2d] packed [m; u] rows (tensor-core path)
@@ -82,7 +83,7 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   L.poff = off;
   off = align_up(off + (size_t)B * 4, 256);
   L.counts = off;
-  off = align_up(off + (size_t)(kMaxWindowPasses + 1) * 4, 256);
+  off = align_up(off + (size_t)2 * (kMaxWindowPasses + 1) * 4, 256);
   L.ge = off;
   off = align_up(off + dd * 4, 256);
   L.r = off;

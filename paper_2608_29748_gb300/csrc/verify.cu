@@ -14,14 +14,18 @@
 //
 // The outputs depend only on rows 0..A_b of each sequence.  The windowed
 // schedule runs the same kernel as a chain of passes over row windows
-// [i0, i1): the finaliser of a sequence whose draft tokens matched every row
-// of the window appends it to the next pass's live list instead of
-// finalising it, and the next pass (launched programmatically dependent)
-// streams only the listed sequences' rows.  Rows past the window holding the
-// first mismatch are never read.  Same keys, same finaliser, same results.
-// The finalisers of a windowed round, and of a one-pass round that packs rows
-// for fewer sequences than there are SMs, only claim their packed rows; the
-// row copies follow in verify_copy_kernel, spread over the whole grid.
+// [i0, i1), with no finalisers and no tickets: a pass only folds keys.  Each
+// later pass (launched programmatically dependent) first rebuilds its live
+// list, the sequences whose draft tokens matched every row so far, from the
+// previous window's keys and the previous live list (every CTA the same list,
+// in sequence order, by a block scan; CTA 0 publishes it for the next pass).
+// The sequences that mismatched in the previous window are decided there and
+// then: accepted length, outputs (spread over the CTAs) and their packed-row
+// offsets, after the rows of the sequences decided in earlier windows.  The
+// pass then streams only the listed sequences' rows.  Rows past the window
+// holding the first mismatch are never read.  verify_finish_kernel decides
+// the sequences of the last window the same way and does the row copies.  A one-pass round that packs rows for fewer sequences than
+// there are SMs leaves its copies to verify_copy_kernel, spread over the grid.
 #include <atomic>
 
 #include "common.cuh"
@@ -62,15 +66,21 @@ struct VerifyParams {
   int32_t* rowmap;
   int32_t* R_count;
   int cond_copy;
-  // Row window of this pass (windowed schedule; [0, K+1) in one pass).
-  int i0, i1;
-  const int32_t* live_in;    // sequences of this pass (NULL: 0..B-1)
-  const uint32_t* count_in;  // their number, written by the previous pass (NULL: B)
-  int32_t* live_out;         // sequences that matched every row of the window (NULL: last pass)
+  // Row window of this pass ([0, K+1) in one pass).  A later pass of the
+  // windowed schedule (i0 > 0) rebuilds its live list from the keys of the
+  // previous window [pi0, i0) of the previous live list.
+  int i0, i1, pi0;
+  int windowed;              // a pass of the windowed schedule: keys only, no finalisers
+  const int32_t* live_in;    // previous pass's live list (NULL: 0..B-1)
+  const uint32_t* count_in;  // its length (NULL: B)
+  const uint32_t* base_in;   // packed rows claimed by the sequences decided before (NULL: 0)
+  int32_t* live_out;         // CTA 0 publishes this pass's live list here
   uint32_t* count_out;
-  uint32_t* pass_counts;     // last pass: counters of every pass, zeroed by its last CTA out
+  uint32_t* base_out;        // ... and the packed rows claimed by the sequences decided so far
+  // verify_finish_kernel: the passes' counters, zeroed with the keys by its last CTA out
+  uint32_t* pass_counts;
   int n_counts;
-  uint32_t* exits;           // last pass: CTAs out (zero between calls)
+  uint32_t* exits;           // CTAs out (zero between calls)
   int defer_copies;          // the finaliser leaves the copies to verify_copy_kernel
   int32_t* pack_off;         // [B] first packed row of each sequence (deferred copies)
 };
@@ -283,23 +293,20 @@ __device__ void finish_sequence(const VerifyParams& p, int b, int A, int rows, c
   if (!p.defer_copies) copy_sequence<T>(p, b, A, s_off, staging);
 }
 
-// Every row of sequence b in the window [i0, i1) has its key (rows before
-// i0 matched their draft tokens in earlier passes): the first mismatch in the
-// window by ballot, then the outputs; a sequence without one, when rows
-// remain, goes on to the next pass instead.
+// Every row of sequence b has its key (one pass): the first mismatch by
+// ballot, then the outputs.
 template <typename T>
 __device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s_A, uint4* staging) {
   const int K = p.K, K1 = K + 1;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int i = threadIdx.x; i < p.i1; i += kThreads)
+  for (int i = threadIdx.x; i < K1; i += kThreads)
     s_t[i] = (int)key_index(__ldcg(&p.keys[(long long)b * K1 + i]));
   __syncthreads();
   if (warp == 0) {
-    int A = p.i1 == K1 ? K : -1;  // -1: every row of the window matched, more rows to read
-    const int hi = min(p.i1, K);
-    for (int base = p.i0; base < hi; base += 32) {
+    int A = K;
+    for (int base = 0; base < K; base += 32) {
       const int i = base + lane;
-      const bool mismatch = (i < hi) && (s_t[i] != p.draft[(long long)b * K + i]);
+      const bool mismatch = (i < K) && (s_t[i] != p.draft[(long long)b * K + i]);
       const unsigned bal = __ballot_sync(0xFFFFFFFFu, mismatch);
       if (bal) {
         A = base + __ffs(bal) - 1;
@@ -310,11 +317,130 @@ __device__ void finalize_sequence(const VerifyParams& p, int b, int* s_t, int* s
   }
   __syncthreads();
   const int A = *s_A;
-  if (threadIdx.x == 0) {
-    p.tickets[b] = 0u;
-    if (A < 0) p.live_out[atomicAdd(p.count_out, 1u)] = b;
+  if (threadIdx.x == 0) p.tickets[b] = 0u;
+  finish_sequence<T>(p, b, A, K1, s_t, s_A + 1, staging);
+}
+
+// Exclusive prefix sum over the CTA (kThreads threads, in thread order) of
+// one value per thread; *total receives the sum.  s_warp holds kThreads / 32
+// + 1 ints.  Every thread of the CTA must call it.
+__device__ __forceinline__ int block_exclusive_scan(int v, int* s_warp, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int y = __shfl_up_sync(0xFFFFFFFFu, x, off);
+    if (lane >= off) x += y;
   }
-  if (A >= 0) finish_sequence<T>(p, b, A, p.i1, s_t, s_A + 1, staging);
+  if (lane == 31) s_warp[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < kThreads / 32 ? s_warp[lane] : 0;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xFFFFFFFFu, w, off);
+      if (lane >= off) w += y;
+    }
+    if (lane < kThreads / 32) s_warp[lane] = w;  // inclusive warp totals
+  }
+  __syncthreads();
+  const int excl = x - v + (warp > 0 ? s_warp[warp - 1] : 0);
+  *total = s_warp[kThreads / 32 - 1];
+  __syncthreads();  // s_warp may be reused by the next call
+  return excl;
+}
+
+// Outputs of sequence b, decided with accepted length A after a windowed
+// pass (every row 0..A has its key): committed tokens, accepted length,
+// bonus, n_b and the first packed row `off` of its n_b conditioned rows.
+// The CTA's threads share the K + 1 committed slots.
+__device__ void write_decided(const VerifyParams& p, int b, int A, int off) {
+  const int K = p.K, K1 = K + 1;
+  for (int i = threadIdx.x; i < K1; i += kThreads) {
+    const long long o = (long long)b * K1 + i;
+    p.committed[o] = i <= A ? (int)key_index(__ldcg(&p.keys[o])) : -1;
+  }
+  if (threadIdx.x == 0) {
+    const int nb = max(0, K - 1 - A);
+    p.accept_len[b] = A;
+    p.bonus[b] = (int)key_index(__ldcg(&p.keys[(long long)b * K1 + A]));
+    if (p.n_out) p.n_out[b] = nb;
+    if (p.R_count) p.pack_off[b] = off;
+  }
+}
+
+// Decides the window [w0, w1) of a windowed verification for the n sequences
+// of `list` (NULL: 0..n-1), the same in every CTA.  s_first[l] = the first
+// row of the window (rows below K only) whose argmax differs from the draft
+// token, as an offset from w0, or w1 - w0 if none: the sequence goes on (to
+// the next window) unless the window ends the block (w1 = K + 1, then A = K).
+// The sequences that end here take consecutive packed rows in list order
+// after `base`; s_off[l] receives their offsets.  Their outputs are written by
+// CTA l mod grid.  Returns the rows they claim; fills s_live (with the going-
+// on sequences, in order) and *n_live when s_live is not NULL.
+__device__ int decide_window(const VerifyParams& p, const int32_t* list, int n, int w0, int w1, int base,
+                             int* s_first, int* s_off, int* s_live, int* n_live, int* s_warp) {
+  const int K = p.K, K1 = K + 1;
+  const int wp = w1 - w0;
+  const bool last = w1 == K1;
+  for (int l = threadIdx.x; l < n; l += kThreads) s_first[l] = wp;
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < n * wp; idx += kThreads) {
+    const int l = idx / wp, r = idx - l * wp, i = w0 + r;
+    const int b = list ? __ldcg(list + l) : l;
+    if (i < K && (int)key_index(__ldcg(&p.keys[(long long)b * K1 + i])) != __ldg(p.draft + (long long)b * K + i))
+      atomicMin(&s_first[l], r);
+  }
+  __syncthreads();
+  int rows = 0, nl = 0;
+  for (int c0 = 0; c0 < n; c0 += kThreads) {
+    const int l = c0 + (int)threadIdx.x;
+    const int first = l < n ? s_first[l] : 0;
+    const bool goes_on = l < n && first == wp && !last;
+    const int A = w0 + min(first, K - w0);  // first == wp in the last window: A = K
+    const int nb = (l < n && !goes_on) ? max(0, K - 1 - A) : 0;
+    int chunk;
+    const int off = block_exclusive_scan(nb, s_warp, &chunk);
+    if (l < n) s_off[l] = base + rows + off;
+    rows += chunk;
+    if (s_live) {
+      const int pos = block_exclusive_scan(goes_on ? 1 : 0, s_warp, &chunk);
+      if (goes_on) s_live[nl + pos] = list ? __ldcg(list + l) : l;
+      nl += chunk;
+    }
+  }
+  __syncthreads();
+  for (int l = blockIdx.x; l < n; l += gridDim.x) {
+    const int first = s_first[l];
+    if (first == wp && !last) continue;  // goes on
+    write_decided(p, list ? __ldcg(list + l) : l, w0 + min(first, K - w0), s_off[l]);
+  }
+  if (n_live) *n_live = nl;
+  return rows;
+}
+
+// Start of a later pass of the windowed schedule: decides the previous
+// window [pi0, i0) for the previous pass's live sequences, then builds this
+// pass's live list in s_live (CTA 0 publishes it, with the packed rows
+// claimed so far, for the next pass and the finish kernel).  s_stage holds 3 B
+// ints.  Returns the list's length.
+__device__ int begin_later_pass(const VerifyParams& p, int* s_stage, int* s_warp) {
+  const int n_prev = p.count_in ? (int)__ldcg(p.count_in) : p.B;
+  const int base = p.base_in ? (int)__ldcg(p.base_in) : 0;
+  int* s_first = s_stage;
+  int* s_off = s_stage + p.B;
+  int* s_live = s_stage + 2 * p.B;
+  int n = 0;
+  const int rows = decide_window(p, p.live_in, n_prev, p.pi0, p.i0, base, s_first, s_off, s_live, &n, s_warp);
+  if (blockIdx.x == 0) {
+    for (int l = threadIdx.x; l < n; l += kThreads) p.live_out[l] = s_live[l];
+    if (threadIdx.x == 0) {
+      *p.count_out = (uint32_t)n;
+      *p.base_out = (uint32_t)(base + rows);
+    }
+  }
+  __syncthreads();
+  return n;
 }
 
 template <typename T, bool VEC>
@@ -327,9 +453,13 @@ __global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams 
   pdl_launch_dependents();  // the next kernel may take SMs as this grid's CTAs finish
 
   long long n_live = p.B;
-  if (p.count_in) {  // a later pass: the previous pass wrote the live list
+  const int* s_list = nullptr;  // the pass's live sequences (NULL: 0..B-1)
+  if (p.windowed && p.i0 > 0) {
+    // a later pass: the previous pass's keys decide which sequences go on
+    __shared__ int s_warp[kThreads / 32 + 1];
     pdl_wait();
-    n_live = (long long)__ldcg(p.count_in);
+    n_live = begin_later_pass(p, reinterpret_cast<int*>(s_stage), s_warp);
+    s_list = reinterpret_cast<int*>(s_stage) + 2 * p.B;
   }
   const long long VV = p.slots_per_row;
   const int K1 = p.K + 1, W = p.i1 - p.i0;
@@ -345,7 +475,7 @@ __global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams 
   while (s < s_end) {
     const long long vrow = s / VV;  // row of the pass: sequence vrow / W, window row vrow % W
     const long long l = vrow / W;
-    const int b = p.live_in ? __ldg(p.live_in + l) : (int)l;
+    const int b = s_list ? s_list[l] : (int)l;
     const int i = p.i0 + (int)(vrow - l * W);
     const long long seg_end = min(s_end, (vrow + 1) * VV);
     const int v0 = (int)(s - vrow * VV), v1 = (int)(seg_end - vrow * VV);
@@ -357,7 +487,7 @@ __global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams 
     if (threadIdx.x == 0) atomicMax(&p.keys[(long long)b * K1 + i], key);
     s = seg_end;
 
-    if (s == s_end || s % per_seq == 0) {
+    if (!p.windowed && (s == s_end || s % per_seq == 0)) {
       // This CTA has folded in all of its rows of sequence b.  The CTAs that
       // own slots of b are those from the owner of its first slot to the
       // owner of its last (every active CTA range is non-empty: G <= T_).
@@ -376,14 +506,6 @@ __global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams 
         finalize_sequence<T>(p, b, s_t, s_A, s_stage);
       }
       __syncthreads();
-    }
-  }
-  // The last pass's last CTA out zeroes the passes' live counters.
-  if (p.exits && threadIdx.x == 0) {
-    __threadfence();
-    if (atomicAdd(p.exits, 1u) == gridDim.x - 1u) {
-      for (int k = 0; k < p.n_counts; ++k) p.pass_counts[k] = 0u;
-      *p.exits = 0u;
     }
   }
 }
@@ -468,8 +590,125 @@ __global__ void __launch_bounds__(kThreads, 2) verify_copy_kernel(const VerifyPa
   }
 }
 
+// The end of a windowed verification, after its last pass.  Decides the
+// sequences of the last window (decide_window over the last pass's live list,
+// the same in every CTA; their outputs spread over the CTAs), sets R, and the
+// last CTA to finish with the keys zeroes them and the passes' counters for
+// the next call.  Then the row copies as in verify_copy_kernel: the
+// unconditioned rows of e~ and the packed [m; u] (and e) rows, each warp one
+// row segment at a time; a sequence decided by an earlier pass gives its
+// accepted length and first packed row from accept_len and pack_off.  s_dyn
+// holds 4 B ints.
+template <typename T, bool CV>
+__global__ void __launch_bounds__(kThreads, 2) verify_finish_kernel(const VerifyParams p) {
+  extern __shared__ int s_dyn[];
+  __shared__ int s_warp[kThreads / 32 + 1];
+  __shared__ int s_last;
+  pdl_launch_dependents();
+  pdl_wait();
+  const int B = p.B, K = p.K, K1 = K + 1, d = p.d;
+  const int n_last = (int)__ldcg(p.count_in);
+  const int base = (int)__ldcg(p.base_in);
+  int* s_first = s_dyn;         // [n_last]
+  int* s_off = s_dyn + B;       // [n_last]
+  int* s_mapA = s_dyn + 2 * B;  // [B]: accepted length of the sequences decided here, -1 for the others
+  int* s_mapO = s_dyn + 3 * B;  // [B]: their first packed row
+  for (int b = threadIdx.x; b < B; b += kThreads) s_mapA[b] = -1;
+  __syncthreads();
+  const int rows = decide_window(p, p.live_in, n_last, p.i0, K1, base, s_first, s_off, nullptr, nullptr, s_warp);
+  for (int l = threadIdx.x; l < n_last; l += kThreads) {
+    const int b = __ldcg(p.live_in + l);
+    s_mapA[b] = p.i0 + min(s_first[l], K - p.i0);
+    s_mapO[b] = s_off[l];
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0 && p.R_count) *p.R_count = base + rows;
+  // every read of the keys above is done: the last CTA out resets them
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(p.exits, 1u) == gridDim.x - 1u;
+  }
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    for (long long i = threadIdx.x; i < (long long)B * K1; i += kThreads) p.keys[i] = 0ull;
+    if (threadIdx.x == 0) {
+      for (int k = 0; k < p.n_counts; ++k) p.pass_counts[k] = 0u;
+      *p.exits = 0u;
+    }
+  }
+  // the row copies
+  constexpr int E = CV ? 16 / (int)sizeof(T) : 1;  // elements per copy slot
+  const int vpr = d / E;
+  const bool pack = p.R_count != nullptr;
+  const int nseg = (p.e_out ? 1 : 0) + (pack ? (p.e_dense ? 3 : 2) : 0);
+  const long long items = (long long)B * K * nseg;
+  const int lane = threadIdx.x & 31;
+  const long long warps = (long long)gridDim.x * (kThreads / 32);
+  const T* e = reinterpret_cast<const T*>(p.e);
+  const T* hD = reinterpret_cast<const T*>(p.hD);
+  const T* hT = reinterpret_cast<const T*>(p.hT);
+  T* e_out = reinterpret_cast<T*>(p.e_out);
+  T* apack = reinterpret_cast<T*>(p.apack);
+  T* epack = reinterpret_cast<T*>(p.epack);
+  for (long long it = (long long)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5); it < items; it += warps) {
+    const long long u = it / nseg;
+    const int seg = (int)(it - u * nseg);
+    const int b = (int)(u / K), j = (int)(u - (long long)b * K);
+    const int Ah = s_mapA[b];
+    const int A = Ah >= 0 ? Ah : __ldcg(p.accept_len + b);
+    const int nb = (K - 1 - A) > 0 ? (K - 1 - A) : 0;
+    const long long pos = (long long)b * K + j;
+    const int kind = p.e_out ? seg : seg + 1;  // 0 e_out row, 1 m half, 2 u half, 3 packed e
+    const T* src;
+    T* dst;
+    if (kind == 0) {
+      if (p.cond_copy == kCondCopyKeep && j < nb) continue;  // the conditioning kernels write it
+      src = (p.cond_copy == kCondCopyM && j < nb) ? hD + (pos + A + 1) * d
+                                                  : e + (long long)b * p.e_batch_stride + (long long)j * p.e_pos_stride;
+      dst = e_out + pos * d;
+    } else {
+      if (j >= nb) continue;
+      const long long row = (long long)(Ah >= 0 ? s_mapO[b] : __ldcg(p.pack_off + b)) + j;
+      if (kind == 1) {
+        src = hD + (pos + A + 1) * d;
+        dst = apack + row * 2 * d;
+        if (lane == 0) p.rowmap[row] = (int32_t)pos;
+      } else if (kind == 2) {
+        src = hT + (pos + A) * d;
+        dst = apack + row * 2 * d + d;
+      } else {
+        src = e + pos * d;
+        dst = epack + row * d;
+      }
+    }
+    if constexpr (CV) {
+      const uint4* s4 = reinterpret_cast<const uint4*>(src);
+      uint4* d4 = reinterpret_cast<uint4*>(dst);
+      for (int v0 = 0; v0 < vpr; v0 += 32 * kCopyBatch) {
+        uint4 x[kCopyBatch];
+#pragma unroll
+        for (int k = 0; k < kCopyBatch; ++k) {
+          const int v = v0 + k * 32 + lane;
+          if (v < vpr) x[k] = __ldcs(s4 + v);
+        }
+#pragma unroll
+        for (int k = 0; k < kCopyBatch; ++k) {
+          const int v = v0 + k * 32 + lane;
+          if (v < vpr) d4[v] = x[k];
+        }
+      }
+    } else {
+      for (int v = lane; v < d; v += 32) dst[v] = src[v];
+    }
+  }
+}
+
 std::atomic<int> g_schedule{RETRACE_VERIFY_AUTO};
 constexpr long long kWindowMinBatchRowBytes = 16ll << 20;  // B * V * element size
+// Largest batch of the windowed schedule: every CTA keeps its decisions and
+// live lists, up to 4 B ints, in 32 KB of shared memory.
+constexpr int kWindowMaxB = kCopyStageBytes / 16;
 
 // Row windows of the windowed schedule: the first kWindowRows rows, then
 // windows half as long again as the one before (fewer, longer passes as the
@@ -497,7 +736,7 @@ int verify_windows(int B, int K, int V, int elem_bytes, bool have_workspace, boo
   const int n = window_bounds(K1, start);
   const int mode = g_schedule.load(std::memory_order_relaxed);
   const long long wave = (long long)B * V * elem_bytes;
-  const bool windowed = have_workspace && !argmax_out && B > 0 && n > 1 &&
+  const bool windowed = have_workspace && !argmax_out && B > 0 && B <= kWindowMaxB && n > 1 &&
                         (mode == RETRACE_VERIFY_WINDOWS || (mode == RETRACE_VERIFY_AUTO && wave >= kWindowMinBatchRowBytes));
   if (windowed) return n;
   start[0] = 0;
@@ -519,6 +758,20 @@ cudaError_t launch_copies(const VerifyArgs& a, const VerifyParams& p, long long 
                   (!a.R_count || (al(a.hD) && al(a.hT) && al(a.apack) && (!a.e_dense || al(a.epack))));
   auto kern = cv ? verify_copy_kernel<T, true> : verify_copy_kernel<T, false>;
   return launch_dependent(kern, dim3((unsigned)grid), dim3(kThreads), 0, stream, 1u, p);
+}
+
+// verify_finish_kernel after the last windowed pass (programmatically
+// dependent), with the 16-byte copy path when every copied tensor allows it.
+template <typename T>
+cudaError_t launch_finish(const VerifyArgs& a, const VerifyParams& p, long long grid, cudaStream_t stream) {
+  const size_t es = sizeof(T);
+  auto al = [](const void* q) { return (uintptr_t)q % 16 == 0; };
+  const bool cv = (a.d * es) % 16 == 0 && (!a.e_out || (al(a.e) && al(a.e_out))) &&
+                  (a.e_pos_stride * (long long)es) % 16 == 0 && (a.e_batch_stride * (long long)es) % 16 == 0 &&
+                  (a.cond_copy != kCondCopyM || al(a.hD)) &&
+                  (!a.R_count || (al(a.hD) && al(a.hT) && al(a.apack) && (!a.e_dense || al(a.epack))));
+  auto kern = cv ? verify_finish_kernel<T, true> : verify_finish_kernel<T, false>;
+  return launch_dependent(kern, dim3((unsigned)grid), dim3(kThreads), (size_t)4 * a.B * sizeof(int), stream, 1u, p);
 }
 
 template <typename T, bool VEC>
@@ -571,6 +824,10 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
   p.cond_copy = a.cond_copy;
   p.i0 = 0;
   p.i1 = a.K + 1;
+  p.pi0 = 0;
+  p.windowed = 0;
+  p.base_in = nullptr;
+  p.base_out = nullptr;
   p.live_in = nullptr;
   p.count_in = nullptr;
   p.live_out = nullptr;
@@ -606,24 +863,27 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
     const long long copy_grid = ((long long)a.B * a.K * 4 + 15) / 16;  // a warp per row segment
     return launch_copies<T>(a, p, copy_grid < grid_full ? copy_grid : grid_full, stream);
   }
-  // Windowed: pass k reads rows [start[k], start[k+1]) of the sequences that
-  // matched every earlier row; each pass after the first waits for its
-  // predecessor inside the kernel (programmatic dependent launch) and sizes
-  // its work from the live count that pass wrote.  The copies of a fused
-  // round follow in one more kernel, balanced over sequences.
-  const bool copies = a.e_out || a.R_count;
-  p.defer_copies = copies ? 1 : 0;
+  // Windowed: pass k reads rows [start[k], start[k+1]) of the sequences whose
+  // draft tokens matched every earlier row.  Each pass after the first waits
+  // for its predecessor inside the kernel (programmatic dependent launch),
+  // rebuilds the live list from the previous window's keys and sizes its
+  // work from it; pass k publishes its list for pass k + 1 (two buffers in
+  // turn).  verify_finish_kernel writes the outputs and does the copies.
+  // Counters: pass_counts[0] CTAs out of the finish kernel, [k] the length of
+  // pass k's live list, [kMaxWindowPasses + 1 + k] the packed rows claimed by
+  // the sequences decided before pass k's window.
+  uint32_t* bases = a.pass_counts + kMaxWindowPasses + 1;
+  p.windowed = 1;
   for (int k = 0; k < n_pass; ++k) {
-    const bool last = k == n_pass - 1;
     p.i0 = start[k];
     p.i1 = start[k + 1];
-    p.live_in = k == 0 ? nullptr : a.live + (size_t)((k - 1) & 1) * a.B;
-    p.count_in = k == 0 ? nullptr : a.pass_counts + k;
-    p.live_out = last ? nullptr : a.live + (size_t)(k & 1) * a.B;
-    p.count_out = last ? nullptr : a.pass_counts + k + 1;
-    p.pass_counts = last ? a.pass_counts + 1 : nullptr;
-    p.n_counts = last ? n_pass - 1 : 0;
-    p.exits = last ? a.pass_counts : nullptr;
+    p.pi0 = k > 0 ? start[k - 1] : 0;
+    p.live_in = k <= 1 ? nullptr : a.live + (size_t)((k - 1) & 1) * a.B;  // pass 0 holds every sequence
+    p.count_in = k <= 1 ? nullptr : a.pass_counts + (k - 1);
+    p.base_in = k <= 1 ? nullptr : bases + (k - 1);
+    p.live_out = k == 0 ? nullptr : a.live + (size_t)(k & 1) * a.B;
+    p.count_out = k == 0 ? nullptr : a.pass_counts + k;
+    p.base_out = k == 0 ? nullptr : bases + k;
     if (k == 0) {
       verify_kernel<T, VEC><<<(unsigned)grid_full, kThreads, kCopyStageBytes, stream>>>(p);
       err = cudaGetLastError();
@@ -633,8 +893,15 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
     }
     if (err != cudaSuccess) return err;
   }
-  if (copies) return launch_copies<T>(a, p, grid_full, stream);
-  return cudaSuccess;
+  // the finish kernel decides the last window [start[n-1], K+1) for the last pass's live list
+  p.i0 = start[n_pass - 1];
+  p.live_in = a.live + (size_t)((n_pass - 1) & 1) * a.B;
+  p.count_in = a.pass_counts + (n_pass - 1);
+  p.base_in = bases + (n_pass - 1);
+  p.pass_counts = a.pass_counts + 1;
+  p.n_counts = 2 * kMaxWindowPasses + 1;  // every live count and base after the exit counter
+  p.exits = a.pass_counts;
+  return launch_finish<T>(a, p, grid_full, stream);
 }
 
 }  // namespace

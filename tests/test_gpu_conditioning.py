@@ -168,11 +168,13 @@ def accept_for_rows(B, K, R):
     return a.cuda()
 
 
-@pytest.mark.parametrize("R", [1, 127, 128, 129, 255, 256, 257, 384, 513])
+@pytest.mark.parametrize("R", [1, 15, 16, 17, 127, 128, 129, 240, 241, 255, 256, 257, 384, 513, 769, 1023, 1200])
 def test_pair_tile_boundaries(rt, R):
-    """Row counts around the 128-row halves and 256-row pairs of the
-    CTA-pair kernel (one CTA's half empty, odd block counts).  B (K-1) = 1200
-    possible rows keeps the call off the small-R path."""
+    """Row counts around the tile edges of the CTA-pair kernel: one to five
+    row tiles of 16 to 256 rows (a multiple of 16 chosen from R), halves of
+    8 to 128 rows in each CTA loaded as boxes of 64, 32, 16 and 8 rows, and
+    the last tile's padding.  B (K-1) = 1200 possible rows keeps the call off
+    the small-R path."""
     B, K, d, dtype = 80, 16, 256, torch.bfloat16
     x = make_inputs(B, K, d, dtype, seed=R, accept=accept_for_rows(B, K, R))
     A = host_int(x["accept"])
