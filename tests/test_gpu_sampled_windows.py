@@ -169,3 +169,42 @@ def test_one_pass_round_many_sequences_equals_windowed(rt):
         for name in ("accept_len", "committed", "bonus", "n", "e_out"):
             assert torch.equal(getattr(o, name), getattr(outs[0], name)), name
     assert ws.check() == 0
+
+
+def test_greedy_and_sampled_windows_share_a_workspace(rt, windows):
+    """Windowed greedy and windowed temperature-T verification alternate on
+    one workspace: each must leave the live lists, pass counters and keys as
+    the other expects, so every call equals the same call on a fresh
+    workspace (and the greedy one equals the oracle)."""
+    import oracle
+    from parity import host_f64
+
+    cfg = CONFIGS[4]
+    g = torch.Generator()
+    g.manual_seed(123)
+    accept = torch.randint(0, cfg.K + 1, (cfg.B,), generator=g)
+    x, s = planted(cfg, accept)
+    T, k, p = s["temperature"], s["top_k"], s["top_p"]
+
+    def greedy(ws):
+        B, K1, _ = x["logits"].shape
+        outs = [torch.full((B,), -7, dtype=torch.int32, device="cuda"),
+                torch.full((B, K1), -7, dtype=torch.int32, device="cuda"),
+                torch.full((B,), -7, dtype=torch.int32, device="cuda")]
+        rt.retrace_verify(x["logits"], s["draft"], *outs, ws)
+        torch.cuda.synchronize()
+        return outs
+
+    def fresh():
+        return rt.Workspace(cfg.B, cfg.K, cfg.V, cfg.d, cfg.torch_dtype)
+
+    ref_g, ref_s = greedy(fresh()), sampled(rt, x, s, fresh(), T, k, p)
+    want = oracle.verify(host_f64(x["logits"]), host_int(s["draft"]))
+    np.testing.assert_array_equal(host_int(ref_g[0]), want["accept_len"])
+    np.testing.assert_array_equal(host_int(ref_g[1]), want["committed"])
+    ws = fresh()
+    for it in range(6):
+        got, ref = (greedy(ws), ref_g) if it % 2 == 0 else (sampled(rt, x, s, ws, T, k, p), ref_s)
+        for a, b in zip(got, ref):
+            assert torch.equal(a, b), it
+    assert ws.check() == 0

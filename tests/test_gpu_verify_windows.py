@@ -166,6 +166,18 @@ def test_windows_workspace_left_clean(rt, windows):
     assert ws.check() == 0
 
 
+def test_windows_batch_limit(rt):
+    """The default schedule verifies in row windows up to B = 2048 sequences
+    (each CTA keeps the live lists and decisions of the whole batch in shared
+    memory) and in one pass above that; both against the oracle, on the
+    smallest rows that still make one row of the batch 16 MiB."""
+    K, V = 8, 4104
+    for B, windowed in ((2048, True), (2049, False)):
+        assert (len(rt.retrace_verify_plan(B, K, V, torch.bfloat16)) > 2) == windowed
+        logits, draft = random_case(B, K, V, torch.bfloat16, seed=B, ties=True)
+        check(rt, logits, draft)
+
+
 def test_windows_in_cuda_graph(rt, windows):
     """Captured once, replayed on new logits written into the same buffer."""
     B, K, V = 128, 16, 30000
