@@ -62,9 +62,9 @@ L2_FLUSH_BYTES = 256 << 20
 # kernel sources it was measured on: `sources` is kernel_sources_hash() at the
 # time, and the line reports null traffic once the sources differ.
 TRAFFIC = {
-    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311331584 + 3026944 + 184293120 + 65792 + 55385600 + 1024
-                                      + 47148032 + 3488512, "sources": "32ff2909d7391a9f"},
-    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 611928576 + 39502080, "sources": "32ff2909d7391a9f"},
+    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311306496 + 2842368 + 184312064 + 70656 + 55401984 + 2560
+                                      + 47180544 + 3741952, "sources": "1992adff287baa27"},
+    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 477912576 + 35674368, "sources": "1992adff287baa27"},
 }
 
 
@@ -514,7 +514,9 @@ def run_gpu(args) -> dict | None:
         copies = " + verify_copy_kernel (copy of unconditioned rows + row packing)"
         passes = "sampled_topk_kernel + sampled_finalize_kernel" if args.sampled else "verify_kernel"
         if n_pass > 1:
-            v_kernel = f"{passes} x{n_pass} passes over row windows {windows}{copies}"
+            finish = (" + verify_finish_kernel (decisions of the last window, copy of unconditioned rows + row "
+                      "packing)")
+            v_kernel = f"{passes} x{n_pass} passes over row windows {windows}{finish}"
         elif verify_launches > (2 if args.sampled else 1):
             v_kernel = f"{passes} (one pass){copies}"
         else:
@@ -535,8 +537,8 @@ def run_gpu(args) -> dict | None:
             "launches": verify_launches,
             "avg_launch_us": round(v_avg_s * 1e6, 2),
             "traffic": None if args.sampled else measured_traffic("verify", cfg.name, args.variant),
-            "traffic_source": "ncu dram read+write of the verification kernels (passes + copy kernel) of one round "
-                              "on this workload",
+            "traffic_source": "ncu dram read+write of the verification kernels (passes + finishing or copy "
+                              "kernel) of one round on this workload",
         }
         if args.variant in ("overwrite", "none"):
             v_roof["kernel"] = v_roof["kernel"].replace("copy of unconditioned rows + row packing",

@@ -234,6 +234,9 @@ retrace_status retrace_gate_fuse(const void* e, int64_t e_batch_stride, int64_t 
  *                           multiple of 8 and V >= 4096, K >= 2, 4d <= 16384).
  *                           Same results bit for bit; other shapes or an
  *                           ablation flag return RETRACE_ERR_UNSUPPORTED.
+ *                           Experimental: measured slower than the default
+ *                           round (about 2.4x the time at B = 256); the
+ *                           default round never takes it.
  * Unknown bits, or two ablation flags together, return
  * RETRACE_ERR_INVALID_ARG. */
 #define RETRACE_ROUND_OVERLAP 0x1u

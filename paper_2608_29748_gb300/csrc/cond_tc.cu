@@ -631,39 +631,25 @@ constexpr uint32_t IDESC_M256_N256 = idesc_bf16_f32(256, 256);
 // weight tiles as well as row blocks (measured: 260 against 264 us for
 // row-block-major order at config 5).
 constexpr int kGroupBlocks = 4;
-constexpr int P_TILE_SLOTS = 3;  // tile indices in flight: the head publishes one tile ahead
+constexpr int P_TILE_SLOTS = 3;  // tile indices in flight: the leader publishes one tile ahead
 
-// Clusters of CL CTAs: CL = 2 is one CTA pair; CL = 4 is two CTA pairs
-// working at once on the same weight tile for two different 256-row blocks,
-// each weight half loaded once and multicast to the CTA at the same position
-// in both pairs (half the L2 reads of the weights).  A stage a producer fills
-// by multicast is then read by both pairs' MMAs, so its empty barrier takes
-// one commit from each pair.  CTA pairs are (0, 1) and (2, 3); the tile queue
-// belongs to cluster rank 0, the stage barriers of a pair to its even CTA.
-template <int CL>
 __global__ void __launch_bounds__(P_THREADS, 1)
     cond_pair_kernel(const __grid_constant__ CUtensorMap tmApack, const __grid_constant__ CUtensorMap tmWc,
                      const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmWv,
                      const __grid_constant__ CUtensorMap tmWg, const CondParams p) {
-  constexpr int NPAIR = CL / 2;                  // CTA pairs per cluster
-  constexpr int WROWS = 128 / NPAIR;             // weight rows each CTA loads per stage
-  constexpr uint16_t ALL = (uint16_t)((1u << CL) - 1u);
   extern __shared__ uint8_t dsmem[];
-  __shared__ __align__(8) uint64_t bar_full[PSTAGES];           // pair leader: the pair's bytes of a stage
-  __shared__ __align__(8) uint64_t bar_empty[PSTAGES];          // stage free (one commit per pair)
-  __shared__ __align__(8) uint64_t bar_tfull[2];                // accumulator ready (both CTAs of the pair)
-  __shared__ __align__(8) uint64_t bar_tempty[2];               // pair leader: eight epilogue warps done
-  __shared__ __align__(8) uint64_t bar_tile_full[P_TILE_SLOTS];   // tile index published (every CTA)
-  __shared__ __align__(8) uint64_t bar_tile_empty[P_TILE_SLOTS];  // cluster rank 0: every reader done
+  __shared__ __align__(8) uint64_t bar_full[PSTAGES];             // leader: both CTAs' bytes of a stage
+  __shared__ __align__(8) uint64_t bar_empty[PSTAGES];            // stage free (leader's commit, both CTAs)
+  __shared__ __align__(8) uint64_t bar_tfull[2];                  // accumulator ready (both CTAs)
+  __shared__ __align__(8) uint64_t bar_tempty[2];                 // leader: eight epilogue warps done
+  __shared__ __align__(8) uint64_t bar_tile_full[P_TILE_SLOTS];   // tile index published (both CTAs)
+  __shared__ __align__(8) uint64_t bar_tile_empty[P_TILE_SLOTS];  // leader: ten readers done
   __shared__ int s_tile[P_TILE_SLOTS];
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t rank = cluster_rank();
-  const uint32_t pair = rank >> 1, prank = rank & 1u;
-  const bool leader = prank == 0;    // this CTA issues its pair's MMAs
-  const bool head = rank == 0;       // this CTA runs the cluster's tile queue
-  const uint16_t pair_mask = (uint16_t)(0x3u << (2 * pair));
+  const bool leader = rank == 0;  // issues the pair's MMAs and runs the tile queue
   const int d = p.d;
   const int nt0 = d / 256, nt1 = d / 128;
   pdl_launch_dependents();
@@ -676,17 +662,16 @@ __global__ void __launch_bounds__(P_THREADS, 1)
   if (tid == 0) {
     s_abort = 0;
     for (int s = 0; s < PSTAGES; ++s) {
-      mbar_init(smem_u32(&bar_full[s]), 1);  // the pair leader's expect_tx
-      mbar_init(smem_u32(&bar_empty[s]), NPAIR);
+      mbar_init(smem_u32(&bar_full[s]), 1);  // the leader's expect_tx
+      mbar_init(smem_u32(&bar_empty[s]), 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&bar_tfull[a]), 1);
-      mbar_init(smem_u32(&bar_tempty[a]), 8);  // four epilogue warps in each CTA of the pair
+      mbar_init(smem_u32(&bar_tempty[a]), 8);  // four epilogue warps in each CTA
     }
     for (int a = 0; a < P_TILE_SLOTS; ++a) {
       mbar_init(smem_u32(&bar_tile_full[a]), 1);
-      // MMA of every pair, 4 epilogue warps of every CTA, producer of every CTA but rank 0
-      mbar_init(smem_u32(&bar_tile_empty[a]), NPAIR + 4 * CL + (CL - 1));
+      mbar_init(smem_u32(&bar_tile_empty[a]), 10);  // MMA + 4 epilogue warps; producer + 4 epilogue warps
     }
     fence_mbar_init();
   }
@@ -707,7 +692,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
-  cluster_sync_all();  // every CTA's barriers initialised before any remote arrive
+  cluster_sync_all();  // both CTAs' barriers initialised before any remote arrive
   tc_fence_after();
   const uint32_t tmem = s_tmem;
   const uint32_t base = (smem_u32(dsmem) + 1023u) & ~1023u;
@@ -717,64 +702,60 @@ __global__ void __launch_bounds__(P_THREADS, 1)
   // every role that reads them waits here first.  The gate-bias GEMV (warps
   // 2-3) reads only the inputs and starts at once.  With R = 0 the queue's
   // first claim already ends every role.
-  int R = 0, T0 = 0, T = 0, groups = 0;
+  int R = 0, T0 = 0, T = 0, pairs_m = 0;
   if (warp != 2 && warp != 3) {
     pdl_wait();
     R = *(volatile const int32_t*)p.R;
-    const int pairs_m = (R + 2 * BM - 1) / (2 * BM);
-    groups = (pairs_m + NPAIR - 1) / NPAIR;  // a cluster tile covers NPAIR pair blocks
-    T0 = p.do_correct ? groups * nt0 : 0;
-    T = T0 + (p.do_gate ? groups * nt1 : 0);
+    pairs_m = (R + 2 * BM - 1) / (2 * BM);
+    T0 = p.do_correct ? pairs_m * nt0 : 0;
+    T = T0 + (p.do_gate ? pairs_m * nt1 : 0);
   }
   // Tile t: correction tiles first, then gate tiles; within each kind, groups
   // of kGroupBlocks pair blocks with the weight tile outer inside a group.
   auto decode = [&](int t, bool* corr, int* m0, int* n0) {
     *corr = t < T0;
     const int tt = *corr ? t : t - T0, nt = *corr ? nt0 : nt1;
-    constexpr int G = kGroupBlocks / NPAIR > 0 ? kGroupBlocks / NPAIR : 1;
-    const int g = tt / (G * nt), w = tt - g * G * nt;
-    const int glen = min(G, groups - g * G);
-    const int cg = g * G + w % glen;  // cluster block group
-    *m0 = (cg * NPAIR + (int)pair) * 2 * BM + (int)prank * BM;  // this CTA's rows
+    const int g = tt / (kGroupBlocks * nt), w = tt - g * kGroupBlocks * nt;
+    const int glen = min(kGroupBlocks, pairs_m - g * kGroupBlocks);
+    const int pb = g * kGroupBlocks + w % glen;  // pair block
+    *m0 = pb * 2 * BM + (int)rank * BM;          // this CTA's rows
     *n0 = (w / glen) * (*corr ? 256 : 128);
   };
-  // barriers of this CTA's pair leader, and of cluster rank 0, seen from here
-  auto pair_lead = [&](const void* local) { return map_rank(smem_u32(local), rank & ~1u); };
-  auto head_addr = [&](const void* local) { return map_rank(smem_u32(local), 0); };
+  // the leader's barriers as seen from either CTA
+  auto leader_addr = [&](const void* local) { return map_rank(smem_u32(local), 0); };
 
   if (warp == 0) {
-    // ---------------- tile hand-off + TMA producer (every CTA) ----------------
+    // ---------------- tile hand-off + TMA producer (both CTAs) ----------------
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      // While more tiles remain than there are clusters, the head publishes
+      // While more tiles remain than there are pairs, the leader publishes
       // tile lt + 1 (from the queue) before it loads tile lt, so the next
-      // index is already waiting in every CTA when its producer and MMA reach
-      // the tile switch; near the end of the queue it claims the next tile at
-      // the switch, so that no cluster holds a tile while others go idle.
+      // index is already waiting in both CTAs when their producers and the MMA
+      // reach the tile switch; near the end of the queue it claims the next
+      // tile at the switch, so that no pair holds a tile while others go idle.
       auto publish = [&](uint32_t l, int t) -> bool {
         const uint32_t slot = l % P_TILE_SLOTS, sph = (l / P_TILE_SLOTS) & 1u;
         if (!mbar_wait_cluster_bounded(smem_u32(&bar_tile_empty[slot]), sph ^ 1u, &s_abort)) return false;
         s_tile[slot] = t;
-        for (uint32_t r = 1; r < CL; ++r) st_remote_u32(map_rank(smem_u32(&s_tile[slot]), r), (uint32_t)t);
+        st_remote_u32(map_rank(smem_u32(&s_tile[slot]), 1), (uint32_t)t);
         mbar_arrive(smem_u32(&bar_tile_full[slot]));
-        for (uint32_t r = 1; r < CL; ++r)
-          mbar_arrive_remote(map_rank(smem_u32(&bar_tile_full[slot]), r));  // release orders the store
+        mbar_arrive_remote(map_rank(smem_u32(&bar_tile_full[slot]), 1));  // release orders the store
         return true;
       };
       auto dequeue = [&]() {
         const int t = (int)atomicAdd(tile_queue, 1u);
         return t < T ? t : -1;
       };
-      const int clusters = (int)(gridDim.x / CL);
-      if (head && !publish(0, dequeue())) ok = false;
+      const int pairs = (int)(gridDim.x / 2);
+      if (leader && !publish(0, dequeue())) ok = false;
       for (uint32_t lt = 0; ok; ++lt) {
         const uint32_t slot = lt % P_TILE_SLOTS, sph = (lt / P_TILE_SLOTS) & 1u;
         int t;
-        bool ahead = false;  // the head published tile lt + 1 already
-        if (head) {
+        bool ahead = false;  // the leader published tile lt + 1 already
+        if (leader) {
           t = s_tile[slot];  // published before
-          ahead = t >= 0 && t + clusters < T;
+          ahead = t >= 0 && t + pairs < T;
           if (ahead && !publish(lt + 1, dequeue())) {
             ok = false;
             break;
@@ -785,7 +766,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
             break;
           }
           t = s_tile[slot];
-          mbar_arrive_remote(head_addr(&bar_tile_empty[slot]));
+          mbar_arrive_remote(leader_addr(&bar_tile_empty[slot]));
         }
         if (t < 0) break;
         bool corr;
@@ -800,32 +781,23 @@ __global__ void __launch_bounds__(P_THREADS, 1)
           }
           fence_proxy_async_global();
         }
-        // this CTA's weight rows: its half of the pair's tile (leader rows
-        // 0..127, follower 128..255), of which it loads the WROWS-row slice of
-        // its pair and multicasts it to the same position in every pair
-        const int wslice = (int)pair * WROWS;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
           const uint32_t s = it % PSTAGES, ph = (it / PSTAGES) & 1u;
           if (!mbar_wait_bounded(smem_u32(&bar_empty[s]), ph ^ 1u, &s_abort)) {
             ok = false;
             break;
           }
-          const uint32_t a_dst = base + s * P_STAGE_BYTES, b_dst = a_dst + P_A_BYTES + (uint32_t)wslice * 128u;
-          const uint32_t full = pair_lead(&bar_full[s]);
-          if (leader) mbar_arrive_expect_tx(smem_u32(&bar_full[s]), 2 * P_STAGE_BYTES);  // the pair's bytes
-          const CUtensorMap* wmap = corr ? &tmWc : (leader ? &tmWv : &tmWg);
-          const int wx = (corr || leader) ? kb * BK : d + kb * BK;
-          const int wy = corr ? n0 + (int)prank * 128 + wslice : n0 + wslice;
+          const uint32_t a_dst = base + s * P_STAGE_BYTES, b_dst = a_dst + P_A_BYTES;
+          const uint32_t full = leader_addr(&bar_full[s]);
+          if (leader) mbar_arrive_expect_tx(smem_u32(&bar_full[s]), 2 * P_STAGE_BYTES);  // both CTAs' bytes
           tma_load_2d_pair(a_dst, corr ? &tmApack : &tmR, kb * BK, m0, full);  // [m; u] or r rows
-          if constexpr (CL == 2) {
-            tma_load_2d_pair(b_dst, wmap, wx, wy, full);  // W_c rows, or W_v (leader) / W_g[:, d:2d] (follower)
-          } else {
-            const uint16_t mc = (uint16_t)((1u << prank) | (1u << (prank + 2)));
-            tma_load_2d_pair_mc(b_dst, wmap, wx, wy, full, mc);
-          }
+          if (corr)  // this CTA's half of the weight tile: rows n0.. (leader) or n0 + 128.. (follower)
+            tma_load_2d_pair(b_dst, &tmWc, kb * BK, n0 + (int)rank * 128, full);
+          else  // W_v rows (leader) and the matching W_g[:, d:2d] rows (follower)
+            tma_load_2d_pair(b_dst, leader ? &tmWv : &tmWg, leader ? kb * BK : d + kb * BK, n0, full);
         }
         if (!ok) break;
-        if (head && !ahead && !publish(lt + 1, dequeue())) ok = false;  // near the end: claim at the switch
+        if (leader && !ahead && !publish(lt + 1, dequeue())) ok = false;  // near the end: claim at the switch
       }
       if (!ok) {
         raise_abort(&s_abort, p.status);
@@ -839,7 +811,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     }
     __syncwarp();
   } else if (warp == 1) {
-    // ---------------- MMA issuer (pair leader) ----------------
+    // ---------------- MMA issuer (leader) ----------------
     if (leader && lane == 0) {
       uint32_t it = 0;
       bool ok = true;
@@ -850,8 +822,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
           break;
         }
         const int t = s_tile[slot];
-        if (head) mbar_arrive(smem_u32(&bar_tile_empty[slot]));
-        else mbar_arrive_remote(head_addr(&bar_tile_empty[slot]));
+        mbar_arrive(smem_u32(&bar_tile_empty[slot]));
         if (t < 0) break;
         const int nkb = t < T0 ? 2 * kb_half : kb_half;
         const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
@@ -874,9 +845,9 @@ __global__ void __launch_bounds__(P_THREADS, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             tc_mma_pair(d_tmem, adesc0 + 2u * k, bdesc0 + 2u * k, IDESC_M256_N256, (kb > 0 || k > 0) ? 1u : 0u);
-          tc_commit_pair(smem_u32(&bar_empty[s]), ALL);  // every CTA that may refill this stage
+          tc_commit_pair(smem_u32(&bar_empty[s]));  // stage free in both CTAs
         }
-        tc_commit_pair(smem_u32(&bar_tfull[acc]), pair_mask);  // accumulator ready (also after a failure)
+        tc_commit_pair(smem_u32(&bar_tfull[acc]));  // accumulator ready (also after a failure)
         if (!ok) break;
       }
       if (!ok) raise_abort(&s_abort, p.status);
@@ -886,7 +857,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     // ---------------- W_g[:, :d] e for the broadcast e (idle warps) ----------------
     if (need_ge) gate_bias_rows(p, d, lane, gemv_next, gemv_done);
   } else {
-    // ---------------- epilogue (warps 4-7 of every CTA) ----------------
+    // ---------------- epilogue (warps 4-7 of both CTAs) ----------------
     const int q = (warp - 4) * 32 + lane;  // tile row = TMEM lane
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     bool have_ge = !need_ge;
@@ -900,8 +871,8 @@ __global__ void __launch_bounds__(P_THREADS, 1)
       const int t = s_tile[slot];
       __syncwarp();
       if (lane == 0) {
-        if (head) mbar_arrive(smem_u32(&bar_tile_empty[slot]));
-        else mbar_arrive_remote(head_addr(&bar_tile_empty[slot]));
+        if (leader) mbar_arrive(smem_u32(&bar_tile_empty[slot]));
+        else mbar_arrive_remote(leader_addr(&bar_tile_empty[slot]));
       }
       if (t < 0) break;
       bool corr;
@@ -943,7 +914,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
       __syncwarp();
       if (lane == 0) {
         if (leader) mbar_arrive(smem_u32(&bar_tempty[acc]));
-        else mbar_arrive_remote(pair_lead(&bar_tempty[acc]));
+        else mbar_arrive_remote(leader_addr(&bar_tempty[acc]));
       }
     }
     // out of tiles: help finish W_g[:, :d] e (the rows left on the counter)
@@ -952,7 +923,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
   // ---------------- teardown ----------------
   tc_fence_before();
   __syncthreads();
-  cluster_sync_all();  // every peer is done with this CTA's shared and tensor memory
+  cluster_sync_all();  // the peer is done with this CTA's shared and tensor memory
   if (warp == 2) {
     tc_fence_after();
     tmem_dealloc_pair(tmem, TMEM_COLS);
@@ -1306,12 +1277,9 @@ cudaError_t launch_pack(const PackArgs& a, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-// Both projections on CTA pairs, in clusters of `cl` CTAs (2 or 4) of which
-// `clusters` run at once.
-static cudaError_t launch_cond_pair(const TcCondArgs& a, int cl, int clusters, cudaStream_t stream) {
+static cudaError_t launch_cond_pair(const TcCondArgs& a, int clusters, cudaStream_t stream) {
   const long long rmax = (long long)a.B * (a.K - 1);
   const uint64_t d = (uint64_t)a.d;
-  const uint32_t wrows = 128u / (uint32_t)(cl / 2);  // weight rows per CTA and stage (the multicast slice)
   CUtensorMap mApack, mWc, mR, mWv, mWg;
   // Maps of operands a call does not use point at a used buffer (never read).
   const void* apack = a.do_correct ? a.apack : a.rpack;
@@ -1320,10 +1288,10 @@ static cudaError_t launch_cond_pair(const TcCondArgs& a, int cl, int clusters, c
   const void* wv = a.do_gate ? a.Wv : a.Wc;
   const void* wg = a.do_gate ? a.Wg : a.Wc;
   if (encode_tensor_map_2d(&mApack, apack, a.do_correct ? 2 * d : d, (uint64_t)rmax, (a.do_correct ? 4 : 2) * d, BK, BM) != CUDA_SUCCESS ||
-      encode_tensor_map_2d(&mWc, wc, a.do_correct ? 2 * d : d, d, (a.do_correct ? 4 : 2) * d, BK, wrows) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWc, wc, a.do_correct ? 2 * d : d, d, (a.do_correct ? 4 : 2) * d, BK, 128) != CUDA_SUCCESS ||
       encode_tensor_map_2d(&mR, rp, d, (uint64_t)rmax, 2 * (a.r_row_stride ? (uint64_t)a.r_row_stride : d), BK, BM) != CUDA_SUCCESS ||
-      encode_tensor_map_2d(&mWv, wv, a.do_gate ? d : 2 * d, d, (a.do_gate ? 2 : 4) * d, BK, wrows) != CUDA_SUCCESS ||
-      encode_tensor_map_2d(&mWg, wg, 2 * d, d, 4 * d, BK, wrows) != CUDA_SUCCESS)
+      encode_tensor_map_2d(&mWv, wv, a.do_gate ? d : 2 * d, d, (a.do_gate ? 2 : 4) * d, BK, 128) != CUDA_SUCCESS ||
+      encode_tensor_map_2d(&mWg, wg, 2 * d, d, 4 * d, BK, 128) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
   CondParams p{};
   p.d = a.d;
@@ -1344,67 +1312,44 @@ static cudaError_t launch_cond_pair(const TcCondArgs& a, int cl, int clusters, c
   p.block_done = a.sync + kSyncBlocks;
   p.block_ready = a.sync + kSyncBlocks + blocks_max(a.B, a.K);
   p.status = a.status;
-  // set-up may overlap the previous kernel's end
-  auto kern = cl == 4 ? cond_pair_kernel<4> : cond_pair_kernel<2>;
-  return launch_dependent(kern, dim3((unsigned)(cl * clusters)), dim3(P_THREADS), P_SMEM_BYTES, stream, (unsigned)cl,
+  // clusters of two CTAs; set-up may overlap the previous kernel's end
+  return launch_dependent(cond_pair_kernel, dim3(2 * (unsigned)clusters), dim3(P_THREADS), P_SMEM_BYTES, stream, 2,
                           mApack, mWc, mR, mWv, mWg, p);
 }
 
-// Clusters of `cl` CTAs of cond_pair_kernel<cl> that fit on the device at
-// once (0: none; -1 cached as "none").
-template <int CL>
-static int max_pair_clusters(int dev, cudaError_t* err) {
+// The CTA-pair kernel: broadcast e (or no gate), and a device that can keep
+// at least one pair of its CTAs resident.  Returns the pair count (0: use
+// cond_kernel).
+static int pair_clusters(const TcCondArgs& a, long long tiles_max_pairs, cudaError_t* err) {
+  *err = cudaSuccess;
+  if (a.do_gate && a.e_dense) return 0;
   static std::atomic<int> max_clusters[64];  // per device; 0: not yet known; -1: none fits
+  int dev = 0;
+  if ((*err = cudaGetDevice(&dev)) != cudaSuccess) return 0;
   if (max_clusters[dev & 63].load(std::memory_order_acquire) == 0) {
-    if ((*err = cudaFuncSetAttribute(cond_pair_kernel<CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     P_SMEM_BYTES)) != cudaSuccess)
+    if ((*err = cudaFuncSetAttribute(cond_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES)) !=
+        cudaSuccess)
       return 0;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(CL, 1, 1);
+    cfg.gridDim = dim3(2, 1, 1);
     cfg.blockDim = dim3(P_THREADS, 1, 1);
     cfg.dynamicSmemBytes = P_SMEM_BYTES;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if ((*err = cudaOccupancyMaxActiveClusters(&n, cond_pair_kernel<CL>, &cfg)) != cudaSuccess) return 0;
+    if ((*err = cudaOccupancyMaxActiveClusters(&n, cond_pair_kernel, &cfg)) != cudaSuccess) return 0;
     max_clusters[dev & 63].store(n > 0 ? n : -1, std::memory_order_release);
   }
   const int n = max_clusters[dev & 63].load(std::memory_order_acquire);
-  return n > 0 ? n : 0;
-}
-
-// The CTA-pair kernel: broadcast e (or no gate), and a device that can keep
-// at least one cluster of its CTAs resident.  Clusters of four (weight tiles
-// multicast to two pairs) when at least two pair blocks of rows are possible
-// and the device holds as many CTAs in clusters of four as in pairs, else
-// pairs.  Sets *cl and returns the cluster count (0: use cond_kernel).
-static int pair_clusters(const TcCondArgs& a, long long tiles_max_pairs, int* cl, cudaError_t* err) {
-  *err = cudaSuccess;
-  if (a.do_gate && a.e_dense) return 0;
-  int dev = 0;
-  if ((*err = cudaGetDevice(&dev)) != cudaSuccess) return 0;
-  const int n2 = max_pair_clusters<2>(dev, err);
-  if (*err != cudaSuccess || n2 <= 0) return 0;
-  const long long pair_blocks = ((long long)a.B * (a.K - 1) + 2 * BM - 1) / (2 * BM);
-  int n = n2;
-  *cl = 2;
-  if (pair_blocks >= 2) {
-    const int n4 = max_pair_clusters<4>(dev, err);
-    if (*err != cudaSuccess) return 0;
-    if (2 * n4 >= n2) {
-      n = n4;
-      *cl = 4;
-    }
-  }
-  // every cluster when the gate-bias GEMV is needed: clusters without tiles compute it
+  if (n <= 0) return 0;
+  // every pair when the gate-bias GEMV is needed: pairs without tiles compute it
   if (a.do_gate) return n;
-  const long long tiles = (tiles_max_pairs + *cl / 2 - 1) / (*cl / 2);
-  return (int)(tiles < n ? tiles : n);
+  return (int)(tiles_max_pairs < n ? tiles_max_pairs : n);
 }
 
 // The small-R path (B (K-1) <= kSwapMaxRows, broadcast e or no gate): each
@@ -1538,10 +1483,9 @@ cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream) {
   const long long tiles_max_pairs =
       (rmax + 2 * BM - 1) / (2 * BM) * ((a.do_correct ? a.d / 256 : 0) + (a.do_gate ? a.d / 128 : 0));
   cudaError_t err;
-  int cl = 2;
-  const int clusters = pair_clusters(a, tiles_max_pairs, &cl, &err);
+  const int clusters = pair_clusters(a, tiles_max_pairs, &err);
   if (err != cudaSuccess) return err;
-  if (clusters > 0) return launch_cond_pair(a, cl, clusters, stream);
+  if (clusters > 0) return launch_cond_pair(a, clusters, stream);
   err = ensure_smem_attr<false>();
   if (err != cudaSuccess) return err;
   const uint64_t d = (uint64_t)a.d;

@@ -170,13 +170,12 @@ __device__ __forceinline__ void tc_mma_pair(uint32_t d_tmem, uint64_t a_desc, ui
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
-// Arrive once on the barrier at `bar` (a CTA-relative offset) in every CTA
-// of the cluster named by `mask` (bit i = cluster rank i) when the MMAs issued
-// so far complete.
-__device__ __forceinline__ void tc_commit_pair(uint32_t bar, uint16_t mask = 0x3) {
+// Arrive once on the barrier at `bar` in both CTAs of the pair when the MMAs
+// issued so far complete.
+__device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
   asm volatile(
       "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
-      "h"(mask)
+      "h"((uint16_t)0x3)
       : "memory");
 }
 // A 2D tile load into this CTA's shared memory that completes on a barrier
@@ -186,19 +185,6 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
       "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(map), "r"(x), "r"(y), "r"(bar)
-      : "memory");
-}
-// The same load delivered to the same shared-memory offset in every CTA of
-// `mask`; each destination CTA's bytes complete on the barrier at the offset
-// of `bar` in that destination's pair leader when `bar` is this CTA's pair
-// leader's barrier (the relation of `bar` to this CTA -- itself or its pair
-// peer -- is applied to every destination).
-__device__ __forceinline__ void tma_load_2d_pair_mc(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar,
-                                                    uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-      "l"(map), "r"(x), "r"(y), "r"(bar), "h"(mask)
       : "memory");
 }
 
