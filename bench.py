@@ -463,6 +463,9 @@ def run_gpu(args) -> dict | None:
     small_r = 0 < rows <= 1024 and (2 * cfg.d // 128) * ((rows + 255) // 256) <= 256
     if cfg.dtype != "bf16" or cfg.d % 256:
         cond_launches = 3  # correction, gate bias, gate (FFMA)
+    elif small_r and rows <= 256:
+        # split-K clusters: correction, gate-bias GEMV, gate (raw: GEMV, gate)
+        cond_launches = 3 if args.variant == "corrected" else 2
     elif small_r:
         cond_launches = 4 if args.variant == "corrected" else 3  # GEMM + reduction each; raw: GEMV, GEMM, reduction
     else:
@@ -599,7 +602,10 @@ def run_gpu(args) -> dict | None:
                 es, d = cfg.elem_bytes, cfg.d
                 cbytes = 5 * d * d * es + R * (2 * d + d + d) * es + R * d * 2
                 c_roof.update({
-                    "kernel": ("small-R GEMMs: swap_gemm_kernel (tcgen05, weights as the 128-row side, split-K) for "
+                    "kernel": ("small-R GEMMs: swap_cluster_kernel (tcgen05, weights as the 128-row side, split-K "
+                               "over a cluster whose partials are summed in distributed shared memory) for each "
+                               "projection, swap_gemv_kernel beside the correction" if rows <= 256 else
+                               "small-R GEMMs: swap_gemm_kernel (tcgen05, weights as the 128-row side, split-K) for "
                                "each projection, each followed by its reduction kernel"),
                     "bound": "hbm", "achieved": round(cbytes / c_avg_s / 1e9, 1), "peak": peaks["hbm_gbs"],
                     "unit": "GB/s", "frac": round(cbytes / c_avg_s / 1e9 / peaks["hbm_gbs"], 4),

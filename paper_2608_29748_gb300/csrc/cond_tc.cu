@@ -1186,6 +1186,11 @@ __global__ void __launch_bounds__(256) swap_reduce_correction_kernel(const SwapR
 __global__ void __launch_bounds__(256) swap_gemv_kernel(const SwapReduceParams p) {
   pdl_launch_dependents();
   gate_bias_rows(p.gemv, p.d, threadIdx.x & 31, p.gemv_next, p.gemv_done);
+  // Complete only after the previous kernel: the next kernel's programmatic
+  // wait, which covers this kernel alone, then covers that one too.  One CTA
+  // waiting is enough (the grid completes with its last CTA); the others
+  // leave and free their SM for the next kernel.
+  if (blockIdx.x == 0) pdl_wait();
 }
 
 // e~ rows of the gated fusion (Eq. 8), broadcast e: v in features 0..d-1 of
@@ -1227,6 +1232,229 @@ __global__ void __launch_bounds__(256) swap_reduce_gate_kernel(const SwapReduceP
     }
     const long long orow = __ldcg(p.rowmap + g);
     *reinterpret_cast<uint4*>(p.e_out + orow * d + n) = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Small R in one N tile (at most 256 rows): split-K clusters, no reduction launch
+// ---------------------------------------------------------------------------
+// The S K-splits of one weight tile run as one cluster of S CTAs.  Each CTA
+// accumulates its k-range in TMEM as swap_gemm_kernel does, moves the fp32
+// partial into its own shared memory (the drained pipeline stages), and after
+// a cluster barrier sums its slice of the rows over the S partials through
+// distributed shared memory, in rank order (results repeat bit for bit), and
+// applies the epilogue: r = m + beta c (Eq. 7) for the correction tiles of
+// W_c, or the gated fusion e~ = e + v sigmoid(g_r + W_g[:, :d] e) (Eq. 8)
+// for the gate tiles, whose 128 weight rows stack 64 rows of W_v over the
+// same 64 rows of W_g[:, d:2d] (v and g_r of a feature in TMEM lanes f and
+// 64 + f).  Nothing goes through global partials and no reduction kernel
+// follows.  The partial is stored row-major ([row][feature]) so that both
+// the TMEM drain and the cluster's reads move whole 128- and 256-byte rows.
+struct SwapClusterParams {
+  const int32_t* R;
+  int d;
+  int nkb;     // 64-deep k-blocks of the GEMM
+  int S;       // K splits = cluster size
+  int gate;    // 0: correction tiles of W_c (128 features); 1: stacked [W_v; W_g,r] tiles (64 features)
+  int tile_n;  // rows of the B box (the largest R rounded to 16, at most 256)
+  uint32_t tmem_cols;
+  uint32_t stage_stride;
+  // correction epilogue
+  const __nv_bfloat16* apack;  // m = the first d columns of each packed row
+  float beta;
+  __nv_bfloat16* r_out;
+  int compact_out;
+  // gate epilogue (broadcast e; ge = W_g[:, :d] e, complete before this launch)
+  const __nv_bfloat16* e;
+  const float* ge;
+  __nv_bfloat16* e_out;
+  const int32_t* rowmap;
+  uint32_t* status;
+};
+
+__global__ void __launch_bounds__(SW_THREADS, 1)
+    swap_cluster_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
+                        const __grid_constant__ CUtensorMap tmB, const SwapClusterParams p) {
+  extern __shared__ uint8_t dsmem[];
+  __shared__ __align__(8) uint64_t bar_full[SW_STAGES];
+  __shared__ __align__(8) uint64_t bar_empty[SW_STAGES];
+  __shared__ __align__(8) uint64_t bar_acc;
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int S = p.S, d = p.d;
+  const uint32_t rank = cluster_rank();
+  const int mt = (int)(blockIdx.x / (unsigned)S);  // weight tile of this cluster
+  pdl_launch_dependents();
+  if (threadIdx.x == 0) {
+    s_abort = 0;
+    for (int s = 0; s < SW_STAGES; ++s) {
+      mbar_init(smem_u32(&bar_full[s]), 1);
+      mbar_init(smem_u32(&bar_empty[s]), 1);
+    }
+    mbar_init(smem_u32(&bar_acc), 1);
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmA2);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 2) {
+    tmem_alloc(smem_u32(&s_tmem), p.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+  const uint32_t base = (smem_u32(dsmem) + 1023u) & ~1023u;
+  // the partial [row][128 features], in the drained pipeline stages (the same offset in every CTA)
+  float* P = reinterpret_cast<float*>(dsmem + (base - smem_u32(dsmem)));
+  const int kb0 = (int)((long long)rank * p.nkb / S), kb1 = (int)((long long)(rank + 1) * p.nkb / S);
+  pdl_wait();  // R and the activation rows come from the previous kernels
+  const int R = *(volatile const int32_t*)p.R;
+  const int nrows = (R + 15) / 16 * 16;  // MMA N (at most tile_n)
+  const bool work = R > 0;
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0 && work) {
+      const uint32_t tx = (uint32_t)(BM * BK * 2) + (uint32_t)p.tile_n * BK * 2;
+      int kb = kb0;
+      for (; kb < kb1; ++kb) {
+        const int i = kb - kb0;
+        const uint32_t s = (uint32_t)(i % SW_STAGES), ph = (uint32_t)((i / SW_STAGES) & 1);
+        if (!mbar_wait_bounded(smem_u32(&bar_empty[s]), ph ^ 1u, &s_abort)) break;
+        const uint32_t a_dst = base + s * p.stage_stride, b_dst = a_dst + (uint32_t)(BM * BK * 2);
+        mbar_arrive_expect_tx(smem_u32(&bar_full[s]), tx);
+        if (p.gate) {  // rows 0-63: W_v rows f0..; rows 64-127: the same rows of W_g[:, d:2d]
+          tma_load_2d(a_dst, &tmA, kb * BK, mt * 64, smem_u32(&bar_full[s]));
+          tma_load_2d(a_dst + (uint32_t)(64 * BK * 2), &tmA2, d + kb * BK, mt * 64, smem_u32(&bar_full[s]));
+        } else {
+          tma_load_2d(a_dst, &tmA, kb * BK, mt * 128, smem_u32(&bar_full[s]));
+        }
+        tma_load_2d(b_dst, &tmB, kb * BK, 0, smem_u32(&bar_full[s]));
+      }
+      if (kb < kb1) {  // a wait expired: flag it, let the copies in flight land
+        raise_abort(&s_abort, p.status);
+        volatile int never = 0;
+        const int first = kb - kb0 > SW_STAGES ? kb - kb0 - SW_STAGES : 0;
+        for (int i = first; i < kb - kb0; ++i)
+          mbar_wait_bounded(smem_u32(&bar_full[i % SW_STAGES]), (uint32_t)((i / SW_STAGES) & 1), &never);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      if (work) {
+        const uint32_t idesc = idesc_bf16_f32(128, nrows);
+        bool ok = true;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          const int i = kb - kb0;
+          const uint32_t s = (uint32_t)(i % SW_STAGES), ph = (uint32_t)((i / SW_STAGES) & 1);
+          if (!mbar_wait_bounded(smem_u32(&bar_full[s]), ph, &s_abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_base = base + s * p.stage_stride, b_base = a_base + (uint32_t)(BM * BK * 2);
+          const uint64_t adesc0 = sw128_kmajor_desc(a_base), bdesc0 = sw128_kmajor_desc(b_base);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            tc_mma_bf16(tmem, adesc0 + 2u * k, bdesc0 + 2u * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+          tc_commit(smem_u32(&bar_empty[s]));
+        }
+        if (!ok) raise_abort(&s_abort, p.status);
+      }
+      tc_commit(smem_u32(&bar_acc));  // accumulator ready (also without work or after a failure)
+    }
+    __syncwarp();
+  } else if (warp >= 4) {
+    // ---------------- epilogue warps: the partial into shared memory ----------------
+    const int q = (warp - 4) * 32 + lane;  // weight row of the tile = TMEM lane = feature
+    const bool ok = warp_wait(smem_u32(&bar_acc), 0u, &s_abort);
+    tc_fence_after();
+    if (!ok && lane == 0) raise_abort(&s_abort, p.status);
+    if (ok && work && !s_abort) {
+      const uint32_t taddr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+      for (int c0 = 0; c0 < nrows; c0 += 32) {
+        float v[32];
+        tmem_ld_32cols(taddr + (uint32_t)c0, v);
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (c0 + j < nrows) P[(c0 + j) * 128 + q] = v[j];  // a warp stores 128 contiguous bytes
+      }
+    }
+  }
+  // ---------------- the cluster's sum and the epilogue ----------------
+  tc_fence_before();
+  __syncthreads();
+  const bool go = work && !s_abort;  // every role is done: the same in every thread of the CTA
+  cluster_sync_all();  // every partial of the cluster is in shared memory
+  if (go) {
+    const float* Pr[8];
+#pragma unroll
+    for (int s = 0; s < 8; ++s) Pr[s] = map_rank_ptr(P, (uint32_t)(s < S ? s : 0));
+    const int g0 = (int)((long long)rank * R / S), g1 = (int)((long long)(rank + 1) * R / S);
+    if (!p.gate) {
+      // r[g, n0 + f] = m + beta * c for this CTA's rows; two features per thread, a warp 256 bytes of a row
+      const int n0 = mt * 128;
+      for (int u = threadIdx.x; u < (g1 - g0) * 64; u += SW_THREADS) {
+        const int g = g0 + u / 64, f = (u % 64) * 2;
+        float2 x[8];
+#pragma unroll
+        for (int s = 0; s < 8; ++s)  // all loads first, then the sums in rank order
+          x[s] = s < S ? *reinterpret_cast<const float2*>(Pr[s] + g * 128 + f) : make_float2(0.f, 0.f);
+        const uint32_t mw = __ldcg(reinterpret_cast<const uint32_t*>(p.apack + (long long)g * 2 * d + n0 + f));
+        const long long orow = p.compact_out ? g : __ldcg(p.rowmap + g);
+        float c0 = 0.f, c1 = 0.f;
+#pragma unroll
+        for (int s = 0; s < 8; ++s) {
+          if (s < S) {
+            c0 += x[s].x;
+            c1 += x[s].y;
+          }
+        }
+        *reinterpret_cast<uint32_t*>(p.r_out + orow * d + n0 + f) =
+            pack_bf16x2(bf16_lo(mw) + p.beta * c0, bf16_hi(mw) + p.beta * c1);
+      }
+    } else {
+      // e~[g, f0 + f] = e + v sigmoid(g_r + ge) for this CTA's rows; two features per thread
+      const int f0 = mt * 64;
+      for (int u = threadIdx.x; u < (g1 - g0) * 32; u += SW_THREADS) {
+        const int g = g0 + u / 32, f = (u % 32) * 2;
+        float2 xv[8], xa[8];
+#pragma unroll
+        for (int s = 0; s < 8; ++s) {  // all loads first, then the sums in rank order
+          xv[s] = s < S ? *reinterpret_cast<const float2*>(Pr[s] + g * 128 + f) : make_float2(0.f, 0.f);
+          xa[s] = s < S ? *reinterpret_cast<const float2*>(Pr[s] + g * 128 + 64 + f) : make_float2(0.f, 0.f);
+        }
+        const float2 gb = __ldcg(reinterpret_cast<const float2*>(p.ge + f0 + f));
+        const uint32_t ew = __ldg(reinterpret_cast<const uint32_t*>(p.e + f0 + f));
+        const long long orow = __ldcg(p.rowmap + g);
+        float v0 = 0.f, v1 = 0.f, a0 = 0.f, a1 = 0.f;
+#pragma unroll
+        for (int s = 0; s < 8; ++s) {
+          if (s < S) {
+            v0 += xv[s].x;
+            v1 += xv[s].y;
+            a0 += xa[s].x;
+            a1 += xa[s].y;
+          }
+        }
+        a0 += gb.x;
+        a1 += gb.y;
+        *reinterpret_cast<uint32_t*>(p.e_out + orow * d + f0 + f) =
+            pack_bf16x2(bf16_lo(ew) + v0 * fast_sigmoid(a0), bf16_hi(ew) + v1 * fast_sigmoid(a1));
+      }
+    }
+  }
+  cluster_sync_all();  // no CTA leaves while the others read its shared memory
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, p.tmem_cols);
   }
 }
 
@@ -1476,10 +1704,153 @@ static cudaError_t launch_cond_swap(const TcCondArgs& a, cudaStream_t stream) {
   return cudaSuccess;
 }
 
+// Clusters of S CTAs of swap_cluster_kernel that the device holds at once
+// with `smem` bytes each (0: none), cached per device, S and shared memory.
+static int swap_cluster_capacity(int dev, int S, int smem, cudaError_t* err) {
+  static std::atomic<int> cache[64][9][17];  // [device][S][smem in 16 KB steps]; 0: not yet known, -1: none
+  std::atomic<int>& slot = cache[dev & 63][S][smem >> 14];
+  int n = slot.load(std::memory_order_acquire);
+  if (n == 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)S, 1, 1);
+    cfg.blockDim = dim3(SW_THREADS, 1, 1);
+    cfg.dynamicSmemBytes = (size_t)smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)S;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int m = 0;
+    if ((*err = cudaOccupancyMaxActiveClusters(&m, swap_cluster_kernel, &cfg)) != cudaSuccess) return 0;
+    n = m > 0 ? m : -1;
+    slot.store(n, std::memory_order_release);
+  }
+  return n > 0 ? n : 0;
+}
+
+// The small-R GEMMs as split-K clusters with the reduction inside
+// (swap_cluster_kernel): one N tile (at most 256 possible rows) and, for
+// each GEMM, a cluster size S <= 8 whose clusters all fit in one wave with
+// one CTA per SM.  Returns cudaErrorNotSupported (nothing launched) where
+// that does not hold.
+static cudaError_t launch_cond_swap_cluster(const TcCondArgs& a, cudaStream_t stream) {
+  const long long rmax = (long long)a.B * (a.K - 1);
+  const int d = a.d;
+  const int rows_max = (int)((rmax + 15) / 16 * 16);
+  if (rows_max > 256 || d % 128 != 0) return cudaErrorNotSupported;
+  const int tile_n = rows_max;
+  DeviceInfo info;
+  cudaError_t err = device_info(&info);
+  if (err != cudaSuccess) return err;
+  const int dev = info.device;
+  const uint32_t stage_stride = (uint32_t)((BM * BK * 2 + tile_n * BK * 2 + 1023) / 1024 * 1024);
+  // at least half of an SM's shared memory: one CTA per SM, so the K splits
+  // of one wave stream over distinct SMs
+  int smem = SW_STAGES * (int)stage_stride + 1024;
+  if (smem < 117 * 1024) smem = 117 * 1024;
+  static std::atomic<int> attr_done[64];
+  if (!attr_done[dev & 63].load(std::memory_order_acquire)) {
+    err = cudaFuncSetAttribute(swap_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               SW_STAGES * (BM * BK * 2 + 256 * BK * 2) + 1024);
+    if (err != cudaSuccess) return err;
+    attr_done[dev & 63].store(1, std::memory_order_release);
+  }
+  // the largest S <= 8 with every cluster of the GEMM resident at once and
+  // at least SW_STAGES k-blocks per split
+  auto pick = [&](int work, int nkb, int* S_out, int* clusters) -> cudaError_t {
+    *S_out = 0;
+    for (int S = 8; S >= 1; --S) {
+      if (nkb / S < SW_STAGES) continue;
+      const int cap = swap_cluster_capacity(dev, S, smem, &err);
+      if (err != cudaSuccess) return err;
+      if (work <= cap) {
+        *S_out = S;
+        *clusters = cap;
+        return cudaSuccess;
+      }
+    }
+    return cudaSuccess;
+  };
+  int Sc = 1, cc = 0, Sg = 1, cg = 0;
+  if (a.do_correct && (err = pick(d / 128, 2 * d / BK, &Sc, &cc)) != cudaSuccess) return err;
+  if (a.do_gate && (err = pick(d / 64, d / BK, &Sg, &cg)) != cudaSuccess) return err;
+  (void)cc;
+  (void)cg;
+  if ((a.do_correct && Sc == 0) || (a.do_gate && Sg == 0)) return cudaErrorNotSupported;
+  uint32_t tmem_cols = 32;
+  while ((int)tmem_cols < tile_n) tmem_cols <<= 1;
+  const uint64_t du = (uint64_t)d;
+  SwapClusterParams sp{};
+  sp.R = a.R;
+  sp.d = d;
+  sp.tile_n = tile_n;
+  sp.tmem_cols = tmem_cols;
+  sp.stage_stride = stage_stride;
+  sp.rowmap = a.rowmap;
+  sp.status = a.status;
+  // W_g[:, :d] e in its own many-warp kernel, launched after the correction
+  // GEMM so that it runs beside it (alone, before the GEMM, it was slower:
+  // its stream is latency-bound); it ends with a programmatic wait, so the
+  // gate launch after it also waits for the correction.
+  auto launch_gemv = [&]() {
+    SwapReduceParams gp{};
+    gp.d = d;
+    gp.gemv.d = d;
+    gp.gemv.e = reinterpret_cast<const __nv_bfloat16*>(a.e);
+    gp.gemv.Wg = reinterpret_cast<const __nv_bfloat16*>(a.Wg);
+    gp.gemv.ge = a.ge;
+    gp.gemv_next = a.sync + kSyncGemvNext;
+    gp.gemv_done = a.sync + kSyncGemvDone;
+    return launch_dependent(swap_gemv_kernel, dim3((unsigned)(info.sm_count * 4)), dim3(256), 0, stream, 1u, gp);
+  };
+  if (a.do_correct) {
+    CUtensorMap mA, mB;
+    if (encode_tensor_map_2d(&mA, a.Wc, 2 * du, du, 4 * du, BK, 128) != CUDA_SUCCESS ||
+        encode_tensor_map_2d(&mB, a.apack, 2 * du, (uint64_t)rmax, 4 * du, BK, (uint32_t)tile_n) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+    SwapClusterParams c = sp;
+    c.nkb = 2 * d / BK;
+    c.S = Sc;
+    c.gate = 0;
+    c.apack = reinterpret_cast<const __nv_bfloat16*>(a.apack);
+    c.beta = a.beta;
+    c.r_out = reinterpret_cast<__nv_bfloat16*>(a.r_out);
+    c.compact_out = a.compact_out;
+    err = launch_dependent(swap_cluster_kernel, dim3((unsigned)(d / 128 * Sc)), dim3(SW_THREADS), (size_t)smem,
+                           stream, (unsigned)Sc, mA, mA, mB, c);
+    if (err != cudaSuccess) return err;
+  }
+  if (a.do_gate) {
+    const uint64_t rstride = 2 * (a.r_row_stride ? (uint64_t)a.r_row_stride : du);
+    CUtensorMap mA, mA2, mB;
+    if (encode_tensor_map_2d(&mA, a.Wv, du, du, 2 * du, BK, 64) != CUDA_SUCCESS ||
+        encode_tensor_map_2d(&mA2, a.Wg, 2 * du, du, 4 * du, BK, 64) != CUDA_SUCCESS ||
+        encode_tensor_map_2d(&mB, a.rpack, du, (uint64_t)rmax, rstride, BK, (uint32_t)tile_n) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+    if ((err = launch_gemv()) != cudaSuccess) return err;
+    SwapClusterParams g = sp;
+    g.nkb = d / BK;
+    g.S = Sg;
+    g.gate = 1;
+    g.e = reinterpret_cast<const __nv_bfloat16*>(a.e);
+    g.ge = a.ge;
+    g.e_out = reinterpret_cast<__nv_bfloat16*>(a.e_out);
+    err = launch_dependent(swap_cluster_kernel, dim3((unsigned)(d / 64 * Sg)), dim3(SW_THREADS), (size_t)smem,
+                           stream, (unsigned)Sg, mA, mA2, mB, g);
+    if (err != cudaSuccess) return err;
+  }
+  return cudaSuccess;
+}
+
 cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream) {
   const long long rmax = (long long)a.B * (a.K - 1);
   if (rmax <= 0 || (!a.do_correct && !a.do_gate)) return cudaSuccess;
-  if (a.part && !(a.do_gate && a.e_dense)) return launch_cond_swap(a, stream);
+  if (a.part && !(a.do_gate && a.e_dense)) {
+    const cudaError_t e1 = launch_cond_swap_cluster(a, stream);
+    return e1 == cudaErrorNotSupported ? launch_cond_swap(a, stream) : e1;
+  }
   const long long tiles_max_pairs =
       (rmax + 2 * BM - 1) / (2 * BM) * ((a.do_correct ? a.d / 256 : 0) + (a.do_gate ? a.d / 128 : 0));
   cudaError_t err;

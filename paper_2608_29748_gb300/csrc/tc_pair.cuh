@@ -53,16 +53,31 @@ __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
+// Non-blocking: has the phase with this parity completed?
+__device__ __forceinline__ bool mbar_test_parity(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // One warp: rows i of ge = W_g[:, :d] e (broadcast e), claimed from a global
 // counter until all d rows are taken; each finished row is counted.  Eight
-// 16-byte loads per lane are in flight (d a multiple of 8).
+// 16-byte loads per lane are in flight (d a multiple of 8).  With a stop
+// barrier (a shared::cta address, not 0) the warp takes no further row once
+// that barrier's phase 0 has completed.
 __device__ void gate_bias_rows(const __nv_bfloat16* e, const __nv_bfloat16* Wg, float* ge, int d, int lane,
-                               uint32_t* next, uint32_t* done) {
+                               uint32_t* next, uint32_t* done, uint32_t stop_bar = 0u) {
   const int vpr = d / 8;
   const uint4* ev = reinterpret_cast<const uint4*>(e);
   for (;;) {
     int i = 0;
-    if (lane == 0) i = (int)atomicAdd(next, 1u);
+    if (lane == 0) i = (stop_bar != 0u && mbar_test_parity(stop_bar, 0u)) ? d : (int)atomicAdd(next, 1u);
     i = __shfl_sync(0xFFFFFFFFu, i, 0);
     if (i >= d) break;
     const uint4* wr = reinterpret_cast<const uint4*>(Wg + (long long)i * 2 * d);
@@ -147,6 +162,14 @@ __device__ __forceinline__ bool warp_wait_cluster(uint32_t bar, uint32_t parity,
   ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
   __syncwarp();
   return ok != 0;
+}
+// The generic address of `p` (this CTA's shared memory) in cluster CTA `rank`:
+// plain loads through it read that CTA's shared memory.
+template <typename T>
+__device__ __forceinline__ const T* map_rank_ptr(const T* p, uint32_t rank) {
+  uint64_t r;
+  asm volatile("mapa.u64 %0, %1, %2;" : "=l"(r) : "l"(reinterpret_cast<uint64_t>(p)), "r"(rank));
+  return reinterpret_cast<const T*>(r);
 }
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
