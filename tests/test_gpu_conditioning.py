@@ -229,3 +229,52 @@ def test_small_r_path(rt, B, K, d):
     e_full = np.broadcast_to(host_f64(x["e_vec"]), (B, K, d))
     want = oracle.gate_fuse(e_full, host_f64(r), n_host, host_f64(x["Wv"]), host_f64(x["Wg"]))
     assert_close(out, want, f"e~, B={B} K={K}")
+
+
+@pytest.mark.parametrize("B,K,d,R", [(1, 2, 256, 1), (1, 17, 512, 15), (2, 9, 256, 16), (17, 2, 1024, 17),
+                                     (8, 16, 4096, 100), (16, 16, 256, 240), (17, 16, 2560, 255),
+                                     (16, 17, 256, 256),
+                                     # more than 256 possible rows: N tiles of 256, split-K partials
+                                     (18, 16, 256, 16), (18, 16, 512, 257), (40, 16, 256, 511),
+                                     (40, 16, 1024, 512), (35, 16, 4096, 513), (64, 16, 2560, 960),
+                                     (64, 17, 256, 1000), (64, 17, 512, 1024)])
+def test_small_r_rows(rt, B, K, d, R):
+    """Exactly R carried rows on the small-R path (B (K-1) <= 1024).  At most
+    256 possible rows the GEMMs run as split-K clusters that sum their
+    partials through distributed shared memory; above that as split-K tiles
+    whose fp32 partials a reduction kernel sums.  R below, at and above
+    multiples of 16 and of 256 (one to four N tiles), cluster sizes that
+    differ between d = 256 and d = 4096: r and e~ against the oracle through
+    both standalone entry points, and repeated bit for bit."""
+    dtype = torch.bfloat16
+    assert B * (K - 1) <= 1024 and R <= B * (K - 1)
+    # carry exactly R rows: sequences reject at once (n_b = K - 1) until R is reached
+    n_want = np.zeros(B, dtype=np.int64)
+    left = R
+    for b in range(B):
+        n_want[b] = min(K - 1, left)
+        left -= n_want[b]
+    accept = torch.tensor([K - 1 - n if n > 0 else K for n in n_want], dtype=torch.int32).cuda()
+    x = make_inputs(B, K, d, dtype, seed=1000 + R + d, accept=accept)
+    A = host_int(x["accept"])
+    n_host = oracle.carried_rows(A, K)
+    assert int(n_host.sum()) == R
+    ws = rt.Workspace(B, K, 8, d, dtype)
+    outs = []
+    for _ in range(2):
+        r = torch.full((B, K, d), 9.0, dtype=dtype, device="cuda")
+        n = torch.empty((B,), dtype=torch.int32, device="cuda")
+        rt.retrace_align_refine(x["hD"], x["hT"], x["accept"], x["Wc"], 0.5, r, n, ws)
+        out = torch.full((B, K, d), 7.0, dtype=dtype, device="cuda")
+        rt.retrace_gate_fuse(x["e_vec"], r, n, x["Wv"], x["Wg"], out, ws)
+        torch.cuda.synchronize()
+        outs.append((r, out))
+    assert ws.check() == 0
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+    r, out = outs[0]
+    m, u = oracle.align(host_f64(x["hD"]), host_f64(x["hT"]), A)
+    r_ref = oracle.correct(m, u, host_f64(x["Wc"]), 0.5, round_r_bf16=False)
+    assert_close(r, r_ref, f"r, R={R} d={d}")
+    e_full = np.broadcast_to(host_f64(x["e_vec"]), (B, K, d))
+    want = oracle.gate_fuse(e_full, host_f64(r), n_host, host_f64(x["Wv"]), host_f64(x["Wg"]))
+    assert_close(out, want, f"e~, R={R} d={d}")
