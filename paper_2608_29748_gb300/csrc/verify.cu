@@ -510,6 +510,68 @@ __global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams 
   }
 }
 
+// One row segment of the copies after verification, by one warp of 32
+// lanes: `kind` 0 is the e~ row of position j (e, or m_j in the overwrite
+// variant), 1 and 2 the m_j and u_j halves of its packed row, 3 its packed e
+// row.  A is sequence b's accepted length, pack0 its first packed row.
+// Nothing is copied where the item does not apply (a conditioned e~ row,
+// which the conditioning kernels write; the packed halves of an
+// unconditioned position).  CV: 16-byte vectors, kCopyBatch in flight per
+// lane; elements otherwise.
+constexpr int kCopyBatch = 8;
+template <typename T, bool CV>
+__device__ __forceinline__ void copy_segment(const VerifyParams& p, int b, int j, int kind, int A, long long pack0) {
+  const int K = p.K, d = p.d;
+  const int nb = (K - 1 - A) > 0 ? (K - 1 - A) : 0;
+  const int lane = threadIdx.x & 31;
+  const long long pos = (long long)b * K + j;
+  const T* e = reinterpret_cast<const T*>(p.e);
+  const T* hD = reinterpret_cast<const T*>(p.hD);
+  const T* hT = reinterpret_cast<const T*>(p.hT);
+  const T* src;
+  T* dst;
+  if (kind == 0) {
+    if (p.cond_copy == kCondCopyKeep && j < nb) return;  // the conditioning kernels write it
+    src = (p.cond_copy == kCondCopyM && j < nb) ? hD + (pos + A + 1) * d
+                                                : e + (long long)b * p.e_batch_stride + (long long)j * p.e_pos_stride;
+    dst = reinterpret_cast<T*>(p.e_out) + pos * d;
+  } else {
+    if (j >= nb) return;
+    const long long row = pack0 + j;
+    if (kind == 1) {
+      src = hD + (pos + A + 1) * d;
+      dst = reinterpret_cast<T*>(p.apack) + row * 2 * d;
+      if (lane == 0) p.rowmap[row] = (int32_t)pos;
+    } else if (kind == 2) {
+      src = hT + (pos + A) * d;
+      dst = reinterpret_cast<T*>(p.apack) + row * 2 * d + d;
+    } else {
+      src = e + pos * d;
+      dst = reinterpret_cast<T*>(p.epack) + row * d;
+    }
+  }
+  if constexpr (CV) {
+    const int vpr = d * (int)sizeof(T) / 16;
+    const uint4* s4 = reinterpret_cast<const uint4*>(src);
+    uint4* d4 = reinterpret_cast<uint4*>(dst);
+    for (int v0 = 0; v0 < vpr; v0 += 32 * kCopyBatch) {
+      uint4 x[kCopyBatch];
+#pragma unroll
+      for (int k = 0; k < kCopyBatch; ++k) {
+        const int v = v0 + k * 32 + lane;
+        if (v < vpr) x[k] = __ldcs(s4 + v);
+      }
+#pragma unroll
+      for (int k = 0; k < kCopyBatch; ++k) {
+        const int v = v0 + k * 32 + lane;
+        if (v < vpr) d4[v] = x[k];
+      }
+    }
+  } else {
+    for (int v = lane; v < d; v += 32) dst[v] = src[v];
+  }
+}
+
 // The copies of a windowed verification, after its last pass (accept_len
 // and the packed-row offsets hold every sequence's values by then).  Work
 // items are row segments: (sequence b, position j, segment), the segments in
@@ -519,74 +581,22 @@ __global__ void __launch_bounds__(kThreads, 2) verify_kernel(const VerifyParams 
 // row.  Each warp takes items in turn and copies one with its 32 lanes, each
 // lane kCopyBatch 16-byte vectors in flight at a time (elements when CV is
 // false); inactive items cost one decode.
-constexpr int kCopyBatch = 8;
 template <typename T, bool CV>
 __global__ void __launch_bounds__(kThreads, 2) verify_copy_kernel(const VerifyParams p) {
   pdl_launch_dependents();
   pdl_wait();
-  const int K = p.K, d = p.d;
-  constexpr int E = CV ? 16 / (int)sizeof(T) : 1;  // elements per copy slot
-  const int vpr = d / E;
+  const int K = p.K;
   const bool pack = p.R_count != nullptr;
   const int nseg = (p.e_out ? 1 : 0) + (pack ? (p.e_dense ? 3 : 2) : 0);
   const long long items = (long long)p.B * K * nseg;
-  const int lane = threadIdx.x & 31;
   const long long warps = (long long)gridDim.x * (kThreads / 32);
-  const T* e = reinterpret_cast<const T*>(p.e);
-  const T* hD = reinterpret_cast<const T*>(p.hD);
-  const T* hT = reinterpret_cast<const T*>(p.hT);
-  T* e_out = reinterpret_cast<T*>(p.e_out);
-  T* apack = reinterpret_cast<T*>(p.apack);
-  T* epack = reinterpret_cast<T*>(p.epack);
   for (long long it = (long long)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5); it < items; it += warps) {
     const long long u = it / nseg;
     const int seg = (int)(it - u * nseg);
     const int b = (int)(u / K), j = (int)(u - (long long)b * K);
+    const int kind = p.e_out ? seg : seg + 1;
     const int A = __ldg(p.accept_len + b);
-    const int nb = (K - 1 - A) > 0 ? (K - 1 - A) : 0;
-    const long long pos = (long long)b * K + j;
-    const int kind = p.e_out ? seg : seg + 1;  // 0 e_out row, 1 m half, 2 u half, 3 packed e
-    const T* src;
-    T* dst;
-    if (kind == 0) {
-      if (p.cond_copy == kCondCopyKeep && j < nb) continue;  // the conditioning kernels write it
-      src = (p.cond_copy == kCondCopyM && j < nb) ? hD + (pos + A + 1) * d
-                                                  : e + (long long)b * p.e_batch_stride + (long long)j * p.e_pos_stride;
-      dst = e_out + pos * d;
-    } else {
-      if (j >= nb) continue;
-      const long long row = (long long)__ldg(p.pack_off + b) + j;
-      if (kind == 1) {
-        src = hD + (pos + A + 1) * d;
-        dst = apack + row * 2 * d;
-        if (lane == 0) p.rowmap[row] = (int32_t)pos;
-      } else if (kind == 2) {
-        src = hT + (pos + A) * d;
-        dst = apack + row * 2 * d + d;
-      } else {
-        src = e + pos * d;
-        dst = epack + row * d;
-      }
-    }
-    if constexpr (CV) {
-      const uint4* s4 = reinterpret_cast<const uint4*>(src);
-      uint4* d4 = reinterpret_cast<uint4*>(dst);
-      for (int v0 = 0; v0 < vpr; v0 += 32 * kCopyBatch) {
-        uint4 x[kCopyBatch];
-#pragma unroll
-        for (int k = 0; k < kCopyBatch; ++k) {
-          const int v = v0 + k * 32 + lane;
-          if (v < vpr) x[k] = __ldcs(s4 + v);
-        }
-#pragma unroll
-        for (int k = 0; k < kCopyBatch; ++k) {
-          const int v = v0 + k * 32 + lane;
-          if (v < vpr) d4[v] = x[k];
-        }
-      }
-    } else {
-      for (int v = lane; v < d; v += 32) dst[v] = src[v];
-    }
+    copy_segment<T, CV>(p, b, j, kind, A, kind > 0 ? (long long)__ldg(p.pack_off + b) : 0ll);
   }
 }
 
@@ -606,7 +616,7 @@ __global__ void __launch_bounds__(kThreads, 2) verify_finish_kernel(const Verify
   __shared__ int s_last;
   pdl_launch_dependents();
   pdl_wait();
-  const int B = p.B, K = p.K, K1 = K + 1, d = p.d;
+  const int B = p.B, K = p.K, K1 = K + 1;
   const int n_last = (int)__ldcg(p.count_in);
   const int base = (int)__ldcg(p.base_in);
   int* s_first = s_dyn;         // [n_last]
@@ -638,69 +648,19 @@ __global__ void __launch_bounds__(kThreads, 2) verify_finish_kernel(const Verify
     }
   }
   // the row copies
-  constexpr int E = CV ? 16 / (int)sizeof(T) : 1;  // elements per copy slot
-  const int vpr = d / E;
   const bool pack = p.R_count != nullptr;
   const int nseg = (p.e_out ? 1 : 0) + (pack ? (p.e_dense ? 3 : 2) : 0);
   const long long items = (long long)B * K * nseg;
-  const int lane = threadIdx.x & 31;
   const long long warps = (long long)gridDim.x * (kThreads / 32);
-  const T* e = reinterpret_cast<const T*>(p.e);
-  const T* hD = reinterpret_cast<const T*>(p.hD);
-  const T* hT = reinterpret_cast<const T*>(p.hT);
-  T* e_out = reinterpret_cast<T*>(p.e_out);
-  T* apack = reinterpret_cast<T*>(p.apack);
-  T* epack = reinterpret_cast<T*>(p.epack);
   for (long long it = (long long)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5); it < items; it += warps) {
     const long long u = it / nseg;
     const int seg = (int)(it - u * nseg);
     const int b = (int)(u / K), j = (int)(u - (long long)b * K);
+    const int kind = p.e_out ? seg : seg + 1;  // 0 e_out row, 1 m half, 2 u half, 3 packed e
     const int Ah = s_mapA[b];
     const int A = Ah >= 0 ? Ah : __ldcg(p.accept_len + b);
-    const int nb = (K - 1 - A) > 0 ? (K - 1 - A) : 0;
-    const long long pos = (long long)b * K + j;
-    const int kind = p.e_out ? seg : seg + 1;  // 0 e_out row, 1 m half, 2 u half, 3 packed e
-    const T* src;
-    T* dst;
-    if (kind == 0) {
-      if (p.cond_copy == kCondCopyKeep && j < nb) continue;  // the conditioning kernels write it
-      src = (p.cond_copy == kCondCopyM && j < nb) ? hD + (pos + A + 1) * d
-                                                  : e + (long long)b * p.e_batch_stride + (long long)j * p.e_pos_stride;
-      dst = e_out + pos * d;
-    } else {
-      if (j >= nb) continue;
-      const long long row = (long long)(Ah >= 0 ? s_mapO[b] : __ldcg(p.pack_off + b)) + j;
-      if (kind == 1) {
-        src = hD + (pos + A + 1) * d;
-        dst = apack + row * 2 * d;
-        if (lane == 0) p.rowmap[row] = (int32_t)pos;
-      } else if (kind == 2) {
-        src = hT + (pos + A) * d;
-        dst = apack + row * 2 * d + d;
-      } else {
-        src = e + pos * d;
-        dst = epack + row * d;
-      }
-    }
-    if constexpr (CV) {
-      const uint4* s4 = reinterpret_cast<const uint4*>(src);
-      uint4* d4 = reinterpret_cast<uint4*>(dst);
-      for (int v0 = 0; v0 < vpr; v0 += 32 * kCopyBatch) {
-        uint4 x[kCopyBatch];
-#pragma unroll
-        for (int k = 0; k < kCopyBatch; ++k) {
-          const int v = v0 + k * 32 + lane;
-          if (v < vpr) x[k] = __ldcs(s4 + v);
-        }
-#pragma unroll
-        for (int k = 0; k < kCopyBatch; ++k) {
-          const int v = v0 + k * 32 + lane;
-          if (v < vpr) d4[v] = x[k];
-        }
-      }
-    } else {
-      for (int v = lane; v < d; v += 32) dst[v] = src[v];
-    }
+    const long long off = kind == 0 ? 0ll : (long long)(Ah >= 0 ? s_mapO[b] : __ldcg(p.pack_off + b));
+    copy_segment<T, CV>(p, b, j, kind, A, off);
   }
 }
 
@@ -750,16 +710,20 @@ int verify_windows(int B, int K, int V, int elem_bytes, bool have_workspace, boo
 
 namespace {
 
+// Copies in 16-byte vectors for every tensor a verification copies.
+inline bool copies_vectorised(const VerifyArgs& a, size_t es) {
+  auto al = [](const void* q) { return (uintptr_t)q % 16 == 0; };
+  return (a.d * es) % 16 == 0 && (!a.e_out || (al(a.e) && al(a.e_out))) &&
+         (a.e_pos_stride * (long long)es) % 16 == 0 && (a.e_batch_stride * (long long)es) % 16 == 0 &&
+         (a.cond_copy != kCondCopyM || al(a.hD)) &&
+         (!a.R_count || (al(a.hD) && al(a.hT) && al(a.apack) && (!a.e_dense || al(a.epack))));
+}
+
 // verify_copy_kernel after the last pass (programmatically dependent): the
 // 16-byte path when every copied tensor allows it.
 template <typename T>
 cudaError_t launch_copies(const VerifyArgs& a, const VerifyParams& p, long long grid, cudaStream_t stream) {
-  const size_t es = sizeof(T);
-  auto al = [](const void* q) { return (uintptr_t)q % 16 == 0; };
-  const bool cv = (a.d * es) % 16 == 0 && (!a.e_out || (al(a.e) && al(a.e_out))) &&
-                  (a.e_pos_stride * (long long)es) % 16 == 0 && (a.e_batch_stride * (long long)es) % 16 == 0 &&
-                  (a.cond_copy != kCondCopyM || al(a.hD)) &&
-                  (!a.R_count || (al(a.hD) && al(a.hT) && al(a.apack) && (!a.e_dense || al(a.epack))));
+  const bool cv = copies_vectorised(a, sizeof(T));
   auto kern = cv ? verify_copy_kernel<T, true> : verify_copy_kernel<T, false>;
   return launch_dependent(kern, dim3((unsigned)grid), dim3(kThreads), 0, stream, 1u, p);
 }
@@ -768,12 +732,7 @@ cudaError_t launch_copies(const VerifyArgs& a, const VerifyParams& p, long long 
 // dependent), with the 16-byte copy path when every copied tensor allows it.
 template <typename T>
 cudaError_t launch_finish(const VerifyArgs& a, const VerifyParams& p, long long grid, cudaStream_t stream) {
-  const size_t es = sizeof(T);
-  auto al = [](const void* q) { return (uintptr_t)q % 16 == 0; };
-  const bool cv = (a.d * es) % 16 == 0 && (!a.e_out || (al(a.e) && al(a.e_out))) &&
-                  (a.e_pos_stride * (long long)es) % 16 == 0 && (a.e_batch_stride * (long long)es) % 16 == 0 &&
-                  (a.cond_copy != kCondCopyM || al(a.hD)) &&
-                  (!a.R_count || (al(a.hD) && al(a.hT) && al(a.apack) && (!a.e_dense || al(a.epack))));
+  const bool cv = copies_vectorised(a, sizeof(T));
   auto kern = cv ? verify_finish_kernel<T, true> : verify_finish_kernel<T, false>;
   return launch_dependent(kern, dim3((unsigned)grid), dim3(kThreads), (size_t)4 * a.B * sizeof(int), stream, 1u, p);
 }
