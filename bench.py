@@ -62,9 +62,9 @@ L2_FLUSH_BYTES = 256 << 20
 # kernel sources it was measured on: `sources` is kernel_sources_hash() at the
 # time, and the line reports null traffic once the sources differ.
 TRAFFIC = {
-    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311306496 + 2842368 + 184312064 + 70656 + 55401984 + 2560
-                                      + 47180544 + 3741952, "sources": "1992adff287baa27"},
-    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 477912576 + 35674368, "sources": "1992adff287baa27"},
+    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311321344 + 2822144 + 184311808 + 85504 + 55400960 + 0
+                                      + 47181312 + 3853824, "sources": "24838df2ab60806b"},
+    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 480060672 + 35517952, "sources": "24838df2ab60806b"},
 }
 
 
