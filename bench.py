@@ -451,8 +451,9 @@ def run_gpu(args) -> dict | None:
     windows = [0, cfg.K + 1] if fused else rt.retrace_verify_plan(cfg.B, cfg.K, cfg.V, cfg.torch_dtype)
     n_pass = len(windows) - 1
     verify_launches = n_pass * (2 if args.sampled else 1) + (1 if n_pass > 1 else 0)
-    # one greedy pass that packs rows for the tensor-core projections hands its
-    # copies to the copy kernel when there are fewer sequences than SMs
+    # one greedy pass that packs rows for the tensor-core projections hands the
+    # decisions and copies to a second kernel when there are fewer sequences
+    # than SMs (the finish kernel; the copy kernel at temperature 1)
     packs = cfg.dtype == "bf16" and (cfg.d % 64 == 0 if args.lowrank
                                      else cfg.d % 256 == 0 and (args.sampled or args.variant in ("corrected", "raw")))
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
@@ -514,7 +515,8 @@ def run_gpu(args) -> dict | None:
             vbytes += d_needed + cfg.B * (cfg.K + 1) * 4
             rbytes += d_rows * cfg.V * cfg.elem_bytes + cfg.B * (cfg.K + 1) * 4
         v_gbs = vbytes / v_avg_s / 1e9
-        copies = " + verify_copy_kernel (copy of unconditioned rows + row packing)"
+        copies = (" + verify_copy_kernel (copy of unconditioned rows + row packing)" if args.sampled else
+                  " (keys only) + verify_finish_kernel (decisions, copy of unconditioned rows + row packing)")
         passes = "sampled_topk_kernel + sampled_finalize_kernel" if args.sampled else "verify_kernel"
         if n_pass > 1:
             finish = (" + verify_finish_kernel (decisions of the last window, copy of unconditioned rows + row "

@@ -617,8 +617,9 @@ __global__ void __launch_bounds__(kThreads, 2) verify_finish_kernel(const Verify
   pdl_launch_dependents();
   pdl_wait();
   const int B = p.B, K = p.K, K1 = K + 1;
-  const int n_last = (int)__ldcg(p.count_in);
-  const int base = (int)__ldcg(p.base_in);
+  // after a single pass (no live lists) every sequence is decided here
+  const int n_last = p.count_in ? (int)__ldcg(p.count_in) : B;
+  const int base = p.base_in ? (int)__ldcg(p.base_in) : 0;
   int* s_first = s_dyn;         // [n_last]
   int* s_off = s_dyn + B;       // [n_last]
   int* s_mapA = s_dyn + 2 * B;  // [B]: accepted length of the sequences decided here, -1 for the others
@@ -627,7 +628,7 @@ __global__ void __launch_bounds__(kThreads, 2) verify_finish_kernel(const Verify
   __syncthreads();
   const int rows = decide_window(p, p.live_in, n_last, p.i0, K1, base, s_first, s_off, nullptr, nullptr, s_warp);
   for (int l = threadIdx.x; l < n_last; l += kThreads) {
-    const int b = __ldcg(p.live_in + l);
+    const int b = p.live_in ? __ldcg(p.live_in + l) : l;
     s_mapA[b] = p.i0 + min(s_first[l], K - p.i0);
     s_mapO[b] = s_off[l];
   }
@@ -817,8 +818,29 @@ cudaError_t launch_typed(const VerifyArgs& a, cudaStream_t stream) {
     if (grid < 1) grid = 1;
     // Row packing for the tensor-core projections with fewer sequences than
     // SMs: each finaliser would copy its sequence's rows on one SM after the
-    // stream has ended, so the copies go to the balanced copy kernel instead.
+    // stream has ended, and the per-sequence arrival tickets of a few
+    // sequences shared by every CTA serialise the end of the pass.  So the
+    // pass only folds keys (as a window [0, K+1) of the windowed schedule),
+    // and verify_finish_kernel decides every sequence, writes the outputs
+    // and does the copies over its grid (target_argmax, every row's argmax,
+    // stays with the finalisers).
     const bool defer = a.R_count && a.B < info.sm_count;
+    if (defer && !a.target_argmax && a.live && a.pass_counts && a.B <= kWindowMaxB) {
+      p.windowed = 1;
+      verify_kernel<T, VEC><<<(unsigned)grid, kThreads, kCopyStageBytes, stream>>>(p);
+      err = cudaGetLastError();
+      if (err != cudaSuccess) return err;
+      p.i0 = 0;
+      p.live_in = nullptr;  // every sequence, no packed rows claimed before
+      p.count_in = nullptr;
+      p.base_in = nullptr;
+      p.pass_counts = a.pass_counts + 1;
+      p.n_counts = 2 * kMaxWindowPasses + 1;
+      p.exits = a.pass_counts;
+      long long fgrid = ((long long)a.B * a.K * 3 + 15) / 16;  // about a warp per row segment
+      if (fgrid > grid_full) fgrid = grid_full;
+      return launch_finish<T>(a, p, fgrid < 1 ? 1 : fgrid, stream);
+    }
     p.defer_copies = defer ? 1 : 0;
     verify_kernel<T, VEC><<<(unsigned)grid, kThreads, kCopyStageBytes, stream>>>(p);
     err = cudaGetLastError();
