@@ -62,9 +62,9 @@ L2_FLUSH_BYTES = 256 << 20
 # kernel sources it was measured on: `sources` is kernel_sources_hash() at the
 # time, and the line reports null traffic once the sources differ.
 TRAFFIC = {
-    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311321344 + 2822144 + 184311808 + 85504 + 55400960 + 0
-                                      + 47181312 + 3853824, "sources": "24838df2ab60806b"},
-    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 480060672 + 35517952, "sources": "24838df2ab60806b"},
+    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311314944 + 2790656 + 184312064 + 451328 + 55402752 + 768
+                                      + 47182336 + 3740928, "sources": "70972efb16841bc9"},
+    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 485058048 + 35867904, "sources": "70972efb16841bc9"},
 }
 
 
