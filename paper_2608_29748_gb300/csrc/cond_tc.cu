@@ -1312,6 +1312,25 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
   // the partial [row][128 features], in the drained pipeline stages (the same offset in every CTA)
   float* P = reinterpret_cast<float*>(dsmem + (base - smem_u32(dsmem)));
   const int kb0 = (int)((long long)rank * p.nkb / S), kb1 = (int)((long long)(rank + 1) * p.nkb / S);
+  // The weight boxes of the first stages are inputs: the producer issues them
+  // before the wait on the previous kernel, and their row boxes after it.
+  const uint32_t tx = (uint32_t)(BM * BK * 2) + (uint32_t)p.tile_n * BK * 2;
+  const int npre = min(SW_STAGES, kb1 - kb0);
+  auto load_a = [&](int kb, uint32_t a_dst, uint32_t bar) {
+    if (p.gate) {  // rows 0-63: W_v rows f0..; rows 64-127: the same rows of W_g[:, d:2d]
+      tma_load_2d(a_dst, &tmA, kb * BK, mt * 64, bar);
+      tma_load_2d(a_dst + (uint32_t)(64 * BK * 2), &tmA2, d + kb * BK, mt * 64, bar);
+    } else {
+      tma_load_2d(a_dst, &tmA, kb * BK, mt * 128, bar);
+    }
+  };
+  if (warp == 0 && lane == 0) {
+    for (int i = 0; i < npre; ++i) {  // every stage is free at the start
+      const uint32_t a_dst = base + (uint32_t)i * p.stage_stride;
+      mbar_arrive_expect_tx(smem_u32(&bar_full[i]), tx);
+      load_a(kb0 + i, a_dst, smem_u32(&bar_full[i]));
+    }
+  }
   pdl_wait();  // R and the activation rows come from the previous kernels
   const int R = *(volatile const int32_t*)p.R;
   const int nrows = (R + 15) / 16 * 16;  // MMA N (at most tile_n)
@@ -1319,28 +1338,32 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
-    if (lane == 0 && work) {
-      const uint32_t tx = (uint32_t)(BM * BK * 2) + (uint32_t)p.tile_n * BK * 2;
-      int kb = kb0;
-      for (; kb < kb1; ++kb) {
-        const int i = kb - kb0;
-        const uint32_t s = (uint32_t)(i % SW_STAGES), ph = (uint32_t)((i / SW_STAGES) & 1);
-        if (!mbar_wait_bounded(smem_u32(&bar_empty[s]), ph ^ 1u, &s_abort)) break;
-        const uint32_t a_dst = base + s * p.stage_stride, b_dst = a_dst + (uint32_t)(BM * BK * 2);
-        mbar_arrive_expect_tx(smem_u32(&bar_full[s]), tx);
-        if (p.gate) {  // rows 0-63: W_v rows f0..; rows 64-127: the same rows of W_g[:, d:2d]
-          tma_load_2d(a_dst, &tmA, kb * BK, mt * 64, smem_u32(&bar_full[s]));
-          tma_load_2d(a_dst + (uint32_t)(64 * BK * 2), &tmA2, d + kb * BK, mt * 64, smem_u32(&bar_full[s]));
-        } else {
-          tma_load_2d(a_dst, &tmA, kb * BK, mt * 128, smem_u32(&bar_full[s]));
+    if (lane == 0) {
+      // the row boxes of the stages issued above (also without work: their
+      // barriers expect them; the boxes stay inside the tensor map)
+      for (int i = 0; i < npre; ++i)
+        tma_load_2d(base + (uint32_t)i * p.stage_stride + (uint32_t)(BM * BK * 2), &tmB, (kb0 + i) * BK, 0,
+                    smem_u32(&bar_full[i]));
+      int kb = kb0 + npre;
+      if (work) {
+        for (; kb < kb1; ++kb) {
+          const int i = kb - kb0;
+          const uint32_t s = (uint32_t)(i % SW_STAGES), ph = (uint32_t)((i / SW_STAGES) & 1);
+          if (!mbar_wait_bounded(smem_u32(&bar_empty[s]), ph ^ 1u, &s_abort)) break;
+          const uint32_t a_dst = base + s * p.stage_stride, b_dst = a_dst + (uint32_t)(BM * BK * 2);
+          mbar_arrive_expect_tx(smem_u32(&bar_full[s]), tx);
+          load_a(kb, a_dst, smem_u32(&bar_full[s]));
+          tma_load_2d(b_dst, &tmB, kb * BK, 0, smem_u32(&bar_full[s]));
         }
-        tma_load_2d(b_dst, &tmB, kb * BK, 0, smem_u32(&bar_full[s]));
       }
-      if (kb < kb1) {  // a wait expired: flag it, let the copies in flight land
-        raise_abort(&s_abort, p.status);
+      if (!work || kb < kb1) {
+        // no MMA consumes the stages (no rows), or a wait expired: let the
+        // copies in flight land before the stages are reused or released
+        if (work) raise_abort(&s_abort, p.status);
         volatile int never = 0;
-        const int first = kb - kb0 > SW_STAGES ? kb - kb0 - SW_STAGES : 0;
-        for (int i = first; i < kb - kb0; ++i)
+        const int issued = kb - kb0;
+        const int first = issued > SW_STAGES ? issued - SW_STAGES : 0;
+        for (int i = first; i < issued; ++i)
           mbar_wait_bounded(smem_u32(&bar_full[i % SW_STAGES]), (uint32_t)((i / SW_STAGES) & 1), &never);
       }
     }
