@@ -1422,55 +1422,67 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
     for (int s = 0; s < 8; ++s) Pr[s] = map_rank_ptr(P, (uint32_t)(s < S ? s : 0));
     const int g0 = (int)((long long)rank * R / S), g1 = (int)((long long)(rank + 1) * R / S);
     if (!p.gate) {
-      // r[g, n0 + f] = m + beta * c for this CTA's rows; two features per thread, a warp 256 bytes of a row
+      // r[g, n0 + f] = m + beta * c for this CTA's rows: four features per
+      // thread (16-byte partial loads, a warp 512 bytes of a row)
       const int n0 = mt * 128;
-      for (int u = threadIdx.x; u < (g1 - g0) * 64; u += SW_THREADS) {
-        const int g = g0 + u / 64, f = (u % 64) * 2;
-        float2 x[8];
+      for (int u = threadIdx.x; u < (g1 - g0) * 32; u += SW_THREADS) {
+        const int g = g0 + u / 32, f = (u % 32) * 4;
+        float4 x[8];
 #pragma unroll
         for (int s = 0; s < 8; ++s)  // all loads first, then the sums in rank order
-          x[s] = s < S ? *reinterpret_cast<const float2*>(Pr[s] + g * 128 + f) : make_float2(0.f, 0.f);
-        const uint32_t mw = __ldcg(reinterpret_cast<const uint32_t*>(p.apack + (long long)g * 2 * d + n0 + f));
+          x[s] = s < S ? *reinterpret_cast<const float4*>(Pr[s] + g * 128 + f) : make_float4(0.f, 0.f, 0.f, 0.f);
+        const uint2 mw = __ldcg(reinterpret_cast<const uint2*>(p.apack + (long long)g * 2 * d + n0 + f));
         const long long orow = p.compact_out ? g : __ldcg(p.rowmap + g);
-        float c0 = 0.f, c1 = 0.f;
+        float c0 = 0.f, c1 = 0.f, c2 = 0.f, c3 = 0.f;
 #pragma unroll
         for (int s = 0; s < 8; ++s) {
           if (s < S) {
             c0 += x[s].x;
             c1 += x[s].y;
+            c2 += x[s].z;
+            c3 += x[s].w;
           }
         }
-        *reinterpret_cast<uint32_t*>(p.r_out + orow * d + n0 + f) =
-            pack_bf16x2(bf16_lo(mw) + p.beta * c0, bf16_hi(mw) + p.beta * c1);
+        *reinterpret_cast<uint2*>(p.r_out + orow * d + n0 + f) =
+            make_uint2(pack_bf16x2(bf16_lo(mw.x) + p.beta * c0, bf16_hi(mw.x) + p.beta * c1),
+                       pack_bf16x2(bf16_lo(mw.y) + p.beta * c2, bf16_hi(mw.y) + p.beta * c3));
       }
     } else {
-      // e~[g, f0 + f] = e + v sigmoid(g_r + ge) for this CTA's rows; two features per thread
+      // e~[g, f0 + f] = e + v sigmoid(g_r + ge) for this CTA's rows: four
+      // features per thread
       const int f0 = mt * 64;
-      for (int u = threadIdx.x; u < (g1 - g0) * 32; u += SW_THREADS) {
-        const int g = g0 + u / 32, f = (u % 32) * 2;
-        float2 xv[8], xa[8];
+      for (int u = threadIdx.x; u < (g1 - g0) * 16; u += SW_THREADS) {
+        const int g = g0 + u / 16, f = (u % 16) * 4;
+        float4 xv[8], xa[8];
 #pragma unroll
         for (int s = 0; s < 8; ++s) {  // all loads first, then the sums in rank order
-          xv[s] = s < S ? *reinterpret_cast<const float2*>(Pr[s] + g * 128 + f) : make_float2(0.f, 0.f);
-          xa[s] = s < S ? *reinterpret_cast<const float2*>(Pr[s] + g * 128 + 64 + f) : make_float2(0.f, 0.f);
+          xv[s] = s < S ? *reinterpret_cast<const float4*>(Pr[s] + g * 128 + f) : make_float4(0.f, 0.f, 0.f, 0.f);
+          xa[s] = s < S ? *reinterpret_cast<const float4*>(Pr[s] + g * 128 + 64 + f) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        const float2 gb = __ldcg(reinterpret_cast<const float2*>(p.ge + f0 + f));
-        const uint32_t ew = __ldg(reinterpret_cast<const uint32_t*>(p.e + f0 + f));
+        const float4 gb = __ldcg(reinterpret_cast<const float4*>(p.ge + f0 + f));
+        const uint2 ew = __ldg(reinterpret_cast<const uint2*>(p.e + f0 + f));
         const long long orow = __ldcg(p.rowmap + g);
-        float v0 = 0.f, v1 = 0.f, a0 = 0.f, a1 = 0.f;
+        float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f, a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
         for (int s = 0; s < 8; ++s) {
           if (s < S) {
             v0 += xv[s].x;
             v1 += xv[s].y;
+            v2 += xv[s].z;
+            v3 += xv[s].w;
             a0 += xa[s].x;
             a1 += xa[s].y;
+            a2 += xa[s].z;
+            a3 += xa[s].w;
           }
         }
         a0 += gb.x;
         a1 += gb.y;
-        *reinterpret_cast<uint32_t*>(p.e_out + orow * d + f0 + f) =
-            pack_bf16x2(bf16_lo(ew) + v0 * fast_sigmoid(a0), bf16_hi(ew) + v1 * fast_sigmoid(a1));
+        a2 += gb.z;
+        a3 += gb.w;
+        *reinterpret_cast<uint2*>(p.e_out + orow * d + f0 + f) =
+            make_uint2(pack_bf16x2(bf16_lo(ew.x) + v0 * fast_sigmoid(a0), bf16_hi(ew.x) + v1 * fast_sigmoid(a1)),
+                       pack_bf16x2(bf16_lo(ew.y) + v2 * fast_sigmoid(a2), bf16_hi(ew.y) + v3 * fast_sigmoid(a3)));
       }
     }
   }
