@@ -62,9 +62,9 @@ L2_FLUSH_BYTES = 256 << 20
 # kernel sources it was measured on: `sources` is kernel_sources_hash() at the
 # time, and the line reports null traffic once the sources differ.
 TRAFFIC = {
-    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311314944 + 2790656 + 184312064 + 451328 + 55402752 + 768
-                                      + 47182336 + 3740928, "sources": "70972efb16841bc9"},
-    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 485058048 + 35867904, "sources": "70972efb16841bc9"},
+    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311306496 + 3006720 + 184319744 + 110336 + 55402496 + 768
+                                      + 47179264 + 3846400, "sources": "cdd24785f661454a"},
+    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 484482560 + 35706880, "sources": "cdd24785f661454a"},
 }
 
 

@@ -611,7 +611,7 @@ __global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
 // CTAs takes a 256-row pair tile, each CTA staging its own 128 rows of A and
 // half of the N = 256 weight tile (correction: W_c rows n0.. and n0+128..;
 // gate: the W_v rows in the leader, the matching W_g[:, d:2d] rows in the
-// follower), so a stage is 32 KB per SM instead of 48 KB and six stages fit.
+// follower), so a stage is 32 KB per SM instead of 48 KB and seven stages fit.
 // The leader's MMA thread issues M256 N256 K16 MMAs that read both CTAs'
 // shared memory and accumulate into both CTAs' tensor memory (each CTA's
 // TMEM lanes are its own 128 rows); its commits arrive on both CTAs'
@@ -619,7 +619,7 @@ __global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
 // bytes of both CTAs' copies.  The leader takes tiles from the global queue
 // and hands each to the follower through the follower's shared memory.  A
 // broadcast e only (per-position e takes cond_kernel).  Every wait is bounded.
-constexpr int PSTAGES = 6;
+constexpr int PSTAGES = 7;
 constexpr int P_THREADS = 256;
 constexpr int P_A_BYTES = BM * BK * 2;   // 16 KB: this CTA's 128 rows
 constexpr int P_B_BYTES = 128 * BK * 2;  // 16 KB: this CTA's half of the weight tile
