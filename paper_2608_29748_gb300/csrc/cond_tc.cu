@@ -611,7 +611,11 @@ __global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
 // CTAs takes a 256-row pair tile, each CTA staging its own 128 rows of A and
 // half of the N = 256 weight tile (correction: W_c rows n0.. and n0+128..;
 // gate: the W_v rows in the leader, the matching W_g[:, d:2d] rows in the
-// follower), so a stage is 32 KB per SM instead of 48 KB and seven stages fit.
+// follower).  A stage is 128 deep in K (two 64-element swizzle boxes per
+// operand, 64 KB per SM): three stages fit.  With 64-deep stages (32 KB,
+// seven of them) the round at B = 256 ran 252.0 against 247.9 us, with
+// 32-deep ones (fourteen) 434 us: each stage costs a fixed handshake (full
+// wait, commit, empty wait, copies issued), which deeper stages amortise.
 // The leader's MMA thread issues M256 N256 K16 MMAs that read both CTAs'
 // shared memory and accumulate into both CTAs' tensor memory (each CTA's
 // TMEM lanes are its own 128 rows); its commits arrive on both CTAs'
@@ -619,10 +623,12 @@ __global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
 // bytes of both CTAs' copies.  The leader takes tiles from the global queue
 // and hands each to the follower through the follower's shared memory.  A
 // broadcast e only (per-position e takes cond_kernel).  Every wait is bounded.
-constexpr int PSTAGES = 7;
+constexpr int PSTAGES = 3;
 constexpr int P_THREADS = 256;
-constexpr int P_A_BYTES = BM * BK * 2;   // 16 KB: this CTA's 128 rows
-constexpr int P_B_BYTES = 128 * BK * 2;  // 16 KB: this CTA's half of the weight tile
+constexpr int PBK = 2 * BK;                      // k-block depth of a stage: two swizzle boxes
+constexpr int P_BOX_BYTES = 128 * BK * 2;        // 16 KB: one 128-row, 64-element box
+constexpr int P_A_BYTES = 2 * P_BOX_BYTES;       // 32 KB: this CTA's 128 rows
+constexpr int P_B_BYTES = 2 * P_BOX_BYTES;       // 32 KB: this CTA's half of the weight tile
 constexpr int P_STAGE_BYTES = P_A_BYTES + P_B_BYTES;
 constexpr int P_SMEM_BYTES = PSTAGES * P_STAGE_BYTES + 1024;  // + slack for 1024-B alignment
 constexpr uint32_t IDESC_M256_N256 = idesc_bf16_f32(256, 256);
@@ -696,7 +702,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = s_tmem;
   const uint32_t base = (smem_u32(dsmem) + 1023u) & ~1023u;
-  const int kb_half = d / BK;
+  const int kb_half = d / PBK;
   // The set-up above may overlap the end of the previous kernel (programmatic
   // dependent launch).  R, the packed rows and the row map are its outputs:
   // every role that reads them waits here first.  The gate-bias GEMV (warps
@@ -790,11 +796,17 @@ __global__ void __launch_bounds__(P_THREADS, 1)
           const uint32_t a_dst = base + s * P_STAGE_BYTES, b_dst = a_dst + P_A_BYTES;
           const uint32_t full = leader_addr(&bar_full[s]);
           if (leader) mbar_arrive_expect_tx(smem_u32(&bar_full[s]), 2 * P_STAGE_BYTES);  // both CTAs' bytes
-          tma_load_2d_pair(a_dst, corr ? &tmApack : &tmR, kb * BK, m0, full);  // [m; u] or r rows
-          if (corr)  // this CTA's half of the weight tile: rows n0.. (leader) or n0 + 128.. (follower)
-            tma_load_2d_pair(b_dst, &tmWc, kb * BK, n0 + (int)rank * 128, full);
-          else  // W_v rows (leader) and the matching W_g[:, d:2d] rows (follower)
-            tma_load_2d_pair(b_dst, leader ? &tmWv : &tmWg, leader ? kb * BK : d + kb * BK, n0, full);
+          // [m; u] or r rows; this CTA's half of the weight tile: W_c rows n0..
+          // (leader) or n0 + 128.. (follower), or the W_v rows (leader) and the
+          // matching W_g[:, d:2d] rows (follower); each as two 64-element boxes
+          const CUtensorMap* mb = corr ? &tmWc : (leader ? &tmWv : &tmWg);
+          const int xb = (corr || leader) ? kb * PBK : d + kb * PBK;
+          const int yb = corr ? n0 + (int)rank * 128 : n0;
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            tma_load_2d_pair(a_dst + (uint32_t)h * P_BOX_BYTES, corr ? &tmApack : &tmR, kb * PBK + h * BK, m0, full);
+            tma_load_2d_pair(b_dst + (uint32_t)h * P_BOX_BYTES, mb, xb + h * BK, yb, full);
+          }
         }
         if (!ok) break;
         if (leader && !ahead && !publish(lt + 1, dequeue())) ok = false;  // near the end: claim at the switch
@@ -840,11 +852,15 @@ __global__ void __launch_bounds__(P_THREADS, 1)
           }
           tc_fence_after();
           const uint32_t a_base = base + s * P_STAGE_BYTES, b_base = a_base + P_A_BYTES;
-          // K16 steps advance the start address by 32 bytes: + 2 in the descriptor's address field
+          // K16 steps advance the start address by 32 bytes (+ 2 in the
+          // descriptor's address field) inside a box, by the box's 16 KB (+ 1024)
+          // from the first box to the second
           const uint64_t adesc0 = sw128_kmajor_desc(a_base), bdesc0 = sw128_kmajor_desc(b_base);
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)
-            tc_mma_pair(d_tmem, adesc0 + 2u * k, bdesc0 + 2u * k, IDESC_M256_N256, (kb > 0 || k > 0) ? 1u : 0u);
+          for (int k = 0; k < PBK / 16; ++k) {
+            const uint64_t step = (uint64_t)((k / (BK / 16)) * (P_BOX_BYTES >> 4) + 2 * (k % (BK / 16)));
+            tc_mma_pair(d_tmem, adesc0 + step, bdesc0 + step, IDESC_M256_N256, (kb > 0 || k > 0) ? 1u : 0u);
+          }
           tc_commit_pair(smem_u32(&bar_empty[s]));  // stage free in both CTAs
         }
         tc_commit_pair(smem_u32(&bar_tfull[acc]));  // accumulator ready (also after a failure)
