@@ -62,9 +62,9 @@ L2_FLUSH_BYTES = 256 << 20
 # kernel sources it was measured on: `sources` is kernel_sources_hash() at the
 # time, and the line reports null traffic once the sources differ.
 TRAFFIC = {
-    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311306496 + 3006720 + 184319744 + 110336 + 55402496 + 768
-                                      + 47179264 + 3846400, "sources": "cdd24785f661454a"},
-    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 484482560 + 35706880, "sources": "cdd24785f661454a"},
+    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311307776 + 2760704 + 184310272 + 181248 + 55402752 + 3840
+                                      + 47180288 + 3880960, "sources": "8c5f885e642229d4"},
+    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 507987200 + 36986880, "sources": "8c5f885e642229d4"},
 }
 
 
