@@ -63,8 +63,8 @@ L2_FLUSH_BYTES = 256 << 20
 # time, and the line reports null traffic once the sources differ.
 TRAFFIC = {
     ("verify", "qwen3-8b-B256-K16"): {"bytes": 311307776 + 2760704 + 184310272 + 181248 + 55402752 + 3840
-                                      + 47180288 + 3880960, "sources": "8c5f885e642229d4"},
-    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 507987200 + 36986880, "sources": "8c5f885e642229d4"},
+                                      + 47180288 + 3880960, "sources": "84b83736dcaf6c47"},
+    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 507987200 + 36986880, "sources": "84b83736dcaf6c47"},
 }
 
 

@@ -612,10 +612,11 @@ __global__ void __launch_bounds__(FUSED ? THREADS_FUSED : THREADS, 1)
 // half of the N = 256 weight tile (correction: W_c rows n0.. and n0+128..;
 // gate: the W_v rows in the leader, the matching W_g[:, d:2d] rows in the
 // follower).  A stage is 128 deep in K (two 64-element swizzle boxes per
-// operand, 64 KB per SM): three stages fit.  With 64-deep stages (32 KB,
-// seven of them) the round at B = 256 ran 252.0 against 247.9 us, with
-// 32-deep ones (fourteen) 434 us: each stage costs a fixed handshake (full
-// wait, commit, empty wait, copies issued), which deeper stages amortise.
+// operand, 64 KB per SM): three stages fit.  Each stage costs a fixed
+// handshake (full wait, commit, empty wait, copies issued), which deeper
+// stages amortise: at B = 256 the kernel took 251.9 us with seven 64-deep
+// stages, 245.3 us with three 128-deep ones, 283 us with two 192-deep ones
+// and 434 us with fourteen 32-deep ones.
 // The leader's MMA thread issues M256 N256 K16 MMAs that read both CTAs'
 // shared memory and accumulate into both CTAs' tensor memory (each CTA's
 // TMEM lanes are its own 128 rows); its commits arrive on both CTAs'
