@@ -62,9 +62,9 @@ L2_FLUSH_BYTES = 256 << 20
 # kernel sources it was measured on: `sources` is kernel_sources_hash() at the
 # time, and the line reports null traffic once the sources differ.
 TRAFFIC = {
-    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311307776 + 2760704 + 184310272 + 181248 + 55402752 + 3840
-                                      + 47180288 + 3880960, "sources": "84b83736dcaf6c47"},
-    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 507987200 + 36986880, "sources": "84b83736dcaf6c47"},
+    ("verify", "qwen3-8b-B256-K16"): {"bytes": 311308288 + 2800384 + 184310272 + 138752 + 55403264 + 0
+                                      + 47179520 + 4033792, "sources": "c403a58964d4ce6e"},
+    ("conditioning", "qwen3-8b-B256-K16"): {"bytes": 509979136 + 37198080, "sources": "c403a58964d4ce6e"},
 }
 
 

@@ -269,6 +269,7 @@ retrace_status enqueue_conditioning(const ConditioningArgs& c, retrace_dtype dty
     a.sync = sync;
     a.status = status_word(ws);
     a.part = swap_part_bytes(B, K, d) ? reinterpret_cast<float*>(reinterpret_cast<char*>(ws) + L.swp) : nullptr;
+    a.split_part = pair_split_bytes(B, K, d, 2) ? reinterpret_cast<float*>(w + L.swp) : nullptr;
     RT_CUDA(launch_cond_tc(a, stream), "conditioning kernel launch");
     if (phase_events) RT_CUDA(cudaEventRecord(phase_events[2], stream), "cudaEventRecord");
   } else {
@@ -446,6 +447,7 @@ retrace_status retrace_gate_fuse(const void* e, int64_t e_batch_stride, int64_t 
     a.sync = sync;
     a.status = status_word(ws);
     a.part = swap_part_bytes(B, K, d) ? reinterpret_cast<float*>(reinterpret_cast<char*>(ws) + L.swp) : nullptr;
+    a.split_part = pair_split_bytes(B, K, d, 2) ? reinterpret_cast<float*>(w + L.swp) : nullptr;
     RT_CUDA(launch_cond_tc(a, stream), "gate kernel launch");
   } else {
     if (!dense) RT_CUDA(launch_gate_bias(Wg, e, d, ge, dtype, stream), "gate bias kernel launch");

@@ -161,6 +161,14 @@ struct CondParams {
   uint32_t* block_done;   // per 128-row block: correction epilogue warps finished
   uint32_t* block_ready;  // per 128-row block: packed rows published (FUSED)
   int max_blocks;         // 128-row blocks of the largest possible R
+  // CTA-pair kernel: the gate tiles of a last wave of at most split_max
+  // tiles run as two K halves on two pairs.  Each half writes its fp32
+  // accumulator to split_part and counts on split_ticket; the half that
+  // counts second adds the other's accumulator to its own and runs the
+  // epilogue.
+  float* split_part;
+  uint32_t* split_ticket;
+  int split_max;
   uint32_t* status;
 };
 
@@ -205,7 +213,10 @@ __device__ __forceinline__ void epilogue_correction(const CondParams& p, uint32_
 // the 128 features n0.., v in accumulator columns 0..127, the r half of the
 // gate in 128..255 (plus W_g[:, :d] e from ge for a broadcast e, the same
 // 32 values for every lane: one 16-byte broadcast load per four features).
-__device__ __forceinline__ void epilogue_gate(const CondParams& p, uint32_t taddr, int g, bool valid, int n0, int d) {
+// With `other` (a split tile), the other K half's accumulator of this row is
+// added first: column c at other[128 c].
+__device__ __forceinline__ void epilogue_gate(const CondParams& p, uint32_t taddr, int g, bool valid, int n0, int d,
+                                              const float* other = nullptr) {
   const long long orow = valid ? __ldcg(p.rowmap + g) : 0;
   const __nv_bfloat16* erow = p.e + (p.e_dense ? (long long)g * d : 0);
   for (int cc = 0; cc < 4; ++cc) {
@@ -214,6 +225,13 @@ __device__ __forceinline__ void epilogue_gate(const CondParams& p, uint32_t tadd
     tmem_ld_32cols(taddr + 128u + (uint32_t)(cc * 32), gt);
     if (valid) {
       const int n = n0 + cc * 32;
+      if (other) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          v[i] += __ldcg(other + (cc * 32 + i) * 128);
+          gt[i] += __ldcg(other + (128 + cc * 32 + i) * 128);
+        }
+      }
       if (!p.e_dense) {
         const float4* gb = reinterpret_cast<const float4*>(p.ge + n);
 #pragma unroll
@@ -709,24 +727,59 @@ __global__ void __launch_bounds__(P_THREADS, 1)
   // every role that reads them waits here first.  The gate-bias GEMV (warps
   // 2-3) reads only the inputs and starts at once.  With R = 0 the queue's
   // first claim already ends every role.
-  int R = 0, T0 = 0, T = 0, pairs_m = 0;
+  int R = 0, T0 = 0, T1 = 0, X = 0, T = 0, pairs_m = 0;
   if (warp != 2 && warp != 3) {
     pdl_wait();
     R = *(volatile const int32_t*)p.R;
     pairs_m = (R + 2 * BM - 1) / (2 * BM);
     T0 = p.do_correct ? pairs_m * nt0 : 0;
-    T = T0 + (p.do_gate ? pairs_m * nt1 : 0);
+    T1 = p.do_gate ? pairs_m * nt1 : 0;
+    // the last wave: work units (a gate tile's worth of MMAs) beyond the
+    // whole waves of the pairs
+    const int last_wave = (2 * T0 + T1) % (int)(gridDim.x / 2);
+    X = last_wave <= p.split_max ? min(last_wave, T1) : 0;
+    T = T0 + T1 + X;
   }
   // Tile t: correction tiles first, then gate tiles; within each kind, groups
   // of kGroupBlocks pair blocks with the weight tile outer inside a group.
-  auto decode = [&](int t, bool* corr, int* m0, int* n0) {
-    *corr = t < T0;
-    const int tt = *corr ? t : t - T0, nt = *corr ? nt0 : nt1;
+  // When the last wave of the queue would keep only a few pairs busy (at
+  // most split_max tiles), its X gate tiles come as two K halves each (2X
+  // queue entries, the halves of a tile next to each other), so that twice
+  // as many pairs share it.  At B = 256 (12 pair blocks, 768 units on 76
+  // pairs, 8 in the last wave) the kernel went from 245.8-247.9 to
+  // 241.7-243.8 us.  Splitting 16 or 38 tiles whatever the last wave made
+  // B = 128 slower (141.4 -> 159.8 us), where splitting 4 or 8 left it
+  // unchanged.
+  struct Tile {
+    bool corr;
+    int m0, n0;    // this CTA's first row; first output column (correction) or feature (gate)
+    int kb0, nkb;  // k-blocks of PBK
+    int split;     // -1, or the split tile (0..X-1) whose K half `half` this is
+    int half;
+  };
+  auto decode = [&](int t) {
+    Tile x;
+    x.corr = t < T0;
+    int tt = x.corr ? t : t - T0;
+    x.kb0 = 0;
+    x.nkb = x.corr ? 2 * kb_half : kb_half;
+    x.split = -1;
+    x.half = 0;
+    if (!x.corr && tt >= T1 - X) {
+      const int j = tt - (T1 - X);
+      x.split = j >> 1;
+      x.half = j & 1;
+      tt = T1 - X + x.split;
+      x.nkb = kb_half / 2;
+      x.kb0 = x.half * x.nkb;
+    }
+    const int nt = x.corr ? nt0 : nt1;
     const int g = tt / (kGroupBlocks * nt), w = tt - g * kGroupBlocks * nt;
     const int glen = min(kGroupBlocks, pairs_m - g * kGroupBlocks);
     const int pb = g * kGroupBlocks + w % glen;  // pair block
-    *m0 = pb * 2 * BM + (int)rank * BM;          // this CTA's rows
-    *n0 = (w / glen) * (*corr ? 256 : 128);
+    x.m0 = pb * 2 * BM + (int)rank * BM;         // this CTA's rows
+    x.n0 = (w / glen) * (x.corr ? 256 : 128);
+    return x;
   };
   // the leader's barriers as seen from either CTA
   auto leader_addr = [&](const void* local) { return map_rank(smem_u32(local), 0); };
@@ -776,10 +829,9 @@ __global__ void __launch_bounds__(P_THREADS, 1)
           mbar_arrive_remote(leader_addr(&bar_tile_empty[slot]));
         }
         if (t < 0) break;
-        bool corr;
-        int m0, n0;
-        decode(t, &corr, &m0, &n0);
-        const int nkb = corr ? 2 * kb_half : kb_half;
+        const Tile x = decode(t);
+        const bool corr = x.corr;
+        const int m0 = x.m0, n0 = x.n0;
         if (!corr && p.do_correct) {
           // the r rows of this CTA's block are written by the correction epilogues
           if (!wait_counter(block_done + m0 / BM, (uint32_t)(4 * nt0), &s_abort)) {
@@ -788,7 +840,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
           }
           fence_proxy_async_global();
         }
-        for (int kb = 0; kb < nkb; ++kb, ++it) {
+        for (int kb = x.kb0; kb < x.kb0 + x.nkb; ++kb, ++it) {
           const uint32_t s = it % PSTAGES, ph = (it / PSTAGES) & 1u;
           if (!mbar_wait_bounded(smem_u32(&bar_empty[s]), ph ^ 1u, &s_abort)) {
             ok = false;
@@ -837,7 +889,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
         const int t = s_tile[slot];
         mbar_arrive(smem_u32(&bar_tile_empty[slot]));
         if (t < 0) break;
-        const int nkb = t < T0 ? 2 * kb_half : kb_half;
+        const int nkb = decode(t).nkb;
         const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
         if (!mbar_wait_cluster_bounded(smem_u32(&bar_tempty[acc]), aph ^ 1u, &s_abort)) {
           ok = false;
@@ -892,9 +944,9 @@ __global__ void __launch_bounds__(P_THREADS, 1)
         else mbar_arrive_remote(leader_addr(&bar_tile_empty[slot]));
       }
       if (t < 0) break;
-      bool corr;
-      int m0, n0;
-      decode(t, &corr, &m0, &n0);
+      const Tile x = decode(t);
+      const bool corr = x.corr;
+      const int m0 = x.m0, n0 = x.n0;
       const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
       ok = warp_wait(smem_u32(&bar_tfull[acc]), aph, &s_abort);
       tc_fence_after();
@@ -924,8 +976,33 @@ __global__ void __launch_bounds__(P_THREADS, 1)
           __syncwarp();
           if (lane == 0) atomicAdd(block_done + m0 / BM, 1u);
         }
-      } else {
+      } else if (x.split < 0) {
         epilogue_gate(p, taddr, g, valid, n0, d);
+      } else {
+        // A K half: this row's accumulator goes to the half's slot ([column][row]
+        // per CTA, so that a warp's stores are contiguous); the warp that counts
+        // second on the ticket of its 32 rows adds the other half's slot and
+        // runs the epilogue.  Fence before the count, fence after it (the
+        // last-arriver pattern): no wait on the other pair.
+        const size_t slot_floats = (size_t)2 * BM * 128;
+        float* own = p.split_part + ((size_t)(x.split * 2 + x.half) * 2 + rank) * slot_floats + q;
+        const float* other = p.split_part + ((size_t)(x.split * 2 + (x.half ^ 1)) * 2 + rank) * slot_floats + q;
+        for (int cc = 0; cc < 8; ++cc) {
+          float c[32];
+          tmem_ld_32cols(taddr + (uint32_t)(cc * 32), c);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) __stcg(own + (cc * 32 + i) * 128, c[i]);
+        }
+        __threadfence();
+        __syncwarp();
+        uint32_t before = 0;
+        if (lane == 0) {
+          before = atomicAdd(p.split_ticket + x.split * 8 + (int)rank * 4 + (warp - 4), 1u);
+          __threadfence();
+        }
+        before = __shfl_sync(0xFFFFFFFFu, before, 0);
+        __syncwarp();
+        if (before == 1u) epilogue_gate(p, taddr, g, valid, n0, d, other);
       }
       tc_fence_before();
       __syncwarp();
@@ -1591,6 +1668,9 @@ static cudaError_t launch_cond_pair(const TcCondArgs& a, int clusters, cudaStrea
   p.sync = a.sync;
   p.block_done = a.sync + kSyncBlocks;
   p.block_ready = a.sync + kSyncBlocks + blocks_max(a.B, a.K);
+  p.split_part = a.split_part;
+  p.split_ticket = a.sync + kSyncBlocks + 2 * blocks_max(a.B, a.K);
+  p.split_max = (a.split_part && a.do_gate) ? kPairSplitTiles : 0;
   p.status = a.status;
   // clusters of two CTAs; set-up may overlap the previous kernel's end
   return launch_dependent(cond_pair_kernel, dim3(2 * (unsigned)clusters), dim3(P_THREADS), P_SMEM_BYTES, stream, 2,

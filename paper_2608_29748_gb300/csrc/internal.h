@@ -6,6 +6,7 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <algorithm>
 #include <atomic>
 
 #include "../../include/retrace.h"
@@ -39,7 +40,8 @@ constexpr int kLowRankLatent = 64;      // rank of the rejected-suffix latents
 constexpr int kLowRankCorrection = 32;  // rank of the target-aware correction
 constexpr int kLowRankSplits = 8;       // split-K parts per half of the [m; u] reduction
 //   skeys    uint64 [B*(2K+1), 64]  sampled verification: top-k keys per target and drafter row
-//   swp      fp32   (small R only)  split partials of the small-R conditioning GEMMs
+//   swp      fp32                   split partials of the small-R conditioning GEMMs, or the
+//                                   K halves of the CTA-pair kernel's split gate tiles
 constexpr int kMaxTopK = 64;            // largest top_k of sampled verification
 constexpr int kWindowRows = 4;          // rows per pass of windowed verification
 constexpr int kMaxWindowPasses = 16;    // most passes of windowed verification
@@ -59,6 +61,17 @@ inline size_t swap_part_bytes(long long B, long long K, long long d) {
   const long long box = rows < 256 ? rows : 256;
   return (size_t)(kSwapMaxCtas * 128 * box * 4);
 }
+// CTA-pair conditioning (every other bf16 shape with d a multiple of 256): a
+// last wave of at most kPairSplitTiles gate tiles runs as two K halves per
+// tile on two pairs.  Each half writes its fp32 accumulator (two CTAs x 128
+// rows x 256 columns) to the same region as the small-R partials, and counts
+// on one ticket per CTA and epilogue warp in the sync area.
+constexpr int kPairSplitTiles = 8;
+inline size_t pair_split_bytes(long long B, long long K, long long d, size_t elem) {
+  const long long rmax = B * (K > 1 ? K - 1 : 0);
+  if (rmax <= 0 || elem != 2 || d <= 0 || d % 256 != 0 || swap_part_bytes(B, K, d) != 0) return 0;
+  return (size_t)kPairSplitTiles * 2 * 2 * 128 * 256 * 4;
+}
 struct WsLayout {
   size_t status, sync, sync_bytes, keys, tickets, live, poff, counts, ge, r, apack, epack, rowmap, lrz, lrt, lrrho, skeys, swp, total;
 };
@@ -72,7 +85,8 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   L.status = off;
   off = align_up(off + 64 * 4, 256);
   L.sync = off;
-  L.sync_bytes = align_up((size_t)(32 + 2 * ((rmax + 255) / 256 * 2)) * 4, 256);  // 2 x blocks_max
+  // 2 x blocks_max, then the split tickets
+  L.sync_bytes = align_up((size_t)(32 + 2 * ((rmax + 255) / 256 * 2) + 8 * kPairSplitTiles) * 4, 256);
   off += L.sync_bytes;
   L.keys = off;
   off = align_up(off + (size_t)(B * (K + 1)) * 8, 256);
@@ -103,7 +117,7 @@ inline WsLayout ws_layout(long long B, long long K, long long d, size_t elem) {
   L.skeys = off;
   off = align_up(off + (size_t)(B * (2 * K + 1)) * kMaxTopK * 8, 256);
   L.swp = off;
-  off = align_up(off + swap_part_bytes(B, K, d), 256);
+  off = align_up(off + std::max(swap_part_bytes(B, K, d), pair_split_bytes(B, K, d, elem)), 256);
   L.total = off;
   return L;
 }
@@ -296,6 +310,8 @@ cudaError_t launch_pack(const PackArgs& a, cudaStream_t stream);
 //   [kSyncChunkNext]  next group of logits chunks to stream (fused round)
 //   [kSyncBlocks ...]            per 128-row block: correction epilogue warps done
 //   [kSyncBlocks + blocks ...]   per 128-row block: packed rows published (fused round)
+//   [kSyncBlocks + 2 blocks ...] per split gate tile, CTA of the pair and epilogue warp:
+//                                K halves finished (CTA-pair kernel; 8 kPairSplitTiles)
 constexpr int kSyncRowCount = 0;
 constexpr int kSyncTileQueue = 1;
 constexpr int kSyncGemvNext = 2;
@@ -336,6 +352,8 @@ struct TcCondArgs {
   uint32_t* status;
   // small-R path (B (K-1) <= kSwapMaxRows): fp32 split partials, swap_part_bytes (NULL: not taken)
   float* part;
+  // CTA-pair path: fp32 accumulators of the split gate tiles, pair_split_bytes (NULL: no split tiles)
+  float* split_part;
 };
 cudaError_t launch_cond_tc(const TcCondArgs& a, cudaStream_t stream);
 // The bounded waits of the pipelined kernels on a caller-controlled condition.

@@ -253,5 +253,24 @@ def test_workspace_holds_small_r_partials(lib):
         part = 256 * 128 * min(256, rows) * 4
         assert ws(B, K, 1000, d, BF16) >= part
     small = ws(64, 17, 1000, 4096, BF16)   # 1024 rows: partials of 32 MiB
-    large = ws(65, 17, 1000, 4096, BF16)   # 1040 rows: the CTA-pair path, no partials
-    assert small - large > 30 << 20
+    large = ws(65, 17, 1000, 4096, BF16)   # 1040 rows: the CTA-pair path, 4 MiB of split-tile halves
+    assert (32 - 4 - 1) << 20 < small - large < (32 - 4) << 20
+    # fp32 takes the FFMA path: neither partial region
+    assert ws(65, 17, 1000, 4096, F32) < ws(64, 17, 1000, 4096, F32) - (30 << 20)
+
+
+def test_workspace_holds_pair_split_halves(lib):
+    """Beyond the small-R path (bf16, d a multiple of 256) the workspace holds
+    the K halves of the CTA-pair kernel's split gate tiles: 8 tiles x 2 halves
+    x 2 CTAs x 128 rows x 256 fp32 columns, and their tickets in the sync area."""
+    ws = lib.retrace_workspace_bytes
+    split = 8 * 2 * 2 * 128 * 256 * 4
+    for B, K, d in ((65, 17, 4096), (256, 16, 4096), (128, 16, 2560 + 256)):
+        rows = B * (K - 1)
+        # r, apack, epack (bf16) and the row map come on top of the split halves
+        assert ws(B, K, 1000, d, BF16) > split + rows * d * 2 * 4
+    # d not a multiple of 256 takes the FFMA path, without split halves: from
+    # d = 4096 to 4224 the d-sized buffers grow by half as much as from 3840 to
+    # 4096, and the split region goes
+    a, b, c = (ws(256, 16, 1000, dd, BF16) for dd in (3840, 4096, 4224))
+    assert abs((c - b) - ((b - a) // 2 - split)) <= 4096
